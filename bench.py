@@ -1,0 +1,363 @@
+"""Benchmark: candidate plans evaluated per second on the burst-arrival window
+(64 sessions, N=2000 activations, D=8 devices, M=8 models, P=16,384 plans per
+GPU), plus the evaluation kernel's achieved HBM bandwidth against the measured
+copy peak.
+
+One step = the whole hot path over one batch: readiness forecast, evaluation
+of every plan, top-k.  Inputs are resident in HBM before the timed region; L2
+is flushed (a 256 MiB write) between timed steps, which are timed one by one
+with CUDA events on the library's stream.  ``e2e`` repeats the step through
+the public call with the plans in pinned host memory, the host-to-device copy
+and the read-back of the top-k inside the timed region.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gpu|reference]
+
+Under torchrun every rank evaluates its own batch (plan indices offset by
+rank * P; weak scaling) and rank 0 prints one JSON line.  ``--impl reference``
+times the CPU oracle on the host cores on a bounded sample of the same batch.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+WORKLOAD = "burst"
+METRIC = "candidate plans evaluated/sec (N=2000,D=8)"
+L2_FLUSH_BYTES = 256 << 20
+
+
+def algorithmic_bytes_per_plan(N: int) -> int:
+    """Compulsory traffic of one plan: place (N B) + order (2N B) + fusion and
+    prefetch bits (2 ceil(N/8) B) read, makespan / p95 / GPU time (3 x 8 B) and
+    status (4 B) written."""
+    return N + 2 * N + 2 * ((N + 7) // 8) + 28
+
+
+def topk_launches(P: int, k: int, tile: int = 2048) -> int:
+    """Kernel launches of one wf_topk call (mirrors the library's pass plan)."""
+    tiles = (P + tile - 1) // tile
+    if tiles == 1:
+        return 2
+    n, launches = tiles * k, 1
+    while n > tile:
+        tiles = (n + tile - 1) // tile
+        n = tiles * k
+        launches += 1
+    return launches + 1
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    for f in ("wf_eval.cu", "wf_internal.cuh"):
+        with open(os.path.join(ROOT, "paper_2609_03335_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def read_peaks() -> dict:
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f)
+    except OSError:
+        return {}
+
+
+def read_traffic(workload: str):
+    """DRAM bytes per launch of the evaluation kernel from the committed ncu
+    summary, only if it was taken on the current kernel source."""
+    path = os.path.join(ROOT, "profiles", "eval_traffic.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+    except OSError:
+        return None, None
+    if d.get("kernel_hash") != kernel_source_hash() or workload not in d.get("per_launch", {}):
+        return None, d.get("kernel_hash")
+    return d["per_launch"][workload], d.get("kernel_hash")
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 50 ms."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = os.path.join("/tmp", f"wf_clocks_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        self.proc.wait()
+        sm, smax, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower() == "active":
+                        reasons.add(n)
+        os.unlink(self.path)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+        load = [s for s in sm if s > 0.5 * max(sm)] or sm
+        return {"sm_mhz": float(np.median(load)), "sm_max_mhz": float(max(smax)),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if os.environ.get("WF_BENCH_BACKEND", "nccl") == "nccl" else "gloo"
+        dist.init_process_group(backend=backend)
+    return rank, world, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda" if dist.get_backend() == "nccl" else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def run_reference(args, rank, world):
+    """The CPU oracle, as it stands, timed on the host cores."""
+    import oracle
+    import wfgen
+    if rank != 0:
+        return
+    w = wfgen.config(WORKLOAD)
+    sample = 1024
+    plans = wfgen.make_plans(w.problem, sample, w.plan_seed)
+    oracle.build()
+    for _ in range(args.warmup):
+        oracle.eval_plans(w.problem, plans, 0, 64)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle.eval_plans(w.problem, plans)
+    dt = (time.perf_counter() - t0) / args.steps
+    value = sample / dt
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "plans/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64",
+        "data": "synthetic",
+        "config": {"workload": f"{WORKLOAD}: 64 sessions, N=2000, D=8, M=8; oracle step = first "
+                               f"{sample} plans of the batch", "P": sample, "N": w.problem.N},
+        "cpu_baseline": {"value": value, "unit": "plans/s", "cores": 1, "kind": "oracle",
+                         "sample": f"first {sample} plans of the burst batch per step, one thread"},
+        "e2e": {"value": value, "unit": "plans/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def run_gpu(args, rank, world, local):
+    import torch
+
+    import wfgen
+    from paper_2609_03335_gb300 import build as pkg_build
+    from paper_2609_03335_gb300 import wf
+    pkg_build.build()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    w = wfgen.config(WORKLOAD)
+    prob, P, k = w.problem, w.P, w.k
+    plans = wfgen.make_plans(prob, P, w.plan_seed, plan_base=rank * P)
+    t0 = time.perf_counter()
+    ctx = wf.Ctx(prob, max_P=P, device=local)
+    torch.cuda.synchronize()
+    ctx_ms = (time.perf_counter() - t0) * 1e3
+    stream = torch.cuda.Stream(device=dev)
+    dp = wf.DevicePlans.from_host(plans, dev)
+    res = wf.Results(P, dev)
+    rel = torch.empty(prob.N, dtype=torch.int64, device=dev)
+    comp = torch.empty_like(rel)
+    ids = torch.empty(k, dtype=torch.int32, device=dev)
+    keys = torch.empty((k, 3), dtype=torch.int64, device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
+    torch.cuda.synchronize()
+
+    def step():
+        wf.wf_forecast_readiness(ctx, rel, comp, stream)
+        wf.wf_eval_plans(ctx, dp, res, stream)
+        wf.wf_topk(ctx, res, P, k, ids, keys, stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            flush.zero_()
+            step()
+    wf.wf_ctx_status(ctx, stream)
+
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    barrier(world)
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        for s in range(args.steps):
+            flush.zero_()
+            e = ev[s]
+            e[0].record(stream)
+            wf.wf_forecast_readiness(ctx, rel, comp, stream)
+            e[1].record(stream)
+            wf.wf_eval_plans(ctx, dp, res, stream)
+            e[2].record(stream)
+            wf.wf_topk(ctx, res, P, k, ids, keys, stream)
+            e[3].record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    wf.wf_ctx_status(ctx, stream)
+    step_ms = [e[0].elapsed_time(e[3]) for e in ev]
+    eval_ms = [e[1].elapsed_time(e[2]) for e in ev]
+    ms_per_step = max_over_ranks(float(np.mean(step_ms)), world)
+    eval_ms_mean = float(np.mean(eval_ms))
+
+    # End to end through the public call: pinned host plans -> device -> top-k -> host.
+    pinned = {a: torch.from_numpy(np.ascontiguousarray(getattr(plans, a))).pin_memory()
+              for a in ("place", "order", "fuse", "prefetch")}
+    e2e_dev = wf.DevicePlans(torch.empty_like(pinned["place"], device=dev),
+                             torch.empty(pinned["order"].shape, dtype=torch.int16, device=dev),
+                             torch.empty(pinned["fuse"].shape, dtype=torch.int32, device=dev),
+                             torch.empty(pinned["prefetch"].shape, dtype=torch.int32, device=dev),
+                             plan_base=rank * P)
+    h2d = sum(t.numel() * t.element_size() for t in pinned.values())
+    ids_h = torch.empty(k, dtype=torch.int32).pin_memory()
+    keys_h = torch.empty((k, 3), dtype=torch.int64).pin_memory()
+    d2h = ids_h.numel() * 4 + keys_h.numel() * 8
+
+    def e2e_step():
+        e2e_dev.place.copy_(pinned["place"], non_blocking=True)
+        e2e_dev.order.copy_(pinned["order"].view(torch.int16), non_blocking=True)
+        e2e_dev.fuse.copy_(pinned["fuse"].view(torch.int32), non_blocking=True)
+        e2e_dev.prefetch.copy_(pinned["prefetch"].view(torch.int32), non_blocking=True)
+        wf.wf_forecast_readiness(ctx, rel, comp, stream)
+        wf.wf_eval_plans(ctx, e2e_dev, res, stream)
+        wf.wf_topk(ctx, res, P, k, ids, keys, stream)
+        ids_h.copy_(ids, non_blocking=True)
+        keys_h.copy_(keys, non_blocking=True)
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            e2e_step()
+    torch.cuda.synchronize()
+    barrier(world)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(args.steps):
+            e2e_step()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    clk = clocks.stop()
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, world)
+    # the host reads the top-k it copied back
+    assert int(ids_h.numpy().min()) >= 0
+
+    bpp = algorithmic_bytes_per_plan(prob.N)
+    achieved = bpp * P / (eval_ms_mean * 1e-3) / 1e9
+    peaks = read_peaks()
+    peak = peaks.get("hbm_gbs")
+    traffic, _ = read_traffic(WORKLOAD)
+    launches = args.steps * (2 + topk_launches(P, k))
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        oracle.build()
+        sample = P
+        t0 = time.perf_counter()
+        oracle.eval_plans(prob, plans, 0, sample)
+        dt = time.perf_counter() - t0
+        cpu = {"value": sample / dt, "unit": "plans/s", "cores": 1, "kind": "oracle",
+               "sample": f"all {sample} plans of the burst batch, one thread, {dt:.2f} s"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": P * world / (ms_per_step * 1e-3), "unit": "plans/s",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64",
+            "data": "synthetic",
+            "config": {"workload": "burst: 64 sessions (Poisson arrivals, mean gap 0.5 s), N=2000, "
+                                   "D=8, M=8, P=16384 plans per GPU, k=32",
+                       "P_per_gpu": P, "N": prob.N, "k": k,
+                       "l2": "flushed between timed steps (256 MiB write)",
+                       "ctx_create_ms": ctx_ms},
+            "e2e": {"value": P * world / (e2e_ms * 1e-3), "unit": "plans/s",
+                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak if peak else None,
+                         "traffic": traffic, "kernel": "eval_det_kernel",
+                         "algorithmic_bytes_per_plan": bpp, "kernel_ms": eval_ms_mean,
+                         "peak_source": "MEASURED_PEAKS.json hbm_gbs (measured copy)" if peak else None},
+            "cpu_baseline": cpu,
+            "clocks": clk,
+            "gpu_launches": launches,
+        }
+        print(json.dumps(line), flush=True)
+    ctx.close()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=("gpu", "reference"), default="gpu")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    rank, world, local = dist_setup()
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+    else:
+        run_gpu(args, rank, world, local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,200 @@
+/*
+ * wf.h -- C ABI of the GB300 batched plan evaluator (libwf.so).
+ *
+ * A *problem* is one window of the activation DAG of concurrent multi-agent
+ * workflows (paper Section 3.2) together with Predictor-style cost tables
+ * (Eq. 1).  A *plan* fixes a device per activation, a dispatch sequence that
+ * orients every resource conflict, and per-activation fusion / prefetch /
+ * retain bits (Eq. 3-10).  The library evaluates batches of plans on one GPU
+ * and ranks them:
+ *
+ *   wf_problem_check        validate a problem on the host (no GPU needed)
+ *   wf_ctx_create           validate, derive and upload a problem (once)
+ *   wf_forecast_readiness   release forecast of every activation (Eq. 2)
+ *   wf_eval_plans           play every plan forward (Eq. 2-11) -> metrics
+ *   wf_topk                 the k best plans by the ranking key
+ *   wf_ctx_destroy, wf_strerror
+ *
+ * Conventions.
+ *   - Times are int64 microseconds, memory int32 MiB; every output is an
+ *     exact integer.
+ *   - Tables are row-major: lat_us and peak_mib are [N][D] (index n*D + d),
+ *     load_us is [M][D].
+ *   - Problem pointers are HOST pointers, read during wf_ctx_create only; the
+ *     caller keeps ownership.  Plan and output pointers are DEVICE pointers
+ *     owned by the caller; the library never frees them.
+ *   - Calls taking a stream (a cudaStream_t passed as void*, NULL = the
+ *     legacy default stream) are asynchronous on it and allocate nothing:
+ *     the context owns every scratch buffer, sized at creation for up to
+ *     max_P plans per call.  One context serves one stream at a time.
+ *   - Return codes: WF_OK (0) or a WF_E* code below.  Problems with single
+ *     plans are data (status bits), never return codes.
+ */
+#ifndef WF_H
+#define WF_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum {
+    WF_OK = 0,
+    WF_EINVAL = 1,    /* a null pointer, a size or stride out of range, a malformed problem */
+    WF_ENOMEM = 2,    /* device or host allocation failed */
+    WF_ECUDA = 3,     /* a CUDA launch or runtime error (see wf_strerror) */
+    WF_ETIMEOUT = 4   /* a bounded device-side wait expired; results are invalid */
+};
+
+/* Plan status bits (wf_eval_out.status). */
+enum {
+    WF_ST_DEVICE = 1u,      /* some place[n] >= D */
+    WF_ST_CAPACITY = 2u,    /* some peak[n][place[n]] > cap[place[n]] (Eq. 8) */
+    WF_ST_PERMUTATION = 4u, /* order is not a permutation of 0..N-1 */
+    WF_ST_TOPOLOGY = 8u     /* an edge u -> v with v dispatched before u (Eq. 9-10);
+                               examined only when WF_ST_PERMUTATION is clear */
+};
+
+typedef struct wf_ctx wf_ctx;
+
+/*
+ * One planning window (Section 3.2) and its cost tables (Eq. 1).
+ *
+ *   N activations (1..65535), D devices (1..32), M models (1..16),
+ *   W sessions (>= 1, every session owns >= 1 activation).
+ *   pred_off[N+1], pred_idx[E=pred_off[N]]: CSR lists of graph predecessors
+ *     (acyclic, no self-loops, no duplicates, never across sessions).
+ *   model[N] < M: deployment identity of each activation (Section 3.2).
+ *   session[N] < W; arrival_us[W] >= 0: session arrival times.
+ *   lat_us[N*D] >= 0: predicted run time of activation n on device d.
+ *   peak_mib[N*D] >= weight_mib[model[n]]: predicted peak memory; the
+ *     activation's KV / request memory is peak - weight.  Every activation
+ *     must fit (peak <= cap) on at least one device.
+ *   weight_mib[M] >= 1, load_us[M*D] >= 0, cap_mib[D] >= 1.
+ *   grant_us >= 0: admission overhead charged once per scheduling unit.
+ *   S >= 0: latency samples per plan (0 = deterministic).  For S > 0 the run
+ *     time of activation n in sample s of plan p is
+ *       (lat * bm_e[zq + (bm_en-1)/2] + 2^15) >> 16,
+ *     h  = mix(mix(mix(seed ^ p) ^ s) ^ n)   (mix = SplitMix64 output),
+ *     zq = floor(bm_r[h & (bm_rn-1)] * bm_c[(h >> 32) & (bm_cn-1)] / 2^18);
+ *     bm_rn and bm_cn must be powers of two, bm_en odd and large enough
+ *     for every zq, bm_e >= 0.  Ignored when S == 0.
+ */
+typedef struct {
+    int32_t N, D, M, W;
+    const int32_t *pred_off;
+    const int32_t *pred_idx;
+    const uint8_t *model;
+    const int32_t *session;
+    const int64_t *arrival_us;
+    const int32_t *lat_us;
+    const int32_t *peak_mib;
+    const int32_t *weight_mib;
+    const int32_t *load_us;
+    const int32_t *cap_mib;
+    int32_t grant_us;
+    int32_t S;
+    uint64_t seed;
+    const int32_t *bm_r, *bm_c, *bm_e;
+    int32_t bm_rn, bm_cn, bm_en;
+} wf_problem;
+
+/*
+ * A batch of P candidate plans (Eq. 6-10), DEVICE pointers, caller-owned.
+ *   place[p*place_stride + n]: device of activation n (uint8).
+ *   order[p*order_stride/2 + i]: activation dispatched at position i (uint16).
+ *   fuse / prefetch / retain[p*bits_stride/4 + (n>>5)] bit (n&31): the
+ *     plan's fusion (Eq. 3-4), prefetch (Eq. 5) and retain bits of n.
+ *     retain may be NULL (every model retained after its units).
+ *   Strides are in bytes and multiples of 16; place_stride >= N,
+ *   order_stride >= 2N, bits_stride >= 4*ceil(N/32).  Base pointers must be
+ *   16-byte aligned.  plan_base is the global index of row 0 (it seeds the
+ *   latency samples, so shards of one batch reproduce the whole batch).
+ */
+typedef struct {
+    int64_t P;
+    int64_t plan_base;
+    const uint8_t *place;
+    int64_t place_stride;
+    const uint16_t *order;
+    int64_t order_stride;
+    const uint32_t *fuse;
+    const uint32_t *prefetch;
+    const uint32_t *retain;
+    int64_t bits_stride;
+} wf_plans;
+
+/* Per-plan results, DEVICE pointers [P], caller-owned. */
+typedef struct {
+    int64_t *makespan_us;  /* last finish - first arrival (Section 4.2) */
+    int64_t *p95_us;       /* nearest-rank 95th percentile of session completion latency */
+    int64_t *gpu_us;       /* summed device occupancy: loading + generating + idle resident (Section 4.3) */
+    uint32_t *status;      /* WF_ST_* bits; a nonzero status sets the three metrics to INT64_MAX */
+} wf_eval_out;
+
+/*
+ * Validate a problem on the host without touching a GPU.  Returns WF_OK or
+ * WF_EINVAL (with a reason retrievable through wf_last_error()).
+ */
+int wf_problem_check(const wf_problem *prob);
+
+/*
+ * Validate *prob, derive the fusible edges of Eq. 3 (succ(u) = {v},
+ * pred(v) = {u}, same model) and the topological levels, and copy every
+ * table to device `device`.  Scratch for up to max_P plans per call is
+ * allocated here (and only here).  On success *out owns all device memory it
+ * allocated.  Returns WF_OK, WF_EINVAL, WF_ENOMEM or WF_ECUDA.
+ */
+int wf_ctx_create(const wf_problem *prob, int device, int64_t max_P, wf_ctx **out);
+
+/*
+ * Release forecast of Eq. 2 over the window, free of contention and loads:
+ *   rel[n]  = max(arrival[session[n]], max over preds v of comp[v])
+ *   comp[n] = rel[n] + min over devices d with peak[n][d] <= cap[d] of lat[n][d]
+ * rel_dev and comp_dev are DEVICE int64 [N].  Asynchronous on `stream`.
+ */
+int wf_forecast_readiness(wf_ctx *ctx, int64_t *rel_dev, int64_t *comp_dev, void *stream);
+
+/*
+ * Evaluate plans->P plans (0 < P <= max_P).  Per plan: the status bits;
+ * then fused chains (Eq. 3-4), releases (Eq. 2, Eq. 7), per-device order
+ * (Eq. 10), least-recently-used reclamation so that resident weights plus
+ * the unit's KV fit at every admission (Eq. 11, Section 3.5), loads and
+ * prefetches on the consumer's device (Eq. 5, Eq. 9), retain / reclaim, and
+ * the three metrics; for S > 0 the floor means over samples and the pooled
+ * p95.  Asynchronous on `stream`.  Returns WF_EINVAL for bad sizes, strides
+ * or alignment, WF_ECUDA for a launch error.
+ */
+int wf_eval_plans(wf_ctx *ctx, const wf_plans *plans, const wf_eval_out *out, void *stream);
+
+/*
+ * The k best of P evaluated plans (1 <= k <= min(P, 1024), P <= max_P) by the
+ * key (status != 0, makespan, p95, gpu, plan index), ascending -- the
+ * single-objective analog of the ranking key of Eq. 12.  ids_dev: DEVICE
+ * int32 [k] plan indices (0-based within the batch); keys_dev: DEVICE int64
+ * [k][3] (makespan, p95, gpu) or NULL.  Asynchronous on `stream`.
+ */
+int wf_topk(wf_ctx *ctx, const wf_eval_out *res, int64_t P, int32_t k,
+            int32_t *ids_dev, int64_t *keys_dev, void *stream);
+
+/*
+ * Synchronize `stream` and report device-side failures of earlier calls on
+ * this context (WF_ETIMEOUT when a bounded wait expired), clearing them.
+ */
+int wf_ctx_status(wf_ctx *ctx, void *stream);
+
+/* Release every device and host allocation of the context (NULL is a no-op). */
+void wf_ctx_destroy(wf_ctx *ctx);
+
+/* Static description of a return code. */
+const char *wf_strerror(int code);
+
+/* Thread-local detail of the last WF_EINVAL / WF_ECUDA on this thread. */
+const char *wf_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* WF_H */

@@ -1,0 +1,370 @@
+// Plan evaluation (rows a3-a11): status bits, then a list-schedule play of
+// each plan over the window with fused chains (Eq. 3-4), releases (Eq. 2,
+// Eq. 7), per-device order (Eq. 10), LRU residency under capacity (Eq. 11),
+// loads / prefetches on the consumer's device (Eq. 5, Eq. 9), retain /
+// reclaim and the metrics of Section 4.2-4.3.
+//
+// Mapping: one thread plays one (plan, sample).  Its mutable state (chain-tail
+// finish times, per-device and per-session state) lives in a scratch row of
+// the context; plans beyond the number of rows are taken in rounds.
+#include <algorithm>
+
+#include "wf_internal.cuh"
+
+namespace {
+
+constexpr int kEvalThreads = 128;
+constexpr int kSampleThreads = 64;
+constexpr int64_t kNone = INT64_MIN;
+
+struct PlanRows {
+    const uint8_t *place;
+    const uint16_t *order;
+    const uint32_t *fuse;
+    const uint32_t *prefetch;
+    const uint32_t *retain;  // NULL = all retained
+};
+
+__device__ __forceinline__ bool bit_at(const uint32_t *row, int32_t n)
+{
+    return (__ldg(row + (n >> 5)) >> (n & 31)) & 1u;
+}
+
+__device__ __forceinline__ PlanRows plan_rows(const wf_plans &pl, int64_t p)
+{
+    PlanRows r;
+    r.place = pl.place + p * pl.place_stride;
+    r.order = (const uint16_t *)((const uint8_t *)pl.order + p * pl.order_stride);
+    r.fuse = (const uint32_t *)((const uint8_t *)pl.fuse + p * pl.bits_stride);
+    r.prefetch = (const uint32_t *)((const uint8_t *)pl.prefetch + p * pl.bits_stride);
+    r.retain = pl.retain ? (const uint32_t *)((const uint8_t *)pl.retain + p * pl.bits_stride) : nullptr;
+    return r;
+}
+
+// Scratch row of one simulation.
+struct Row {
+    int64_t *ctail;   // [N] finish time of chain tails (also holds int32 positions for the status check)
+    int64_t *tfree;   // [D] device free time
+    int64_t *occ;     // [D] start of the current occupancy interval, kNone if empty
+    int64_t *gpu;     // [D] closed occupancy
+    int64_t *comp;    // [W] latest finish per session
+    int32_t *used;    // [D] resident weights
+    int32_t *nres;    // [D] resident model count
+    int32_t *stamp;   // [D][M] last dispatch position + 1 using the model, 0 = not resident
+};
+
+__device__ __forceinline__ size_t up8(size_t x) { return (x + 7) & ~(size_t)7; }
+
+__device__ __forceinline__ Row row_at(const wf_dev_problem &dp, uint8_t *base)
+{
+    Row r;
+    size_t o = 0;
+    r.ctail = (int64_t *)(base + o); o += up8(8 * (size_t)dp.N);
+    r.tfree = (int64_t *)(base + o); o += 8 * (size_t)dp.D;
+    r.occ = (int64_t *)(base + o); o += 8 * (size_t)dp.D;
+    r.gpu = (int64_t *)(base + o); o += 8 * (size_t)dp.D;
+    r.comp = (int64_t *)(base + o); o += 8 * (size_t)dp.W;
+    r.used = (int32_t *)(base + o); o += up8(4 * (size_t)dp.D);
+    r.nres = (int32_t *)(base + o); o += up8(4 * (size_t)dp.D);
+    r.stamp = (int32_t *)(base + o);
+    return r;
+}
+
+// Status bits (Eq. 8-10).  Uses the ctail area as an int32 position table.
+__device__ uint32_t plan_status(const wf_dev_problem &dp, const PlanRows &pr, Row &row)
+{
+    const int32_t N = dp.N, D = dp.D;
+    uint32_t st = 0;
+    for (int32_t n = 0; n < N; ++n) {
+        const int32_t d = pr.place[n];
+        if (d >= D) st |= WF_ST_DEVICE;
+        else if (dp.peak[(int64_t)n * D + d] > dp.cap[d]) st |= WF_ST_CAPACITY;
+    }
+    int32_t *pos = (int32_t *)row.ctail;
+    for (int32_t n = 0; n < N; ++n) pos[n] = -1;
+    for (int32_t i = 0; i < N; ++i) {
+        const int32_t h = pr.order[i];
+        if (h >= N || pos[h] >= 0) { st |= WF_ST_PERMUTATION; continue; }
+        pos[h] = i;
+    }
+    if (!(st & WF_ST_PERMUTATION)) {
+        for (int32_t v = 0; v < N && !(st & WF_ST_TOPOLOGY); ++v)
+            for (int32_t e = dp.pred_off[v]; e < dp.pred_off[v + 1]; ++e)
+                if (pos[dp.pred_idx[e]] > pos[v]) { st |= WF_ST_TOPOLOGY; break; }
+    }
+    return st;
+}
+
+// SplitMix64 output function (Steele, Lea, Flood 2014).
+__device__ __forceinline__ uint64_t splitmix(uint64_t x)
+{
+    x += 0x9E3779B97F4A7C15ull;
+    x = (x ^ (x >> 30)) * 0xBF58476D1CE4E5B9ull;
+    x = (x ^ (x >> 27)) * 0x94D049BB133111EBull;
+    return x ^ (x >> 31);
+}
+
+// Run time of activation n on device d; for a latency sample, scaled by the
+// multiplier drawn from (plan, sample, n) through the integer Box-Muller
+// tables (an arithmetic right shift of the signed product is the floor).
+template <bool kStoch>
+__device__ __forceinline__ int64_t run_time(const wf_dev_problem &dp, int32_t n, int32_t d, uint64_t key)
+{
+    const int64_t base = dp.lat[(int64_t)n * dp.D + d];
+    if (!kStoch) return base;
+    const uint64_t h = splitmix(key ^ (uint64_t)n);
+    const int64_t r = dp.bm_r[h & (uint64_t)(dp.bm_rn - 1)];
+    const int64_t c = dp.bm_c[(h >> 32) & (uint64_t)(dp.bm_cn - 1)];
+    const int64_t zq = (r * c) >> 18;
+    const int64_t mult = dp.bm_e[zq + ((dp.bm_en - 1) >> 1)];
+    return (base * mult + 32768) >> 16;
+}
+
+// One play of a valid plan.  Returns makespan and GPU time; per-session
+// completion latencies are left in row.comp.
+template <bool kStoch>
+__device__ void play(const wf_dev_problem &dp, const PlanRows &pr, Row &row, uint64_t key,
+                     int64_t *makespan, int64_t *gpu_total)
+{
+    const int32_t N = dp.N, D = dp.D, M = dp.M, W = dp.W;
+    for (int32_t d = 0; d < D; ++d) {
+        row.tfree[d] = 0; row.occ[d] = kNone; row.gpu[d] = 0; row.used[d] = 0; row.nres[d] = 0;
+    }
+    for (int32_t k = 0; k < D * M; ++k) row.stamp[k] = 0;
+    for (int32_t w = 0; w < W; ++w) row.comp[w] = kNone;
+    int64_t end = 0;
+
+    for (int32_t i = 0; i < N; ++i) {
+        const int32_t h = pr.order[i];
+        const int32_t d = pr.place[h];
+        // A chain member runs inside its head's unit (Eq. 3, Eq. 9).
+        const int32_t fp = dp.fprev[h];
+        if (fp >= 0 && bit_at(pr.fuse, h) && pr.place[fp] == d) continue;
+
+        const int32_t m = dp.model[h];
+        const int32_t w = dp.session[h];
+        const int64_t arr = dp.arrival[w];
+        int64_t rel = arr;  // Eq. 2 / Eq. 7: the heads' predecessors are chain tails
+        for (int32_t e = dp.pred_off[h]; e < dp.pred_off[h + 1]; ++e)
+            rel = max(rel, row.ctail[dp.pred_idx[e]]);
+
+        // Extend the chain; admission KV is the largest on it, run time the sum (Eq. 4).
+        const int32_t wm = dp.weight[m];
+        int32_t tail = h;
+        int64_t kv = dp.peak[(int64_t)h * D + d] - wm;
+        int64_t run = run_time<kStoch>(dp, h, d, key);
+        for (int32_t s = dp.fnext[h]; s >= 0 && bit_at(pr.fuse, s) && pr.place[s] == d; s = dp.fnext[s]) {
+            kv = max(kv, (int64_t)dp.peak[(int64_t)s * D + d] - wm);
+            run += run_time<kStoch>(dp, s, d, key);
+            tail = s;
+        }
+
+        // Eq. 11 with LRU reclamation of other models.
+        int32_t *st = row.stamp + d * M;
+        const bool hit = st[m] != 0;
+        const int64_t need = hit ? kv : wm + kv;
+        while (row.used[d] + need > dp.cap[d]) {
+            int32_t victim = -1, vs = INT32_MAX;
+            for (int32_t k = 0; k < M; ++k)
+                if (k != m && st[k] != 0 && st[k] < vs) { vs = st[k]; victim = k; }
+            if (victim < 0) { atomicExch(dp.err, 2); break; }  // unreachable for a valid plan
+            row.used[d] -= dp.weight[victim];
+            row.nres[d] -= 1;
+            st[victim] = 0;
+        }
+        const int64_t tf = row.tfree[d];
+        int64_t start;
+        if (hit) {
+            start = max(tf, rel);
+        } else {
+            const int64_t ls = max(tf, bit_at(pr.prefetch, h) ? arr : rel);
+            if (row.occ[d] == kNone) row.occ[d] = ls;
+            row.used[d] += wm;
+            row.nres[d] += 1;
+            start = max(ls + dp.load[m * D + d], rel);
+        }
+        const int64_t c = start + dp.grant + run;
+        row.ctail[tail] = c;
+        row.tfree[d] = c;
+        st[m] = i + 1;
+        end = max(end, c);
+        row.comp[w] = max(row.comp[w], c);
+        if (pr.retain && !bit_at(pr.retain, tail)) {
+            row.used[d] -= wm;
+            row.nres[d] -= 1;
+            st[m] = 0;
+            if (row.nres[d] == 0) {
+                row.gpu[d] += c - row.occ[d];
+                row.occ[d] = kNone;
+            }
+        }
+    }
+    int64_t g = 0;
+    for (int32_t d = 0; d < D; ++d) {
+        if (row.occ[d] != kNone) row.gpu[d] += end - row.occ[d];
+        g += row.gpu[d];
+    }
+    for (int32_t w = 0; w < W; ++w) row.comp[w] -= dp.arrival[w];
+    *makespan = end - dp.first_arrival;
+    *gpu_total = g;
+}
+
+// r-th smallest (0-based) of v[0..n), reordering v (Hoare quickselect).
+__device__ int64_t select_rank(int64_t *v, int32_t n, int32_t r)
+{
+    int32_t lo = 0, hi = n - 1;
+    while (lo < hi) {
+        const int64_t pivot = v[lo + (hi - lo) / 2];
+        int32_t i = lo, j = hi;
+        while (i <= j) {
+            while (v[i] < pivot) ++i;
+            while (v[j] > pivot) --j;
+            if (i <= j) { int64_t t = v[i]; v[i] = v[j]; v[j] = t; ++i; --j; }
+        }
+        if (r <= j) hi = j;
+        else if (r >= i) lo = i;
+        else return v[r];
+    }
+    return v[r];
+}
+
+__device__ __forceinline__ int32_t p95_rank(int64_t n) { return (int32_t)((95 * n + 99) / 100 - 1); }
+
+__global__ void __launch_bounds__(kEvalThreads)
+eval_det_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, uint8_t *scratch, size_t row_bytes,
+                int64_t rows)
+{
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (t >= rows) return;
+    Row row = row_at(dp, scratch + (size_t)t * row_bytes);
+    for (int64_t p = t; p < pl.P; p += rows) {
+        const PlanRows pr = plan_rows(pl, p);
+        const uint32_t st = plan_status(dp, pr, row);
+        out.status[p] = st;
+        if (st) {
+            out.makespan_us[p] = out.p95_us[p] = out.gpu_us[p] = WF_INF64;
+            continue;
+        }
+        int64_t mk, g;
+        play<false>(dp, pr, row, 0, &mk, &g);
+        out.makespan_us[p] = mk;
+        out.gpu_us[p] = g;
+        out.p95_us[p] = select_rank(row.comp, dp.W, p95_rank(dp.W));
+    }
+}
+
+// Stochastic latencies: one CTA per plan, one thread per sample; the pooled
+// S x W completions of the plan go to a per-CTA pool for the p95 selection.
+__global__ void __launch_bounds__(kSampleThreads)
+eval_stoch_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, uint8_t *scratch, size_t row_bytes,
+                  int64_t *pool_base, int64_t ctas)
+{
+    __shared__ unsigned long long s_mk, s_gpu;
+    __shared__ uint32_t s_status;
+    __shared__ uint32_t s_hist[256];
+    __shared__ uint64_t s_prefix;
+    __shared__ int32_t s_rank;
+    const int64_t cta = blockIdx.x;
+    const int32_t S = dp.S, W = dp.W;
+    Row row = row_at(dp, scratch + (size_t)(cta * blockDim.x + threadIdx.x) * row_bytes);
+    int64_t *pool = pool_base + cta * (int64_t)S * W;
+    for (int64_t p = cta; p < pl.P; p += ctas) {
+        const PlanRows pr = plan_rows(pl, p);
+        if (threadIdx.x == 0) {
+            s_mk = 0; s_gpu = 0;
+            s_status = plan_status(dp, pr, row);
+        }
+        __syncthreads();
+        const uint32_t st = s_status;
+        if (st) {
+            if (threadIdx.x == 0) {
+                out.status[p] = st;
+                out.makespan_us[p] = out.p95_us[p] = out.gpu_us[p] = WF_INF64;
+            }
+            __syncthreads();
+            continue;
+        }
+        const uint64_t gp = (uint64_t)(pl.plan_base + p);
+        for (int32_t s = threadIdx.x; s < S; s += blockDim.x) {
+            const uint64_t key = splitmix(splitmix(dp.seed ^ gp) ^ (uint64_t)s);
+            int64_t mk, g;
+            play<true>(dp, pr, row, key, &mk, &g);
+            atomicAdd(&s_mk, (unsigned long long)mk);
+            atomicAdd(&s_gpu, (unsigned long long)g);
+            for (int32_t w = 0; w < W; ++w) pool[(int64_t)s * W + w] = row.comp[w];
+        }
+        __syncthreads();
+        // Nearest-rank p95 of the pooled non-negative completions: radix
+        // select, 8 bits per pass from the most significant byte.
+        const int64_t n = (int64_t)S * W;
+        if (threadIdx.x == 0) { s_prefix = 0; s_rank = p95_rank(n); }
+        __syncthreads();
+        for (int shift = 56; shift >= 0; shift -= 8) {
+            for (int b = threadIdx.x; b < 256; b += blockDim.x) s_hist[b] = 0;
+            __syncthreads();
+            const uint64_t hi_mask = shift == 56 ? 0 : (~0ull << (shift + 8));
+            for (int64_t i = threadIdx.x; i < n; i += blockDim.x) {
+                const uint64_t v = (uint64_t)pool[i];
+                if ((v & hi_mask) == s_prefix) atomicAdd(&s_hist[(v >> shift) & 255u], 1u);
+            }
+            __syncthreads();
+            if (threadIdx.x == 0) {
+                int32_t r = s_rank;
+                int b = 0;
+                while ((int32_t)s_hist[b] <= r) { r -= s_hist[b]; ++b; }
+                s_rank = r;
+                s_prefix |= (uint64_t)b << shift;
+            }
+            __syncthreads();
+        }
+        if (threadIdx.x == 0) {
+            out.status[p] = 0;
+            out.makespan_us[p] = (int64_t)(s_mk / (unsigned long long)S);
+            out.gpu_us[p] = (int64_t)(s_gpu / (unsigned long long)S);
+            out.p95_us[p] = (int64_t)s_prefix;
+        }
+        __syncthreads();
+    }
+}
+
+}  // namespace
+
+size_t wf_eval_row_bytes(const wf_dev_problem &dp)
+{
+    size_t b = ((8 * (size_t)dp.N + 7) & ~(size_t)7) + 8 * 3 * (size_t)dp.D + 8 * (size_t)dp.W +
+               2 * ((4 * (size_t)dp.D + 7) & ~(size_t)7) + 4 * (size_t)dp.D * dp.M;
+    return (b + 127) & ~(size_t)127;
+}
+
+static size_t sample_cta_bytes(const wf_dev_problem &dp)
+{
+    const size_t pool = (8 * (size_t)dp.S * dp.W + 127) & ~(size_t)127;
+    return kSampleThreads * wf_eval_row_bytes(dp) + pool;
+}
+
+size_t wf_eval_scratch_bytes(const wf_dev_problem &dp, int64_t max_P, int64_t *units)
+{
+    const size_t budget = (size_t)1 << 30;
+    const size_t unit = dp.S == 0 ? wf_eval_row_bytes(dp) : sample_cta_bytes(dp);
+    const int64_t floor_units = dp.S == 0 ? 1024 : 16;
+    *units = std::min<int64_t>(max_P, std::max<int64_t>((int64_t)(budget / unit), floor_units));
+    return unit * (size_t)*units;
+}
+
+int wf_launch_eval(wf_ctx *ctx, const wf_plans *plans, const wf_eval_out *out, cudaStream_t st)
+{
+    const wf_dev_problem &dp = ctx->dp;
+    uint8_t *scratch = (uint8_t *)ctx->eval_scratch;
+    const int64_t units = std::min<int64_t>(ctx->eval_threads, plans->P);
+    if (dp.S == 0) {
+        const int64_t blocks = (units + kEvalThreads - 1) / kEvalThreads;
+        eval_det_kernel<<<(unsigned)blocks, kEvalThreads, 0, st>>>(dp, *plans, *out, scratch,
+                                                                    ctx->eval_row_bytes, units);
+    } else {
+        // Per-thread rows of every CTA first, then one completion pool per CTA.
+        int64_t *pool = (int64_t *)(scratch + (size_t)units * kSampleThreads * ctx->eval_row_bytes);
+        eval_stoch_kernel<<<(unsigned)units, kSampleThreads, 0, st>>>(dp, *plans, *out, scratch,
+                                                                      ctx->eval_row_bytes, pool, units);
+    }
+    return wf_cuda_check(cudaGetLastError(), "eval launch");
+}

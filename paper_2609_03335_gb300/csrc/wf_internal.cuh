@@ -1,0 +1,64 @@
+// Internal definitions shared by the library's translation units.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cstdint>
+
+#include "../../include/wf.h"
+
+#define WF_INF64 INT64_MAX
+
+// Device-resident copy of a problem plus derived tables.  Owned by wf_ctx.
+struct wf_dev_problem {
+    int32_t N, D, M, W, E;
+    int32_t grant;
+    int32_t S;
+    uint64_t seed;
+    int32_t bm_rn, bm_cn, bm_en;
+    int64_t first_arrival;      // min over sessions of arrival_us
+    const int32_t *pred_off;    // [N+1]
+    const int32_t *pred_idx;    // [E]
+    const int32_t *fnext;       // [N] fusible successor (Eq. 3) or -1
+    const int32_t *fprev;       // [N] fusible predecessor (Eq. 3) or -1
+    const uint8_t *model;       // [N]
+    const int32_t *session;     // [N]
+    const int64_t *arrival;     // [W]
+    const int32_t *lat;         // [N][D]
+    const int32_t *peak;        // [N][D]
+    const int32_t *weight;      // [M]
+    const int32_t *load;        // [M][D]
+    const int32_t *cap;         // [D]
+    const int32_t *lev_off;     // [nlev+1] topological levels
+    const int32_t *lev_nodes;   // [N]
+    int32_t nlev;
+    const int32_t *bm_r, *bm_c, *bm_e;
+    int *err;                   // device error word (0 = ok)
+};
+
+struct wf_ctx {
+    int device;
+    int64_t max_P;
+    wf_dev_problem dp;
+    void *tables;               // one device allocation holding every table
+    size_t tables_bytes;
+    void *eval_scratch;         // per-simulation state (and sample pools)
+    size_t eval_scratch_bytes;
+    int64_t eval_threads;       // launch units (plans, or sample CTAs) the scratch holds
+    size_t eval_row_bytes;
+    void *topk_scratch;
+    size_t topk_scratch_bytes;
+    int *err;
+};
+
+// Error plumbing (wf_ctx.cu).
+int wf_set_error(int code, const char *fmt, ...);
+int wf_cuda_check(cudaError_t e, const char *what);
+
+// Launchers (one per translation unit).
+int wf_launch_forecast(wf_ctx *ctx, int64_t *rel, int64_t *comp, cudaStream_t st);
+int wf_launch_eval(wf_ctx *ctx, const wf_plans *plans, const wf_eval_out *out, cudaStream_t st);
+int wf_launch_topk(wf_ctx *ctx, const wf_eval_out *res, int64_t P, int32_t k, int32_t *ids,
+                   int64_t *keys, cudaStream_t st);
+size_t wf_eval_row_bytes(const wf_dev_problem &dp);
+size_t wf_eval_scratch_bytes(const wf_dev_problem &dp, int64_t max_P, int64_t *units);
+size_t wf_topk_scratch_bytes(int64_t max_P);

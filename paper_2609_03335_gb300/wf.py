@@ -1,0 +1,282 @@
+"""ctypes binding of libwf.so (include/wf.h): argument marshalling only.
+
+The functions carry the C ABI's names.  Problem arrays are host numpy arrays;
+plan, result and output arrays are device tensors (torch supplies device
+memory and streams).  Every step of the evaluation runs in the library's CUDA
+kernels; if the library is missing this module raises instead of falling
+back to anything else.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libwf.so")
+
+WF_OK, WF_EINVAL, WF_ENOMEM, WF_ECUDA, WF_ETIMEOUT = 0, 1, 2, 3, 4
+ST_DEVICE, ST_CAPACITY, ST_PERMUTATION, ST_TOPOLOGY = 1, 2, 4, 8
+INT64_MAX = np.iinfo(np.int64).max
+
+# Every entry point declared in include/wf.h.
+EXPORTS = ("wf_problem_check", "wf_ctx_create", "wf_forecast_readiness", "wf_eval_plans",
+           "wf_topk", "wf_ctx_status", "wf_ctx_destroy", "wf_strerror", "wf_last_error")
+
+
+class WfError(RuntimeError):
+    def __init__(self, code: int, where: str, detail: str = ""):
+        super().__init__(f"{where}: {_strerror(code)} ({code}) {detail}".strip())
+        self.code = code
+
+
+class wf_problem(ctypes.Structure):
+    _fields_ = [("N", ctypes.c_int32), ("D", ctypes.c_int32), ("M", ctypes.c_int32),
+                ("W", ctypes.c_int32),
+                ("pred_off", ctypes.c_void_p), ("pred_idx", ctypes.c_void_p),
+                ("model", ctypes.c_void_p), ("session", ctypes.c_void_p),
+                ("arrival_us", ctypes.c_void_p), ("lat_us", ctypes.c_void_p),
+                ("peak_mib", ctypes.c_void_p), ("weight_mib", ctypes.c_void_p),
+                ("load_us", ctypes.c_void_p), ("cap_mib", ctypes.c_void_p),
+                ("grant_us", ctypes.c_int32), ("S", ctypes.c_int32), ("seed", ctypes.c_uint64),
+                ("bm_r", ctypes.c_void_p), ("bm_c", ctypes.c_void_p), ("bm_e", ctypes.c_void_p),
+                ("bm_rn", ctypes.c_int32), ("bm_cn", ctypes.c_int32), ("bm_en", ctypes.c_int32)]
+
+
+class wf_plans(ctypes.Structure):
+    _fields_ = [("P", ctypes.c_int64), ("plan_base", ctypes.c_int64),
+                ("place", ctypes.c_void_p), ("place_stride", ctypes.c_int64),
+                ("order", ctypes.c_void_p), ("order_stride", ctypes.c_int64),
+                ("fuse", ctypes.c_void_p), ("prefetch", ctypes.c_void_p),
+                ("retain", ctypes.c_void_p), ("bits_stride", ctypes.c_int64)]
+
+
+class wf_eval_out(ctypes.Structure):
+    _fields_ = [("makespan_us", ctypes.c_void_p), ("p95_us", ctypes.c_void_p),
+                ("gpu_us", ctypes.c_void_p), ("status", ctypes.c_void_p)]
+
+
+_lib = None
+
+
+def load_library():
+    """Load libwf.so (raises if it was not built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"libwf.so not built ({LIB_PATH}); run __graft_entry__.build()")
+    lib = ctypes.CDLL(LIB_PATH)
+    p, i32, i64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
+    sig = {
+        "wf_problem_check": ([p], ctypes.c_int),
+        "wf_ctx_create": ([p, ctypes.c_int, i64, p], ctypes.c_int),
+        "wf_forecast_readiness": ([p, p, p, p], ctypes.c_int),
+        "wf_eval_plans": ([p, p, p, p], ctypes.c_int),
+        "wf_topk": ([p, p, i64, i32, p, p, p], ctypes.c_int),
+        "wf_ctx_status": ([p, p], ctypes.c_int),
+        "wf_ctx_destroy": ([p], None),
+        "wf_strerror": ([ctypes.c_int], ctypes.c_char_p),
+        "wf_last_error": ([], ctypes.c_char_p),
+    }
+    for name, (args, res) in sig.items():
+        f = getattr(lib, name)
+        f.argtypes = args
+        f.restype = res
+    _lib = lib
+    return lib
+
+
+def _strerror(code: int) -> str:
+    try:
+        return load_library().wf_strerror(code).decode()
+    except Exception:
+        return "error"
+
+
+def _check(code: int, where: str):
+    if code != WF_OK:
+        detail = load_library().wf_last_error().decode()
+        raise WfError(code, where, detail)
+
+
+def _stream_handle(stream) -> int | None:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream or None
+    if isinstance(stream, int):
+        return stream or None
+    return stream.cuda_stream or None
+
+
+class HostProblem:
+    """A problem marshalled into a wf_problem (keeps the host arrays alive)."""
+
+    def __init__(self, prob):
+        def a(x, dt):
+            return np.ascontiguousarray(np.asarray(x, dtype=dt))
+        self.keep = dict(
+            pred_off=a(prob.pred_off, np.int32), pred_idx=a(prob.pred_idx, np.int32),
+            model=a(prob.model, np.uint8), session=a(prob.session, np.int32),
+            arrival_us=a(prob.arrival_us, np.int64), lat_us=a(prob.lat_us, np.int32),
+            peak_mib=a(prob.peak_mib, np.int32), weight_mib=a(prob.weight_mib, np.int32),
+            load_us=a(prob.load_us, np.int32), cap_mib=a(prob.cap_mib, np.int32),
+            bm_r=a(getattr(prob, "bm_r", np.zeros(0)), np.int32),
+            bm_c=a(getattr(prob, "bm_c", np.zeros(0)), np.int32),
+            bm_e=a(getattr(prob, "bm_e", np.zeros(0)), np.int32))
+        k = self.keep
+        ptr = {n: (v.ctypes.data if v.size else None) for n, v in k.items()}
+        self.c = wf_problem(int(prob.N), int(prob.D), int(prob.M), int(prob.W),
+                            ptr["pred_off"], ptr["pred_idx"], ptr["model"], ptr["session"],
+                            ptr["arrival_us"], ptr["lat_us"], ptr["peak_mib"], ptr["weight_mib"],
+                            ptr["load_us"], ptr["cap_mib"], int(prob.grant_us), int(prob.S),
+                            int(prob.seed) & ((1 << 64) - 1), ptr["bm_r"], ptr["bm_c"], ptr["bm_e"],
+                            int(k["bm_r"].size), int(k["bm_c"].size), int(k["bm_e"].size))
+        self.N, self.D, self.M, self.W, self.S = (int(prob.N), int(prob.D), int(prob.M),
+                                                  int(prob.W), int(prob.S))
+
+
+def wf_problem_check(prob) -> int:
+    """Host-side validation; returns the WF_* code (no GPU needed)."""
+    hp = prob if isinstance(prob, HostProblem) else HostProblem(prob)
+    return int(load_library().wf_problem_check(ctypes.byref(hp.c)))
+
+
+def wf_last_error() -> str:
+    return load_library().wf_last_error().decode()
+
+
+def wf_strerror(code: int) -> str:
+    return _strerror(code)
+
+
+class Ctx:
+    """Owns a wf_ctx (device copy of one problem + scratch for max_P plans)."""
+
+    def __init__(self, prob, max_P: int, device: int = 0):
+        self.host = prob if isinstance(prob, HostProblem) else HostProblem(prob)
+        self.max_P = int(max_P)
+        self.device = int(device)
+        self.ptr = ctypes.c_void_p()
+        _check(load_library().wf_ctx_create(ctypes.byref(self.host.c), self.device, self.max_P,
+                                            ctypes.byref(self.ptr)), "wf_ctx_create")
+
+    @property
+    def N(self):
+        return self.host.N
+
+    def close(self):
+        if self.ptr:
+            load_library().wf_ctx_destroy(self.ptr)
+            self.ptr = ctypes.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def wf_ctx_create(prob, device: int = 0, max_P: int = 1) -> Ctx:
+    return Ctx(prob, max_P, device)
+
+
+def wf_ctx_destroy(ctx: Ctx):
+    ctx.close()
+
+
+def wf_ctx_status(ctx: Ctx, stream=None):
+    _check(load_library().wf_ctx_status(ctx.ptr, _stream_handle(stream)), "wf_ctx_status")
+
+
+def wf_forecast_readiness(ctx: Ctx, rel, comp, stream=None):
+    """rel, comp: device int64 tensors [N]."""
+    _check(load_library().wf_forecast_readiness(ctx.ptr, rel.data_ptr(), comp.data_ptr(),
+                                                _stream_handle(stream)), "wf_forecast_readiness")
+
+
+class DevicePlans:
+    """Plan arrays on the device (torch tensors) and their wf_plans view."""
+
+    def __init__(self, place, order, fuse, prefetch, retain=None, plan_base: int = 0):
+        self.place, self.order, self.fuse, self.prefetch, self.retain = place, order, fuse, prefetch, retain
+        self.P = int(place.shape[0])
+        self.plan_base = int(plan_base)
+
+    @staticmethod
+    def from_host(plans, device="cuda", non_blocking=False):
+        import torch
+
+        def t(x):
+            if x is None:
+                return None
+            h = torch.from_numpy(np.ascontiguousarray(x))
+            return h.to(device, non_blocking=non_blocking)
+        return DevicePlans(t(plans.place), t(plans.order.view(np.int16)), t(plans.fuse.view(np.int32)),
+                           t(plans.prefetch.view(np.int32)), t(None if plans.retain is None
+                                                               else plans.retain.view(np.int32)),
+                           plan_base=getattr(plans, "plan_base", 0))
+
+    def c(self, P: int | None = None, offset: int = 0) -> wf_plans:
+        P = self.P - offset if P is None else P
+        ps = self.place.stride(0)
+        os_ = self.order.stride(0) * 2
+        bs = self.fuse.stride(0) * 4
+        return wf_plans(P, self.plan_base + offset,
+                        self.place.data_ptr() + offset * ps, ps,
+                        self.order.data_ptr() + offset * os_, os_,
+                        self.fuse.data_ptr() + offset * bs, self.prefetch.data_ptr() + offset * bs,
+                        None if self.retain is None else self.retain.data_ptr() + offset * bs, bs)
+
+
+class Results:
+    """Per-plan outputs on the device."""
+
+    def __init__(self, P: int, device="cuda"):
+        import torch
+        self.makespan = torch.empty(P, dtype=torch.int64, device=device)
+        self.p95 = torch.empty(P, dtype=torch.int64, device=device)
+        self.gpu = torch.empty(P, dtype=torch.int64, device=device)
+        self.status = torch.empty(P, dtype=torch.int32, device=device)
+
+    def c(self, offset: int = 0) -> wf_eval_out:
+        return wf_eval_out(self.makespan.data_ptr() + 8 * offset, self.p95.data_ptr() + 8 * offset,
+                           self.gpu.data_ptr() + 8 * offset, self.status.data_ptr() + 4 * offset)
+
+    def numpy(self):
+        return (self.makespan.cpu().numpy(), self.p95.cpu().numpy(), self.gpu.cpu().numpy(),
+                self.status.cpu().numpy().view(np.uint32))
+
+
+def wf_eval_plans(ctx: Ctx, plans: DevicePlans, out: Results, stream=None, P: int | None = None,
+                  offset: int = 0):
+    pl = plans.c(P, offset)
+    oc = out.c(offset)
+    _check(load_library().wf_eval_plans(ctx.ptr, ctypes.byref(pl), ctypes.byref(oc),
+                                        _stream_handle(stream)), "wf_eval_plans")
+
+
+def wf_topk(ctx: Ctx, res: Results, P: int, k: int, ids, keys=None, stream=None):
+    """ids: device int32 [k]; keys: device int64 [k, 3] or None."""
+    oc = res.c()
+    _check(load_library().wf_topk(ctx.ptr, ctypes.byref(oc), int(P), int(k), ids.data_ptr(),
+                                  None if keys is None else keys.data_ptr(), _stream_handle(stream)),
+           "wf_topk")
+
+
+def evaluate(ctx: Ctx, plans, k: int, stream=None):
+    """End-to-end public call: host plans in (numpy / pinned), forecast, evaluation
+    and top-k on the device, and the top-k ids and keys back on the host."""
+    import torch
+    dev = torch.device("cuda", ctx.device)
+    dp = plans if isinstance(plans, DevicePlans) else DevicePlans.from_host(plans, dev, non_blocking=True)
+    res = Results(dp.P, dev)
+    rel = torch.empty(ctx.N, dtype=torch.int64, device=dev)
+    comp = torch.empty_like(rel)
+    ids = torch.empty(k, dtype=torch.int32, device=dev)
+    keys = torch.empty((k, 3), dtype=torch.int64, device=dev)
+    wf_forecast_readiness(ctx, rel, comp, stream)
+    wf_eval_plans(ctx, dp, res, stream)
+    wf_topk(ctx, res, dp.P, k, ids, keys, stream)
+    return ids.cpu().numpy(), keys.cpu().numpy()

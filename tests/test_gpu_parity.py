@@ -1,0 +1,195 @@
+"""Bit-exact parity of the CUDA path (through the C ABI) with the CPU oracle.
+
+Every quantity is an integer, so every comparison is exact equality.
+"""
+import numpy as np
+import pytest
+
+import oracle
+import wfgen
+from golden_util import fixture_names, load, plans_of, problem_of
+from gpu_util import assert_same, gpu_eval, oracle_eval
+from randprob import random_problem
+
+pytestmark = pytest.mark.gpu
+
+
+def inject_invalid(plans, prob, rng, frac=0.1):
+    """Corrupt a fraction of the plans in every way the status bits name."""
+    N, D = prob.N, prob.D
+    fits = prob.fits()
+    P = plans.P
+    idx = rng.choice(P, size=max(4, int(frac * P)), replace=False)
+    for j, p in enumerate(idx):
+        kind = j % 5
+        if kind == 0:
+            plans.place[p, rng.integers(N)] = D + rng.integers(0, 255 - D + 1)
+        elif kind == 1:
+            bad = np.argwhere(~fits)
+            if len(bad):
+                n, d = bad[rng.integers(len(bad))]
+                plans.place[p, n] = d
+        elif kind == 2:
+            i, j2 = rng.choice(N, size=2, replace=N < 2)
+            plans.order[p, i] = plans.order[p, j2]
+        elif kind == 3:
+            plans.order[p, rng.integers(N)] = N + rng.integers(0, 65535 - N + 1)
+        else:
+            # swap a node with its predecessor's position (against an edge)
+            v = int(rng.choice(np.nonzero(np.diff(prob.pred_off) > 0)[0]))
+            u = int(prob.pred_idx[prob.pred_off[v]])
+            pos = np.empty(N, int)
+            pos[plans.order[p, :N]] = np.arange(N)
+            plans.order[p, pos[u]], plans.order[p, pos[v]] = v, u
+    return idx
+
+
+@pytest.mark.parametrize("name", ["tiny", "mix", "burst"])
+def test_named_workload_full_parity(name):
+    w = wfgen.config(name)
+    plans = wfgen.make_plans(w.problem, w.P, w.plan_seed)
+    got = gpu_eval(w.problem, plans, k=w.k, forecast=True)
+    want = oracle_eval(w.problem, plans)
+    assert_same(got, want)
+    ids, keys = oracle.topk(want["makespan"], want["p95"], want["gpu"], want["status"], w.k)
+    assert np.array_equal(got["ids"], ids) and np.array_equal(got["keys"], keys)
+    rel, comp = oracle.forecast(w.problem)
+    assert np.array_equal(got["rel"], rel) and np.array_equal(got["comp"], comp)
+
+
+def test_stochastic_workload_full_parity():
+    w = wfgen.config("stochastic")
+    plans = wfgen.make_plans(w.problem, w.P, w.plan_seed)
+    got = gpu_eval(w.problem, plans, k=w.k)
+    want = oracle_eval(w.problem, plans)
+    assert_same(got, want)
+    ids, keys = oracle.topk(want["makespan"], want["p95"], want["gpu"], want["status"], w.k)
+    assert np.array_equal(got["ids"], ids) and np.array_equal(got["keys"], keys)
+
+
+def test_large_window_parity():
+    """Full size (P=131072, N=8192, D=16); the oracle checks every plan."""
+    w = wfgen.config("large")
+    plans = wfgen.make_plans(w.problem, w.P, w.plan_seed)
+    got = gpu_eval(w.problem, plans, k=w.k, forecast=True)
+    want = oracle_eval(w.problem, plans)
+    assert_same(got, want)
+    ids, keys = oracle.topk(want["makespan"], want["p95"], want["gpu"], want["status"], w.k)
+    assert np.array_equal(got["ids"], ids) and np.array_equal(got["keys"], keys)
+    rel, comp = oracle.forecast(w.problem)
+    assert np.array_equal(got["rel"], rel) and np.array_equal(got["comp"], comp)
+
+
+@pytest.mark.parametrize("name", fixture_names())
+def test_golden_windows_on_gpu(name):
+    fx = load(name)
+    for case in fx["cases"]:
+        prob = problem_of(fx, case)
+        plans = plans_of(fx, [case])
+        got = gpu_eval(prob, plans)
+        exp = case["expect"]
+        assert got["status"][0] == exp["status"], case["label"]
+        if exp["status"] == 0:
+            assert (got["makespan"][0], got["p95"][0], got["gpu"][0]) == \
+                (exp["makespan"], exp["p95"], exp["gpu"]), case["label"]
+
+
+@pytest.mark.parametrize("seed", range(8))
+def test_random_windows_with_invalid_plans_retain_and_grant(seed):
+    rng = np.random.default_rng(4000 + seed)
+    prob = random_problem(rng, n_sessions=int(rng.integers(1, 9)), sizes=(4, 12),
+                          D=int(rng.integers(1, 9)), M=int(rng.integers(1, 9)))
+    P = int(rng.integers(1, 700))
+    plans = wfgen.make_plans(prob, P, seed, p_fuse=float(rng.uniform(0, 1)),
+                             p_prefetch=float(rng.uniform(0, 1)),
+                             p_retain=float(rng.uniform(0.3, 1)) if seed % 2 else None)
+    if P >= 8:
+        inject_invalid(plans, prob, rng)
+    k = int(rng.integers(1, min(P, 64) + 1))
+    got = gpu_eval(prob, plans, k=k, forecast=True)
+    want = oracle_eval(prob, plans)
+    assert_same(got, want)
+    ids, keys = oracle.topk(want["makespan"], want["p95"], want["gpu"], want["status"], k)
+    assert np.array_equal(got["ids"], ids) and np.array_equal(got["keys"], keys)
+    rel, comp = oracle.forecast(prob)
+    assert np.array_equal(got["rel"], rel) and np.array_equal(got["comp"], comp)
+
+
+@pytest.mark.parametrize("seed", range(3))
+def test_random_stochastic_windows(seed):
+    rng = np.random.default_rng(4100 + seed)
+    prob = random_problem(rng, n_sessions=int(rng.integers(1, 6)), D=int(rng.integers(1, 6)))
+    r, c, e = wfgen.box_muller_tables()
+    prob = prob.with_(S=int(rng.integers(1, 100)), seed=int(rng.integers(0, 2**63)), bm_r=r, bm_c=c, bm_e=e)
+    plans = wfgen.make_plans(prob, int(rng.integers(1, 300)), seed, plan_base=int(rng.integers(0, 10**6)),
+                             p_retain=0.7 if seed % 2 else None)
+    if plans.P >= 8:
+        inject_invalid(plans, prob, rng)
+    got = gpu_eval(prob, plans)
+    assert_same(got, oracle_eval(prob, plans))
+
+
+def test_ties_break_by_plan_index():
+    w = wfgen.config("tiny")
+    base = wfgen.make_plans(w.problem, 64, 3)
+    plans = wfgen.Plans.empty(256, w.problem.N)
+    for a in ("place", "order", "fuse", "prefetch"):
+        getattr(plans, a)[:] = np.tile(getattr(base, a), (4, 1))
+    got = gpu_eval(w.problem, plans, k=40)
+    want = oracle_eval(w.problem, plans)
+    assert_same(got, want)
+    ids, _ = oracle.topk(want["makespan"], want["p95"], want["gpu"], want["status"], 40)
+    assert np.array_equal(got["ids"], ids)
+
+
+def test_sub_batches_reproduce_the_batch():
+    """Evaluating row ranges with an offset equals evaluating the whole batch."""
+    import torch
+    from gpu_util import lib
+    wf = lib()
+    w = wfgen.config("mix")
+    plans = wfgen.make_plans(w.problem, 3000, 5, p_retain=0.5)
+    ctx = wf.Ctx(w.problem, max_P=3000)
+    dp = wf.DevicePlans.from_host(plans, "cuda")
+    whole = wf.Results(3000)
+    wf.wf_eval_plans(ctx, dp, whole)
+    parts = wf.Results(3000)
+    for lo, hi in ((0, 1), (1, 1000), (1000, 2999), (2999, 3000)):
+        wf.wf_eval_plans(ctx, dp, parts, P=hi - lo, offset=lo)
+    torch.cuda.synchronize()
+    for a, b in zip(whole.numpy(), parts.numpy()):
+        assert np.array_equal(a, b)
+
+
+def test_single_node_and_extreme_shapes():
+    rng = np.random.default_rng(17)
+    one = wfgen.Problem(N=1, D=1, M=1, W=1, pred_off=np.zeros(2, np.int32),
+                        pred_idx=np.zeros(0, np.int32), model=np.zeros(1, np.uint8),
+                        session=np.zeros(1, np.int32), arrival_us=np.array([5], np.int64),
+                        lat_us=np.array([7], np.int32), peak_mib=np.array([3], np.int32),
+                        weight_mib=np.array([2], np.int32), load_us=np.array([11], np.int32),
+                        cap_mib=np.array([4], np.int32), grant_us=1)
+    plans = wfgen.make_plans(one, 3, 0)
+    got = gpu_eval(one, plans, k=3)
+    assert got["makespan"].tolist() == [19, 19, 19]  # load 11 + grant 1 + run 7
+    assert got["ids"].tolist() == [0, 1, 2]
+    # 32 devices, 16 models, tight memory
+    prob = random_problem(rng, n_sessions=12, sizes=(6, 14), D=32, M=16)
+    plans = wfgen.make_plans(prob, 777, 1, p_retain=0.5)
+    got = gpu_eval(prob, plans, k=1)
+    assert_same(got, oracle_eval(prob, plans))
+
+
+def test_long_chain_window():
+    """A 20000-activation window (chains of one model, heavy fusion)."""
+    N = 20000
+    n_sess = 40
+    sizes = wfgen.split_sizes(N, n_sess)
+    sess = [wfgen.fam_softdev(s) for s in sizes]
+    rng = np.random.default_rng(23)
+    prob = wfgen.assemble("long", sess, np.zeros(n_sess, np.int64), wfgen.DEV_BURST,
+                          [3, 6, 8, 14], rng)
+    plans = wfgen.make_plans(prob, 512, 2, p_fuse=0.9)
+    got = gpu_eval(prob, plans, k=16)
+    want = oracle_eval(prob, plans)
+    assert_same(got, want)
