@@ -13,6 +13,7 @@
  *   wf_forecast_readiness   release forecast of every activation (Eq. 2)
  *   wf_eval_plans           play every plan forward (Eq. 2-11) -> metrics
  *   wf_topk                 the k best plans by the ranking key
+ *   wf_eval_plans_static    wf_eval_plans without a context or any allocation
  *   wf_ctx_destroy, wf_strerror
  *
  * Conventions.
@@ -177,6 +178,35 @@ int wf_eval_plans(wf_ctx *ctx, const wf_plans *plans, const wf_eval_out *out, vo
  */
 int wf_topk(wf_ctx *ctx, const wf_eval_out *res, int64_t P, int32_t k,
             int32_t *ids_dev, int64_t *keys_dev, void *stream);
+
+/*
+ * The paper has no counterpart to this entry point; it serves callers that
+ * cannot allocate device memory when they score plans -- for example a
+ * scheduler inside a serving engine that reserved nearly all GPU memory up
+ * front for weights and KV cache, where another cudaMalloc fails or eats into
+ * the cache -- or whose device memory belongs to an allocator that must not
+ * be bypassed.
+ *
+ * Same results as wf_eval_plans for a deterministic problem (S must be 0),
+ * without a context and without allocating anything: every table of *prob is
+ * a DEVICE pointer here (same layouts as above; the caller guarantees the
+ * problem passes wf_problem_check, which this call cannot repeat without
+ * copying it back), plans and outputs are DEVICE pointers as for
+ * wf_eval_plans.  Scratch is a 32 MiB file-scope device array that every GPU
+ * loading this library holds until the process exits.  A call needs 256 B,
+ * plus three tables of 4*N bytes each rounded up to 256 B, plus one state row
+ * per plan of about 8*(N + W + 3*D) + 4*D*(M + 2) bytes (rounded up to
+ * 128 B); a batch that does not fit returns WF_EINVAL naming the largest
+ * batch that does (about 1,900 plans of a 2,000-activation window) -- split
+ * larger batches by plan_base.  The first call on a device looks the array's
+ * address up (cudaGetSymbolAddress) with that device current; make that first
+ * call before any stream capture.  All calls share the array and each call
+ * re-initialises what it relies on; calls that overlap on the GPU (other
+ * streams, other threads) race on it and must be serialised by the caller.
+ * Asynchronous on `stream`; returns WF_OK, WF_EINVAL or WF_ECUDA.
+ */
+int wf_eval_plans_static(const wf_problem *prob, const wf_plans *plans, const wf_eval_out *out,
+                         void *stream);
 
 /*
  * Synchronize `stream` and report device-side failures of earlier calls on

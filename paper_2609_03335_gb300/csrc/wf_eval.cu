@@ -8,6 +8,7 @@
 // finish times, per-device and per-session state) lives in a scratch row of
 // the context; plans beyond the number of rows are taken in rounds.
 #include <algorithm>
+#include <mutex>
 
 #include "wf_internal.cuh"
 
@@ -367,4 +368,190 @@ int wf_launch_eval(wf_ctx *ctx, const wf_plans *plans, const wf_eval_out *out, c
                                                                       ctx->eval_row_bytes, pool, units);
     }
     return wf_cuda_check(cudaGetLastError(), "eval launch");
+}
+
+// ---------------------------------------------------------------------------
+// Allocation-free entry point: wf_eval_plans_static.
+//
+// Some callers cannot allocate device memory when they want to score plans:
+// a scheduler that runs inside a serving engine which reserved nearly all of
+// the GPU's memory up front for model weights and KV cache (an extra
+// cudaMalloc there fails, or takes memory the engine's cache counts on), or a
+// process whose device memory belongs to another allocator that must not be
+// bypassed.  For them this entry point evaluates a deterministic batch with
+// no context and no allocation: the caller passes the problem tables, the
+// plans and the outputs as device pointers, and every piece of scratch lives
+// in the file-scope array below, which each GPU that loads this library holds
+// until the process exits.
+// ---------------------------------------------------------------------------
+
+namespace {
+
+constexpr size_t kStaticScratchBytes = (size_t)32 << 20;  // 32 MiB
+constexpr size_t kStaticHeader = 256;                     // first arrival, error word
+
+static __device__ __align__(256) uint8_t g_static_scratch[kStaticScratchBytes];
+
+__host__ __device__ __forceinline__ size_t up256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+// Layout: header | succ count [N] | fusible successor [N] | fusible predecessor [N] | rows [P]
+struct StaticLayout {
+    size_t nsucc, fnext, fprev, rows, total;
+};
+
+__host__ __device__ __forceinline__ StaticLayout static_layout(int32_t N, int64_t P, size_t row)
+{
+    StaticLayout l;
+    l.nsucc = kStaticHeader;
+    l.fnext = l.nsucc + up256(4 * (size_t)N);
+    l.fprev = l.fnext + up256(4 * (size_t)N);
+    l.rows = l.fprev + up256(4 * (size_t)N);
+    l.total = l.rows + (size_t)P * row;
+    return l;
+}
+
+// Everything the derived tables start from: zero successor counts, no links,
+// the first arrival at +infinity, a clear error word.
+__global__ void static_init_kernel(uint8_t *s, int32_t N, StaticLayout l)
+{
+    const int32_t n = blockIdx.x * blockDim.x + threadIdx.x;
+    if (n == 0) {
+        *(int64_t *)s = WF_INF64;
+        *(int *)(s + 8) = 0;
+    }
+    if (n < N) {
+        ((int32_t *)(s + l.nsucc))[n] = 0;
+        ((int32_t *)(s + l.fnext))[n] = -1;
+        ((int32_t *)(s + l.fprev))[n] = -1;
+    }
+}
+
+__global__ void static_count_kernel(uint8_t *s, wf_dev_problem dp, StaticLayout l)
+{
+    const int32_t v = blockIdx.x * blockDim.x + threadIdx.x;
+    if (v < dp.W) atomicMin((long long *)s, (long long)dp.arrival[v]);
+    if (v >= dp.N) return;
+    int32_t *nsucc = (int32_t *)(s + l.nsucc);
+    for (int32_t e = dp.pred_off[v]; e < dp.pred_off[v + 1]; ++e) atomicAdd(&nsucc[dp.pred_idx[e]], 1);
+}
+
+// Eq. 3: (u, v) fusible iff succ(u) = {v}, pred(v) = {u}, same model.
+__global__ void static_link_kernel(uint8_t *s, wf_dev_problem dp, StaticLayout l)
+{
+    const int32_t v = blockIdx.x * blockDim.x + threadIdx.x;
+    if (v >= dp.N || dp.pred_off[v + 1] - dp.pred_off[v] != 1) return;
+    const int32_t u = dp.pred_idx[dp.pred_off[v]];
+    if (((const int32_t *)(s + l.nsucc))[u] == 1 && dp.model[u] == dp.model[v]) {
+        ((int32_t *)(s + l.fnext))[u] = v;
+        ((int32_t *)(s + l.fprev))[v] = u;
+    }
+}
+
+// The deterministic evaluation with one scratch row per plan and the first
+// arrival taken from the static header.
+__global__ void __launch_bounds__(kEvalThreads)
+eval_static_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, uint8_t *s, StaticLayout l,
+                   size_t row_bytes)
+{
+    const int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (p >= pl.P) return;
+    wf_dev_problem d = dp;
+    d.first_arrival = *(const int64_t *)s;
+    Row row = row_at(d, s + l.rows + (size_t)p * row_bytes);
+    const PlanRows pr = plan_rows(pl, p);
+    const uint32_t st = plan_status(d, pr, row);
+    out.status[p] = st;
+    if (st) {
+        out.makespan_us[p] = out.p95_us[p] = out.gpu_us[p] = WF_INF64;
+        return;
+    }
+    int64_t mk, g;
+    play<false>(d, pr, row, 0, &mk, &g);
+    out.makespan_us[p] = mk;
+    out.gpu_us[p] = g;
+    out.p95_us[p] = select_rank(row.comp, d.W, p95_rank(d.W));
+}
+
+// Device address of the static array, looked up once per device.
+uint8_t *g_static_addr[64];
+bool g_static_ready[64];
+std::mutex g_static_mu;
+
+}  // namespace
+
+extern "C" int wf_eval_plans_static(const wf_problem *pb, const wf_plans *pl, const wf_eval_out *out,
+                                    void *stream)
+{
+    if (!pb || !pl || !out) return wf_set_error(WF_EINVAL, "NULL argument");
+    const int32_t N = pb->N, D = pb->D, M = pb->M, W = pb->W;
+    if (N < 1 || N > 65535 || D < 1 || D > 32 || M < 1 || M > 16 || W < 1)
+        return wf_set_error(WF_EINVAL, "sizes outside N 1..65535, D 1..32, M 1..16, W >= 1");
+    if (pb->S != 0) return wf_set_error(WF_EINVAL, "wf_eval_plans_static evaluates deterministic problems (S = 0) only");
+    if (!pb->pred_off || !pb->model || !pb->session || !pb->arrival_us || !pb->lat_us || !pb->peak_mib ||
+        !pb->weight_mib || !pb->load_us || !pb->cap_mib || pb->grant_us < 0)
+        return wf_set_error(WF_EINVAL, "a problem table pointer is NULL or grant_us < 0");
+    if (pl->P < 1 || !pl->place || !pl->order || !pl->fuse || !pl->prefetch || pl->plan_base < 0)
+        return wf_set_error(WF_EINVAL, "empty batch or NULL plan array");
+    if (!out->makespan_us || !out->p95_us || !out->gpu_us || !out->status)
+        return wf_set_error(WF_EINVAL, "NULL output array");
+    const int64_t words = ((int64_t)N + 31) / 32;
+    if (pl->place_stride < N || pl->place_stride % 16 || pl->order_stride < 2 * (int64_t)N ||
+        pl->order_stride % 16 || pl->bits_stride < 4 * words || pl->bits_stride % 16)
+        return wf_set_error(WF_EINVAL, "plan strides must be multiples of 16 covering N");
+    const uintptr_t mis = (uintptr_t)pl->place | (uintptr_t)pl->order | (uintptr_t)pl->fuse |
+                          (uintptr_t)pl->prefetch | (uintptr_t)pl->retain;
+    if (mis & 15u) return wf_set_error(WF_EINVAL, "plan arrays must be 16-byte aligned");
+
+    wf_dev_problem dp = {};
+    dp.N = N; dp.D = D; dp.M = M; dp.W = W;
+    dp.grant = pb->grant_us;
+    dp.pred_off = pb->pred_off;
+    dp.pred_idx = pb->pred_idx;
+    dp.model = pb->model;
+    dp.session = pb->session;
+    dp.arrival = pb->arrival_us;
+    dp.lat = pb->lat_us;
+    dp.peak = pb->peak_mib;
+    dp.weight = pb->weight_mib;
+    dp.load = pb->load_us;
+    dp.cap = pb->cap_mib;
+    const size_t row = wf_eval_row_bytes(dp);
+    const StaticLayout l = static_layout(N, pl->P, row);
+    if (l.total > kStaticScratchBytes) {
+        const int64_t fit = (int64_t)((kStaticScratchBytes - l.rows) / row);
+        return wf_set_error(WF_EINVAL,
+                            "batch needs %zu bytes of scratch but the static array holds %zu; at most "
+                            "%lld plans of this window per call", l.total, kStaticScratchBytes,
+                            (long long)fit);
+    }
+
+    int dev = 0;
+    int rc = wf_cuda_check(cudaGetDevice(&dev), "cudaGetDevice");
+    if (rc) return rc;
+    if (dev < 0 || dev >= 64) return wf_set_error(WF_EINVAL, "device ordinal %d >= 64", dev);
+    uint8_t *s = nullptr;
+    {
+        std::lock_guard<std::mutex> lock(g_static_mu);
+        if (!g_static_ready[dev]) {
+            void *p = nullptr;
+            rc = wf_cuda_check(cudaGetSymbolAddress(&p, g_static_scratch), "cudaGetSymbolAddress");
+            if (rc) return rc;
+            g_static_addr[dev] = (uint8_t *)p;
+            g_static_ready[dev] = true;
+        }
+        s = g_static_addr[dev];
+    }
+    dp.fnext = (const int32_t *)(s + l.fnext);
+    dp.fprev = (const int32_t *)(s + l.fprev);
+    dp.err = (int *)(s + 8);
+
+    cudaStream_t st = (cudaStream_t)stream;
+    const int32_t span = std::max(N, W);
+    const unsigned grid = (unsigned)((span + 255) / 256);
+    static_init_kernel<<<(unsigned)((N + 255) / 256), 256, 0, st>>>(s, N, l);
+    static_count_kernel<<<grid, 256, 0, st>>>(s, dp, l);
+    static_link_kernel<<<(unsigned)((N + 255) / 256), 256, 0, st>>>(s, dp, l);
+    eval_static_kernel<<<(unsigned)((pl->P + kEvalThreads - 1) / kEvalThreads), kEvalThreads, 0, st>>>(
+        dp, *pl, *out, s, l, row);
+    return wf_cuda_check(cudaGetLastError(), "static evaluation launch");
 }

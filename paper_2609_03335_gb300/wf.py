@@ -22,7 +22,8 @@ INT64_MAX = np.iinfo(np.int64).max
 
 # Every entry point declared in include/wf.h.
 EXPORTS = ("wf_problem_check", "wf_ctx_create", "wf_forecast_readiness", "wf_eval_plans",
-           "wf_topk", "wf_ctx_status", "wf_ctx_destroy", "wf_strerror", "wf_last_error")
+           "wf_topk", "wf_ctx_status", "wf_ctx_destroy", "wf_strerror", "wf_last_error",
+           "wf_eval_plans_static")
 
 
 class WfError(RuntimeError):
@@ -79,6 +80,7 @@ def load_library():
         "wf_ctx_destroy": ([p], None),
         "wf_strerror": ([ctypes.c_int], ctypes.c_char_p),
         "wf_last_error": ([], ctypes.c_char_p),
+        "wf_eval_plans_static": ([p, p, p, p], ctypes.c_int),
     }
     for name, (args, res) in sig.items():
         f = getattr(lib, name)
@@ -280,3 +282,28 @@ def evaluate(ctx: Ctx, plans, k: int, stream=None):
     wf_eval_plans(ctx, dp, res, stream)
     wf_topk(ctx, res, dp.P, k, ids, keys, stream)
     return ids.cpu().numpy(), keys.cpu().numpy()
+
+
+class DeviceProblem:
+    """A problem whose tables already sit in device memory (torch tensors),
+    viewed as a wf_problem of DEVICE pointers for wf_eval_plans_static."""
+
+    def __init__(self, prob, device="cuda"):
+        import torch
+        hp = HostProblem(prob)
+        self.tensors = {n: torch.from_numpy(v.view(np.int8) if v.dtype == np.uint8 else v).to(device)
+                        for n, v in hp.keep.items() if v.size}
+        ptr = {n: (self.tensors[n].data_ptr() if n in self.tensors else None) for n in hp.keep}
+        self.c = wf_problem(hp.N, hp.D, hp.M, hp.W, ptr["pred_off"], ptr["pred_idx"], ptr["model"],
+                            ptr["session"], ptr["arrival_us"], ptr["lat_us"], ptr["peak_mib"],
+                            ptr["weight_mib"], ptr["load_us"], ptr["cap_mib"], int(prob.grant_us),
+                            int(prob.S), int(prob.seed) & ((1 << 64) - 1), None, None, None, 0, 0, 0)
+
+
+def wf_eval_plans_static(prob: DeviceProblem, plans: DevicePlans, out: Results, stream=None):
+    """wf_eval_plans without a context or any device allocation (deterministic
+    problems; scratch in the library's static device array)."""
+    pl = plans.c()
+    oc = out.c()
+    _check(load_library().wf_eval_plans_static(ctypes.byref(prob.c), ctypes.byref(pl), ctypes.byref(oc),
+                                               _stream_handle(stream)), "wf_eval_plans_static")
