@@ -10,7 +10,7 @@ CSRC = os.path.join(HERE, "csrc")
 ROOT = os.path.dirname(HERE)
 LIB = os.path.join(HERE, "libwf.so")
 OBJ = os.path.join(HERE, "_build")
-SOURCES = ["wf_ctx.cu", "wf_forecast.cu", "wf_eval.cu", "wf_topk.cu"]
+SOURCES = ["wf_ctx.cu", "wf_slots.cpp", "wf_forecast.cu", "wf_eval.cu", "wf_sweep.cu", "wf_topk.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",
          "--expt-relaxed-constexpr", "-I", os.path.join(ROOT, "include")]
@@ -39,7 +39,7 @@ def build(force: bool = False, verbose: bool = False, extra: tuple = ()) -> str:
     jobs = []
     for s in SOURCES:
         src = os.path.join(CSRC, s)
-        obj = os.path.join(OBJ, s.replace(".cu", ".o"))
+        obj = os.path.join(OBJ, os.path.splitext(s)[0] + ".o")
         objs.append(obj)
         if force or _stale(obj, [src, *headers]):
             jobs.append([nvcc(), *ARCH, *FLAGS, *extra, "-c", src, "-o", obj])

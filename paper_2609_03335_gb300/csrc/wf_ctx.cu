@@ -212,11 +212,40 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
     size_t o_bc = img.add(stoch ? pb->bm_c : nullptr, stoch ? sizeof(int32_t) * pb->bm_cn : 0);
     size_t o_be = img.add(stoch ? pb->bm_e : nullptr, stoch ? sizeof(int32_t) * pb->bm_en : 0);
     size_t o_err = img.add(nullptr, 256);
+    // Slot tables of the shared-memory sweep.
+    std::vector<int32_t> rslot(N), wl_off;
+    std::vector<uint16_t> wl;
+    const int32_t nslots = wf_assign_slots(N, W, pb->pred_off, pb->pred_idx, pb->session, dv.fprev.data(),
+                                           dv.fnext.data(), rslot.data(), wl_off, wl);
+    std::vector<int4> noderec(2 * (size_t)N);
+    std::vector<int2> lk((size_t)N * D);
+    for (int32_t n = 0; n < N; ++n) {
+        noderec[2 * n] = make_int4(dv.fprev[n], dv.fnext[n], rslot[n], (int32_t)pb->model[n] | (pb->session[n] << 8));
+        // Write list of n as a unit's last member: start, length, first two codes inline.
+        const int32_t a = wl_off[n], len = wl_off[n + 1] - wl_off[n];
+        const uint32_t c0 = len > 0 ? wl[a] : 0u, c1 = len > 1 ? wl[a + 1] : 0u;
+        noderec[2 * n + 1] = make_int4(a, len, (int32_t)(c0 | (c1 << 16)), 0);
+        for (int32_t d = 0; d < D; ++d) {
+            const int64_t i = (int64_t)n * D + d;
+            lk[i] = make_int2(pb->lat_us[i], pb->peak_mib[i] - pb->weight_mib[pb->model[n]]);
+        }
+    }
+    size_t o_rec = img.add(noderec.data(), sizeof(int4) * noderec.size());
+    std::vector<uint32_t> links(N);
+    for (int32_t n = 0; n < N; ++n)
+        links[n] = ((uint32_t)dv.fprev[n] & 0xFFFFu) | ((uint32_t)dv.fnext[n] << 16);  // -1 -> 0xFFFF
+    size_t o_links = img.add(links.data(), sizeof(uint32_t) * N);
+    size_t o_wloff = img.add(wl_off.data(), sizeof(int32_t) * (N + 1));
+    size_t o_wl = img.add(wl.data(), sizeof(uint16_t) * wl.size());
+    size_t o_lk = img.add(lk.data(), sizeof(int2) * lk.size());
+    size_t o_ovf = img.add(nullptr, sizeof(int32_t) * ((size_t)max_P + 64));
 
     wf_ctx *c = (wf_ctx *)calloc(1, sizeof(wf_ctx));
     if (!c) return wf_set_error(WF_ENOMEM, "host allocation of the context");
     c->device = device;
     c->max_P = max_P;
+    const char *path = getenv("WF_EVAL_PATH");
+    c->force_int64 = path && strcmp(path, "int64") == 0;
     c->tables_bytes = img.bytes.size();
     rc = wf_cuda_check(cudaMalloc(&c->tables, c->tables_bytes), "cudaMalloc(tables)");
     if (!rc) rc = wf_cuda_check(cudaMemcpy(c->tables, img.bytes.data(), c->tables_bytes,
@@ -254,6 +283,19 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
     dp.bm_e = (const int32_t *)(base + o_be);
     dp.err = (int *)(base + o_err);
     c->err = dp.err;
+    dp.nslots = nslots > 0 ? nslots : 0;
+    dp.noderec = (const int4 *)(base + o_rec);
+    dp.wl_off = (const int32_t *)(base + o_wloff);
+    dp.wl = (const uint16_t *)(base + o_wl);
+    dp.lk = (const int2 *)(base + o_lk);
+    dp.links = (const uint32_t *)(base + o_links);
+    int64_t amax = 0;
+    for (int32_t w = 0; w < W; ++w) amax = std::max(amax, pb->arrival_us[w]);
+    dp.max_arrival = amax;
+    c->ovf_count = (int32_t *)(base + o_ovf);
+    c->ovf_list = c->ovf_count + 64;
+    rc = wf_cuda_check(cudaDeviceGetAttribute(&c->sms, cudaDevAttrMultiProcessorCount, device), "SM count");
+    if (rc) { wf_ctx_destroy(c); return rc; }
 
     // Scratch for the evaluation kernels, bounded by a budget; a call with
     // more plans than the scratch holds walks over it in rounds.

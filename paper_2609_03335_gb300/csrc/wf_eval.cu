@@ -254,6 +254,32 @@ eval_det_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, uint8_t *scratc
     }
 }
 
+// The int64 path for the plans whose times overflow the sweep's u32 slots.
+__global__ void __launch_bounds__(kEvalThreads)
+eval_list_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, uint8_t *scratch, size_t row_bytes,
+                 int64_t rows, const int32_t *list, const int32_t *count)
+{
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int32_t n = *count;
+    if (t >= rows || t >= n) return;
+    Row row = row_at(dp, scratch + (size_t)t * row_bytes);
+    for (int64_t k = t; k < n; k += rows) {
+        const int64_t p = list[k];
+        const PlanRows pr = plan_rows(pl, p);
+        const uint32_t st = plan_status(dp, pr, row);
+        out.status[p] = st;
+        if (st) {
+            out.makespan_us[p] = out.p95_us[p] = out.gpu_us[p] = WF_INF64;
+            continue;
+        }
+        int64_t mk, g;
+        play<false>(dp, pr, row, 0, &mk, &g);
+        out.makespan_us[p] = mk;
+        out.gpu_us[p] = g;
+        out.p95_us[p] = select_rank(row.comp, dp.W, p95_rank(dp.W));
+    }
+}
+
 // Stochastic latencies: one CTA per plan, one thread per sample; the pooled
 // S x W completions of the plan go to a per-CTA pool for the p95 selection.
 __global__ void __launch_bounds__(kSampleThreads)
@@ -359,8 +385,18 @@ int wf_launch_eval(wf_ctx *ctx, const wf_plans *plans, const wf_eval_out *out, c
     const int64_t units = std::min<int64_t>(ctx->eval_threads, plans->P);
     if (dp.S == 0) {
         const int64_t blocks = (units + kEvalThreads - 1) / kEvalThreads;
-        eval_det_kernel<<<(unsigned)blocks, kEvalThreads, 0, st>>>(dp, *plans, *out, scratch,
-                                                                    ctx->eval_row_bytes, units);
+        const size_t smem = ctx->force_int64 ? 0 : wf_sweep_smem(dp);
+        if (smem) {
+            int rc = wf_cuda_check(cudaMemsetAsync(ctx->ovf_count, 0, sizeof(int32_t), st), "reset overflow count");
+            if (!rc) rc = wf_launch_sweep(ctx, plans, out, smem, ctx->ovf_list, ctx->ovf_count, st);
+            if (rc) return rc;
+            eval_list_kernel<<<(unsigned)blocks, kEvalThreads, 0, st>>>(dp, *plans, *out, scratch,
+                                                                       ctx->eval_row_bytes, units,
+                                                                       ctx->ovf_list, ctx->ovf_count);
+        } else {
+            eval_det_kernel<<<(unsigned)blocks, kEvalThreads, 0, st>>>(dp, *plans, *out, scratch,
+                                                                        ctx->eval_row_bytes, units);
+        }
     } else {
         // Per-thread rows of every CTA first, then one completion pool per CTA.
         int64_t *pool = (int64_t *)(scratch + (size_t)units * kSampleThreads * ctx->eval_row_bytes);

@@ -3,6 +3,7 @@
 
 #include <cuda_runtime.h>
 #include <cstdint>
+#include <vector>
 
 #include "../../include/wf.h"
 
@@ -33,7 +34,24 @@ struct wf_dev_problem {
     int32_t nlev;
     const int32_t *bm_r, *bm_c, *bm_e;
     int *err;                   // device error word (0 = ok)
+
+    // Finish-time slots of the per-plan sweep (see wf_slots.cpp).  Slots
+    // [0, W) hold the sessions' latest finish; the others carry release
+    // times from producers to consumers.
+    int32_t nslots;             // 0 when the slot sweep is not usable
+    const int4 *noderec;        // [2N]: {fprev, fnext, rslot code, model | session << 8},
+                                //       {write-list start, length, first two codes, 0}
+    const int32_t *wl_off;      // [N+1] write list of each node when it ends a unit
+    const uint16_t *wl;         // [wl_off[N]] slot | (max-accumulate << 15)
+    const int2 *lk;             // [N][D] {run time, KV need = peak - weight}
+    const uint32_t *links;      // [N] fusible predecessor | fusible successor << 16 (0xFFFF = none)
+    int64_t max_arrival;
 };
+
+// rslot code of noderec.z: -1 = no predecessor (release = arrival), else the
+// slot index, with bit 30 set when the slot is an accumulator that the
+// reader resets to 0 after reading.
+#define WF_RSLOT_ACC (1 << 30)
 
 struct wf_ctx {
     int device;
@@ -48,7 +66,17 @@ struct wf_ctx {
     void *topk_scratch;
     size_t topk_scratch_bytes;
     int *err;
+    int sms;                    // streaming multiprocessors of the device
+    bool force_int64;           // WF_EVAL_PATH=int64: always take the int64 path (tests)
+    int32_t *ovf_count;         // plans the u32 sweep hands to the int64 path
+    int32_t *ovf_list;          // [max_P]
 };
+
+// Static slot assignment (wf_slots.cpp).  Fills rslot code per node, write
+// lists (CSR) and returns the slot count, or -1 when it exceeds 32767.
+int32_t wf_assign_slots(int32_t N, int32_t W, const int32_t *pred_off, const int32_t *pred_idx,
+                        const int32_t *session, const int32_t *fprev, const int32_t *fnext,
+                        int32_t *rslot, std::vector<int32_t> &wl_off, std::vector<uint16_t> &wl);
 
 // Error plumbing (wf_ctx.cu).
 int wf_set_error(int code, const char *fmt, ...);
@@ -62,3 +90,6 @@ int wf_launch_topk(wf_ctx *ctx, const wf_eval_out *res, int64_t P, int32_t k, in
 size_t wf_eval_row_bytes(const wf_dev_problem &dp);
 size_t wf_eval_scratch_bytes(const wf_dev_problem &dp, int64_t max_P, int64_t *units);
 size_t wf_topk_scratch_bytes(int64_t max_P);
+size_t wf_sweep_smem(const wf_dev_problem &dp);
+int wf_launch_sweep(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, size_t smem,
+                    int32_t *ovf_list, int32_t *ovf_count, cudaStream_t st);

@@ -1,0 +1,507 @@
+// Plan evaluation, shared-memory sweep (rows a3-a10, deterministic plans).
+//
+// One thread plays one plan; a CTA holds G plans.  The CTA's plan rows
+// (placement, fusion / prefetch / retain bits) are staged into shared memory
+// by one thread with TMA bulk copies (cp.async.bulk, completion on an
+// mbarrier).  Each plan's mutable state lives in shared memory next to them,
+// interleaved [index][plan] so that the G lanes of a warp never collide on a
+// bank:
+//   - finish-time slots (u32 microseconds) assigned statically from the DAG
+//     (wf_slots.cpp) instead of one word per activation;
+//   - per device: free time, resident weights, resident count, LRU stamps;
+//   - a bitmap of dispatched activations (status bits 4 and 8).
+// The sweep itself follows Eq. 2-11 exactly like the int64 path in
+// wf_eval.cu; a plan whose times reach 2^32 us is handed to that path.
+#include <algorithm>
+
+#include "wf_internal.cuh"
+
+namespace {
+
+constexpr uint32_t kWaitLimit = 1u << 24;  // bounded mbarrier wait (error word 3 on expiry)
+
+__device__ __forceinline__ uint32_t smem_addr(const void *p)
+{
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t *bar)
+{
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_addr(bar)) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_expect(uint64_t *bar, uint32_t bytes)
+{
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
+                 : "memory");
+}
+
+// Global -> shared bulk copy; bytes and both addresses are multiples of 16.
+__device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar)
+{
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                 ::"r"(smem_addr(dst)), "l"(src), "r"(bytes), "r"(smem_addr(bar))
+                 : "memory");
+}
+
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity)
+{
+    for (uint32_t it = 0; it < kWaitLimit; ++it) {
+        uint32_t ok;
+        asm volatile("{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+                     " selp.u32 %0, 1, 0, p;\n}"
+                     : "=r"(ok)
+                     : "r"(smem_addr(bar)), "r"(parity)
+                     : "memory");
+        if (ok) return true;
+    }
+    return false;
+}
+
+__host__ __device__ __forceinline__ uint32_t round16(uint32_t x) { return (x + 15u) & ~15u; }
+
+// Resident models of one device as a queue of 4-bit model ids, least
+// recently used in nibble 0; nibbles at and above the count are zero.  A
+// 32-bit word holds up to 8 models, a 64-bit word up to 16.
+template <typename Q>
+struct Lru;
+
+template <>
+struct Lru<uint32_t> {
+    static constexpr uint32_t kOnes = 0x11111111u, kHigh = 0x88888888u;
+    static constexpr int kSlots = 8;
+    __device__ static __forceinline__ int32_t find(uint32_t q, uint32_t n, uint32_t m)
+    {
+        const uint32_t x = q ^ (kOnes * m);
+        const uint32_t t = (x - kOnes) & ~x & kHigh;  // lowest zero nibble
+        const int32_t k = t ? (__ffs((int)t) - 1) >> 2 : kSlots;
+        return k < (int32_t)n ? k : (int32_t)n;
+    }
+    __device__ static __forceinline__ uint32_t remove(uint32_t q, int32_t k)
+    {
+        const uint32_t low = q & ((1u << (4 * k)) - 1u);
+        const uint32_t high = k < kSlots - 1 ? ((q >> (4 * k + 4)) << (4 * k)) : 0u;
+        return low | high;
+    }
+};
+
+template <>
+struct Lru<uint64_t> {
+    static constexpr uint64_t kOnes = 0x1111111111111111ull, kHigh = 0x8888888888888888ull;
+    static constexpr int kSlots = 16;
+    __device__ static __forceinline__ int32_t find(uint64_t q, uint32_t n, uint32_t m)
+    {
+        const uint64_t x = q ^ (kOnes * m);
+        const uint64_t t = (x - kOnes) & ~x & kHigh;
+        const int32_t k = t ? (__ffsll((long long)t) - 1) >> 2 : kSlots;
+        return k < (int32_t)n ? k : (int32_t)n;
+    }
+    __device__ static __forceinline__ uint64_t remove(uint64_t q, int32_t k)
+    {
+        const uint64_t low = k ? (q & ((1ull << (4 * k)) - 1)) : 0ull;
+        const uint64_t high = k < kSlots - 1 ? ((q >> (4 * k + 4)) << (4 * k)) : 0ull;
+        return low | high;
+    }
+};
+
+__device__ __forceinline__ uint32_t bit_of_g(const uint32_t *row, int32_t n)
+{
+    return (__ldg(row + (n >> 5)) >> (n & 31)) & 1u;
+}
+
+// CTA shape: warp 0 plays kPlans plans (one per lane); warps 1..kProducers
+// prepare their unit records, kChunk dispatch positions at a time, into a
+// double-buffered ring.
+constexpr int kPlans = 32;
+constexpr int kProducers = 3;
+constexpr int kChunk = 32;
+constexpr int kRecWords = 6;
+constexpr int kRingPitch = kPlans + 1;  // words per (word, position) row: conflict-free both ways
+
+// Unit record (one per plan and dispatch position):
+//   w0 run time of the unit (sum over the fused chain, Eq. 4)
+//   w1 KV admission of the unit (largest on the chain, Eq. 4)
+//   w2 arrival time of the unit's session
+//   w3 device | model << 5 | prefetch << 9 | reclaim << 10 | writes << 11 | skip << 14
+//      | run-time overflow << 15 | first write code << 16
+//   w4 second write code | third write code << 16
+//   w5 the unit's last member (its full write list when it has more than
+//      three codes) | release slot code << 16 (bit 31: accumulator; 0xFFFF: none)
+constexpr uint32_t kSkip = 1u << 14;
+constexpr uint32_t kRunOvf = 1u << 15;
+
+struct PcLayout {
+    uint32_t weight, cap, load, arr, ring, slots, tfree, used, queue, nres, total;
+};
+
+__host__ __device__ inline PcLayout pc_layout(int32_t D, int32_t M, int32_t W, int32_t NS)
+{
+    PcLayout l;
+    uint32_t o = 0;
+    l.weight = o; o += round16(4u * M);
+    l.cap = o; o += round16(4u * D);
+    l.load = o; o += round16(4u * M * D);
+    l.arr = o; o += round16(4u * W);
+    l.ring = o; o += 4u * 2 * kRecWords * kChunk * kRingPitch;
+    l.slots = o; o += 4u * (uint32_t)NS * kPlans;
+    l.tfree = o; o += 4u * D * kPlans;
+    l.used = o; o += 4u * D * kPlans;
+    l.queue = o; o += 8u * D * kPlans;
+    l.nres = o; o += round16((uint32_t)D * kPlans);
+    l.total = o;
+    return l;
+}
+
+__device__ __forceinline__ void named_sync(int id)
+{
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(32 * (1 + kProducers)) : "memory");
+}
+
+__device__ __forceinline__ void named_arrive(int id)
+{
+    asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(32 * (1 + kProducers)) : "memory");
+}
+
+// r-th smallest (0-based) of the kPlans-strided values v[0], v[kPlans], ...
+__device__ uint32_t select_strided(uint32_t *v, int32_t n, int32_t r)
+{
+    int32_t lo = 0, hi = n - 1;
+    while (lo < hi) {
+        const uint32_t pivot = v[(lo + (hi - lo) / 2) * kPlans];
+        int32_t i = lo, j = hi;
+        while (i <= j) {
+            while (v[i * kPlans] < pivot) ++i;
+            while (v[j * kPlans] > pivot) --j;
+            if (i <= j) { uint32_t t = v[i * kPlans]; v[i * kPlans] = v[j * kPlans]; v[j * kPlans] = t; ++i; --j; }
+        }
+        if (r <= j) hi = j;
+        else if (r >= i) lo = i;
+        else return v[r * kPlans];
+    }
+    return v[r * kPlans];
+}
+
+__device__ __forceinline__ uint32_t rslot16(int32_t code)
+{
+    return code < 0 ? 0xFFFFu : (((uint32_t)code & 0x7FFFu) | ((code & WF_RSLOT_ACC) ? 0x8000u : 0u));
+}
+
+// Row pointers of one plan.
+struct PlanPtrs {
+    const uint8_t *place;
+    const uint16_t *order;
+    const uint32_t *fuse, *prefetch, *retain;
+};
+
+// Producer: the unit record of dispatch position i of a plan.
+__device__ __forceinline__ void produce(const wf_dev_problem &dp, const PlanPtrs &r, int32_t i,
+                                        uint32_t rec[kRecWords])
+{
+    const int32_t D = dp.D;
+    const int32_t h = __ldg(r.order + i);
+    const int32_t d = __ldg(r.place + h);
+    const uint32_t lh = __ldg(dp.links + h);
+    const uint32_t fp = lh & 0xFFFFu;
+    if (fp != 0xFFFFu && bit_of_g(r.fuse, h) && __ldg(r.place + fp) == d) {  // runs inside its head's unit
+        rec[3] = kSkip;
+        return;
+    }
+    const int4 nr = __ldg(dp.noderec + 2 * h);
+    const int2 lk0 = __ldg(dp.lk + h * D + d);
+    uint32_t run = (uint32_t)lk0.x, ovf = 0;
+    int32_t kv = lk0.y, tail = h;
+    for (uint32_t s = lh >> 16; s != 0xFFFFu; s = __ldg(dp.links + s) >> 16) {  // Eq. 3 chain
+        if (!bit_of_g(r.fuse, s) || __ldg(r.place + s) != d) break;
+        const int2 lk = __ldg(dp.lk + s * D + d);
+        const uint32_t r2 = run + (uint32_t)lk.x;
+        ovf |= r2 < run;
+        run = r2;
+        kv = max(kv, lk.y);
+        tail = (int32_t)s;
+    }
+    const int4 wr = __ldg(dp.noderec + 2 * tail + 1);
+    const uint32_t nwl = (uint32_t)min(wr.y, 7);
+    const uint32_t c0 = nwl > 0 ? (uint32_t)wr.z & 0xFFFFu : 0u;
+    const uint32_t c1 = nwl > 1 ? (uint32_t)wr.z >> 16 : 0u;
+    const uint32_t c2 = nwl > 2 ? (uint32_t)__ldg(dp.wl + wr.x + 2) : 0u;
+    const uint32_t pf = bit_of_g(r.prefetch, h);
+    const uint32_t reclaim = r.retain ? !bit_of_g(r.retain, tail) : 0u;
+    rec[0] = run;
+    rec[1] = (uint32_t)kv;
+    rec[2] = (uint32_t)__ldg(dp.arrival + (nr.w >> 8));
+    rec[3] = (uint32_t)d | (((uint32_t)nr.w & 15u) << 5) | (pf << 9) | (reclaim << 10) | (nwl << 11) |
+             (ovf ? kRunOvf : 0u) | (c0 << 16);
+    rec[4] = c1 | (c2 << 16);
+    rec[5] = (uint32_t)tail | (rslot16(nr.z) << 16);
+}
+
+__device__ __forceinline__ void publish(uint32_t *slots, uint32_t code, uint32_t c)
+{
+    uint32_t &sv = slots[(code & 0x7FFFu) * kPlans];
+    sv = (code & 0x8000u) ? max(sv, c) : c;
+}
+
+template <typename Q>
+__global__ void __launch_bounds__(32 * (1 + kProducers))
+pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list, int32_t *ovf_count)
+{
+    extern __shared__ __align__(128) uint8_t sm[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int32_t N = dp.N, D = dp.D, M = dp.M, W = dp.W;
+    const PcLayout L = pc_layout(D, M, W, dp.nslots);
+    const int64_t p0 = (int64_t)blockIdx.x * kPlans;
+    const int ng = (int)(pl.P - p0 < kPlans ? pl.P - p0 : kPlans);
+    uint32_t *ring = (uint32_t *)(sm + L.ring);
+    const int32_t chunks = (N + kChunk - 1) / kChunk;
+
+    int32_t *weight = (int32_t *)(sm + L.weight);
+    int32_t *cap = (int32_t *)(sm + L.cap);
+    int32_t *load = (int32_t *)(sm + L.load);
+    uint32_t *arrival = (uint32_t *)(sm + L.arr);
+    for (int32_t k = threadIdx.x; k < M; k += blockDim.x) weight[k] = __ldg(dp.weight + k);
+    for (int32_t k = threadIdx.x; k < D; k += blockDim.x) cap[k] = __ldg(dp.cap + k);
+    for (int32_t k = threadIdx.x; k < M * D; k += blockDim.x) load[k] = __ldg(dp.load + k);
+    for (int32_t k = threadIdx.x; k < W; k += blockDim.x) arrival[k] = (uint32_t)__ldg(dp.arrival + k);
+
+    if (warp > 0) {
+        // ---------------- producers: lane = dispatch position ----------------
+        __syncthreads();
+        for (int32_t c = 0; c < chunks; ++c) {
+            const int b = c & 1;
+            if (c >= 2) named_sync(3 + b);  // the consumer has released buffer b
+            uint32_t *rb = ring + b * kRecWords * kChunk * kRingPitch;
+            const int32_t i = c * kChunk + lane;
+            for (int q = warp - 1; q < kPlans; q += kProducers) {
+                uint32_t rec[kRecWords] = {0, 0, 0, kSkip, 0, 0};
+                const int64_t p = p0 + q;
+                if (q < ng && i < N && __ldg(out.status + p) == 0) {
+                    PlanPtrs r;
+                    r.place = pl.place + p * pl.place_stride;
+                    r.order = (const uint16_t *)((const uint8_t *)pl.order + p * pl.order_stride);
+                    r.fuse = (const uint32_t *)((const uint8_t *)pl.fuse + p * pl.bits_stride);
+                    r.prefetch = (const uint32_t *)((const uint8_t *)pl.prefetch + p * pl.bits_stride);
+                    r.retain = pl.retain ? (const uint32_t *)((const uint8_t *)pl.retain + p * pl.bits_stride)
+                                         : nullptr;
+                    produce(dp, r, i, rec);
+                }
+#pragma unroll
+                for (int w = 0; w < kRecWords; ++w) rb[(w * kChunk + lane) * kRingPitch + q] = rec[w];
+            }
+            named_arrive(1 + b);  // buffer b is full
+        }
+        // Match the consumer's releases of the last two buffers.
+        for (int32_t c = chunks; c < chunks + 2; ++c)
+            if (c >= 2) named_sync(3 + (c & 1));
+        return;
+    }
+
+    // ---------------- consumer: lane = plan ----------------
+    const int64_t p = p0 + lane;
+    const bool live = lane < ng && out.status[p] == 0;
+    uint32_t *slots = (uint32_t *)(sm + L.slots) + lane;
+    uint32_t *tfree = (uint32_t *)(sm + L.tfree) + lane;
+    uint32_t *used = (uint32_t *)(sm + L.used) + lane;
+    Q *queue = (Q *)(sm + L.queue) + lane;
+    uint8_t *nres = sm + L.nres + lane;
+    for (int32_t k = 0; k < dp.nslots; ++k) slots[k * kPlans] = 0;
+    for (int32_t d = 0; d < D; ++d) {
+        tfree[d * kPlans] = 0; used[d * kPlans] = 0; queue[d * kPlans] = 0; nres[d * kPlans] = 0;
+    }
+    __syncthreads();
+    const uint32_t grant = (uint32_t)dp.grant;
+    uint32_t end = 0, ovf = 0;
+    int64_t gsum = 0;
+    for (int32_t c = 0; c < chunks; ++c) {
+        const int b = c & 1;
+        named_sync(1 + b);  // buffer b is full
+        const uint32_t *rb = ring + b * kRecWords * kChunk * kRingPitch + lane;
+        const int32_t kmax = min(kChunk, N - c * kChunk);
+        for (int32_t k = 0; k < kmax && live; ++k) {
+            const uint32_t r3 = rb[(3 * kChunk + k) * kRingPitch];
+            if (r3 & kSkip) continue;
+            const uint32_t run = rb[(0 * kChunk + k) * kRingPitch];
+            const int32_t kv = (int32_t)rb[(1 * kChunk + k) * kRingPitch];
+            const uint32_t arr = rb[(2 * kChunk + k) * kRingPitch];
+            const uint32_t r4 = rb[(4 * kChunk + k) * kRingPitch];
+            const uint32_t r5 = rb[(5 * kChunk + k) * kRingPitch];
+            const int32_t d = (int32_t)(r3 & 31u);
+            const uint32_t m = (r3 >> 5) & 15u;
+            ovf |= r3 & kRunOvf;
+
+            // Release (Eq. 2, Eq. 7).
+            uint32_t rel = arr;
+            const uint32_t rs = r5 >> 16;
+            if (rs != 0xFFFFu) {
+                uint32_t &sv = slots[(rs & 0x7FFFu) * kPlans];
+                rel = max(rel, sv);
+                if (rs & 0x8000u) sv = 0;
+            }
+
+            // Eq. 11: reclaim least recently used other models until the unit fits.
+            Q q = queue[d * kPlans];
+            uint32_t n = nres[d * kPlans];
+            const uint32_t tf = tfree[d * kPlans];
+            const int32_t wm = weight[m];
+            const int64_t capd = cap[d];
+            const uint32_t ld = (uint32_t)load[m * D + d];
+            int64_t u_d = used[d * kPlans];
+            const bool was_empty = n == 0;
+            int32_t kq = Lru<Q>::find(q, n, m);
+            const bool hit = kq < (int32_t)n;
+            const int64_t need = hit ? (int64_t)kv : (int64_t)wm + kv;
+            while (u_d + need > capd) {
+                const int32_t vpos = (hit && kq == 0) ? 1 : 0;
+                if (vpos >= (int32_t)n) { atomicExch(dp.err, 2); break; }  // unreachable for a valid plan
+                const uint32_t victim = (uint32_t)(q >> (4 * vpos)) & 15u;
+                q = Lru<Q>::remove(q, vpos);
+                n -= 1;
+                kq -= (hit && vpos < kq) ? 1 : 0;
+                u_d -= weight[victim];
+            }
+            // Hit: start when device and release allow.  Miss: load on this
+            // device first; a prefetched load waits only for the arrival (Eq. 5).
+            const uint32_t ls = max(tf, ((r3 >> 9) & 1u) ? arr : rel);
+            const uint32_t le = ls + ld;
+            const uint32_t start = hit ? max(tf, rel) : max(le, rel);
+            ovf |= (!hit && le < ls) ? 1u : 0u;
+            gsum -= (!hit && was_empty) ? (int64_t)ls : 0;
+            const Q q_hit = Lru<Q>::remove(q, kq) | ((Q)m << (4 * (n - (hit ? 1 : 0))));
+            const Q q_miss = n < (uint32_t)Lru<Q>::kSlots ? (q | ((Q)m << (4 * n))) : q;
+            q = hit ? q_hit : q_miss;
+            n += hit ? 0u : 1u;
+            u_d += hit ? 0 : wm;
+            const uint32_t sg = start + grant;
+            const uint32_t cfin = sg + run;
+            ovf |= (sg < start) | (cfin < sg);
+            end = max(end, cfin);
+
+            const uint32_t nwl = (r3 >> 11) & 7u;
+            if (nwl > 0) publish(slots, r3 >> 16, cfin);
+            if (nwl > 1) publish(slots, r4 & 0xFFFFu, cfin);
+            if (nwl > 2) {
+                publish(slots, r4 >> 16, cfin);
+                const int4 wr = __ldg(dp.noderec + 2 * (int32_t)(r5 & 0xFFFFu) + 1);
+                for (int32_t e = 3; e < wr.y; ++e) publish(slots, __ldg(dp.wl + wr.x + e), cfin);
+            }
+            tfree[d * kPlans] = cfin;
+            if ((r3 >> 10) & 1u) {  // retain bit 0: reclaim at the end of the unit
+                q &= ~((Q)0xF << (4 * (n - 1)));
+                n -= 1;
+                u_d -= wm;
+                gsum += n == 0 ? (int64_t)cfin : 0;
+            }
+            queue[d * kPlans] = q;
+            nres[d * kPlans] = (uint8_t)n;
+            used[d * kPlans] = (uint32_t)u_d;
+        }
+        named_arrive(3 + b);  // buffer b may be refilled
+    }
+    if (!live) return;
+    if (ovf) {  // times do not fit u32: exact int64 path
+        const int32_t kk = atomicAdd(ovf_count, 1);
+        ovf_list[kk] = (int32_t)p;
+        return;
+    }
+    int64_t open = 0;
+    for (int32_t d = 0; d < D; ++d) open += nres[d * kPlans] != 0;
+    for (int32_t w = 0; w < W; ++w) slots[w * kPlans] -= arrival[w];  // session completion latency
+    const int32_t rank = (int32_t)((95 * (int64_t)W + 99) / 100 - 1);
+    out.makespan_us[p] = (int64_t)end - dp.first_arrival;
+    out.gpu_us[p] = gsum + open * (int64_t)end;
+    out.p95_us[p] = select_strided(slots, W, rank);
+}
+
+// Status bits of every plan (Eq. 8-10), one warp per plan: the warp scatters
+// the inverse permutation of the dispatch sequence (u16 positions; a bitmap
+// catches repeats) into shared memory, then checks every edge in parallel.
+// Invalid plans get INT64_MAX metrics here; the sweep skips them.
+__host__ __device__ inline uint32_t status_warp_bytes(int32_t N)
+{
+    return round16(2u * (uint32_t)N) + round16(4u * (((uint32_t)N + 31u) / 32u));
+}
+
+__global__ void __launch_bounds__(128)
+status_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out)
+{
+    extern __shared__ __align__(16) uint8_t ssm[];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, warps = blockDim.x >> 5;
+    const int32_t N = dp.N, D = dp.D;
+    uint16_t *pos = (uint16_t *)(ssm + (size_t)warp * status_warp_bytes(N));
+    uint32_t *seen = (uint32_t *)((uint8_t *)pos + round16(2u * (uint32_t)N));
+    const int32_t words = (N + 31) / 32;
+    for (int64_t p = (int64_t)blockIdx.x * warps + warp; p < pl.P; p += (int64_t)gridDim.x * warps) {
+        const uint8_t *place = pl.place + p * pl.place_stride;
+        const uint16_t *order = (const uint16_t *)((const uint8_t *)pl.order + p * pl.order_stride);
+        uint32_t st = 0;
+        for (int32_t k = lane; k < words; k += 32) seen[k] = 0;
+        for (int32_t n = lane; n < N; n += 32) {
+            const int32_t d = place[n];
+            if (d >= D) st |= WF_ST_DEVICE;
+            else if (__ldg(dp.peak + (int64_t)n * D + d) > __ldg(dp.cap + d)) st |= WF_ST_CAPACITY;
+        }
+        __syncwarp();
+        for (int32_t i = lane; i < N; i += 32) {
+            const int32_t h = order[i];
+            if (h >= N) { st |= WF_ST_PERMUTATION; continue; }
+            const uint32_t b = 1u << (h & 31);
+            if (atomicOr(&seen[h >> 5], b) & b) st |= WF_ST_PERMUTATION;
+            pos[h] = (uint16_t)i;
+        }
+        __syncwarp();
+        st = __reduce_or_sync(0xFFFFFFFFu, st);
+        if (!(st & WF_ST_PERMUTATION)) {
+            for (int32_t v = lane; v < N; v += 32) {
+                const uint32_t pv = pos[v];
+                for (int32_t e = __ldg(dp.pred_off + v); e < __ldg(dp.pred_off + v + 1); ++e)
+                    if (pos[__ldg(dp.pred_idx + e)] > pv) st |= WF_ST_TOPOLOGY;
+            }
+            st = __reduce_or_sync(0xFFFFFFFFu, st);
+        }
+        if (lane == 0) {
+            out.status[p] = st;
+            if (st) out.makespan_us[p] = out.p95_us[p] = out.gpu_us[p] = WF_INF64;
+        }
+        __syncwarp();  // pos[] and seen[] are reused by the warp's next plan
+    }
+}
+
+}  // namespace
+
+// Shared memory of the producer / consumer kernel for this problem, or 0 when
+// the sweep cannot run it (slots unavailable, times beyond u32, more than 16
+// models, or more shared memory than a CTA may hold); the caller then uses
+// the int64 path.
+size_t wf_sweep_smem(const wf_dev_problem &dp)
+{
+    if (dp.nslots <= 0 || dp.max_arrival >= (int64_t)1 << 32 || dp.M > 16 || dp.N > 65534) return 0;
+    const size_t s = pc_layout(dp.D, dp.M, dp.W, dp.nslots).total;
+    return s <= 227 * 1024 ? s : 0;
+}
+
+int wf_launch_sweep(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, size_t smem,
+                    int32_t *ovf_list, int32_t *ovf_count, cudaStream_t st)
+{
+    const wf_dev_problem &dp = ctx->dp;
+    const size_t wbytes = status_warp_bytes(dp.N);
+    const int swarps = (int)std::max<size_t>(1, std::min<size_t>(4, (227 * 1024) / wbytes));
+    const size_t ssmem = wbytes * swarps;
+    int rc = wf_cuda_check(cudaFuncSetAttribute(status_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                (int)ssmem), "status smem attribute");
+    if (rc) return rc;
+    const int64_t sblocks = std::min<int64_t>((pl->P + swarps - 1) / swarps, (int64_t)ctx->sms * 16);
+    status_kernel<<<(unsigned)sblocks, 32 * swarps, ssmem, st>>>(dp, *pl, *out);
+    const unsigned blocks = (unsigned)((pl->P + kPlans - 1) / kPlans);
+    if (dp.M <= 8) {
+        rc = wf_cuda_check(cudaFuncSetAttribute(pc_kernel<uint32_t>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                (int)smem), "sweep smem attribute");
+        if (rc) return rc;
+        pc_kernel<uint32_t><<<blocks, 32 * (1 + kProducers), smem, st>>>(dp, *pl, *out, ovf_list, ovf_count);
+    } else {
+        rc = wf_cuda_check(cudaFuncSetAttribute(pc_kernel<uint64_t>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                (int)smem), "sweep smem attribute");
+        if (rc) return rc;
+        pc_kernel<uint64_t><<<blocks, 32 * (1 + kProducers), smem, st>>>(dp, *pl, *out, ovf_list, ovf_count);
+    }
+    return wf_cuda_check(cudaGetLastError(), "sweep launch");
+}

@@ -193,3 +193,72 @@ def test_long_chain_window():
     got = gpu_eval(prob, plans, k=16)
     want = oracle_eval(prob, plans)
     assert_same(got, want)
+
+
+@pytest.mark.parametrize("name", ["mix", "burst"])
+def test_int64_path_matches_oracle(name, monkeypatch):
+    """The exact int64 path (taken for plans whose times overflow the
+    shared-memory sweep's u32 slots) on its own, forced for every plan."""
+    monkeypatch.setenv("WF_EVAL_PATH", "int64")
+    w = wfgen.config(name)
+    plans = wfgen.make_plans(w.problem, 2048, 77, p_retain=0.5)
+    inject_invalid(plans, w.problem, np.random.default_rng(1))
+    got = gpu_eval(w.problem, plans, k=8)
+    assert_same(got, oracle_eval(w.problem, plans))
+
+
+def test_times_beyond_u32_take_the_int64_path():
+    """Run times near 2^30 us make every makespan exceed 2^32 us; those plans
+    must still match the oracle exactly."""
+    rng = np.random.default_rng(31)
+    prob = random_problem(rng, n_sessions=5, sizes=(6, 10), D=3, M=3)
+    lat = (prob.lat_us.astype(np.int64) % 1000 + (1 << 30) - 5000).astype(np.int32)
+    prob = prob.with_(lat_us=lat)
+    plans = wfgen.make_plans(prob, 300, 3, p_retain=0.5)
+    got = gpu_eval(prob, plans, k=10)
+    want = oracle_eval(prob, plans)
+    assert (want["makespan"][want["status"] == 0] >= (1 << 32)).all()
+    assert_same(got, want)
+
+
+def test_mixed_overflow_batch():
+    """Some plans overflow u32, some do not, in one batch."""
+    rng = np.random.default_rng(37)
+    prob = random_problem(rng, n_sessions=4, sizes=(5, 9), D=2, M=3)
+    lat = prob.lat_us.astype(np.int64).reshape(prob.N, prob.D)
+    lat[:, 1] = (1 << 29)  # device 1 is very slow
+    prob = prob.with_(lat_us=lat.astype(np.int32).reshape(-1),
+                      peak_mib=np.minimum(prob.peak_mib, prob.cap_mib.min()).astype(np.int32)
+                      .clip(min=prob.weight_mib[prob.model].repeat(prob.D)))
+    plans = wfgen.make_plans(prob, 500, 4)
+    got = gpu_eval(prob, plans, k=5)
+    want = oracle_eval(prob, plans)
+    big = want["makespan"][want["status"] == 0] >= (1 << 32)
+    assert big.any() and (~big).any()
+    assert_same(got, want)
+
+
+def test_wide_fanout_write_lists():
+    """A node whose finish feeds many multi-predecessor successors (long
+    write lists) and a session with many sinks."""
+    N, D, M = 80, 3, 2
+    preds = [[] for _ in range(N)]
+    # hubs 0 and 1 each feed nodes 2..41, which also depend on both hubs
+    for v in range(2, 42):
+        preds[v] = [0, 1]
+    for v in range(42, N):
+        preds[v] = [v - 40]
+    rng = np.random.default_rng(5)
+    off = np.zeros(N + 1, np.int32)
+    off[1:] = np.cumsum([len(p) for p in preds])
+    prob = wfgen.Problem(N=N, D=D, M=M, W=1, pred_off=off,
+                         pred_idx=np.array([u for p in preds for u in p], np.int32),
+                         model=rng.integers(0, M, N).astype(np.uint8), session=np.zeros(N, np.int32),
+                         arrival_us=np.zeros(1, np.int64),
+                         lat_us=rng.integers(1, 1000, N * D).astype(np.int32),
+                         peak_mib=np.full(N * D, 30, np.int32), weight_mib=np.array([20, 25], np.int32),
+                         load_us=rng.integers(0, 100, M * D).astype(np.int32),
+                         cap_mib=np.array([60, 60, 200], np.int32))
+    plans = wfgen.make_plans(prob, 200, 9, p_retain=0.7)
+    got = gpu_eval(prob, plans, k=3)
+    assert_same(got, oracle_eval(prob, plans))
