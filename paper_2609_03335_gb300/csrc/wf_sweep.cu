@@ -110,10 +110,11 @@ __device__ __forceinline__ uint32_t bit_of_g(const uint32_t *row, int32_t n)
     return (__ldg(row + (n >> 5)) >> (n & 31)) & 1u;
 }
 
-// CTA shape: warp 0 plays kPlans plans (one per lane); warps 1..kProducers
+// CTA shape: warp 0 plays kPlans plans (one per lane, 16 so that four CTAs and
+// four consumer warps fit an SM); warps 1..kProducers
 // prepare their unit records, kChunk dispatch positions at a time, into a
 // double-buffered ring.
-constexpr int kPlans = 32;
+constexpr int kPlans = 16;
 constexpr int kProducers = 3;
 constexpr int kChunk = 32;
 constexpr int kRecWords = 6;
@@ -297,16 +298,20 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list, in
     }
 
     // ---------------- consumer: lane = plan ----------------
+    // Lanes at or beyond kPlans own no plan and touch no per-plan state.
+    const bool mine = lane < kPlans;
     const int64_t p = p0 + lane;
-    const bool live = lane < ng && out.status[p] == 0;
+    const bool live = mine && lane < ng && out.status[p] == 0;
     uint32_t *slots = (uint32_t *)(sm + L.slots) + lane;
     uint32_t *tfree = (uint32_t *)(sm + L.tfree) + lane;
     uint32_t *used = (uint32_t *)(sm + L.used) + lane;
     Q *queue = (Q *)(sm + L.queue) + lane;
     uint8_t *nres = sm + L.nres + lane;
-    for (int32_t k = 0; k < dp.nslots; ++k) slots[k * kPlans] = 0;
-    for (int32_t d = 0; d < D; ++d) {
-        tfree[d * kPlans] = 0; used[d * kPlans] = 0; queue[d * kPlans] = 0; nres[d * kPlans] = 0;
+    if (mine) {
+        for (int32_t k = 0; k < dp.nslots; ++k) slots[k * kPlans] = 0;
+        for (int32_t d = 0; d < D; ++d) {
+            tfree[d * kPlans] = 0; used[d * kPlans] = 0; queue[d * kPlans] = 0; nres[d * kPlans] = 0;
+        }
     }
     __syncthreads();
     const uint32_t grant = (uint32_t)dp.grant;
@@ -342,14 +347,14 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list, in
             Q q = queue[d * kPlans];
             uint32_t n = nres[d * kPlans];
             const uint32_t tf = tfree[d * kPlans];
-            const int32_t wm = weight[m];
-            const int64_t capd = cap[d];
+            const uint32_t wm = (uint32_t)weight[m];
+            const uint32_t capd = (uint32_t)cap[d];
             const uint32_t ld = (uint32_t)load[m * D + d];
-            int64_t u_d = used[d * kPlans];
+            uint32_t u_d = used[d * kPlans];  // used + need <= cap + peak < 2^32
             const bool was_empty = n == 0;
             int32_t kq = Lru<Q>::find(q, n, m);
             const bool hit = kq < (int32_t)n;
-            const int64_t need = hit ? (int64_t)kv : (int64_t)wm + kv;
+            const uint32_t need = hit ? (uint32_t)kv : wm + (uint32_t)kv;
             while (u_d + need > capd) {
                 const int32_t vpos = (hit && kq == 0) ? 1 : 0;
                 if (vpos >= (int32_t)n) { atomicExch(dp.err, 2); break; }  // unreachable for a valid plan
@@ -357,7 +362,7 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list, in
                 q = Lru<Q>::remove(q, vpos);
                 n -= 1;
                 kq -= (hit && vpos < kq) ? 1 : 0;
-                u_d -= weight[victim];
+                u_d -= (uint32_t)weight[victim];
             }
             // Hit: start when device and release allow.  Miss: load on this
             // device first; a prefetched load waits only for the arrival (Eq. 5).
@@ -370,7 +375,7 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list, in
             const Q q_miss = n < (uint32_t)Lru<Q>::kSlots ? (q | ((Q)m << (4 * n))) : q;
             q = hit ? q_hit : q_miss;
             n += hit ? 0u : 1u;
-            u_d += hit ? 0 : wm;
+            u_d += hit ? 0u : wm;
             const uint32_t sg = start + grant;
             const uint32_t cfin = sg + run;
             ovf |= (sg < start) | (cfin < sg);
@@ -393,7 +398,7 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list, in
             }
             queue[d * kPlans] = q;
             nres[d * kPlans] = (uint8_t)n;
-            used[d * kPlans] = (uint32_t)u_d;
+            used[d * kPlans] = u_d;
         }
         named_arrive(3 + b);  // buffer b may be refilled
     }
