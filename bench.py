@@ -58,7 +58,7 @@ def topk_launches(P: int, k: int, tile: int = 2048) -> int:
 
 def kernel_source_hash() -> str:
     h = hashlib.sha256()
-    for f in ("wf_eval.cu", "wf_internal.cuh"):
+    for f in ("wf_eval.cu", "wf_sweep.cu", "wf_internal.cuh"):
         with open(os.path.join(ROOT, "paper_2609_03335_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
@@ -302,7 +302,9 @@ def run_gpu(args, rank, world, local):
     peaks = read_peaks()
     peak = peaks.get("hbm_gbs")
     traffic, _ = read_traffic(WORKLOAD)
-    launches = args.steps * (2 + topk_launches(P, k))
+    # forecast, status, sweep, overflow pass, top-k passes (the overflow-count
+    # reset is a memset, not a kernel)
+    launches = args.steps * (4 + topk_launches(P, k))
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -330,7 +332,8 @@ def run_gpu(args, rank, world, local):
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak if peak else None,
-                         "traffic": traffic, "kernel": "eval_det_kernel",
+                         "traffic": traffic,
+                         "kernel": "wf_eval_plans = status_kernel + pc_kernel<uint32_t> + eval_list_kernel",
                          "algorithmic_bytes_per_plan": bpp, "kernel_ms": eval_ms_mean,
                          "peak_source": "MEASURED_PEAKS.json hbm_gbs (measured copy)" if peak else None},
             "cpu_baseline": cpu,

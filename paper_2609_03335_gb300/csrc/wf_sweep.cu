@@ -110,19 +110,25 @@ __device__ __forceinline__ uint32_t bit_of_g(const uint32_t *row, int32_t n)
     return (__ldg(row + (n >> 5)) >> (n & 31)) & 1u;
 }
 
-// CTA shape: warp 0 plays kPlans plans (one per lane, 16 so that four CTAs and
-// four consumer warps fit an SM); warps 1..kProducers
-// prepare their unit records, kChunk dispatch positions at a time, into a
-// double-buffered ring.
+// CTA shape, a three-stage pipeline over kChunk dispatch positions at a time:
+// warps 2..kProducers+1 prepare the unit records of kPlans plans (lane =
+// position) into a ring of kBuffers buffers; warp 1 settles model residency
+// (lane = plan: hits, reclamations, occupancy changes); warp 0 plays the
+// timing (lane = plan: releases, starts, finishes, slots).  16 plans per CTA
+// lets four CTAs share an SM.
 constexpr int kPlans = 16;
 constexpr int kProducers = 3;
-constexpr int kChunk = 32;
+constexpr int kChunk = 16;
+constexpr int kPlansPerIter = 32 / kChunk;  // plans a producer warp covers per iteration
+constexpr int kBuffers = 3;
+constexpr int kWarps = 2 + kProducers;
 constexpr int kRecWords = 6;
 constexpr int kRingPitch = kPlans + 1;  // words per (word, position) row: conflict-free both ways
 
 // Unit record (one per plan and dispatch position):
 //   w0 run time of the unit (sum over the fused chain, Eq. 4)
-//   w1 KV admission of the unit (largest on the chain, Eq. 4)
+//   w1 KV admission of the unit (largest on the chain, Eq. 4); the residency
+//      stage overwrites it with hit | was-empty << 1 | emptied-by-reclaim << 2
 //   w2 arrival time of the unit's session
 //   w3 device | model << 5 | prefetch << 9 | reclaim << 10 | writes << 11 | skip << 14
 //      | run-time overflow << 15 | first write code << 16
@@ -133,7 +139,7 @@ constexpr uint32_t kSkip = 1u << 14;
 constexpr uint32_t kRunOvf = 1u << 15;
 
 struct PcLayout {
-    uint32_t weight, cap, load, arr, ring, slots, tfree, used, queue, nres, total;
+    uint32_t weight, cap, load, arr, ring, slots, tfree, used, queue, nres, open, total;
 };
 
 __host__ __device__ inline PcLayout pc_layout(int32_t D, int32_t M, int32_t W, int32_t NS)
@@ -144,24 +150,30 @@ __host__ __device__ inline PcLayout pc_layout(int32_t D, int32_t M, int32_t W, i
     l.cap = o; o += round16(4u * D);
     l.load = o; o += round16(4u * M * D);
     l.arr = o; o += round16(4u * W);
-    l.ring = o; o += 4u * 2 * kRecWords * kChunk * kRingPitch;
+    l.ring = o; o += 4u * kBuffers * kRecWords * kChunk * kRingPitch;
     l.slots = o; o += 4u * (uint32_t)NS * kPlans;
     l.tfree = o; o += 4u * D * kPlans;
     l.used = o; o += 4u * D * kPlans;
     l.queue = o; o += 8u * D * kPlans;
     l.nres = o; o += round16((uint32_t)D * kPlans);
+    l.open = o; o += 4u * kPlans;
     l.total = o;
     return l;
 }
 
-__device__ __forceinline__ void named_sync(int id)
+// Named barriers: kFullP + b (producers -> residency), kFullR + b (residency
+// -> timing), kEmpty + b (timing -> producers) for ring buffer b; kOpen
+// (residency -> timing, once at the end).
+constexpr int kFullP = 1, kFullR = kFullP + kBuffers, kEmpty = kFullR + kBuffers, kOpen = kEmpty + kBuffers;
+
+__device__ __forceinline__ void named_sync(int id, int threads)
 {
-    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(32 * (1 + kProducers)) : "memory");
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
 }
 
-__device__ __forceinline__ void named_arrive(int id)
+__device__ __forceinline__ void named_arrive(int id, int threads)
 {
-    asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(32 * (1 + kProducers)) : "memory");
+    asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(threads) : "memory");
 }
 
 // r-th smallest (0-based) of the kPlans-strided values v[0], v[kPlans], ...
@@ -244,7 +256,7 @@ __device__ __forceinline__ void publish(uint32_t *slots, uint32_t code, uint32_t
 }
 
 template <typename Q>
-__global__ void __launch_bounds__(32 * (1 + kProducers))
+__global__ void __launch_bounds__(32 * kWarps)
 pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list, int32_t *ovf_count)
 {
     extern __shared__ __align__(128) uint8_t sm[];
@@ -255,6 +267,7 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list, in
     const int ng = (int)(pl.P - p0 < kPlans ? pl.P - p0 : kPlans);
     uint32_t *ring = (uint32_t *)(sm + L.ring);
     const int32_t chunks = (N + kChunk - 1) / kChunk;
+    constexpr int kProdThreads = 32 * kProducers;
 
     int32_t *weight = (int32_t *)(sm + L.weight);
     int32_t *cap = (int32_t *)(sm + L.cap);
@@ -265,121 +278,162 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list, in
     for (int32_t k = threadIdx.x; k < M * D; k += blockDim.x) load[k] = __ldg(dp.load + k);
     for (int32_t k = threadIdx.x; k < W; k += blockDim.x) arrival[k] = (uint32_t)__ldg(dp.arrival + k);
 
-    if (warp > 0) {
+    // Lanes at or beyond kPlans own no plan and touch no per-plan state.
+    const bool mine = lane < kPlans;
+    const int64_t p = p0 + lane;
+    const bool live = warp < 2 && mine && lane < ng && out.status[p] == 0;
+
+    if (warp >= 2) {
         // ---------------- producers: lane = dispatch position ----------------
         __syncthreads();
         for (int32_t c = 0; c < chunks; ++c) {
-            const int b = c & 1;
-            if (c >= 2) named_sync(3 + b);  // the consumer has released buffer b
+            const int b = c % kBuffers;
+            if (c >= kBuffers) named_sync(kEmpty + b, kProdThreads + 32);  // timing released buffer b
             uint32_t *rb = ring + b * kRecWords * kChunk * kRingPitch;
-            const int32_t i = c * kChunk + lane;
-            for (int q = warp - 1; q < kPlans; q += kProducers) {
+            const int pos = lane % kChunk, sub = lane / kChunk;
+            const int32_t i = c * kChunk + pos;
+            for (int q0 = (warp - 2) * kPlansPerIter; q0 < kPlans; q0 += kProducers * kPlansPerIter) {
+                const int q = q0 + sub;
+                if (q >= kPlans) continue;
                 uint32_t rec[kRecWords] = {0, 0, 0, kSkip, 0, 0};
-                const int64_t p = p0 + q;
-                if (q < ng && i < N && __ldg(out.status + p) == 0) {
+                const int64_t pq = p0 + q;
+                if (q < ng && i < N && __ldg(out.status + pq) == 0) {
                     PlanPtrs r;
-                    r.place = pl.place + p * pl.place_stride;
-                    r.order = (const uint16_t *)((const uint8_t *)pl.order + p * pl.order_stride);
-                    r.fuse = (const uint32_t *)((const uint8_t *)pl.fuse + p * pl.bits_stride);
-                    r.prefetch = (const uint32_t *)((const uint8_t *)pl.prefetch + p * pl.bits_stride);
-                    r.retain = pl.retain ? (const uint32_t *)((const uint8_t *)pl.retain + p * pl.bits_stride)
+                    r.place = pl.place + pq * pl.place_stride;
+                    r.order = (const uint16_t *)((const uint8_t *)pl.order + pq * pl.order_stride);
+                    r.fuse = (const uint32_t *)((const uint8_t *)pl.fuse + pq * pl.bits_stride);
+                    r.prefetch = (const uint32_t *)((const uint8_t *)pl.prefetch + pq * pl.bits_stride);
+                    r.retain = pl.retain ? (const uint32_t *)((const uint8_t *)pl.retain + pq * pl.bits_stride)
                                          : nullptr;
                     produce(dp, r, i, rec);
                 }
 #pragma unroll
-                for (int w = 0; w < kRecWords; ++w) rb[(w * kChunk + lane) * kRingPitch + q] = rec[w];
+                for (int w = 0; w < kRecWords; ++w) rb[(w * kChunk + pos) * kRingPitch + q] = rec[w];
             }
-            named_arrive(1 + b);  // buffer b is full
+            named_arrive(kFullP + b, kProdThreads + 32);  // buffer b is full
         }
-        // Match the consumer's releases of the last two buffers.
-        for (int32_t c = chunks; c < chunks + 2; ++c)
-            if (c >= 2) named_sync(3 + (c & 1));
+        // Match the timing stage's releases of the last buffers.
+        for (int32_t c = chunks; c < chunks + kBuffers; ++c)
+            if (c >= kBuffers) named_sync(kEmpty + c % kBuffers, kProdThreads + 32);
         return;
     }
 
-    // ---------------- consumer: lane = plan ----------------
-    // Lanes at or beyond kPlans own no plan and touch no per-plan state.
-    const bool mine = lane < kPlans;
-    const int64_t p = p0 + lane;
-    const bool live = mine && lane < ng && out.status[p] == 0;
+    if (warp == 1) {
+        // ---------------- residency: lane = plan (Eq. 11, Section 3.5) ----------------
+        uint32_t *used = (uint32_t *)(sm + L.used) + lane;
+        Q *queue = (Q *)(sm + L.queue) + lane;
+        uint8_t *nres = sm + L.nres + lane;
+        if (mine)
+            for (int32_t d = 0; d < D; ++d) { used[d * kPlans] = 0; queue[d * kPlans] = 0; nres[d * kPlans] = 0; }
+        __syncthreads();
+        for (int32_t c = 0; c < chunks; ++c) {
+            const int b = c % kBuffers;
+            named_sync(kFullP + b, kProdThreads + 32);
+            uint32_t *rb = ring + b * kRecWords * kChunk * kRingPitch + lane;
+            const int32_t kmax = min(kChunk, N - c * kChunk);
+            for (int32_t k = 0; k < kmax && live; ++k) {
+                const uint32_t r3 = rb[(3 * kChunk + k) * kRingPitch];
+                if (r3 & kSkip) continue;
+                uint32_t &r1 = rb[(1 * kChunk + k) * kRingPitch];
+                const int32_t d = (int32_t)(r3 & 31u);
+                const uint32_t m = (r3 >> 5) & 15u;
+                Q q = queue[d * kPlans];
+                uint32_t n = nres[d * kPlans];
+                uint32_t u_d = used[d * kPlans];  // used + need <= cap + peak < 2^32
+                const uint32_t wm = (uint32_t)weight[m];
+                const uint32_t capd = (uint32_t)cap[d];
+                const bool was_empty = n == 0;
+                int32_t kq = Lru<Q>::find(q, n, m);
+                const bool hit = kq < (int32_t)n;
+                const uint32_t need = hit ? r1 : wm + r1;
+                // Reclaim the least recently used other models until the unit fits.
+                while (u_d + need > capd) {
+                    const int32_t vpos = (hit && kq == 0) ? 1 : 0;
+                    if (vpos >= (int32_t)n) { atomicExch(dp.err, 2); break; }  // unreachable for a valid plan
+                    const uint32_t victim = (uint32_t)(q >> (4 * vpos)) & 15u;
+                    q = Lru<Q>::remove(q, vpos);
+                    n -= 1;
+                    kq -= (hit && vpos < kq) ? 1 : 0;
+                    u_d -= (uint32_t)weight[victim];
+                }
+                const Q q_hit = Lru<Q>::remove(q, kq) | ((Q)m << (4 * (n - (hit ? 1 : 0))));
+                const Q q_miss = n < (uint32_t)Lru<Q>::kSlots ? (q | ((Q)m << (4 * n))) : q;
+                q = hit ? q_hit : q_miss;  // m becomes the most recently used
+                n += hit ? 0u : 1u;
+                u_d += hit ? 0u : wm;
+                uint32_t emptied = 0;
+                if ((r3 >> 10) & 1u) {  // retain bit 0: reclaim at the end of the unit
+                    q &= ~((Q)0xF << (4 * (n - 1)));
+                    n -= 1;
+                    u_d -= wm;
+                    emptied = n == 0;
+                }
+                queue[d * kPlans] = q;
+                nres[d * kPlans] = (uint8_t)n;
+                used[d * kPlans] = u_d;
+                r1 = (hit ? 1u : 0u) | (was_empty ? 2u : 0u) | (emptied << 2);
+            }
+            named_arrive(kFullR + b, 64);
+        }
+        uint32_t *open = (uint32_t *)(sm + L.open);
+        if (live) {
+            uint32_t o = 0;
+            for (int32_t d = 0; d < D; ++d) o += nres[d * kPlans] != 0;
+            open[lane] = o;
+        }
+        named_arrive(kOpen, 64);
+        return;
+    }
+
+    // ---------------- timing: lane = plan (Eq. 2, 5, 7, 10) ----------------
     uint32_t *slots = (uint32_t *)(sm + L.slots) + lane;
     uint32_t *tfree = (uint32_t *)(sm + L.tfree) + lane;
-    uint32_t *used = (uint32_t *)(sm + L.used) + lane;
-    Q *queue = (Q *)(sm + L.queue) + lane;
-    uint8_t *nres = sm + L.nres + lane;
     if (mine) {
         for (int32_t k = 0; k < dp.nslots; ++k) slots[k * kPlans] = 0;
-        for (int32_t d = 0; d < D; ++d) {
-            tfree[d * kPlans] = 0; used[d * kPlans] = 0; queue[d * kPlans] = 0; nres[d * kPlans] = 0;
-        }
+        for (int32_t d = 0; d < D; ++d) tfree[d * kPlans] = 0;
     }
     __syncthreads();
     const uint32_t grant = (uint32_t)dp.grant;
     uint32_t end = 0, ovf = 0;
     int64_t gsum = 0;
     for (int32_t c = 0; c < chunks; ++c) {
-        const int b = c & 1;
-        named_sync(1 + b);  // buffer b is full
+        const int b = c % kBuffers;
+        named_sync(kFullR + b, 64);
         const uint32_t *rb = ring + b * kRecWords * kChunk * kRingPitch + lane;
         const int32_t kmax = min(kChunk, N - c * kChunk);
         for (int32_t k = 0; k < kmax && live; ++k) {
             const uint32_t r3 = rb[(3 * kChunk + k) * kRingPitch];
             if (r3 & kSkip) continue;
             const uint32_t run = rb[(0 * kChunk + k) * kRingPitch];
-            const int32_t kv = (int32_t)rb[(1 * kChunk + k) * kRingPitch];
+            const uint32_t fl = rb[(1 * kChunk + k) * kRingPitch];
             const uint32_t arr = rb[(2 * kChunk + k) * kRingPitch];
             const uint32_t r4 = rb[(4 * kChunk + k) * kRingPitch];
             const uint32_t r5 = rb[(5 * kChunk + k) * kRingPitch];
             const int32_t d = (int32_t)(r3 & 31u);
             const uint32_t m = (r3 >> 5) & 15u;
+            const bool hit = fl & 1u;
             ovf |= r3 & kRunOvf;
 
-            // Release (Eq. 2, Eq. 7).
-            uint32_t rel = arr;
+            uint32_t rel = arr;  // release (Eq. 2, Eq. 7)
             const uint32_t rs = r5 >> 16;
             if (rs != 0xFFFFu) {
                 uint32_t &sv = slots[(rs & 0x7FFFu) * kPlans];
                 rel = max(rel, sv);
                 if (rs & 0x8000u) sv = 0;
             }
-
-            // Eq. 11: reclaim least recently used other models until the unit fits.
-            Q q = queue[d * kPlans];
-            uint32_t n = nres[d * kPlans];
-            const uint32_t tf = tfree[d * kPlans];
-            const uint32_t wm = (uint32_t)weight[m];
-            const uint32_t capd = (uint32_t)cap[d];
-            const uint32_t ld = (uint32_t)load[m * D + d];
-            uint32_t u_d = used[d * kPlans];  // used + need <= cap + peak < 2^32
-            const bool was_empty = n == 0;
-            int32_t kq = Lru<Q>::find(q, n, m);
-            const bool hit = kq < (int32_t)n;
-            const uint32_t need = hit ? (uint32_t)kv : wm + (uint32_t)kv;
-            while (u_d + need > capd) {
-                const int32_t vpos = (hit && kq == 0) ? 1 : 0;
-                if (vpos >= (int32_t)n) { atomicExch(dp.err, 2); break; }  // unreachable for a valid plan
-                const uint32_t victim = (uint32_t)(q >> (4 * vpos)) & 15u;
-                q = Lru<Q>::remove(q, vpos);
-                n -= 1;
-                kq -= (hit && vpos < kq) ? 1 : 0;
-                u_d -= (uint32_t)weight[victim];
-            }
             // Hit: start when device and release allow.  Miss: load on this
             // device first; a prefetched load waits only for the arrival (Eq. 5).
+            const uint32_t tf = tfree[d * kPlans];
             const uint32_t ls = max(tf, ((r3 >> 9) & 1u) ? arr : rel);
-            const uint32_t le = ls + ld;
+            const uint32_t le = ls + (uint32_t)load[m * D + d];
             const uint32_t start = hit ? max(tf, rel) : max(le, rel);
             ovf |= (!hit && le < ls) ? 1u : 0u;
-            gsum -= (!hit && was_empty) ? (int64_t)ls : 0;
-            const Q q_hit = Lru<Q>::remove(q, kq) | ((Q)m << (4 * (n - (hit ? 1 : 0))));
-            const Q q_miss = n < (uint32_t)Lru<Q>::kSlots ? (q | ((Q)m << (4 * n))) : q;
-            q = hit ? q_hit : q_miss;
-            n += hit ? 0u : 1u;
-            u_d += hit ? 0u : wm;
+            gsum -= (!hit && (fl & 2u)) ? (int64_t)ls : 0;  // an empty device becomes occupied
             const uint32_t sg = start + grant;
             const uint32_t cfin = sg + run;
             ovf |= (sg < start) | (cfin < sg);
             end = max(end, cfin);
+            gsum += (fl & 4u) ? (int64_t)cfin : 0;  // the device empties after the unit
 
             const uint32_t nwl = (r3 >> 11) & 7u;
             if (nwl > 0) publish(slots, r3 >> 16, cfin);
@@ -390,26 +444,17 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list, in
                 for (int32_t e = 3; e < wr.y; ++e) publish(slots, __ldg(dp.wl + wr.x + e), cfin);
             }
             tfree[d * kPlans] = cfin;
-            if ((r3 >> 10) & 1u) {  // retain bit 0: reclaim at the end of the unit
-                q &= ~((Q)0xF << (4 * (n - 1)));
-                n -= 1;
-                u_d -= wm;
-                gsum += n == 0 ? (int64_t)cfin : 0;
-            }
-            queue[d * kPlans] = q;
-            nres[d * kPlans] = (uint8_t)n;
-            used[d * kPlans] = u_d;
         }
-        named_arrive(3 + b);  // buffer b may be refilled
+        named_arrive(kEmpty + b, kProdThreads + 32);  // buffer b may be refilled
     }
+    named_sync(kOpen, 64);  // the residency stage's final device counts
     if (!live) return;
     if (ovf) {  // times do not fit u32: exact int64 path
         const int32_t kk = atomicAdd(ovf_count, 1);
         ovf_list[kk] = (int32_t)p;
         return;
     }
-    int64_t open = 0;
-    for (int32_t d = 0; d < D; ++d) open += nres[d * kPlans] != 0;
+    const int64_t open = ((const uint32_t *)(sm + L.open))[lane];
     for (int32_t w = 0; w < W; ++w) slots[w * kPlans] -= arrival[w];  // session completion latency
     const int32_t rank = (int32_t)((95 * (int64_t)W + 99) / 100 - 1);
     out.makespan_us[p] = (int64_t)end - dp.first_arrival;
@@ -501,12 +546,12 @@ int wf_launch_sweep(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, siz
         rc = wf_cuda_check(cudaFuncSetAttribute(pc_kernel<uint32_t>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                 (int)smem), "sweep smem attribute");
         if (rc) return rc;
-        pc_kernel<uint32_t><<<blocks, 32 * (1 + kProducers), smem, st>>>(dp, *pl, *out, ovf_list, ovf_count);
+        pc_kernel<uint32_t><<<blocks, 32 * kWarps, smem, st>>>(dp, *pl, *out, ovf_list, ovf_count);
     } else {
         rc = wf_cuda_check(cudaFuncSetAttribute(pc_kernel<uint64_t>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                 (int)smem), "sweep smem attribute");
         if (rc) return rc;
-        pc_kernel<uint64_t><<<blocks, 32 * (1 + kProducers), smem, st>>>(dp, *pl, *out, ovf_list, ovf_count);
+        pc_kernel<uint64_t><<<blocks, 32 * kWarps, smem, st>>>(dp, *pl, *out, ovf_list, ovf_count);
     }
     return wf_cuda_check(cudaGetLastError(), "sweep launch");
 }
