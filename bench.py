@@ -43,17 +43,9 @@ def algorithmic_bytes_per_plan(N: int) -> int:
     return N + 2 * N + 2 * ((N + 7) // 8) + 28
 
 
-def topk_launches(P: int, k: int, tile: int = 2048) -> int:
-    """Kernel launches of one wf_topk call (mirrors the library's pass plan)."""
-    tiles = (P + tile - 1) // tile
-    if tiles == 1:
-        return 2
-    n, launches = tiles * k, 1
-    while n > tile:
-        tiles = (n + tile - 1) // tile
-        n = tiles * k
-        launches += 1
-    return launches + 1
+def topk_launches(P: int, k: int) -> int:
+    """Kernel launches of one wf_topk call: select, compact, final."""
+    return 3
 
 
 def kernel_source_hash() -> str:
@@ -252,6 +244,8 @@ def run_gpu(args, rank, world, local):
     wf.wf_ctx_status(ctx, stream)
     step_ms = [e[0].elapsed_time(e[3]) for e in ev]
     eval_ms = [e[1].elapsed_time(e[2]) for e in ev]
+    forecast_ms = float(np.mean([e[0].elapsed_time(e[1]) for e in ev]))
+    topk_ms = float(np.mean([e[2].elapsed_time(e[3]) for e in ev]))
     ms_per_step = max_over_ranks(float(np.mean(step_ms)), world)
     eval_ms_mean = float(np.mean(eval_ms))
 
@@ -327,7 +321,8 @@ def run_gpu(args, rank, world, local):
                                    "D=8, M=8, P=16384 plans per GPU, k=32",
                        "P_per_gpu": P, "N": prob.N, "k": k,
                        "l2": "flushed between timed steps (256 MiB write)",
-                       "ctx_create_ms": ctx_ms},
+                       "ctx_create_ms": ctx_ms,
+                       "stage_ms": {"forecast": forecast_ms, "eval": eval_ms_mean, "topk": topk_ms}},
             "e2e": {"value": P * world / (e2e_ms * 1e-3), "unit": "plans/s",
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",

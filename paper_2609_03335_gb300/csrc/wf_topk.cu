@@ -1,15 +1,21 @@
 // Top-k of evaluated plans (row a12) by the key (status != 0, makespan, p95,
-// gpu, plan index): each CTA sorts a tile of candidates in shared memory
-// (bitonic network) and keeps its k best; passes repeat until one tile holds
-// every survivor.
+// gpu, plan index), ascending.
+//
+//  1. select: one CTA finds T, the k-th smallest of the 64-bit keys
+//     (status != 0) << 63 | makespan, by radix selection (8 bits a pass);
+//  2. compact: every plan whose 64-bit key is at most T becomes a candidate
+//     (all ties with T included, so the full key decides among them);
+//  3. final: one CTA sorts the candidates by the full key in shared memory
+//     (bitonic network) and writes the first k; more candidates than one
+//     tile (massive ties) are folded tile by tile into the running best k.
 #include <algorithm>
 
 #include "wf_internal.cuh"
 
 namespace {
 
-constexpr int kTile = 2048;          // candidates per CTA
-constexpr int kTopkThreads = 1024;   // two candidates per thread
+constexpr int kTile = 2048;
+constexpr int kThreads = 1024;
 
 struct Cand {
     int64_t mk, p95, gpu;
@@ -35,65 +41,128 @@ __device__ __forceinline__ Cand padding()
     return c;
 }
 
-__device__ void bitonic_sort(Cand *s)
+__device__ __forceinline__ uint64_t key64(const wf_eval_out &res, int64_t p)
 {
-    for (int size = 2; size <= kTile; size <<= 1) {
+    return ((uint64_t)(res.status[p] != 0) << 63) | (uint64_t)res.makespan_us[p];
+}
+
+// Scratch words: [0] T (u64), [1] candidate count, then the candidates.
+struct TopkScratch {
+    unsigned long long *T;
+    unsigned int *count;
+    Cand *cand;
+};
+
+__device__ __forceinline__ TopkScratch scratch_of(void *base)
+{
+    TopkScratch s;
+    s.T = (unsigned long long *)base;
+    s.count = (unsigned int *)((uint8_t *)base + 8);
+    s.cand = (Cand *)((uint8_t *)base + 64);
+    return s;
+}
+
+constexpr int64_t kSelectShared = 20480;  // keys staged in shared memory up to this many plans
+
+template <bool kStaged>
+__global__ void __launch_bounds__(kThreads)
+select_kernel(wf_eval_out res, int64_t P, int32_t k, void *scr)
+{
+    extern __shared__ unsigned long long keys[];
+    __shared__ unsigned int hist[256];
+    __shared__ unsigned long long prefix;
+    __shared__ long long rank;
+    const TopkScratch s = scratch_of(scr);
+    if (threadIdx.x == 0) { prefix = 0; rank = k - 1; *s.count = 0; }
+    if (kStaged)
+        for (int64_t p = threadIdx.x; p < P; p += blockDim.x) keys[p] = key64(res, p);
+    __syncthreads();
+    for (int shift = 56; shift >= 0; shift -= 8) {
+        for (int b = threadIdx.x; b < 256; b += blockDim.x) hist[b] = 0;
+        __syncthreads();
+        const unsigned long long hi = shift == 56 ? 0ull : (~0ull << (shift + 8));
+        const unsigned long long pre = prefix;
+        for (int64_t p = threadIdx.x; p < P; p += blockDim.x) {
+            const uint64_t v = kStaged ? keys[p] : key64(res, p);
+            if ((v & hi) == pre) atomicAdd(&hist[(v >> shift) & 255u], 1u);
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            long long r = rank;
+            int b = 0;
+            while ((long long)hist[b] <= r) { r -= hist[b]; ++b; }
+            rank = r;
+            prefix |= (unsigned long long)b << shift;
+        }
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) *s.T = prefix;
+}
+
+__global__ void compact_kernel(wf_eval_out res, int64_t P, void *scr)
+{
+    const TopkScratch s = scratch_of(scr);
+    const unsigned long long T = *s.T;
+    for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < P; p += (int64_t)gridDim.x * blockDim.x) {
+        if (key64(res, p) > T) continue;
+        Cand c;
+        c.mk = res.makespan_us[p];
+        c.p95 = res.p95_us[p];
+        c.gpu = res.gpu_us[p];
+        c.id = (int32_t)p;
+        c.bad = res.status[p] != 0 ? 1u : 0u;
+        s.cand[atomicAdd(s.count, 1u)] = c;
+    }
+}
+
+// Sorts t[0, len) ascending; len is a power of two, at most kTile.
+__device__ void bitonic_sort(Cand *t, int len)
+{
+    for (int size = 2; size <= len; size <<= 1) {
         for (int stride = size >> 1; stride > 0; stride >>= 1) {
             __syncthreads();
-            for (int t = threadIdx.x; t < kTile / 2; t += blockDim.x) {
-                const int i = 2 * stride * (t / stride) + (t % stride);
+            for (int u = threadIdx.x; u < len / 2; u += blockDim.x) {
+                const int i = 2 * stride * (u / stride) + (u % stride);
                 const int j = i + stride;
                 const bool up = (i & size) == 0;
-                Cand a = s[i], b = s[j];
-                if (before(b, a) == up) { s[i] = b; s[j] = a; }
+                const Cand a = t[i], b = t[j];
+                if (before(b, a) == up) { t[i] = b; t[j] = a; }
             }
         }
     }
     __syncthreads();
 }
 
-// First pass: candidates straight from the result arrays.
-__global__ void __launch_bounds__(kTopkThreads)
-topk_from_results(wf_eval_out res, int64_t P, int32_t k, Cand *dst)
+__global__ void __launch_bounds__(kThreads)
+final_kernel(int32_t k, void *scr, int32_t *ids, int64_t *keys)
 {
-    extern __shared__ Cand s[];
-    const int64_t base = (int64_t)blockIdx.x * kTile;
-    for (int t = threadIdx.x; t < kTile; t += blockDim.x) {
-        const int64_t p = base + t;
-        Cand c = padding();
-        if (p < P) {
-            c.mk = res.makespan_us[p];
-            c.p95 = res.p95_us[p];
-            c.gpu = res.gpu_us[p];
-            c.id = (int32_t)p;
-            c.bad = res.status[p] != 0 ? 1u : 0u;
+    extern __shared__ Cand t[];
+    const TopkScratch s = scratch_of(scr);
+    const int64_t n = *s.count;
+    // One network of the smallest power-of-two size that holds every candidate
+    // when they fit a tile; otherwise the running best k occupy t[0, k) and
+    // each round fills the rest of a full tile with new candidates.
+    int len = 64;
+    while (len < n && len < kTile) len <<= 1;
+    int64_t next = 0;
+    bool first = true;
+    while (first || next < n) {
+        const int base = first ? 0 : k;
+        for (int u = threadIdx.x; u < len - base; u += blockDim.x) {
+            const int64_t c = next + u;
+            t[base + u] = c < n ? s.cand[c] : padding();
         }
-        s[t] = c;
+        next += len - base;
+        first = false;
+        bitonic_sort(t, len);
     }
-    bitonic_sort(s);
-    for (int t = threadIdx.x; t < k; t += blockDim.x) dst[(int64_t)blockIdx.x * k + t] = s[t];
-}
-
-// Later passes: candidates from the previous pass.
-__global__ void __launch_bounds__(kTopkThreads)
-topk_from_cands(const Cand *src, int64_t n, int32_t k, Cand *dst, int32_t *ids, int64_t *keys)
-{
-    extern __shared__ Cand s[];
-    const int64_t base = (int64_t)blockIdx.x * kTile;
-    for (int t = threadIdx.x; t < kTile; t += blockDim.x)
-        s[t] = base + t < n ? src[base + t] : padding();
-    bitonic_sort(s);
-    if (ids) {  // final pass: one CTA
-        for (int t = threadIdx.x; t < k; t += blockDim.x) {
-            ids[t] = s[t].id;
-            if (keys) {
-                keys[3 * t] = s[t].mk;
-                keys[3 * t + 1] = s[t].p95;
-                keys[3 * t + 2] = s[t].gpu;
-            }
+    for (int u = threadIdx.x; u < k; u += blockDim.x) {
+        ids[u] = t[u].id;
+        if (keys) {
+            keys[3 * u] = t[u].mk;
+            keys[3 * u + 1] = t[u].p95;
+            keys[3 * u + 2] = t[u].gpu;
         }
-    } else {
-        for (int t = threadIdx.x; t < k; t += blockDim.x) dst[(int64_t)blockIdx.x * k + t] = s[t];
     }
 }
 
@@ -101,46 +170,27 @@ topk_from_cands(const Cand *src, int64_t n, int32_t k, Cand *dst, int32_t *ids, 
 
 size_t wf_topk_scratch_bytes(int64_t max_P)
 {
-    const int64_t tiles = (max_P + kTile - 1) / kTile + 1;
-    return 2 * (size_t)tiles * 1024 * sizeof(Cand);
+    return 64 + sizeof(Cand) * (size_t)max_P;
 }
 
 int wf_launch_topk(wf_ctx *ctx, const wf_eval_out *res, int64_t P, int32_t k, int32_t *ids,
                    int64_t *keys, cudaStream_t st)
 {
     const size_t smem = kTile * sizeof(Cand);
-    static bool attr_set = false;
-    if (!attr_set) {
-        int rc = wf_cuda_check(cudaFuncSetAttribute(topk_from_results,
-                                                    cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
-                               "topk smem attribute");
-        if (!rc) rc = wf_cuda_check(cudaFuncSetAttribute(topk_from_cands,
-                                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
-                                    "topk smem attribute");
+    int rc = wf_cuda_check(cudaFuncSetAttribute(final_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                (int)smem), "topk smem attribute");
+    if (rc) return rc;
+    if (P <= kSelectShared) {
+        const size_t ks = 8 * (size_t)P;
+        rc = wf_cuda_check(cudaFuncSetAttribute(select_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                (int)ks), "topk select smem attribute");
         if (rc) return rc;
-        attr_set = true;
+        select_kernel<true><<<1, kThreads, ks, st>>>(*res, P, k, ctx->topk_scratch);
+    } else {
+        select_kernel<false><<<1, kThreads, 0, st>>>(*res, P, k, ctx->topk_scratch);
     }
-    Cand *buf[2];
-    const int64_t half = (int64_t)(ctx->topk_scratch_bytes / 2 / sizeof(Cand));
-    buf[0] = (Cand *)ctx->topk_scratch;
-    buf[1] = buf[0] + half;
-    int64_t tiles = (P + kTile - 1) / kTile;
-    if (tiles == 1) {
-        // One tile: sort the results directly into the output.
-        topk_from_results<<<1, kTopkThreads, smem, st>>>(*res, P, k, buf[0]);
-        topk_from_cands<<<1, kTopkThreads, smem, st>>>(buf[0], k, k, nullptr, ids, keys);
-        return wf_cuda_check(cudaGetLastError(), "topk launch");
-    }
-    topk_from_results<<<(unsigned)tiles, kTopkThreads, smem, st>>>(*res, P, k, buf[0]);
-    int64_t n = tiles * k;
-    int cur = 0;
-    while (n > kTile) {
-        tiles = (n + kTile - 1) / kTile;
-        topk_from_cands<<<(unsigned)tiles, kTopkThreads, smem, st>>>(buf[cur], n, k, buf[cur ^ 1],
-                                                                      nullptr, nullptr);
-        cur ^= 1;
-        n = tiles * k;
-    }
-    topk_from_cands<<<1, kTopkThreads, smem, st>>>(buf[cur], n, k, nullptr, ids, keys);
+    const int64_t blocks = std::min<int64_t>((P + 255) / 256, (int64_t)ctx->sms * 8);
+    compact_kernel<<<(unsigned)blocks, 256, 0, st>>>(*res, P, ctx->topk_scratch);
+    final_kernel<<<1, kThreads, smem, st>>>(k, ctx->topk_scratch, ids, keys);
     return wf_cuda_check(cudaGetLastError(), "topk launch");
 }

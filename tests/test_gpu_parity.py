@@ -190,9 +190,13 @@ def test_long_chain_window():
     prob = wfgen.assemble("long", sess, np.zeros(n_sess, np.int64), wfgen.DEV_BURST,
                           [3, 6, 8, 14], rng)
     plans = wfgen.make_plans(prob, 512, 2, p_fuse=0.9)
-    got = gpu_eval(prob, plans, k=16)
+    got = gpu_eval(prob, plans, k=16, forecast=True)  # beyond the shared-memory forecast
     want = oracle_eval(prob, plans)
     assert_same(got, want)
+    ids, keys = oracle.topk(want["makespan"], want["p95"], want["gpu"], want["status"], 16)
+    assert np.array_equal(got["ids"], ids) and np.array_equal(got["keys"], keys)
+    rel, comp = oracle.forecast(prob)
+    assert np.array_equal(got["rel"], rel) and np.array_equal(got["comp"], comp)
 
 
 @pytest.mark.parametrize("name", ["mix", "burst"])
@@ -262,3 +266,22 @@ def test_wide_fanout_write_lists():
     plans = wfgen.make_plans(prob, 200, 9, p_retain=0.7)
     got = gpu_eval(prob, plans, k=3)
     assert_same(got, oracle_eval(prob, plans))
+
+
+def test_topk_with_massive_ties():
+    """More tied candidates than one sorting tile: 3000 copies of one plan
+    plus distinct plans; the tie-break by plan index must hold."""
+    w = wfgen.config("mix")
+    base = wfgen.make_plans(w.problem, 200, 8)
+    P = 3200
+    plans = wfgen.Plans.empty(P, w.problem.N)
+    best = 0
+    for a in ("place", "order", "fuse", "prefetch"):
+        arr = getattr(plans, a)
+        arr[:3000] = getattr(base, a)[best]
+        arr[3000:] = getattr(base, a)[:200]
+    for k in (1, 37, 1024):
+        got = gpu_eval(w.problem, plans, k=k)
+        want = oracle_eval(w.problem, plans)
+        ids, keys = oracle.topk(want["makespan"], want["p95"], want["gpu"], want["status"], k)
+        assert np.array_equal(got["ids"], ids) and np.array_equal(got["keys"], keys)
