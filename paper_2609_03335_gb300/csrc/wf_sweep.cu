@@ -213,14 +213,18 @@ __device__ __forceinline__ void produce(const wf_dev_problem &dp, const PlanPtrs
 {
     const int32_t D = dp.D;
     const int32_t h = __ldg(r.order + i);
+    // Loads that depend on h alone go out together, ahead of any branch.
     const int32_t d = __ldg(r.place + h);
     const uint32_t lh = __ldg(dp.links + h);
+    const uint32_t fw = __ldg(r.fuse + (h >> 5));
+    const uint32_t pw = __ldg(r.prefetch + (h >> 5));
+    const int4 nr = __ldg(dp.noderec + 2 * h);
+    int4 wr = __ldg(dp.noderec + 2 * h + 1);
     const uint32_t fp = lh & 0xFFFFu;
-    if (fp != 0xFFFFu && bit_of_g(r.fuse, h) && __ldg(r.place + fp) == d) {  // runs inside its head's unit
+    if (fp != 0xFFFFu && ((fw >> (h & 31)) & 1u) && __ldg(r.place + fp) == d) {  // runs inside its head's unit
         rec[3] = kSkip;
         return;
     }
-    const int4 nr = __ldg(dp.noderec + 2 * h);
     const int2 lk0 = __ldg(dp.lk + h * D + d);
     uint32_t run = (uint32_t)lk0.x, ovf = 0;
     int32_t kv = lk0.y, tail = h;
@@ -233,12 +237,12 @@ __device__ __forceinline__ void produce(const wf_dev_problem &dp, const PlanPtrs
         kv = max(kv, lk.y);
         tail = (int32_t)s;
     }
-    const int4 wr = __ldg(dp.noderec + 2 * tail + 1);
+    if (tail != h) wr = __ldg(dp.noderec + 2 * tail + 1);
     const uint32_t nwl = (uint32_t)min(wr.y, 7);
     const uint32_t c0 = nwl > 0 ? (uint32_t)wr.z & 0xFFFFu : 0u;
     const uint32_t c1 = nwl > 1 ? (uint32_t)wr.z >> 16 : 0u;
     const uint32_t c2 = nwl > 2 ? (uint32_t)__ldg(dp.wl + wr.x + 2) : 0u;
-    const uint32_t pf = bit_of_g(r.prefetch, h);
+    const uint32_t pf = (pw >> (h & 31)) & 1u;
     const uint32_t reclaim = r.retain ? !bit_of_g(r.retain, tail) : 0u;
     rec[0] = run;
     rec[1] = (uint32_t)kv;
@@ -343,23 +347,23 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list, in
                 const uint32_t wm = (uint32_t)weight[m];
                 const uint32_t capd = (uint32_t)cap[d];
                 const bool was_empty = n == 0;
-                int32_t kq = Lru<Q>::find(q, n, m);
+                const int32_t kq = Lru<Q>::find(q, n, m);
                 const bool hit = kq < (int32_t)n;
+                // Take the unit's own model out of the queue; the reclamation
+                // victims are then exactly its first e entries (least recently
+                // used first), and the unit's model goes back in at the end.
+                if (hit) { q = Lru<Q>::remove(q, kq); n -= 1; }
                 const uint32_t need = hit ? r1 : wm + r1;
-                // Reclaim the least recently used other models until the unit fits.
-                while (u_d + need > capd) {
-                    const int32_t vpos = (hit && kq == 0) ? 1 : 0;
-                    if (vpos >= (int32_t)n) { atomicExch(dp.err, 2); break; }  // unreachable for a valid plan
-                    const uint32_t victim = (uint32_t)(q >> (4 * vpos)) & 15u;
-                    q = Lru<Q>::remove(q, vpos);
-                    n -= 1;
-                    kq -= (hit && vpos < kq) ? 1 : 0;
-                    u_d -= (uint32_t)weight[victim];
+                uint32_t e = 0;
+                while (u_d + need > capd && e < n) {
+                    u_d -= (uint32_t)weight[(uint32_t)(q >> (4 * e)) & 15u];
+                    ++e;
                 }
-                const Q q_hit = Lru<Q>::remove(q, kq) | ((Q)m << (4 * (n - (hit ? 1 : 0))));
-                const Q q_miss = n < (uint32_t)Lru<Q>::kSlots ? (q | ((Q)m << (4 * n))) : q;
-                q = hit ? q_hit : q_miss;  // m becomes the most recently used
-                n += hit ? 0u : 1u;
+                if (u_d + need > capd) atomicExch(dp.err, 2);  // unreachable for a valid plan
+                q = e < (uint32_t)Lru<Q>::kSlots ? (q >> (4 * e)) : (Q)0;
+                n -= e;
+                q |= (Q)m << (4 * n);  // the unit's model is now the most recently used
+                n += 1;
                 u_d += hit ? 0u : wm;
                 uint32_t emptied = 0;
                 if ((r3 >> 10) & 1u) {  // retain bit 0: reclaim at the end of the unit
