@@ -284,7 +284,7 @@ eval_list_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, uint8_t *scrat
 // S x W completions of the plan go to a per-CTA pool for the p95 selection.
 __global__ void __launch_bounds__(kSampleThreads)
 eval_stoch_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, uint8_t *scratch, size_t row_bytes,
-                  int64_t *pool_base, int64_t ctas)
+                  int64_t *pool_base, int64_t ctas, const int32_t *list, const int32_t *list_len)
 {
     __shared__ unsigned long long s_mk, s_gpu;
     __shared__ uint32_t s_status;
@@ -295,7 +295,11 @@ eval_stoch_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, uint8_t *scra
     const int32_t S = dp.S, W = dp.W;
     Row row = row_at(dp, scratch + (size_t)(cta * blockDim.x + threadIdx.x) * row_bytes);
     int64_t *pool = pool_base + cta * (int64_t)S * W;
-    for (int64_t p = cta; p < pl.P; p += ctas) {
+    // Every plan of the batch, or only those listed (plans whose times left
+    // the 32-bit range of the shared-memory sweep).
+    const int64_t total = list ? (int64_t)*list_len : pl.P;
+    for (int64_t j = cta; j < total; j += ctas) {
+        const int64_t p = list ? (int64_t)list[j] : j;
         const PlanRows pr = plan_rows(pl, p);
         if (threadIdx.x == 0) {
             s_mk = 0; s_gpu = 0;
@@ -400,8 +404,20 @@ int wf_launch_eval(wf_ctx *ctx, const wf_plans *plans, const wf_eval_out *out, c
     } else {
         // Per-thread rows of every CTA first, then one completion pool per CTA.
         int64_t *pool = (int64_t *)(scratch + (size_t)units * kSampleThreads * ctx->eval_row_bytes);
-        eval_stoch_kernel<<<(unsigned)units, kSampleThreads, 0, st>>>(dp, *plans, *out, scratch,
-                                                                      ctx->eval_row_bytes, pool, units);
+        const size_t smem = ctx->force_int64 ? 0 : wf_stoch_smem(dp);
+        if (smem) {
+            int rc = wf_cuda_check(cudaMemsetAsync(ctx->ovf_count, 0, sizeof(int32_t), st), "reset overflow count");
+            if (!rc) rc = wf_launch_stoch(ctx, plans, out, smem, ctx->ovf_list, ctx->ovf_count, st);
+            if (rc) return rc;
+            const int64_t lunits = std::min<int64_t>(units, (int64_t)ctx->sms * 4);
+            eval_stoch_kernel<<<(unsigned)lunits, kSampleThreads, 0, st>>>(dp, *plans, *out, scratch,
+                                                                           ctx->eval_row_bytes, pool, lunits,
+                                                                           ctx->ovf_list, ctx->ovf_count);
+        } else {
+            eval_stoch_kernel<<<(unsigned)units, kSampleThreads, 0, st>>>(dp, *plans, *out, scratch,
+                                                                          ctx->eval_row_bytes, pool, units,
+                                                                          nullptr, nullptr);
+        }
     }
     return wf_cuda_check(cudaGetLastError(), "eval launch");
 }

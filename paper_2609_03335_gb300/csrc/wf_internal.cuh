@@ -91,5 +91,8 @@ size_t wf_eval_row_bytes(const wf_dev_problem &dp);
 size_t wf_eval_scratch_bytes(const wf_dev_problem &dp, int64_t max_P, int64_t *units);
 size_t wf_topk_scratch_bytes(int64_t max_P);
 size_t wf_sweep_smem(const wf_dev_problem &dp);
+size_t wf_stoch_smem(const wf_dev_problem &dp);
+int wf_launch_stoch(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, size_t smem,
+                    int32_t *ovf_list, int32_t *ovf_count, cudaStream_t st);
 int wf_launch_sweep(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, size_t smem,
                     int32_t *ovf_list, int32_t *ovf_count, cudaStream_t st);

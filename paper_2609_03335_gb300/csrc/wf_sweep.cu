@@ -1,63 +1,29 @@
-// Plan evaluation, shared-memory sweep (rows a3-a10, deterministic plans).
+// Plan evaluation in shared memory (rows a3-a11).
 //
-// One thread plays one plan; a CTA holds G plans.  The CTA's plan rows
-// (placement, fusion / prefetch / retain bits) are staged into shared memory
-// by one thread with TMA bulk copies (cp.async.bulk, completion on an
-// mbarrier).  Each plan's mutable state lives in shared memory next to them,
-// interleaved [index][plan] so that the G lanes of a warp never collide on a
-// bank:
+// Deterministic plans (pc_kernel): a CTA plays 16 plans as a three-stage warp
+// pipeline over 16 dispatch positions at a time.  Producer warps turn each
+// (plan, position) into a unit record (Eq. 3-4 chain, write list, release
+// slot); one residency warp settles LRU model residency under capacity
+// (Eq. 11) with lane = plan; one timing warp plays releases, loads, starts and
+// finishes (Eq. 2, 5, 7, 10) with lane = plan.  Records pass through a ring of
+// three buffers guarded by named barriers.  Per-plan state lives in shared
+// memory, interleaved [index][plan]:
 //   - finish-time slots (u32 microseconds) assigned statically from the DAG
 //     (wf_slots.cpp) instead of one word per activation;
-//   - per device: free time, resident weights, resident count, LRU stamps;
-//   - a bitmap of dispatched activations (status bits 4 and 8).
-// The sweep itself follows Eq. 2-11 exactly like the int64 path in
-// wf_eval.cu; a plan whose times reach 2^32 us is handed to that path.
+//   - per device: free time, resident weights, resident count, LRU queue.
+// Status bits (Eq. 8-10) come first from status_kernel, a warp per plan.
+//
+// Stochastic latencies (stoch_kernel): one plan per CTA, the same pipeline
+// with one producer warp, residency settled once for all samples, and 64
+// timing lanes, one per sample.
+//
+// Times are u32; a plan whose times reach 2^32 us is listed for the exact
+// int64 path in wf_eval.cu.
 #include <algorithm>
 
 #include "wf_internal.cuh"
 
 namespace {
-
-constexpr uint32_t kWaitLimit = 1u << 24;  // bounded mbarrier wait (error word 3 on expiry)
-
-__device__ __forceinline__ uint32_t smem_addr(const void *p)
-{
-    return (uint32_t)__cvta_generic_to_shared(p);
-}
-
-__device__ __forceinline__ void mbar_init(uint64_t *bar)
-{
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_addr(bar)) : "memory");
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-}
-
-__device__ __forceinline__ void mbar_expect(uint64_t *bar, uint32_t bytes)
-{
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
-                 : "memory");
-}
-
-// Global -> shared bulk copy; bytes and both addresses are multiples of 16.
-__device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar)
-{
-    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
-                 ::"r"(smem_addr(dst)), "l"(src), "r"(bytes), "r"(smem_addr(bar))
-                 : "memory");
-}
-
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity)
-{
-    for (uint32_t it = 0; it < kWaitLimit; ++it) {
-        uint32_t ok;
-        asm volatile("{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-                     " selp.u32 %0, 1, 0, p;\n}"
-                     : "=r"(ok)
-                     : "r"(smem_addr(bar)), "r"(parity)
-                     : "memory");
-        if (ok) return true;
-    }
-    return false;
-}
 
 __host__ __device__ __forceinline__ uint32_t round16(uint32_t x) { return (x + 15u) & ~15u; }
 
@@ -209,10 +175,11 @@ struct PlanPtrs {
 
 // Producer: the unit record of dispatch position i of a plan.
 __device__ __forceinline__ void produce(const wf_dev_problem &dp, const PlanPtrs &r, int32_t i,
-                                        uint32_t rec[kRecWords])
+                                        uint32_t rec[kRecWords], int32_t *head = nullptr)
 {
     const int32_t D = dp.D;
     const int32_t h = __ldg(r.order + i);
+    if (head) *head = h;
     // Loads that depend on h alone go out together, ahead of any branch.
     const int32_t d = __ldg(r.place + h);
     const uint32_t lh = __ldg(dp.links + h);
@@ -466,6 +433,296 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list, in
     out.p95_us[p] = select_strided(slots, W, rank);
 }
 
+// ---------------------------------------------------------------------------
+// Stochastic latencies (row a11): one plan per CTA.  Model residency does not
+// depend on times, so one residency lane settles it for every sample; the
+// timing warps play kSamples samples at once (lane = sample), each drawing
+// its run-time multipliers from (plan, sample, node) through SplitMix64 and
+// the integer Box-Muller tables; then the CTA reduces the floor means and the
+// pooled nearest-rank p95 over samples x sessions.
+// ---------------------------------------------------------------------------
+constexpr int kSamples = 64;                  // timing lanes (two warps)
+constexpr int kSChunk = 32;                   // positions per chunk (one producer warp)
+constexpr int kSRec = kRecWords + 1;          // + head node
+constexpr int kSWarps = kSamples / 32 + 2;    // timing warps, residency warp, producer warp
+constexpr int kSTiming = kSamples;            // threads of the timing stage
+// Named barriers of this kernel (ids reuse those of the deterministic one).
+constexpr int kSFullP = 1, kSFullR = kSFullP + kBuffers, kSEmpty = kSFullR + kBuffers, kSOpen = kSEmpty + kBuffers,
+              kSRed = kSOpen + 1;
+
+struct StochLayout {
+    uint32_t weight, cap, load, arr, ring, slots, tfree, used, queue, nres, hist, red, total;
+};
+
+__host__ __device__ inline StochLayout stoch_layout(int32_t D, int32_t M, int32_t W, int32_t NS)
+{
+    StochLayout l;
+    uint32_t o = 0;
+    l.weight = o; o += round16(4u * M);
+    l.cap = o; o += round16(4u * D);
+    l.load = o; o += round16(4u * M * D);
+    l.arr = o; o += round16(4u * W);
+    l.ring = o; o += 4u * kBuffers * kSRec * kSChunk;
+    l.slots = o; o += 4u * (uint32_t)NS * kSamples;
+    l.tfree = o; o += 4u * D * kSamples;
+    l.used = o; o += round16(4u * D);
+    l.queue = o; o += 8u * D;
+    l.nres = o; o += round16((uint32_t)D);
+    l.hist = o; o += 4u * 256 + 16;
+    l.red = o; o += 8u * 2 * kSamples + 16;
+    l.total = o;
+    return l;
+}
+
+__device__ __forceinline__ uint64_t splitmix64(uint64_t x)
+{
+    x += 0x9E3779B97F4A7C15ull;
+    x = (x ^ (x >> 30)) * 0xBF58476D1CE4E5B9ull;
+    x = (x ^ (x >> 27)) * 0x94D049BB133111EBull;
+    return x ^ (x >> 31);
+}
+
+template <typename Q>
+__global__ void __launch_bounds__(32 * kSWarps)
+stoch_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list, int32_t *ovf_count)
+{
+    extern __shared__ __align__(128) uint8_t sm[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int32_t N = dp.N, D = dp.D, M = dp.M, W = dp.W, S = dp.S;
+    const StochLayout L = stoch_layout(D, M, W, dp.nslots);
+    const int64_t p = blockIdx.x;
+    if (out.status[p] != 0) return;  // uniform over the CTA: the status kernel marked the plan invalid
+    uint32_t *ring = (uint32_t *)(sm + L.ring);
+    const int32_t chunks = (N + kSChunk - 1) / kSChunk;
+    int32_t *weight = (int32_t *)(sm + L.weight);
+    int32_t *cap = (int32_t *)(sm + L.cap);
+    int32_t *load = (int32_t *)(sm + L.load);
+    uint32_t *arrival = (uint32_t *)(sm + L.arr);
+    for (int32_t k = threadIdx.x; k < M; k += blockDim.x) weight[k] = __ldg(dp.weight + k);
+    for (int32_t k = threadIdx.x; k < D; k += blockDim.x) cap[k] = __ldg(dp.cap + k);
+    for (int32_t k = threadIdx.x; k < M * D; k += blockDim.x) load[k] = __ldg(dp.load + k);
+    for (int32_t k = threadIdx.x; k < W; k += blockDim.x) arrival[k] = (uint32_t)__ldg(dp.arrival + k);
+    const int tw = kSTiming / 32;  // timing warps are 0 .. tw-1
+
+    if (warp == tw + 1) {
+        // ---------------- producer: lane = dispatch position ----------------
+        __syncthreads();
+        PlanPtrs r;
+        r.place = pl.place + p * pl.place_stride;
+        r.order = (const uint16_t *)((const uint8_t *)pl.order + p * pl.order_stride);
+        r.fuse = (const uint32_t *)((const uint8_t *)pl.fuse + p * pl.bits_stride);
+        r.prefetch = (const uint32_t *)((const uint8_t *)pl.prefetch + p * pl.bits_stride);
+        r.retain = pl.retain ? (const uint32_t *)((const uint8_t *)pl.retain + p * pl.bits_stride) : nullptr;
+        for (int32_t c = 0; c < chunks; ++c) {
+            const int b = c % kBuffers;
+            if (c >= kBuffers) named_sync(kSEmpty + b, kSTiming + 32);
+            uint32_t *rb = ring + b * kSRec * kSChunk;
+            const int32_t i = c * kSChunk + lane;
+            uint32_t rec[kRecWords] = {0, 0, 0, kSkip, 0, 0};
+            int32_t head = 0;
+            if (i < N) produce(dp, r, i, rec, &head);
+#pragma unroll
+            for (int w = 0; w < kRecWords; ++w) rb[w * kSChunk + lane] = rec[w];
+            rb[kRecWords * kSChunk + lane] = (uint32_t)head;
+            named_arrive(kSFullP + b, 64);
+        }
+        for (int32_t c = chunks; c < chunks + kBuffers; ++c)
+            if (c >= kBuffers) named_sync(kSEmpty + c % kBuffers, kSTiming + 32);
+        return;
+    }
+
+    if (warp == tw) {
+        // ---------------- residency, once for all samples (lane 0) ----------------
+        uint32_t *usedp = (uint32_t *)(sm + L.used);
+        Q *queuep = (Q *)(sm + L.queue);
+        uint8_t *nresp = sm + L.nres;
+        __syncthreads();
+        Q q[1];
+        if (lane == 0)
+            for (int32_t d = 0; d < D; ++d) { usedp[d] = 0; queuep[d] = 0; nresp[d] = 0; }
+        for (int32_t c = 0; c < chunks; ++c) {
+            const int b = c % kBuffers;
+            named_sync(kSFullP + b, 64);
+            uint32_t *rb = ring + b * kSRec * kSChunk;
+            const int32_t kmax = min(kSChunk, N - c * kSChunk);
+            for (int32_t k = 0; k < kmax && lane == 0; ++k) {
+                const uint32_t r3 = rb[3 * kSChunk + k];
+                if (r3 & kSkip) continue;
+                uint32_t &r1 = rb[1 * kSChunk + k];
+                const int32_t d = (int32_t)(r3 & 31u);
+                const uint32_t m = (r3 >> 5) & 15u;
+                q[0] = queuep[d];
+                uint32_t n = nresp[d];
+                uint32_t u_d = usedp[d];
+                const uint32_t wm = (uint32_t)weight[m];
+                const uint32_t capd = (uint32_t)cap[d];
+                const bool was_empty = n == 0;
+                const int32_t kq = Lru<Q>::find(q[0], n, m);
+                const bool hit = kq < (int32_t)n;
+                if (hit) { q[0] = Lru<Q>::remove(q[0], kq); n -= 1; }
+                const uint32_t need = hit ? r1 : wm + r1;
+                uint32_t e = 0;
+                while (u_d + need > capd && e < n) {
+                    u_d -= (uint32_t)weight[(uint32_t)(q[0] >> (4 * e)) & 15u];
+                    ++e;
+                }
+                if (u_d + need > capd) atomicExch(dp.err, 2);  // unreachable for a valid plan
+                q[0] = e < (uint32_t)Lru<Q>::kSlots ? (q[0] >> (4 * e)) : (Q)0;
+                n -= e;
+                q[0] |= (Q)m << (4 * n);
+                n += 1;
+                u_d += hit ? 0u : wm;
+                uint32_t emptied = 0;
+                if ((r3 >> 10) & 1u) {
+                    q[0] &= ~((Q)0xF << (4 * (n - 1)));
+                    n -= 1;
+                    u_d -= wm;
+                    emptied = n == 0;
+                }
+                queuep[d] = q[0];
+                nresp[d] = (uint8_t)n;
+                usedp[d] = u_d;
+                r1 = (hit ? 1u : 0u) | (was_empty ? 2u : 0u) | (emptied << 2);
+            }
+            named_arrive(kSFullR + b, kSTiming + 32);
+        }
+        uint32_t *hist = (uint32_t *)(sm + L.hist);
+        if (lane == 0) {
+            uint32_t o = 0;
+            for (int32_t d = 0; d < D; ++d) o += nresp[d] != 0;
+            hist[256] = o;  // devices still occupied at the end (same for every sample)
+        }
+        named_arrive(kSOpen, kSTiming + 32);
+        return;
+    }
+
+    // ---------------- timing: lane = sample ----------------
+    const int t = threadIdx.x;  // 0 .. kSamples-1
+    const bool live = t < S;
+    uint32_t *slots = (uint32_t *)(sm + L.slots) + t;
+    uint32_t *tfree = (uint32_t *)(sm + L.tfree) + t;
+    for (int32_t k = 0; k < dp.nslots; ++k) slots[k * kSamples] = 0;
+    for (int32_t d = 0; d < D; ++d) tfree[d * kSamples] = 0;
+    __syncthreads();
+    const uint64_t key = splitmix64(splitmix64(dp.seed ^ (uint64_t)(pl.plan_base + p)) ^ (uint64_t)t);
+    const uint64_t rmask = (uint64_t)(dp.bm_rn - 1), cmask = (uint64_t)(dp.bm_cn - 1);
+    const int64_t zoff = (dp.bm_en - 1) >> 1;
+    const uint32_t grant = (uint32_t)dp.grant;
+    uint32_t end = 0, ovf = 0;
+    int64_t gsum = 0;
+    for (int32_t c = 0; c < chunks; ++c) {
+        const int b = c % kBuffers;
+        named_sync(kSFullR + b, kSTiming + 32);
+        const uint32_t *rb = ring + b * kSRec * kSChunk;
+        const int32_t kmax = min(kSChunk, N - c * kSChunk);
+        for (int32_t k = 0; k < kmax && live; ++k) {
+            const uint32_t r3 = rb[3 * kSChunk + k];
+            if (r3 & kSkip) continue;
+            const uint32_t fl = rb[1 * kSChunk + k];
+            const uint32_t arr = rb[2 * kSChunk + k];
+            const uint32_t r4 = rb[4 * kSChunk + k];
+            const uint32_t r5 = rb[5 * kSChunk + k];
+            const int32_t d = (int32_t)(r3 & 31u);
+            const uint32_t m = (r3 >> 5) & 15u;
+            const bool hit = fl & 1u;
+            // Sampled run time of the unit: every member's multiplier (Eq. 4 sum).
+            const int32_t tail = (int32_t)(r5 & 0xFFFFu);
+            uint64_t run = 0;
+            for (int32_t j = (int32_t)rb[kRecWords * kSChunk + k];; j = (int32_t)(__ldg(dp.links + j) >> 16)) {
+                const uint64_t hh = splitmix64(key ^ (uint64_t)j);
+                const int64_t prod = (int64_t)__ldg(dp.bm_r + (hh & rmask)) * (int64_t)__ldg(dp.bm_c + ((hh >> 32) & cmask));
+                const int64_t mult = __ldg(dp.bm_e + ((prod >> 18) + zoff));
+                run += ((uint64_t)(uint32_t)__ldg(&dp.lk[j * D + d].x) * (uint64_t)mult + 32768u) >> 16;
+                if (j == tail) break;
+            }
+            ovf |= run >> 32 ? 1u : 0u;
+            uint32_t rel = arr;
+            const uint32_t rs = r5 >> 16;
+            if (rs != 0xFFFFu) {
+                uint32_t &sv = slots[(rs & 0x7FFFu) * kSamples];
+                rel = max(rel, sv);
+                if (rs & 0x8000u) sv = 0;
+            }
+            const uint32_t tf = tfree[d * kSamples];
+            const uint32_t ls = max(tf, ((r3 >> 9) & 1u) ? arr : rel);
+            const uint32_t le = ls + (uint32_t)load[m * D + d];
+            const uint32_t start = hit ? max(tf, rel) : max(le, rel);
+            ovf |= (!hit && le < ls) ? 1u : 0u;
+            gsum -= (!hit && (fl & 2u)) ? (int64_t)ls : 0;
+            const uint32_t sg = start + grant;
+            const uint32_t cfin = sg + (uint32_t)run;
+            ovf |= (sg < start) | (cfin < sg);
+            end = max(end, cfin);
+            gsum += (fl & 4u) ? (int64_t)cfin : 0;
+            const uint32_t nwl = (r3 >> 11) & 7u;
+            uint32_t *sl = slots;
+            if (nwl > 0) { uint32_t &sv = sl[((r3 >> 16) & 0x7FFFu) * kSamples]; sv = (r3 >> 31) ? max(sv, cfin) : cfin; }
+            if (nwl > 1) { uint32_t &sv = sl[(r4 & 0x7FFFu) * kSamples]; sv = ((r4 >> 15) & 1u) ? max(sv, cfin) : cfin; }
+            if (nwl > 2) {
+                { uint32_t &sv = sl[((r4 >> 16) & 0x7FFFu) * kSamples]; sv = (r4 >> 31) ? max(sv, cfin) : cfin; }
+                const int4 wr = __ldg(dp.noderec + 2 * tail + 1);
+                for (int32_t e = 3; e < wr.y; ++e) {
+                    const uint32_t code = __ldg(dp.wl + wr.x + e);
+                    uint32_t &sv = sl[(code & 0x7FFFu) * kSamples];
+                    sv = (code & 0x8000u) ? max(sv, cfin) : cfin;
+                }
+            }
+            tfree[d * kSamples] = cfin;
+        }
+        named_arrive(kSEmpty + b, kSTiming + 32);
+    }
+    named_sync(kSOpen, kSTiming + 32);
+    uint32_t *hist = (uint32_t *)(sm + L.hist);
+    const int64_t open = hist[256];
+    // Per-sample results, then the floor means and the pooled p95 over S x W.
+    int64_t *red = (int64_t *)(sm + L.red);
+    const int64_t mk = live ? (int64_t)end - dp.first_arrival : 0;
+    const int64_t g = live ? gsum + open * (int64_t)end : 0;
+    red[t] = mk;
+    red[kSamples + t] = g;
+    if (live) for (int32_t w = 0; w < W; ++w) slots[w * kSamples] -= arrival[w];
+    uint32_t *flag = hist + 257;
+    if (t == 0) *flag = 0;
+    named_sync(kSRed, kSTiming);
+    if (live && ovf) atomicOr(flag, 1u);
+    named_sync(kSRed, kSTiming);
+    if (*flag) {  // some sample's times do not fit u32: exact int64 path for the plan
+        if (t == 0) ovf_list[atomicAdd(ovf_count, 1)] = (int32_t)p;
+        return;
+    }
+    // Nearest-rank p95 of the pooled completions: radix select, 8 bits a pass.
+    const int64_t n = (int64_t)S * W;
+    uint32_t *meta = hist + 258;  // [0] prefix, [1] rank
+    if (t == 0) { meta[0] = 0; meta[1] = (uint32_t)((95 * n + 99) / 100 - 1); }
+    for (int shift = 24; shift >= 0; shift -= 8) {
+        for (int k = t; k < 256; k += kSTiming) hist[k] = 0;
+        named_sync(kSRed, kSTiming);
+        const uint32_t hi = shift == 24 ? 0u : (~0u << (shift + 8));
+        const uint32_t pre = meta[0];
+        if (live)
+            for (int32_t w = 0; w < W; ++w) {
+                const uint32_t v = slots[w * kSamples];
+                if ((v & hi) == pre) atomicAdd(&hist[(v >> shift) & 255u], 1u);
+            }
+        named_sync(kSRed, kSTiming);
+        if (t == 0) {
+            uint32_t r = meta[1];
+            int bin = 0;
+            while (hist[bin] <= r) { r -= hist[bin]; ++bin; }
+            meta[1] = r;
+            meta[0] |= (uint32_t)bin << shift;
+        }
+        named_sync(kSRed, kSTiming);
+    }
+    if (t == 0) {
+        int64_t smk = 0, sg = 0;
+        for (int k = 0; k < S; ++k) { smk += red[k]; sg += red[kSamples + k]; }
+        out.makespan_us[p] = smk / S;
+        out.gpu_us[p] = sg / S;
+        out.p95_us[p] = (int64_t)meta[0];
+    }
+}
+
 // Status bits of every plan (Eq. 8-10), one warp per plan: the warp scatters
 // the inverse permutation of the dispatch sequence (u16 positions; a bitmap
 // catches repeats) into shared memory, then checks every edge in parallel.
@@ -520,12 +777,56 @@ status_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out)
     }
 }
 
+int launch_status(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, cudaStream_t st)
+{
+    const wf_dev_problem &dp = ctx->dp;
+    const size_t wbytes = status_warp_bytes(dp.N);
+    const int swarps = (int)std::max<size_t>(1, std::min<size_t>(4, (227 * 1024) / wbytes));
+    const size_t ssmem = wbytes * swarps;
+    int rc = wf_cuda_check(cudaFuncSetAttribute(status_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                (int)ssmem), "status smem attribute");
+    if (rc) return rc;
+    const int64_t sblocks = std::min<int64_t>((pl->P + swarps - 1) / swarps, (int64_t)ctx->sms * 16);
+    status_kernel<<<(unsigned)sblocks, 32 * swarps, ssmem, st>>>(dp, *pl, *out);
+    return WF_OK;
+}
+
 }  // namespace
 
 // Shared memory of the producer / consumer kernel for this problem, or 0 when
 // the sweep cannot run it (slots unavailable, times beyond u32, more than 16
 // models, or more shared memory than a CTA may hold); the caller then uses
 // the int64 path.
+size_t wf_stoch_smem(const wf_dev_problem &dp)
+{
+    if (dp.nslots <= 0 || dp.max_arrival >= (int64_t)1 << 32 || dp.M > 16 || dp.N > 65534 ||
+        dp.S < 1 || dp.S > kSamples)
+        return 0;
+    const size_t s = stoch_layout(dp.D, dp.M, dp.W, dp.nslots).total;
+    return s <= 227 * 1024 ? s : 0;
+}
+
+int wf_launch_stoch(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, size_t smem,
+                    int32_t *ovf_list, int32_t *ovf_count, cudaStream_t st)
+{
+    const wf_dev_problem &dp = ctx->dp;
+    int rc = launch_status(ctx, pl, out, st);
+    if (rc) return rc;
+    const unsigned blocks = (unsigned)pl->P;
+    if (dp.M <= 8) {
+        rc = wf_cuda_check(cudaFuncSetAttribute(stoch_kernel<uint32_t>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                (int)smem), "stochastic smem attribute");
+        if (rc) return rc;
+        stoch_kernel<uint32_t><<<blocks, 32 * kSWarps, smem, st>>>(dp, *pl, *out, ovf_list, ovf_count);
+    } else {
+        rc = wf_cuda_check(cudaFuncSetAttribute(stoch_kernel<uint64_t>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                (int)smem), "stochastic smem attribute");
+        if (rc) return rc;
+        stoch_kernel<uint64_t><<<blocks, 32 * kSWarps, smem, st>>>(dp, *pl, *out, ovf_list, ovf_count);
+    }
+    return wf_cuda_check(cudaGetLastError(), "stochastic launch");
+}
+
 size_t wf_sweep_smem(const wf_dev_problem &dp)
 {
     if (dp.nslots <= 0 || dp.max_arrival >= (int64_t)1 << 32 || dp.M > 16 || dp.N > 65534) return 0;
@@ -537,14 +838,8 @@ int wf_launch_sweep(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, siz
                     int32_t *ovf_list, int32_t *ovf_count, cudaStream_t st)
 {
     const wf_dev_problem &dp = ctx->dp;
-    const size_t wbytes = status_warp_bytes(dp.N);
-    const int swarps = (int)std::max<size_t>(1, std::min<size_t>(4, (227 * 1024) / wbytes));
-    const size_t ssmem = wbytes * swarps;
-    int rc = wf_cuda_check(cudaFuncSetAttribute(status_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                (int)ssmem), "status smem attribute");
+    int rc = launch_status(ctx, pl, out, st);
     if (rc) return rc;
-    const int64_t sblocks = std::min<int64_t>((pl->P + swarps - 1) / swarps, (int64_t)ctx->sms * 16);
-    status_kernel<<<(unsigned)sblocks, 32 * swarps, ssmem, st>>>(dp, *pl, *out);
     const unsigned blocks = (unsigned)((pl->P + kPlans - 1) / kPlans);
     if (dp.M <= 8) {
         rc = wf_cuda_check(cudaFuncSetAttribute(pc_kernel<uint32_t>, cudaFuncAttributeMaxDynamicSharedMemorySize,

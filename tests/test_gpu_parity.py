@@ -129,6 +129,54 @@ def test_random_stochastic_windows(seed):
     assert_same(got, oracle_eval(prob, plans))
 
 
+@pytest.mark.parametrize("S", [1, 2, 31, 63, 64, 65])
+def test_stochastic_sample_counts(S):
+    """Sample counts around the width of the per-plan sample block (64 lanes)
+    and beyond it (the int64 path evaluates S > 64)."""
+    rng = np.random.default_rng(4200 + S)
+    prob = random_problem(rng, n_sessions=4, D=3)
+    r, c, e = wfgen.box_muller_tables()
+    prob = prob.with_(S=S, seed=int(rng.integers(0, 2**63)), bm_r=r, bm_c=c, bm_e=e)
+    plans = wfgen.make_plans(prob, 200, S, plan_base=int(rng.integers(0, 10**6)), p_retain=0.6)
+    inject_invalid(plans, prob, rng)
+    got = gpu_eval(prob, plans, k=7)
+    want = oracle_eval(prob, plans)
+    assert_same(got, want)
+    ids, keys = oracle.topk(want["makespan"], want["p95"], want["gpu"], want["status"], 7)
+    assert np.array_equal(got["ids"], ids) and np.array_equal(got["keys"], keys)
+
+
+def test_stochastic_int64_path_matches_oracle(monkeypatch):
+    """The per-sample int64 path on its own, forced for every plan."""
+    monkeypatch.setenv("WF_EVAL_PATH", "int64")
+    w = wfgen.config("stochastic")
+    plans = wfgen.make_plans(w.problem, 512, 91, p_retain=0.5)
+    inject_invalid(plans, w.problem, np.random.default_rng(2))
+    got = gpu_eval(w.problem, plans, k=8)
+    assert_same(got, oracle_eval(w.problem, plans))
+
+
+def test_stochastic_mixed_overflow_batch():
+    """Sampled times beyond 2^32 us for some plans (two activations are very
+    slow on device 1), within it for the others: the plans that overflow go to
+    the int64 path."""
+    rng = np.random.default_rng(41)
+    prob = random_problem(rng, n_sessions=4, sizes=(5, 9), D=2, M=3)
+    lat = prob.lat_us.astype(np.int64).reshape(prob.N, prob.D)
+    lat[:2, 1] = (1 << 31) - 1
+    r, c, e = wfgen.box_muller_tables()
+    prob = prob.with_(lat_us=lat.astype(np.int32).reshape(-1),
+                      peak_mib=np.minimum(prob.peak_mib, prob.cap_mib.min()).astype(np.int32)
+                      .clip(min=prob.weight_mib[prob.model].repeat(prob.D)),
+                      S=16, seed=99, bm_r=r, bm_c=c, bm_e=e)
+    plans = wfgen.make_plans(prob, 400, 6)
+    got = gpu_eval(prob, plans, k=5)
+    want = oracle_eval(prob, plans)
+    mk = want["makespan"][want["status"] == 0]
+    assert (mk >= (1 << 32)).any() and (mk < (1 << 31)).any()
+    assert_same(got, want)
+
+
 def test_ties_break_by_plan_index():
     w = wfgen.config("tiny")
     base = wfgen.make_plans(w.problem, 64, 3)
