@@ -238,6 +238,18 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
     size_t o_wloff = img.add(wl_off.data(), sizeof(int32_t) * (N + 1));
     size_t o_wl = img.add(wl.data(), sizeof(uint16_t) * wl.size());
     size_t o_lk = img.add(lk.data(), sizeof(int2) * lk.size());
+    // Status tables: the devices each activation fits on (Eq. 8), padded to a
+    // multiple of four entries, and every edge packed as pred | succ << 16.
+    std::vector<uint32_t> fitmask(((size_t)N + 3) & ~(size_t)3, 0u);
+    for (int32_t n = 0; n < N; ++n)
+        for (int32_t d = 0; d < D; ++d)
+            if (pb->peak_mib[(int64_t)n * D + d] <= pb->cap_mib[d]) fitmask[n] |= 1u << d;
+    size_t o_fit = img.add(fitmask.data(), sizeof(uint32_t) * fitmask.size());
+    std::vector<uint32_t> edges(E);
+    for (int32_t v = 0; v < N; ++v)
+        for (int32_t e = pb->pred_off[v]; e < pb->pred_off[v + 1]; ++e)
+            edges[e] = (uint32_t)pb->pred_idx[e] | ((uint32_t)v << 16);
+    size_t o_edges = img.add(edges.data(), sizeof(uint32_t) * E);
     size_t o_ovf = img.add(nullptr, sizeof(int32_t) * ((size_t)max_P + 64));
 
     wf_ctx *c = (wf_ctx *)calloc(1, sizeof(wf_ctx));
@@ -289,6 +301,8 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
     dp.wl = (const uint16_t *)(base + o_wl);
     dp.lk = (const int2 *)(base + o_lk);
     dp.links = (const uint32_t *)(base + o_links);
+    dp.fitmask = (const uint32_t *)(base + o_fit);
+    dp.edges = (const uint32_t *)(base + o_edges);
     int64_t amax = 0;
     for (int32_t w = 0; w < W; ++w) amax = std::max(amax, pb->arrival_us[w]);
     dp.max_arrival = amax;

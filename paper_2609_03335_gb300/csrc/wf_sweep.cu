@@ -89,20 +89,29 @@ constexpr int kPlansPerIter = 32 / kChunk;  // plans a producer warp covers per 
 constexpr int kBuffers = 3;
 constexpr int kWarps = 2 + kProducers;
 constexpr int kRecWords = 6;
-constexpr int kRingPitch = kPlans + 1;  // words per (word, position) row: conflict-free both ways
+// Words per (word, position) row of the ring.  A producer store covers
+// kChunk positions x (32 / kChunk) plans; with the pitch = 32 / kChunk
+// (mod 2 * 32 / kChunk) those 32 words fall in 32 distinct banks, and the
+// consumers' plan-major loads are contiguous.
+constexpr int kRingPitch = kPlans + 32 / kChunk;
 
 // Unit record (one per plan and dispatch position):
-//   w0 run time of the unit (sum over the fused chain, Eq. 4)
+//   w0 run time of the unit (sum over the fused chain, Eq. 4) plus the grant,
+//      saturated at 2^32 - 1 (a saturated unit sends its plan to the int64 path)
 //   w1 KV admission of the unit (largest on the chain, Eq. 4); the residency
-//      stage overwrites it with hit | was-empty << 1 | emptied-by-reclaim << 2
+//      stage overwrites it with the load time the unit waits for (0 on a hit)
 //   w2 arrival time of the unit's session
 //   w3 device | model << 5 | prefetch << 9 | reclaim << 10 | writes << 11 | skip << 14
-//      | run-time overflow << 15 | first write code << 16
+//      | first write code << 16; the residency stage clears the prefetch bit
+//      on a hit and sets kWasEmpty (bit 10) and kEmptied (bit 15) for timing
 //   w4 second write code | third write code << 16
 //   w5 the unit's last member (its full write list when it has more than
 //      three codes) | release slot code << 16 (bit 31: accumulator; 0xFFFF: none)
 constexpr uint32_t kSkip = 1u << 14;
-constexpr uint32_t kRunOvf = 1u << 15;
+constexpr uint32_t kPrefetch = 1u << 9;
+constexpr uint32_t kWasEmpty = 1u << 10;   // after residency: a miss on an empty device
+constexpr uint32_t kEmptied = 1u << 15;    // after residency: the unit's reclaim empties the device
+constexpr uint32_t kRunCap = 0xFFFFFFFFu;  // saturation of w0
 
 struct PcLayout {
     uint32_t weight, cap, load, arr, ring, slots, tfree, used, queue, nres, open, total;
@@ -120,7 +129,7 @@ __host__ __device__ inline PcLayout pc_layout(int32_t D, int32_t M, int32_t W, i
     l.slots = o; o += 4u * (uint32_t)NS * kPlans;
     l.tfree = o; o += 4u * D * kPlans;
     l.used = o; o += 4u * D * kPlans;
-    l.queue = o; o += 8u * D * kPlans;
+    l.queue = o; o += (M <= 8 ? 4u : 8u) * D * kPlans;  // Lru<uint32_t> or Lru<uint64_t>
     l.nres = o; o += round16((uint32_t)D * kPlans);
     l.open = o; o += 4u * kPlans;
     l.total = o;
@@ -161,9 +170,13 @@ __device__ uint32_t select_strided(uint32_t *v, int32_t n, int32_t r)
     return v[r * kPlans];
 }
 
-__device__ __forceinline__ uint32_t rslot16(int32_t code)
+// Two extra slots follow a plan's nslots slots: a sink that absorbs writes
+// with no reader (index nslots) and a slot that always holds 0 (nslots + 1),
+// the release slot of a node without predecessors.  With them every unit
+// reads one release slot and writes its first two codes without branching.
+__device__ __forceinline__ uint32_t rslot16(int32_t code, uint32_t zero)
 {
-    return code < 0 ? 0xFFFFu : (((uint32_t)code & 0x7FFFu) | ((code & WF_RSLOT_ACC) ? 0x8000u : 0u));
+    return code < 0 ? zero : (((uint32_t)code & 0x7FFFu) | ((code & WF_RSLOT_ACC) ? 0x8000u : 0u));
 }
 
 // Row pointers of one plan.
@@ -193,7 +206,7 @@ __device__ __forceinline__ void produce(const wf_dev_problem &dp, const PlanPtrs
         return;
     }
     const int2 lk0 = __ldg(dp.lk + h * D + d);
-    uint32_t run = (uint32_t)lk0.x, ovf = 0;
+    uint32_t run = (uint32_t)lk0.x + (uint32_t)dp.grant, ovf = 0;  // both < 2^31: no wrap
     int32_t kv = lk0.y, tail = h;
     for (uint32_t s = lh >> 16; s != 0xFFFFu; s = __ldg(dp.links + s) >> 16) {  // Eq. 3 chain
         if (!bit_of_g(r.fuse, s) || __ldg(r.place + s) != d) break;
@@ -206,18 +219,19 @@ __device__ __forceinline__ void produce(const wf_dev_problem &dp, const PlanPtrs
     }
     if (tail != h) wr = __ldg(dp.noderec + 2 * tail + 1);
     const uint32_t nwl = (uint32_t)min(wr.y, 7);
-    const uint32_t c0 = nwl > 0 ? (uint32_t)wr.z & 0xFFFFu : 0u;
-    const uint32_t c1 = nwl > 1 ? (uint32_t)wr.z >> 16 : 0u;
+    const uint32_t trash = (uint32_t)dp.nslots;
+    const uint32_t c0 = nwl > 0 ? (uint32_t)wr.z & 0xFFFFu : trash;
+    const uint32_t c1 = nwl > 1 ? (uint32_t)wr.z >> 16 : trash;
     const uint32_t c2 = nwl > 2 ? (uint32_t)__ldg(dp.wl + wr.x + 2) : 0u;
     const uint32_t pf = (pw >> (h & 31)) & 1u;
     const uint32_t reclaim = r.retain ? !bit_of_g(r.retain, tail) : 0u;
-    rec[0] = run;
+    rec[0] = ovf ? kRunCap : run;
     rec[1] = (uint32_t)kv;
     rec[2] = (uint32_t)__ldg(dp.arrival + (nr.w >> 8));
     rec[3] = (uint32_t)d | (((uint32_t)nr.w & 15u) << 5) | (pf << 9) | (reclaim << 10) | (nwl << 11) |
-             (ovf ? kRunOvf : 0u) | (c0 << 16);
+             (c0 << 16);
     rec[4] = c1 | (c2 << 16);
-    rec[5] = (uint32_t)tail | (rslot16(nr.z) << 16);
+    rec[5] = (uint32_t)tail | (rslot16(nr.z, trash + 1) << 16);
 }
 
 __device__ __forceinline__ void publish(uint32_t *slots, uint32_t code, uint32_t c)
@@ -233,7 +247,7 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list, in
     extern __shared__ __align__(128) uint8_t sm[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int32_t N = dp.N, D = dp.D, M = dp.M, W = dp.W;
-    const PcLayout L = pc_layout(D, M, W, dp.nslots);
+    const PcLayout L = pc_layout(D, M, W, dp.nslots + 2);
     const int64_t p0 = (int64_t)blockIdx.x * kPlans;
     const int ng = (int)(pl.P - p0 < kPlans ? pl.P - p0 : kPlans);
     uint32_t *ring = (uint32_t *)(sm + L.ring);
@@ -319,7 +333,8 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list, in
                 // Take the unit's own model out of the queue; the reclamation
                 // victims are then exactly its first e entries (least recently
                 // used first), and the unit's model goes back in at the end.
-                if (hit) { q = Lru<Q>::remove(q, kq); n -= 1; }
+                q = hit ? Lru<Q>::remove(q, hit ? kq : 0) : q;  // (an index below the queue length)
+                n -= hit ? 1u : 0u;
                 const uint32_t need = hit ? r1 : wm + r1;
                 uint32_t e = 0;
                 while (u_d + need > capd && e < n) {
@@ -342,7 +357,11 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list, in
                 queue[d * kPlans] = q;
                 nres[d * kPlans] = (uint8_t)n;
                 used[d * kPlans] = u_d;
-                r1 = (hit ? 1u : 0u) | (was_empty ? 2u : 0u) | (emptied << 2);
+                // For timing: the load to wait for (none on a hit, Eq. 5) and
+                // the occupancy changes of section 4.3.
+                r1 = hit ? 0u : (uint32_t)load[m * D + d];
+                rb[(3 * kChunk + k) * kRingPitch] = (r3 & ~(kPrefetch | kWasEmpty)) | (hit ? 0u : (r3 & kPrefetch)) |
+                                                    (was_empty ? kWasEmpty : 0u) | (emptied ? kEmptied : 0u);
             }
             named_arrive(kFullR + b, 64);
         }
@@ -360,11 +379,13 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list, in
     uint32_t *slots = (uint32_t *)(sm + L.slots) + lane;
     uint32_t *tfree = (uint32_t *)(sm + L.tfree) + lane;
     if (mine) {
-        for (int32_t k = 0; k < dp.nslots; ++k) slots[k * kPlans] = 0;
+        for (int32_t k = 0; k < dp.nslots + 2; ++k) slots[k * kPlans] = 0;
         for (int32_t d = 0; d < D; ++d) tfree[d * kPlans] = 0;
     }
     __syncthreads();
-    const uint32_t grant = (uint32_t)dp.grant;
+    const uint32_t trash = (uint32_t)dp.nslots;
+    // Times are u32.  A plan is handed to the int64 path when a sum carries
+    // out, or when a finish reaches 2^32 - 1 (which a saturated w0 forces).
     uint32_t end = 0, ovf = 0;
     int64_t gsum = 0;
     for (int32_t c = 0; c < chunks; ++c) {
@@ -376,48 +397,40 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list, in
             const uint32_t r3 = rb[(3 * kChunk + k) * kRingPitch];
             if (r3 & kSkip) continue;
             const uint32_t run = rb[(0 * kChunk + k) * kRingPitch];
-            const uint32_t fl = rb[(1 * kChunk + k) * kRingPitch];
+            const uint32_t ld = rb[(1 * kChunk + k) * kRingPitch];
             const uint32_t arr = rb[(2 * kChunk + k) * kRingPitch];
             const uint32_t r4 = rb[(4 * kChunk + k) * kRingPitch];
             const uint32_t r5 = rb[(5 * kChunk + k) * kRingPitch];
-            const int32_t d = (int32_t)(r3 & 31u);
-            const uint32_t m = (r3 >> 5) & 15u;
-            const bool hit = fl & 1u;
-            ovf |= r3 & kRunOvf;
+            uint32_t *tf_d = tfree + (r3 & 31u) * kPlans;
 
-            uint32_t rel = arr;  // release (Eq. 2, Eq. 7)
+            // Release (Eq. 2, Eq. 7); an accumulator slot is reset by its reader.
             const uint32_t rs = r5 >> 16;
-            if (rs != 0xFFFFu) {
-                uint32_t &sv = slots[(rs & 0x7FFFu) * kPlans];
-                rel = max(rel, sv);
-                if (rs & 0x8000u) sv = 0;
-            }
-            // Hit: start when device and release allow.  Miss: load on this
-            // device first; a prefetched load waits only for the arrival (Eq. 5).
-            const uint32_t tf = tfree[d * kPlans];
-            const uint32_t ls = max(tf, ((r3 >> 9) & 1u) ? arr : rel);
-            const uint32_t le = ls + (uint32_t)load[m * D + d];
-            const uint32_t start = hit ? max(tf, rel) : max(le, rel);
-            ovf |= (!hit && le < ls) ? 1u : 0u;
-            gsum -= (!hit && (fl & 2u)) ? (int64_t)ls : 0;  // an empty device becomes occupied
-            const uint32_t sg = start + grant;
-            const uint32_t cfin = sg + run;
-            ovf |= (sg < start) | (cfin < sg);
+            const uint32_t rel = max(arr, slots[(rs & 0x7FFFu) * kPlans]);
+            slots[((rs & 0x8000u) ? (rs & 0x7FFFu) : trash) * kPlans] = 0;
+            // A miss loads on this device first (ld > 0 only on a miss); a
+            // prefetched load waits only for the arrival (Eq. 5).  On a hit
+            // the residency stage cleared the prefetch bit and ld is 0.
+            const uint32_t ls = max(*tf_d, (r3 & kPrefetch) ? arr : rel);
+            const uint32_t le = ls + ld;
+            const uint32_t start = max(le, rel);
+            const uint32_t cfin = start + run;
+            ovf |= (le < ls) | (cfin < start);
             end = max(end, cfin);
-            gsum += (fl & 4u) ? (int64_t)cfin : 0;  // the device empties after the unit
+            if (r3 & kWasEmpty) gsum -= ls;   // an empty device becomes occupied
+            if (r3 & kEmptied) gsum += cfin;  // the device empties after the unit
 
-            const uint32_t nwl = (r3 >> 11) & 7u;
-            if (nwl > 0) publish(slots, r3 >> 16, cfin);
-            if (nwl > 1) publish(slots, r4 & 0xFFFFu, cfin);
-            if (nwl > 2) {
+            publish(slots, r3 >> 16, cfin);  // the sink when the unit writes nothing
+            publish(slots, r4 & 0xFFFFu, cfin);
+            if (((r3 >> 11) & 7u) > 2) {
                 publish(slots, r4 >> 16, cfin);
                 const int4 wr = __ldg(dp.noderec + 2 * (int32_t)(r5 & 0xFFFFu) + 1);
                 for (int32_t e = 3; e < wr.y; ++e) publish(slots, __ldg(dp.wl + wr.x + e), cfin);
             }
-            tfree[d * kPlans] = cfin;
+            *tf_d = cfin;
         }
         named_arrive(kEmpty + b, kProdThreads + 32);  // buffer b may be refilled
     }
+    ovf |= end == kRunCap;
     named_sync(kOpen, 64);  // the residency stage's final device counts
     if (!live) return;
     if (ovf) {  // times do not fit u32: exact int64 path
@@ -489,7 +502,7 @@ stoch_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list,
     extern __shared__ __align__(128) uint8_t sm[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int32_t N = dp.N, D = dp.D, M = dp.M, W = dp.W, S = dp.S;
-    const StochLayout L = stoch_layout(D, M, W, dp.nslots);
+    const StochLayout L = stoch_layout(D, M, W, dp.nslots + 2);
     const int64_t p = blockIdx.x;
     if (out.status[p] != 0) return;  // uniform over the CTA: the status kernel marked the plan invalid
     uint32_t *ring = (uint32_t *)(sm + L.ring);
@@ -601,7 +614,7 @@ stoch_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list,
     const bool live = t < S;
     uint32_t *slots = (uint32_t *)(sm + L.slots) + t;
     uint32_t *tfree = (uint32_t *)(sm + L.tfree) + t;
-    for (int32_t k = 0; k < dp.nslots; ++k) slots[k * kSamples] = 0;
+    for (int32_t k = 0; k < dp.nslots + 2; ++k) slots[k * kSamples] = 0;
     for (int32_t d = 0; d < D; ++d) tfree[d * kSamples] = 0;
     __syncthreads();
     const uint64_t key = splitmix64(splitmix64(dp.seed ^ (uint64_t)(pl.plan_base + p)) ^ (uint64_t)t);
@@ -723,13 +736,16 @@ stoch_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list,
     }
 }
 
-// Status bits of every plan (Eq. 8-10), one warp per plan: the warp scatters
-// the inverse permutation of the dispatch sequence (u16 positions; a bitmap
-// catches repeats) into shared memory, then checks every edge in parallel.
-// Invalid plans get INT64_MAX metrics here; the sweep skips them.
+// Status bits of every plan (Eq. 8-10), one warp per plan.  Four nodes per
+// lane check placement and fit (one fit mask per node); the warp scatters the
+// inverse of the dispatch sequence (u16 positions) into shared memory and
+// reads it back: a repeated node leaves some position with another position's
+// entry, so every in-range sequence that reads back intact is a permutation.
+// The edges (pred | succ << 16) are then checked 32 at a time.  Invalid plans
+// get INT64_MAX metrics here; the sweep skips them.
 __host__ __device__ inline uint32_t status_warp_bytes(int32_t N)
 {
-    return round16(2u * (uint32_t)N) + round16(4u * (((uint32_t)N + 31u) / 32u));
+    return round16(2u * (uint32_t)N);
 }
 
 __global__ void __launch_bounds__(128)
@@ -737,35 +753,47 @@ status_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out)
 {
     extern __shared__ __align__(16) uint8_t ssm[];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, warps = blockDim.x >> 5;
-    const int32_t N = dp.N, D = dp.D;
+    const int32_t N = dp.N, D = dp.D, E = dp.E;
     uint16_t *pos = (uint16_t *)(ssm + (size_t)warp * status_warp_bytes(N));
-    uint32_t *seen = (uint32_t *)((uint8_t *)pos + round16(2u * (uint32_t)N));
-    const int32_t words = (N + 31) / 32;
     for (int64_t p = (int64_t)blockIdx.x * warps + warp; p < pl.P; p += (int64_t)gridDim.x * warps) {
         const uint8_t *place = pl.place + p * pl.place_stride;
         const uint16_t *order = (const uint16_t *)((const uint8_t *)pl.order + p * pl.order_stride);
         uint32_t st = 0;
-        for (int32_t k = lane; k < words; k += 32) seen[k] = 0;
-        for (int32_t n = lane; n < N; n += 32) {
-            const int32_t d = place[n];
-            if (d >= D) st |= WF_ST_DEVICE;
-            else if (__ldg(dp.peak + (int64_t)n * D + d) > __ldg(dp.cap + d)) st |= WF_ST_CAPACITY;
+        // Rows start 16-byte aligned and hold at least N entries; a word read
+        // past N stays inside the row's padding to 4 bytes only when used
+        // below N, so lanes mask the entries at or beyond N.
+        for (int32_t n4 = 4 * lane; n4 < N; n4 += 128) {
+            const uint32_t pw = __ldg((const uint32_t *)(place + n4));
+            const uint4 fm = __ldg((const uint4 *)(dp.fitmask + n4));
+            const uint32_t f[4] = {fm.x, fm.y, fm.z, fm.w};
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const uint32_t d = (pw >> (8 * j)) & 255u;
+                if (n4 + j < N) st |= d >= (uint32_t)D ? WF_ST_DEVICE : (((f[j] >> d) & 1u) ? 0u : WF_ST_CAPACITY);
+            }
+        }
+        for (int32_t i = 2 * lane; i < N; i += 64) {
+            const uint32_t ow = __ldg((const uint32_t *)(order + i));
+            const uint32_t h0 = ow & 0xFFFFu, h1 = ow >> 16;
+            if (h0 < (uint32_t)N) pos[h0] = (uint16_t)i;
+            else st |= WF_ST_PERMUTATION;
+            if (i + 1 < N) {
+                if (h1 < (uint32_t)N) pos[h1] = (uint16_t)(i + 1);
+                else st |= WF_ST_PERMUTATION;
+            }
         }
         __syncwarp();
-        for (int32_t i = lane; i < N; i += 32) {
-            const int32_t h = order[i];
-            if (h >= N) { st |= WF_ST_PERMUTATION; continue; }
-            const uint32_t b = 1u << (h & 31);
-            if (atomicOr(&seen[h >> 5], b) & b) st |= WF_ST_PERMUTATION;
-            pos[h] = (uint16_t)i;
+        for (int32_t i = 2 * lane; i < N; i += 64) {
+            const uint32_t ow = __ldg((const uint32_t *)(order + i));
+            const uint32_t h0 = ow & 0xFFFFu, h1 = ow >> 16;
+            if (h0 < (uint32_t)N && pos[h0] != (uint16_t)i) st |= WF_ST_PERMUTATION;
+            if (i + 1 < N && h1 < (uint32_t)N && pos[h1] != (uint16_t)(i + 1)) st |= WF_ST_PERMUTATION;
         }
-        __syncwarp();
         st = __reduce_or_sync(0xFFFFFFFFu, st);
         if (!(st & WF_ST_PERMUTATION)) {
-            for (int32_t v = lane; v < N; v += 32) {
-                const uint32_t pv = pos[v];
-                for (int32_t e = __ldg(dp.pred_off + v); e < __ldg(dp.pred_off + v + 1); ++e)
-                    if (pos[__ldg(dp.pred_idx + e)] > pv) st |= WF_ST_TOPOLOGY;
+            for (int32_t e = lane; e < E; e += 32) {
+                const uint32_t uv = __ldg(dp.edges + e);
+                if (pos[uv & 0xFFFFu] > pos[uv >> 16]) st |= WF_ST_TOPOLOGY;
             }
             st = __reduce_or_sync(0xFFFFFFFFu, st);
         }
@@ -773,7 +801,7 @@ status_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out)
             out.status[p] = st;
             if (st) out.makespan_us[p] = out.p95_us[p] = out.gpu_us[p] = WF_INF64;
         }
-        __syncwarp();  // pos[] and seen[] are reused by the warp's next plan
+        __syncwarp();  // pos[] is reused by the warp's next plan
     }
 }
 
@@ -799,10 +827,10 @@ int launch_status(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, cudaS
 // the int64 path.
 size_t wf_stoch_smem(const wf_dev_problem &dp)
 {
-    if (dp.nslots <= 0 || dp.max_arrival >= (int64_t)1 << 32 || dp.M > 16 || dp.N > 65534 ||
+    if (dp.nslots <= 0 || dp.nslots > 32765 || dp.max_arrival >= (int64_t)1 << 32 || dp.M > 16 || dp.N > 65534 ||
         dp.S < 1 || dp.S > kSamples)
         return 0;
-    const size_t s = stoch_layout(dp.D, dp.M, dp.W, dp.nslots).total;
+    const size_t s = stoch_layout(dp.D, dp.M, dp.W, dp.nslots + 2).total;
     return s <= 227 * 1024 ? s : 0;
 }
 
@@ -829,8 +857,9 @@ int wf_launch_stoch(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, siz
 
 size_t wf_sweep_smem(const wf_dev_problem &dp)
 {
-    if (dp.nslots <= 0 || dp.max_arrival >= (int64_t)1 << 32 || dp.M > 16 || dp.N > 65534) return 0;
-    const size_t s = pc_layout(dp.D, dp.M, dp.W, dp.nslots).total;
+    if (dp.nslots <= 0 || dp.nslots > 32765 || dp.max_arrival >= (int64_t)1 << 32 || dp.M > 16 || dp.N > 65534)
+        return 0;
+    const size_t s = pc_layout(dp.D, dp.M, dp.W, dp.nslots + 2).total;
     return s <= 227 * 1024 ? s : 0;
 }
 

@@ -273,6 +273,21 @@ def test_times_beyond_u32_take_the_int64_path():
     assert_same(got, want)
 
 
+def test_fused_run_time_beyond_u32():
+    """Fused chains of near-2^31 us members: a unit's summed run time alone
+    leaves 32 bits, with a start of 0 on some plans."""
+    rng = np.random.default_rng(43)
+    prob = random_problem(rng, n_sessions=3, sizes=(6, 9), D=2, M=2)
+    lat = np.full(prob.N * prob.D, (1 << 31) - 1, np.int32)
+    prob = prob.with_(lat_us=lat, arrival_us=np.zeros(prob.W, np.int64),
+                      load_us=np.zeros_like(prob.load_us), grant_us=0)
+    plans = wfgen.make_plans(prob, 300, 8, p_fuse=0.95)
+    got = gpu_eval(prob, plans, k=4)
+    want = oracle_eval(prob, plans)
+    assert (want["makespan"][want["status"] == 0] >= (1 << 32)).all()
+    assert_same(got, want)
+
+
 def test_mixed_overflow_batch():
     """Some plans overflow u32, some do not, in one batch."""
     rng = np.random.default_rng(37)
