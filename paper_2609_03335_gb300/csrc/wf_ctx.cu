@@ -250,7 +250,7 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
         for (int32_t e = pb->pred_off[v]; e < pb->pred_off[v + 1]; ++e)
             edges[e] = (uint32_t)pb->pred_idx[e] | ((uint32_t)v << 16);
     size_t o_edges = img.add(edges.data(), sizeof(uint32_t) * E);
-    size_t o_ovf = img.add(nullptr, sizeof(int32_t) * ((size_t)max_P + 64));
+    size_t o_ovf = img.add(nullptr, sizeof(int32_t) * (2 * (size_t)max_P + 64));
 
     wf_ctx *c = (wf_ctx *)calloc(1, sizeof(wf_ctx));
     if (!c) return wf_set_error(WF_ENOMEM, "host allocation of the context");
@@ -308,6 +308,7 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
     dp.max_arrival = amax;
     c->ovf_count = (int32_t *)(base + o_ovf);
     c->ovf_list = c->ovf_count + 64;
+    c->ovf_list2 = c->ovf_list + max_P;
     rc = wf_cuda_check(cudaDeviceGetAttribute(&c->sms, cudaDevAttrMultiProcessorCount, device), "SM count");
     if (rc) { wf_ctx_destroy(c); return rc; }
 
@@ -320,6 +321,10 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
         c->topk_scratch_bytes = wf_topk_scratch_bytes(max_P);
         rc = wf_cuda_check(cudaMalloc(&c->topk_scratch, c->topk_scratch_bytes), "cudaMalloc(topk scratch)");
     }
+    if (!rc) rc = wf_cuda_check(cudaMallocHost(&c->h_ovf, sizeof(int32_t)), "cudaMallocHost(overflow count)");
+    if (!rc) rc = wf_cuda_check(cudaEventCreateWithFlags(&c->ovf_event, cudaEventDisableTiming), "cudaEventCreate");
+    if (!rc) rc = wf_cuda_check(cudaEventCreateWithFlags(&c->sweep_done, cudaEventDisableTiming), "cudaEventCreate");
+    if (!rc) rc = wf_cuda_check(cudaStreamCreateWithFlags(&c->side, cudaStreamNonBlocking), "cudaStreamCreate");
     if (rc) { wf_ctx_destroy(c); return rc; }
     *out = c;
     return WF_OK;
@@ -334,6 +339,11 @@ extern "C" void wf_ctx_destroy(wf_ctx *c)
     if (c->tables) cudaFree(c->tables);
     if (c->eval_scratch) cudaFree(c->eval_scratch);
     if (c->topk_scratch) cudaFree(c->topk_scratch);
+    if (c->side) cudaStreamSynchronize(c->side);
+    if (c->side) cudaStreamDestroy(c->side);
+    if (c->ovf_event) cudaEventDestroy(c->ovf_event);
+    if (c->sweep_done) cudaEventDestroy(c->sweep_done);
+    if (c->h_ovf) cudaFreeHost(c->h_ovf);
     if (prev >= 0) cudaSetDevice(prev);
     free(c);
 }

@@ -389,14 +389,48 @@ int wf_launch_eval(wf_ctx *ctx, const wf_plans *plans, const wf_eval_out *out, c
     const int64_t units = std::min<int64_t>(ctx->eval_threads, plans->P);
     if (dp.S == 0) {
         const int64_t blocks = (units + kEvalThreads - 1) / kEvalThreads;
-        const size_t smem = ctx->force_int64 ? 0 : wf_sweep_smem(dp);
-        if (smem) {
-            int rc = wf_cuda_check(cudaMemsetAsync(ctx->ovf_count, 0, sizeof(int32_t), st), "reset overflow count");
-            if (!rc) rc = wf_launch_sweep(ctx, plans, out, smem, ctx->ovf_list, ctx->ovf_count, st);
+        const wf_sweep_cfg cfg = ctx->force_int64 ? wf_sweep_cfg{0, 0, 0} : wf_sweep_config(dp);
+        if (cfg.smem32 || cfg.smem64) {
+            // Path choice: the u32 sweep's hand-off count of an earlier call,
+            // if it has arrived (never waited for).
+            if (ctx->wide_pending) {
+                const cudaError_t q = cudaEventQuery(ctx->ovf_event);
+                if (q == cudaSuccess) {
+                    ctx->prefer_wide = 2 * (int64_t)*ctx->h_ovf > ctx->wide_P;
+                    ctx->wide_pending = false;
+                } else if (q == cudaErrorNotReady) {
+                    (void)cudaGetLastError();
+                } else {
+                    return wf_cuda_check(q, "overflow count event");
+                }
+            }
+            const bool wide_first = ctx->prefer_wide && cfg.smem64;
+            int rc = wf_cuda_check(cudaMemsetAsync(ctx->ovf_count, 0, 2 * sizeof(int32_t), st), "reset overflow counts");
+            const int32_t *rest = nullptr, *rest_count = nullptr;
+            if (!rc) rc = wf_launch_sweep(ctx, plans, out, cfg, wide_first, ctx->ovf_count, ctx->ovf_list,
+                                          ctx->ovf_list2, st, &rest, &rest_count);
             if (rc) return rc;
+            cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+            rc = wf_cuda_check(cudaStreamIsCapturing(st, &cs), "stream capture status");
+            if (rc) return rc;
+            if (cfg.smem32 && !wide_first && !ctx->wide_pending && cs == cudaStreamCaptureStatusNone) {
+                // The read-back runs on the context's side stream after the
+                // sweeps, so the caller's stream never waits for it.  A later
+                // call may reset the count before the copy runs; the value
+                // only picks the path, never a result.
+                rc = wf_cuda_check(cudaEventRecord(ctx->sweep_done, st), "sweep event");
+                if (!rc) rc = wf_cuda_check(cudaStreamWaitEvent(ctx->side, ctx->sweep_done, 0), "side stream wait");
+                if (!rc) rc = wf_cuda_check(cudaMemcpyAsync(ctx->h_ovf, ctx->ovf_count, sizeof(int32_t),
+                                                            cudaMemcpyDeviceToHost, ctx->side),
+                                            "overflow count read-back");
+                if (!rc) rc = wf_cuda_check(cudaEventRecord(ctx->ovf_event, ctx->side), "overflow count event");
+                if (rc) return rc;
+                ctx->wide_pending = true;
+                ctx->wide_P = plans->P;
+            }
             eval_list_kernel<<<(unsigned)blocks, kEvalThreads, 0, st>>>(dp, *plans, *out, scratch,
                                                                        ctx->eval_row_bytes, units,
-                                                                       ctx->ovf_list, ctx->ovf_count);
+                                                                       rest, rest_count);
         } else {
             eval_det_kernel<<<(unsigned)blocks, kEvalThreads, 0, st>>>(dp, *plans, *out, scratch,
                                                                         ctx->eval_row_bytes, units);

@@ -70,8 +70,19 @@ struct wf_ctx {
     int *err;
     int sms;                    // streaming multiprocessors of the device
     bool force_int64;           // WF_EVAL_PATH=int64: always take the int64 path (tests)
-    int32_t *ovf_count;         // plans the u32 sweep hands to the int64 path
-    int32_t *ovf_list;          // [max_P]
+    int32_t *ovf_count;         // [2]: plans the u32 sweep hands on, plans left for the int64 path
+    int32_t *ovf_list;          // [max_P] the u32 sweep's hand-offs (and the stochastic sweep's)
+    int32_t *ovf_list2;         // [max_P] plans for the int64 path
+    // Path choice from an earlier call: when more than half of a batch left
+    // 32 bits, later calls start with the u64 sweep.  The count is read back
+    // through pinned memory and an event, never waited for.
+    bool prefer_wide;
+    bool wide_pending;
+    int64_t wide_P;
+    int32_t *h_ovf;             // pinned host copy of ovf_count[0]
+    cudaEvent_t sweep_done;     // recorded on the caller's stream after the sweeps
+    cudaEvent_t ovf_event;      // recorded on side after the read-back
+    cudaStream_t side;          // the read-back's own stream, off the caller's critical path
 };
 
 // Static slot assignment (wf_slots.cpp).  Fills rslot code per node, write
@@ -92,9 +103,19 @@ int wf_launch_topk(wf_ctx *ctx, const wf_eval_out *res, int64_t P, int32_t k, in
 size_t wf_eval_row_bytes(const wf_dev_problem &dp);
 size_t wf_eval_scratch_bytes(const wf_dev_problem &dp, int64_t max_P, int64_t *units);
 size_t wf_topk_scratch_bytes(int64_t max_P);
-size_t wf_sweep_smem(const wf_dev_problem &dp);
+// The shared-memory sweeps that apply to a problem: u32 times with 16 plans
+// per CTA, and u64 times with plans64 plans per CTA (0 bytes = not usable).
+struct wf_sweep_cfg {
+    size_t smem32;
+    size_t smem64;
+    int plans64;
+};
+wf_sweep_cfg wf_sweep_config(const wf_dev_problem &dp);
 size_t wf_stoch_smem(const wf_dev_problem &dp);
 int wf_launch_stoch(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, size_t smem,
                     int32_t *ovf_list, int32_t *ovf_count, cudaStream_t st);
-int wf_launch_sweep(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, size_t smem,
-                    int32_t *ovf_list, int32_t *ovf_count, cudaStream_t st);
+// Status pass, then the sweeps (u32 first unless wide_first); on return
+// *rest_list / *rest_count name the plans left for the int64 path.
+int wf_launch_sweep(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, const wf_sweep_cfg &cfg,
+                    bool wide_first, int32_t *counts, int32_t *list1, int32_t *list2, cudaStream_t st,
+                    const int32_t **rest_list, const int32_t **rest_count);

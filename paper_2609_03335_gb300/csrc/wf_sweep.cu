@@ -77,23 +77,27 @@ __device__ __forceinline__ uint32_t bit_of_g(const uint32_t *row, int32_t n)
 }
 
 // CTA shape, a three-stage pipeline over kChunk dispatch positions at a time:
-// warps 2..kProducers+1 prepare the unit records of kPlans plans (lane =
+// warps 2..kProducers+1 prepare the unit records of kP plans (lane =
 // position) into a ring of kBuffers buffers; warp 1 settles model residency
 // (lane = plan: hits, reclamations, occupancy changes); warp 0 plays the
-// timing (lane = plan: releases, starts, finishes, slots).  16 plans per CTA
-// lets four CTAs share an SM.
-constexpr int kPlans = 16;
-constexpr int kProducers = 3;
+// timing (lane = plan: releases, starts, finishes, slots).  With u32 times
+// and 16 plans per CTA, four CTAs share an SM at 2,000 activations; the u64
+// variant holds fewer plans per CTA when its slots need the room.
 constexpr int kChunk = 16;
 constexpr int kPlansPerIter = 32 / kChunk;  // plans a producer warp covers per iteration
 constexpr int kBuffers = 3;
-constexpr int kWarps = 2 + kProducers;
 constexpr int kRecWords = 6;
-// Words per (word, position) row of the ring.  A producer store covers
-// kChunk positions x (32 / kChunk) plans; with the pitch = 32 / kChunk
-// (mod 2 * 32 / kChunk) those 32 words fall in 32 distinct banks, and the
-// consumers' plan-major loads are contiguous.
-constexpr int kRingPitch = kPlans + 32 / kChunk;
+
+template <int kP>
+struct PcShape {
+    static constexpr int kProducers = kP >= 6 ? 3 : 2;
+    static constexpr int kWarps = 2 + kProducers;
+    // Words per (word, position) row of the ring.  A producer store covers 16
+    // positions x 2 plans; a pitch of 2 (mod 4) puts those 32 words in 32
+    // distinct banks, and the consumers' plan-major loads are contiguous.
+    static constexpr int kPitch = ((kP + 1) | 3) - 1;
+    static_assert(kChunk == 16 && kP >= 1 && kP <= 32, "ring pitch assumes 16 positions per chunk");
+};
 
 // Unit record (one per plan and dispatch position):
 //   w0 run time of the unit (sum over the fused chain, Eq. 4) plus the grant,
@@ -114,24 +118,28 @@ constexpr uint32_t kEmptied = 1u << 15;    // after residency: the unit's reclai
 constexpr uint32_t kRunCap = 0xFFFFFFFFu;  // saturation of w0
 
 struct PcLayout {
-    uint32_t weight, cap, load, arr, ring, slots, tfree, used, queue, nres, open, total;
+    uint32_t weight, cap, load, arr, ring, slots, tfree, used, queue, nres, open, flag, total;
 };
 
+// Shared memory of a CTA of kP plans with TT times and NS slots per plan.
+template <int kP, typename TT>
 __host__ __device__ inline PcLayout pc_layout(int32_t D, int32_t M, int32_t W, int32_t NS)
 {
+    constexpr uint32_t t = sizeof(TT);
     PcLayout l;
     uint32_t o = 0;
     l.weight = o; o += round16(4u * M);
     l.cap = o; o += round16(4u * D);
     l.load = o; o += round16(4u * M * D);
     l.arr = o; o += round16(4u * W);
-    l.ring = o; o += 4u * kBuffers * kRecWords * kChunk * kRingPitch;
-    l.slots = o; o += 4u * (uint32_t)NS * kPlans;
-    l.tfree = o; o += 4u * D * kPlans;
-    l.used = o; o += 4u * D * kPlans;
-    l.queue = o; o += (M <= 8 ? 4u : 8u) * D * kPlans;  // Lru<uint32_t> or Lru<uint64_t>
-    l.nres = o; o += round16((uint32_t)D * kPlans);
-    l.open = o; o += 4u * kPlans;
+    l.ring = o; o += round16(4u * kBuffers * kRecWords * kChunk * PcShape<kP>::kPitch);
+    l.slots = o; o += round16(t * (uint32_t)NS * kP);
+    l.tfree = o; o += round16(t * D * kP);
+    l.used = o; o += round16(4u * D * kP);
+    l.queue = o; o += round16((M <= 8 ? 4u : 8u) * D * kP);  // Lru<uint32_t> or Lru<uint64_t>
+    l.nres = o; o += round16((uint32_t)D * kP);
+    l.open = o; o += round16(4u * kP);
+    l.flag = o; o += 16;
     l.total = o;
     return l;
 }
@@ -151,23 +159,24 @@ __device__ __forceinline__ void named_arrive(int id, int threads)
     asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(threads) : "memory");
 }
 
-// r-th smallest (0-based) of the kPlans-strided values v[0], v[kPlans], ...
-__device__ uint32_t select_strided(uint32_t *v, int32_t n, int32_t r)
+// r-th smallest (0-based) of the kS-strided values v[0], v[kS], ...
+template <typename TT, int kS>
+__device__ TT select_strided(TT *v, int32_t n, int32_t r)
 {
     int32_t lo = 0, hi = n - 1;
     while (lo < hi) {
-        const uint32_t pivot = v[(lo + (hi - lo) / 2) * kPlans];
+        const TT pivot = v[(lo + (hi - lo) / 2) * kS];
         int32_t i = lo, j = hi;
         while (i <= j) {
-            while (v[i * kPlans] < pivot) ++i;
-            while (v[j * kPlans] > pivot) --j;
-            if (i <= j) { uint32_t t = v[i * kPlans]; v[i * kPlans] = v[j * kPlans]; v[j * kPlans] = t; ++i; --j; }
+            while (v[i * kS] < pivot) ++i;
+            while (v[j * kS] > pivot) --j;
+            if (i <= j) { TT t = v[i * kS]; v[i * kS] = v[j * kS]; v[j * kS] = t; ++i; --j; }
         }
         if (r <= j) hi = j;
         else if (r >= i) lo = i;
-        else return v[r * kPlans];
+        else return v[r * kS];
     }
-    return v[r * kPlans];
+    return v[r * kS];
 }
 
 // Two extra slots follow a plan's nslots slots: a sink that absorbs writes
@@ -234,25 +243,37 @@ __device__ __forceinline__ void produce(const wf_dev_problem &dp, const PlanPtrs
     rec[5] = (uint32_t)tail | (rslot16(nr.z, trash + 1) << 16);
 }
 
-__device__ __forceinline__ void publish(uint32_t *slots, uint32_t code, uint32_t c)
+template <typename TT, int kS>
+__device__ __forceinline__ void publish(TT *slots, uint32_t code, TT c)
 {
-    uint32_t &sv = slots[(code & 0x7FFFu) * kPlans];
+    TT &sv = slots[(code & 0x7FFFu) * kS];
     sv = (code & 0x8000u) ? max(sv, c) : c;
 }
 
-template <typename Q>
-__global__ void __launch_bounds__(32 * kWarps)
-pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list, int32_t *ovf_count)
+// The sweep of groups of kP plans: every plan of the batch (in_list NULL, plan
+// = group * kP + q) or the listed ones (plan = in_list[group * kP + q] below
+// *in_count).  CTA b plays groups b, b + gridDim.x, ...  TT = uint32_t: a plan whose times leave 32 bits is appended to
+// ovf_list; once every plan of a CTA has, its stages run on without loads.
+// TT = uint64_t: only a unit whose summed run time reaches 2^32 - 1 sends its
+// plan to ovf_list.
+template <typename Q, typename TT, int kP>
+__global__ void __launch_bounds__(32 * PcShape<kP>::kWarps)
+pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_list, const int32_t *in_count,
+          int32_t *ovf_list, int32_t *ovf_count)
 {
+    using S = PcShape<kP>;
+    constexpr int kPitch = S::kPitch;
+    constexpr int kProdThreads = 32 * S::kProducers;
+    constexpr bool kNarrow = sizeof(TT) == 4;
     extern __shared__ __align__(128) uint8_t sm[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int32_t N = dp.N, D = dp.D, M = dp.M, W = dp.W;
-    const PcLayout L = pc_layout(D, M, W, dp.nslots + 2);
-    const int64_t p0 = (int64_t)blockIdx.x * kPlans;
-    const int ng = (int)(pl.P - p0 < kPlans ? pl.P - p0 : kPlans);
+    const PcLayout L = pc_layout<kP, TT>(D, M, W, dp.nslots + 2);
+    const int64_t total = in_list ? (int64_t)*in_count : pl.P;
+    if ((int64_t)blockIdx.x * kP >= total) return;  // the whole CTA: no plan
     uint32_t *ring = (uint32_t *)(sm + L.ring);
     const int32_t chunks = (N + kChunk - 1) / kChunk;
-    constexpr int kProdThreads = 32 * kProducers;
+    volatile uint32_t *gave_up = (volatile uint32_t *)(sm + L.flag);
 
     int32_t *weight = (int32_t *)(sm + L.weight);
     int32_t *cap = (int32_t *)(sm + L.cap);
@@ -262,69 +283,74 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list, in
     for (int32_t k = threadIdx.x; k < D; k += blockDim.x) cap[k] = __ldg(dp.cap + k);
     for (int32_t k = threadIdx.x; k < M * D; k += blockDim.x) load[k] = __ldg(dp.load + k);
     for (int32_t k = threadIdx.x; k < W; k += blockDim.x) arrival[k] = (uint32_t)__ldg(dp.arrival + k);
+    // (each role's first __syncthreads below publishes these tables)
 
-    // Lanes at or beyond kPlans own no plan and touch no per-plan state.
-    const bool mine = lane < kPlans;
-    const int64_t p = p0 + lane;
+  for (int64_t j0 = (int64_t)blockIdx.x * kP; j0 < total; j0 += (int64_t)gridDim.x * kP) {
+    const int ng = (int)(total - j0 < kP ? total - j0 : kP);
+    if (threadIdx.x == 0) *gave_up = 0;
+
+    // Lanes at or beyond kP own no plan and touch no per-plan state.
+    const bool mine = lane < kP;
+    const int64_t p = (mine && lane < ng) ? (in_list ? (int64_t)in_list[j0 + lane] : j0 + lane) : 0;
     const bool live = warp < 2 && mine && lane < ng && out.status[p] == 0;
 
     if (warp >= 2) {
         // ---------------- producers: lane = dispatch position ----------------
         __syncthreads();
+        const int pos = lane % kChunk, sub = lane / kChunk;
         for (int32_t c = 0; c < chunks; ++c) {
             const int b = c % kBuffers;
             if (c >= kBuffers) named_sync(kEmpty + b, kProdThreads + 32);  // timing released buffer b
-            uint32_t *rb = ring + b * kRecWords * kChunk * kRingPitch;
-            const int pos = lane % kChunk, sub = lane / kChunk;
+            const bool quit = kNarrow && *gave_up;
+            uint32_t *rb = ring + b * kRecWords * kChunk * kPitch;
             const int32_t i = c * kChunk + pos;
-            for (int q0 = (warp - 2) * kPlansPerIter; q0 < kPlans; q0 += kProducers * kPlansPerIter) {
+            for (int q0 = (warp - 2) * kPlansPerIter; q0 < kP; q0 += S::kProducers * kPlansPerIter) {
                 const int q = q0 + sub;
-                if (q >= kPlans) continue;
+                if (q >= kP) continue;
                 uint32_t rec[kRecWords] = {0, 0, 0, kSkip, 0, 0};
-                const int64_t pq = p0 + q;
-                if (q < ng && i < N && __ldg(out.status + pq) == 0) {
-                    PlanPtrs r;
-                    r.place = pl.place + pq * pl.place_stride;
-                    r.order = (const uint16_t *)((const uint8_t *)pl.order + pq * pl.order_stride);
-                    r.fuse = (const uint32_t *)((const uint8_t *)pl.fuse + pq * pl.bits_stride);
-                    r.prefetch = (const uint32_t *)((const uint8_t *)pl.prefetch + pq * pl.bits_stride);
-                    r.retain = pl.retain ? (const uint32_t *)((const uint8_t *)pl.retain + pq * pl.bits_stride)
-                                         : nullptr;
-                    produce(dp, r, i, rec);
+                if (q < ng && i < N && !quit) {
+                    const int64_t pq = in_list ? (int64_t)__ldg(in_list + j0 + q) : j0 + q;
+                    if (__ldg(out.status + pq) == 0) {
+                        PlanPtrs r;
+                        r.place = pl.place + pq * pl.place_stride;
+                        r.order = (const uint16_t *)((const uint8_t *)pl.order + pq * pl.order_stride);
+                        r.fuse = (const uint32_t *)((const uint8_t *)pl.fuse + pq * pl.bits_stride);
+                        r.prefetch = (const uint32_t *)((const uint8_t *)pl.prefetch + pq * pl.bits_stride);
+                        r.retain = pl.retain ? (const uint32_t *)((const uint8_t *)pl.retain + pq * pl.bits_stride)
+                                             : nullptr;
+                        produce(dp, r, i, rec);
+                    }
                 }
 #pragma unroll
-                for (int w = 0; w < kRecWords; ++w) rb[(w * kChunk + pos) * kRingPitch + q] = rec[w];
+                for (int w = 0; w < kRecWords; ++w) rb[(w * kChunk + pos) * kPitch + q] = rec[w];
             }
             named_arrive(kFullP + b, kProdThreads + 32);  // buffer b is full
         }
         // Match the timing stage's releases of the last buffers.
         for (int32_t c = chunks; c < chunks + kBuffers; ++c)
             if (c >= kBuffers) named_sync(kEmpty + c % kBuffers, kProdThreads + 32);
-        return;
-    }
-
-    if (warp == 1) {
+    } else if (warp == 1) {
         // ---------------- residency: lane = plan (Eq. 11, Section 3.5) ----------------
         uint32_t *used = (uint32_t *)(sm + L.used) + lane;
         Q *queue = (Q *)(sm + L.queue) + lane;
         uint8_t *nres = sm + L.nres + lane;
         if (mine)
-            for (int32_t d = 0; d < D; ++d) { used[d * kPlans] = 0; queue[d * kPlans] = 0; nres[d * kPlans] = 0; }
+            for (int32_t d = 0; d < D; ++d) { used[d * kP] = 0; queue[d * kP] = 0; nres[d * kP] = 0; }
         __syncthreads();
         for (int32_t c = 0; c < chunks; ++c) {
             const int b = c % kBuffers;
             named_sync(kFullP + b, kProdThreads + 32);
-            uint32_t *rb = ring + b * kRecWords * kChunk * kRingPitch + lane;
+            uint32_t *rb = ring + b * kRecWords * kChunk * kPitch + lane;
             const int32_t kmax = min(kChunk, N - c * kChunk);
             for (int32_t k = 0; k < kmax && live; ++k) {
-                const uint32_t r3 = rb[(3 * kChunk + k) * kRingPitch];
+                const uint32_t r3 = rb[(3 * kChunk + k) * kPitch];
                 if (r3 & kSkip) continue;
-                uint32_t &r1 = rb[(1 * kChunk + k) * kRingPitch];
+                uint32_t &r1 = rb[(1 * kChunk + k) * kPitch];
                 const int32_t d = (int32_t)(r3 & 31u);
                 const uint32_t m = (r3 >> 5) & 15u;
-                Q q = queue[d * kPlans];
-                uint32_t n = nres[d * kPlans];
-                uint32_t u_d = used[d * kPlans];  // used + need <= cap + peak < 2^32
+                Q q = queue[d * kP];
+                uint32_t n = nres[d * kP];
+                uint32_t u_d = used[d * kP];  // used + need <= cap + peak < 2^32
                 const uint32_t wm = (uint32_t)weight[m];
                 const uint32_t capd = (uint32_t)cap[d];
                 const bool was_empty = n == 0;
@@ -354,96 +380,102 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list, in
                     u_d -= wm;
                     emptied = n == 0;
                 }
-                queue[d * kPlans] = q;
-                nres[d * kPlans] = (uint8_t)n;
-                used[d * kPlans] = u_d;
+                queue[d * kP] = q;
+                nres[d * kP] = (uint8_t)n;
+                used[d * kP] = u_d;
                 // For timing: the load to wait for (none on a hit, Eq. 5) and
                 // the occupancy changes of section 4.3.
                 r1 = hit ? 0u : (uint32_t)load[m * D + d];
-                rb[(3 * kChunk + k) * kRingPitch] = (r3 & ~(kPrefetch | kWasEmpty)) | (hit ? 0u : (r3 & kPrefetch)) |
-                                                    (was_empty ? kWasEmpty : 0u) | (emptied ? kEmptied : 0u);
+                rb[(3 * kChunk + k) * kPitch] = (r3 & ~(kPrefetch | kWasEmpty)) | (hit ? 0u : (r3 & kPrefetch)) |
+                                                (was_empty ? kWasEmpty : 0u) | (emptied ? kEmptied : 0u);
             }
             named_arrive(kFullR + b, 64);
         }
         uint32_t *open = (uint32_t *)(sm + L.open);
         if (live) {
             uint32_t o = 0;
-            for (int32_t d = 0; d < D; ++d) o += nres[d * kPlans] != 0;
+            for (int32_t d = 0; d < D; ++d) o += nres[d * kP] != 0;
             open[lane] = o;
         }
         named_arrive(kOpen, 64);
-        return;
-    }
-
+    } else {
     // ---------------- timing: lane = plan (Eq. 2, 5, 7, 10) ----------------
-    uint32_t *slots = (uint32_t *)(sm + L.slots) + lane;
-    uint32_t *tfree = (uint32_t *)(sm + L.tfree) + lane;
+    TT *slots = (TT *)(sm + L.slots) + lane;
+    TT *tfree = (TT *)(sm + L.tfree) + lane;
     if (mine) {
-        for (int32_t k = 0; k < dp.nslots + 2; ++k) slots[k * kPlans] = 0;
-        for (int32_t d = 0; d < D; ++d) tfree[d * kPlans] = 0;
+        for (int32_t k = 0; k < dp.nslots + 2; ++k) slots[k * kP] = 0;
+        for (int32_t d = 0; d < D; ++d) tfree[d * kP] = 0;
     }
     __syncthreads();
     const uint32_t trash = (uint32_t)dp.nslots;
-    // Times are u32.  A plan is handed to the int64 path when a sum carries
-    // out, or when a finish reaches 2^32 - 1 (which a saturated w0 forces).
-    uint32_t end = 0, ovf = 0;
+    // u32 times: a plan is handed on when a sum carries out, or when a finish
+    // reaches 2^32 - 1 (which a saturated w0 forces).  u64 times cannot wrap;
+    // only a saturated w0 is handed on.
+    TT end = 0;
+    uint32_t ovf = 0;
     int64_t gsum = 0;
     for (int32_t c = 0; c < chunks; ++c) {
         const int b = c % kBuffers;
         named_sync(kFullR + b, 64);
-        const uint32_t *rb = ring + b * kRecWords * kChunk * kRingPitch + lane;
+        const uint32_t *rb = ring + b * kRecWords * kChunk * kPitch + lane;
         const int32_t kmax = min(kChunk, N - c * kChunk);
         for (int32_t k = 0; k < kmax && live; ++k) {
-            const uint32_t r3 = rb[(3 * kChunk + k) * kRingPitch];
+            const uint32_t r3 = rb[(3 * kChunk + k) * kPitch];
             if (r3 & kSkip) continue;
-            const uint32_t run = rb[(0 * kChunk + k) * kRingPitch];
-            const uint32_t ld = rb[(1 * kChunk + k) * kRingPitch];
-            const uint32_t arr = rb[(2 * kChunk + k) * kRingPitch];
-            const uint32_t r4 = rb[(4 * kChunk + k) * kRingPitch];
-            const uint32_t r5 = rb[(5 * kChunk + k) * kRingPitch];
-            uint32_t *tf_d = tfree + (r3 & 31u) * kPlans;
+            const uint32_t run = rb[(0 * kChunk + k) * kPitch];
+            const uint32_t ld = rb[(1 * kChunk + k) * kPitch];
+            const uint32_t arr = rb[(2 * kChunk + k) * kPitch];
+            const uint32_t r4 = rb[(4 * kChunk + k) * kPitch];
+            const uint32_t r5 = rb[(5 * kChunk + k) * kPitch];
+            TT *tf_d = tfree + (r3 & 31u) * kP;
 
             // Release (Eq. 2, Eq. 7); an accumulator slot is reset by its reader.
             const uint32_t rs = r5 >> 16;
-            const uint32_t rel = max(arr, slots[(rs & 0x7FFFu) * kPlans]);
-            slots[((rs & 0x8000u) ? (rs & 0x7FFFu) : trash) * kPlans] = 0;
+            const TT rel = max((TT)arr, slots[(rs & 0x7FFFu) * kP]);
+            slots[((rs & 0x8000u) ? (rs & 0x7FFFu) : trash) * kP] = 0;
             // A miss loads on this device first (ld > 0 only on a miss); a
             // prefetched load waits only for the arrival (Eq. 5).  On a hit
             // the residency stage cleared the prefetch bit and ld is 0.
-            const uint32_t ls = max(*tf_d, (r3 & kPrefetch) ? arr : rel);
-            const uint32_t le = ls + ld;
-            const uint32_t start = max(le, rel);
-            const uint32_t cfin = start + run;
-            ovf |= (le < ls) | (cfin < start);
+            const TT ls = max(*tf_d, (r3 & kPrefetch) ? (TT)arr : rel);
+            const TT le = ls + ld;
+            const TT start = max(le, rel);
+            const TT cfin = start + run;
+            if (kNarrow) ovf |= (le < ls) | (cfin < start);
+            else ovf |= run == kRunCap;
             end = max(end, cfin);
-            if (r3 & kWasEmpty) gsum -= ls;   // an empty device becomes occupied
-            if (r3 & kEmptied) gsum += cfin;  // the device empties after the unit
+            if (r3 & kWasEmpty) gsum -= (int64_t)ls;   // an empty device becomes occupied
+            if (r3 & kEmptied) gsum += (int64_t)cfin;  // the device empties after the unit
 
-            publish(slots, r3 >> 16, cfin);  // the sink when the unit writes nothing
-            publish(slots, r4 & 0xFFFFu, cfin);
+            publish<TT, kP>(slots, r3 >> 16, cfin);  // the sink when the unit writes nothing
+            publish<TT, kP>(slots, r4 & 0xFFFFu, cfin);
             if (((r3 >> 11) & 7u) > 2) {
-                publish(slots, r4 >> 16, cfin);
+                publish<TT, kP>(slots, r4 >> 16, cfin);
                 const int4 wr = __ldg(dp.noderec + 2 * (int32_t)(r5 & 0xFFFFu) + 1);
-                for (int32_t e = 3; e < wr.y; ++e) publish(slots, __ldg(dp.wl + wr.x + e), cfin);
+                for (int32_t e = 3; e < wr.y; ++e) publish<TT, kP>(slots, __ldg(dp.wl + wr.x + e), cfin);
             }
             *tf_d = cfin;
         }
+        // Once every plan of the CTA has left 32 bits, the producers stop
+        // loading (they see the flag at their next wait on this buffer).
+        if (kNarrow && __all_sync(0xFFFFFFFFu, !live || ovf) && lane == 0) *gave_up = 1;
         named_arrive(kEmpty + b, kProdThreads + 32);  // buffer b may be refilled
     }
-    ovf |= end == kRunCap;
+    if (kNarrow) ovf |= end == (TT)kRunCap;
     named_sync(kOpen, 64);  // the residency stage's final device counts
-    if (!live) return;
-    if (ovf) {  // times do not fit u32: exact int64 path
+    if (live && ovf) {  // handed to the next path
         const int32_t kk = atomicAdd(ovf_count, 1);
         ovf_list[kk] = (int32_t)p;
-        return;
+    } else if (live) {
+        const int64_t open = ((const uint32_t *)(sm + L.open))[lane];
+        for (int32_t w = 0; w < W; ++w) slots[w * kP] -= arrival[w];  // session completion latency
+        const int32_t rank = (int32_t)((95 * (int64_t)W + 99) / 100 - 1);
+        out.makespan_us[p] = (int64_t)end - dp.first_arrival;
+        out.gpu_us[p] = gsum + open * (int64_t)end;
+        out.p95_us[p] = (int64_t)select_strided<TT, kP>(slots, W, rank);
     }
-    const int64_t open = ((const uint32_t *)(sm + L.open))[lane];
-    for (int32_t w = 0; w < W; ++w) slots[w * kPlans] -= arrival[w];  // session completion latency
-    const int32_t rank = (int32_t)((95 * (int64_t)W + 99) / 100 - 1);
-    out.makespan_us[p] = (int64_t)end - dp.first_arrival;
-    out.gpu_us[p] = gsum + open * (int64_t)end;
-    out.p95_us[p] = select_strided(slots, W, rank);
+    }
+    __syncthreads();  // the group's shared state is free for the next group
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -855,31 +887,87 @@ int wf_launch_stoch(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, siz
     return wf_cuda_check(cudaGetLastError(), "stochastic launch");
 }
 
-size_t wf_sweep_smem(const wf_dev_problem &dp)
+namespace {
+
+bool sweep_usable(const wf_dev_problem &dp)
 {
-    if (dp.nslots <= 0 || dp.nslots > 32765 || dp.max_arrival >= (int64_t)1 << 32 || dp.M > 16 || dp.N > 65534)
-        return 0;
-    const size_t s = pc_layout(dp.D, dp.M, dp.W, dp.nslots + 2).total;
-    return s <= 227 * 1024 ? s : 0;
+    return dp.nslots > 0 && dp.nslots <= 32765 && dp.max_arrival < ((int64_t)1 << 32) && dp.M <= 16 &&
+           dp.N <= 65534;
 }
 
-int wf_launch_sweep(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, size_t smem,
-                    int32_t *ovf_list, int32_t *ovf_count, cudaStream_t st)
+// Plans per SM at this shared-memory size (228 KB per SM, 1 KB reserved per CTA).
+int plans_per_sm(size_t smem, int kp)
+{
+    return smem <= 227 * 1024 ? kp * (int)((228 * 1024) / (smem + 1024)) : 0;
+}
+
+template <typename Q, typename TT, int kP>
+int launch_pc(const wf_dev_problem &dp, int sms, const wf_plans *pl, const wf_eval_out *out, size_t smem,
+              const int32_t *in_list, const int32_t *in_count, int32_t *list, int32_t *count, cudaStream_t st)
+{
+    int rc = wf_cuda_check(cudaFuncSetAttribute(pc_kernel<Q, TT, kP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                (int)smem), "sweep smem attribute");
+    if (rc) return rc;
+    // Every plan: a CTA per group.  A list (of unknown length): at most as
+    // many CTAs as are resident at once, each walking over groups.
+    int64_t blocks = (pl->P + kP - 1) / kP;
+    if (in_list) {
+        const int64_t per_sm = std::max<int64_t>(1, std::min<int64_t>(8, (228 * 1024) / (int64_t)(smem + 1024)));
+        blocks = std::min<int64_t>(blocks, per_sm * sms);
+    }
+    pc_kernel<Q, TT, kP><<<(unsigned)blocks, 32 * PcShape<kP>::kWarps, smem, st>>>(dp, *pl, *out, in_list, in_count, list,
+                                                                          count);
+    return wf_cuda_check(cudaGetLastError(), "sweep launch");
+}
+
+template <typename TT>
+int launch_pc_q(const wf_ctx *ctx, int kp, const wf_plans *pl, const wf_eval_out *out, size_t smem,
+                const int32_t *in_list, const int32_t *in_count, int32_t *list, int32_t *count, cudaStream_t st)
 {
     const wf_dev_problem &dp = ctx->dp;
+    const int sms = ctx->sms;
+    if (kp == 16)
+        return dp.M <= 8 ? launch_pc<uint32_t, TT, 16>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
+                         : launch_pc<uint64_t, TT, 16>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
+    return dp.M <= 8 ? launch_pc<uint32_t, TT, 6>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
+                     : launch_pc<uint64_t, TT, 6>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
+}
+
+}  // namespace
+
+wf_sweep_cfg wf_sweep_config(const wf_dev_problem &dp)
+{
+    wf_sweep_cfg c = {0, 0, 0};
+    if (!sweep_usable(dp)) return c;
+    const int32_t NS = dp.nslots + 2;
+    const size_t s32 = pc_layout<16, uint32_t>(dp.D, dp.M, dp.W, NS).total;
+    if (s32 <= 227 * 1024) c.smem32 = s32;
+    // The u64 sweep: 16 plans per CTA, or 6 where that keeps more plans per SM.
+    const size_t s16 = pc_layout<16, uint64_t>(dp.D, dp.M, dp.W, NS).total;
+    const size_t s6 = pc_layout<6, uint64_t>(dp.D, dp.M, dp.W, NS).total;
+    const int a = plans_per_sm(s16, 16), b = plans_per_sm(s6, 6);
+    if (a > 0 && a >= b) { c.smem64 = s16; c.plans64 = 16; }
+    else if (b > 0) { c.smem64 = s6; c.plans64 = 6; }
+    return c;
+}
+
+int wf_launch_sweep(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, const wf_sweep_cfg &cfg,
+                    bool wide_first, int32_t *counts, int32_t *list1, int32_t *list2, cudaStream_t st,
+                    const int32_t **rest_list, const int32_t **rest_count)
+{
     int rc = launch_status(ctx, pl, out, st);
     if (rc) return rc;
-    const unsigned blocks = (unsigned)((pl->P + kPlans - 1) / kPlans);
-    if (dp.M <= 8) {
-        rc = wf_cuda_check(cudaFuncSetAttribute(pc_kernel<uint32_t>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                (int)smem), "sweep smem attribute");
+    if (cfg.smem32 && !(wide_first && cfg.smem64)) {
+        // u32 times for every plan; the plans that leave 32 bits go on to the
+        // u64 sweep, and from there (or straight) to the int64 path.
+        rc = launch_pc_q<uint32_t>(ctx, 16, pl, out, cfg.smem32, nullptr, nullptr, list1, counts, st);
         if (rc) return rc;
-        pc_kernel<uint32_t><<<blocks, 32 * kWarps, smem, st>>>(dp, *pl, *out, ovf_list, ovf_count);
+        if (!cfg.smem64) { *rest_list = list1; *rest_count = counts; return WF_OK; }
+        rc = launch_pc_q<uint64_t>(ctx, cfg.plans64, pl, out, cfg.smem64, list1, counts, list2, counts + 1, st);
     } else {
-        rc = wf_cuda_check(cudaFuncSetAttribute(pc_kernel<uint64_t>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                (int)smem), "sweep smem attribute");
-        if (rc) return rc;
-        pc_kernel<uint64_t><<<blocks, 32 * kWarps, smem, st>>>(dp, *pl, *out, ovf_list, ovf_count);
+        rc = launch_pc_q<uint64_t>(ctx, cfg.plans64, pl, out, cfg.smem64, nullptr, nullptr, list2, counts + 1, st);
     }
-    return wf_cuda_check(cudaGetLastError(), "sweep launch");
+    *rest_list = list2;
+    *rest_count = counts + 1;
+    return rc;
 }

@@ -288,6 +288,30 @@ def test_fused_run_time_beyond_u32():
     assert_same(got, want)
 
 
+def test_repeated_calls_after_overflow():
+    """A context whose batches leave 32 bits starts later calls with the u64
+    sweep; every call gives the oracle's results."""
+    import torch
+    from gpu_util import lib
+    wf = lib()
+    rng = np.random.default_rng(47)
+    prob = random_problem(rng, n_sessions=6, sizes=(6, 12), D=3, M=3)
+    lat = (prob.lat_us.astype(np.int64) % 1000 + (1 << 30) - 5000).astype(np.int32)
+    prob = prob.with_(lat_us=lat)
+    plans = wfgen.make_plans(prob, 700, 9, p_retain=0.4)
+    want = oracle_eval(prob, plans)
+    assert (want["makespan"][want["status"] == 0] >= (1 << 32)).all()
+    ctx = wf.Ctx(prob, max_P=plans.P)
+    dp = wf.DevicePlans.from_host(plans, "cuda")
+    for _ in range(3):
+        res = wf.Results(plans.P)
+        wf.wf_eval_plans(ctx, dp, res)
+        torch.cuda.synchronize()
+        mk, p95, gpu, st = res.numpy()
+        assert np.array_equal(mk, want["makespan"]) and np.array_equal(p95, want["p95"])
+        assert np.array_equal(gpu, want["gpu"]) and np.array_equal(st, want["status"])
+
+
 def test_mixed_overflow_batch():
     """Some plans overflow u32, some do not, in one batch."""
     rng = np.random.default_rng(37)
