@@ -73,7 +73,9 @@ def _setup(lib):
     lib.orc_splitmix64.restype = ctypes.c_uint64
     lib.orc_multiplier.argtypes = [p, ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint64]
     lib.orc_multiplier.restype = ctypes.c_int64
-    for f in ("orc_fusible_next", "orc_forecast", "orc_status", "orc_eval_plan", "orc_eval_batch"):
+    lib.orc_mutate.argtypes = [p, p, i64, p, i64, p, p, p, i64, i64, p, i64, p, i64, p, p, p, i64, i64,
+                               ctypes.c_uint64, i64, ctypes.c_int32]
+    for f in ("orc_fusible_next", "orc_forecast", "orc_status", "orc_eval_plan", "orc_eval_batch", "orc_mutate"):
         getattr(lib, f).restype = ctypes.c_int
     return lib
 
@@ -248,3 +250,89 @@ def splitmix64(x: int) -> int:
 def multiplier(prob, plan: int, sample: int, node: int) -> int:
     op = OracleProblem(prob)
     return int(op.lib.orc_multiplier(ctypes.byref(op.c), plan, sample, node))
+
+
+class PlanRows:
+    """A batch of plan rows (the layout of the evaluator's inputs)."""
+
+    def __init__(self, P: int, N: int, with_retain: bool, plan_base: int = 0):
+        words = (N + 31) // 32
+        self.P, self.N, self.plan_base = P, N, plan_base
+        self.place = np.zeros((P, N), np.uint8)
+        self.order = np.zeros((P, N), np.uint16)
+        self.fuse = np.zeros((P, words), np.uint32)
+        self.prefetch = np.zeros((P, words), np.uint32)
+        self.retain = np.zeros((P, words), np.uint32) if with_retain else None
+
+    @staticmethod
+    def copy_of(plans, N: int):
+        """Rows 0..P-1 of any batch with the same fields (padding dropped)."""
+        words = (N + 31) // 32
+        retain = getattr(plans, "retain", None)
+        out = PlanRows(plans.P, N, retain is not None, int(getattr(plans, "plan_base", 0)))
+        out.place[:] = plans.place[:, :N]
+        out.order[:] = plans.order[:, :N]
+        out.fuse[:] = plans.fuse[:, :words]
+        out.prefetch[:] = plans.prefetch[:, :words]
+        if retain is not None:
+            out.retain[:] = retain[:, :words]
+        return out
+
+
+def mutate(prob, parents, n_children: int, seed: int, round_: int, n_ops: int, plan_base: int = 0):
+    """Children of a parent batch: child c copies parent c mod P and takes
+    n_ops point changes (move / fuse flip / prefetch flip / adjacent swap)
+    decoded from SplitMix64 of (seed, round, c, step)."""
+    op = OracleProblem(prob)
+    N = op.N
+    par = {a: np.ascontiguousarray(getattr(parents, a)) for a in ("place", "order", "fuse", "prefetch")}
+    ret = None if parents.retain is None else np.ascontiguousarray(parents.retain)
+    ch = PlanRows(n_children, N, ret is not None, plan_base)
+    rc = op.lib.orc_mutate(ctypes.byref(op.c), par["place"].ctypes.data, par["place"].shape[1],
+                           par["order"].ctypes.data, par["order"].shape[1] * 2,
+                           par["fuse"].ctypes.data, par["prefetch"].ctypes.data,
+                           None if ret is None else ret.ctypes.data, par["fuse"].shape[1] * 4, parents.P,
+                           ch.place.ctypes.data, N, ch.order.ctypes.data, 2 * N,
+                           ch.fuse.ctypes.data, ch.prefetch.ctypes.data,
+                           None if ch.retain is None else ch.retain.ctypes.data, ch.fuse.shape[1] * 4,
+                           n_children, seed & ((1 << 64) - 1), round_, n_ops)
+    if rc != 0:
+        raise RuntimeError(f"oracle mutate failed ({rc})")
+    return ch
+
+
+def merge_elite(elite_metrics, child_metrics, k: int):
+    """The k best of elite (indices 0..k-1) and children (k, k+1, ...) by the
+    top-k key, kept in place: elite slots whose plan stays keep it; the
+    leaving slots, in ascending order, take the entering children in key
+    order.  Returns [(slot, child)] and the elite's new metrics."""
+    union = [np.concatenate([np.asarray(e), np.asarray(c)]) for e, c in zip(elite_metrics, child_metrics)]
+    ids, _ = topk(union[0], union[1], union[2], union[3], k)
+    ids = [int(i) for i in ids]
+    entering = [i - k for i in ids if i >= k]
+    kept = set(i for i in ids if i < k)
+    leaving = [s for s in range(k) if s not in kept]
+    pairs = list(zip(leaving, entering))
+    new = [np.asarray(e).copy() for e in elite_metrics]
+    for s, c in pairs:
+        for a in range(4):
+            new[a][s] = np.asarray(child_metrics[a])[c]
+    return pairs, new
+
+
+def local_search(prob, elite, elite_metrics, n_children: int, seed: int, round0: int, rounds: int,
+                 n_ops: int, children_plan_base: int = 0, threads: int = 1):
+    """rounds x (children of the elite -> evaluate -> keep the k best in
+    place).  Returns the final elite rows and metrics."""
+    k = elite.P
+    cur = PlanRows.copy_of(elite, int(prob.N))
+    met = [np.asarray(m).copy() for m in elite_metrics]
+    for r in range(rounds):
+        ch = mutate(prob, cur, n_children, seed, round0 + r, n_ops, children_plan_base)
+        cm = eval_plans(prob, ch, threads=threads)
+        pairs, met = merge_elite(met, cm, k)
+        for s, c in pairs:
+            for a in ("place", "order", "fuse", "prefetch", "retain"):
+                if getattr(cur, a) is not None:
+                    getattr(cur, a)[s] = getattr(ch, a)[c]
+    return cur, met

@@ -482,3 +482,87 @@ int orc_eval_batch(const orc_problem *pb, const int32_t *fnext,
     }
     return 0;
 }
+
+/*
+ * Local search around the best plans (the scheduler's re-ranking of its
+ * uncommitted decisions after new information, Section 3.5): each child is a
+ * copy of a parent with n_ops point changes.  Child c (0-based within the
+ * call) copies parent c mod n_parents; change s of child c is decoded from
+ *   h = mix(mix(mix(seed ^ round) ^ c) ^ s),  x = bits 8..39 of h,  y = bits 40..63:
+ *   h mod 4 = 0  move:     n = x mod N; the device becomes the (y mod f)-th
+ *                          (0-based, ascending) of the f devices whose
+ *                          capacity holds peak[n][d] (Eq. 8);
+ *             1  fuse:     n = x mod N; flip the fuse bit of n (Eq. 3);
+ *             2  prefetch: n = x mod N; flip the prefetch bit of n (Eq. 5);
+ *             3  swap:     i = x mod (N - 1); exchange dispatch positions i
+ *                          and i + 1 unless the node at i is a graph
+ *                          predecessor of the node at i + 1 (Eq. 10 keeps
+ *                          the sequence topological); no change when N = 1
+ *                          or the node at i + 1 is not an activation.
+ * Retain bits are copied unchanged.  Rows are addressed with byte strides.
+ */
+static int is_pred(const orc_problem *pb, int32_t u, int32_t v)
+{
+    for (int32_t e = pb->pred_off[v]; e < pb->pred_off[v + 1]; ++e)
+        if (pb->pred_idx[e] == u) return 1;
+    return 0;
+}
+
+int orc_mutate(const orc_problem *pb,
+               const uint8_t *place, int64_t place_stride,
+               const uint16_t *order, int64_t order_stride,
+               const uint32_t *fuse, const uint32_t *prefetch, const uint32_t *retain, int64_t bits_stride,
+               int64_t n_parents,
+               uint8_t *c_place, int64_t c_place_stride,
+               uint16_t *c_order, int64_t c_order_stride,
+               uint32_t *c_fuse, uint32_t *c_prefetch, uint32_t *c_retain, int64_t c_bits_stride,
+               int64_t n_children, uint64_t seed, int64_t round, int32_t n_ops)
+{
+    const int32_t N = pb->N, D = pb->D, words = (N + 31) / 32;
+    for (int64_t c = 0; c < n_children; ++c) {
+        const int64_t p = c % n_parents;
+        const uint8_t *pp = place + p * place_stride;
+        const uint16_t *po = (const uint16_t *)((const uint8_t *)order + p * order_stride);
+        const uint32_t *pf = (const uint32_t *)((const uint8_t *)fuse + p * bits_stride);
+        const uint32_t *pr = (const uint32_t *)((const uint8_t *)prefetch + p * bits_stride);
+        uint8_t *cp = c_place + c * c_place_stride;
+        uint16_t *co = (uint16_t *)((uint8_t *)c_order + c * c_order_stride);
+        uint32_t *cf = (uint32_t *)((uint8_t *)c_fuse + c * c_bits_stride);
+        uint32_t *cr = (uint32_t *)((uint8_t *)c_prefetch + c * c_bits_stride);
+        memcpy(cp, pp, (size_t)N);
+        memcpy(co, po, 2 * (size_t)N);
+        memcpy(cf, pf, 4 * (size_t)words);
+        memcpy(cr, pr, 4 * (size_t)words);
+        if (retain)
+            memcpy((uint8_t *)c_retain + c * c_bits_stride, (const uint8_t *)retain + p * bits_stride,
+                   4 * (size_t)words);
+        for (int32_t s = 0; s < n_ops; ++s) {
+            const uint64_t h = orc_splitmix64(orc_splitmix64(orc_splitmix64(seed ^ (uint64_t)round) ^ (uint64_t)c) ^
+                                              (uint64_t)s);
+            const uint32_t x = (uint32_t)(h >> 8);
+            const uint32_t y = (uint32_t)(h >> 40);
+            const int op = (int)(h & 3u);
+            if (op == 3) {
+                if (N < 2) continue;
+                const int32_t i = (int32_t)(x % (uint32_t)(N - 1));
+                const int32_t u = co[i], v = co[i + 1];
+                if (v < N && !(u < N && is_pred(pb, u, v))) { co[i] = (uint16_t)v; co[i + 1] = (uint16_t)u; }
+                continue;
+            }
+            const int32_t n = (int32_t)(x % (uint32_t)N);
+            if (op == 0) {
+                int32_t f = 0;
+                for (int32_t d = 0; d < D; ++d) f += pb->peak[(int64_t)n * D + d] <= pb->cap[d];
+                if (f == 0) continue;
+                int32_t r = (int32_t)(y % (uint32_t)f);
+                for (int32_t d = 0; d < D; ++d)
+                    if (pb->peak[(int64_t)n * D + d] <= pb->cap[d] && r-- == 0) { cp[n] = (uint8_t)d; break; }
+            } else if (op == 1) {
+                cf[n >> 5] ^= 1u << (n & 31);
+            } else {
+                cr[n >> 5] ^= 1u << (n & 31);
+            }
+        }
+    }
+    return 0;
+}

@@ -50,10 +50,13 @@ MUTANTS = {
     "status_place_ge": ("if (place[n] >= D) st |= 1u;", "if (place[n] > D) st |= 1u;"),
     "release_ignores_preds": ("rel = imax64(rel, c[pb->pred_idx[e]]);", "rel = imax64(rel, 0);"),
     "chain_reuses_start": ("t += L[(int64_t)n * D + d];", "t = start + L[(int64_t)n * D + d];"),
+    "swap_crosses_edges": ("if (v < N && !(u < N && is_pred(pb, u, v)))", "if (v < N)"),
+    "move_ignores_capacity": ("if (pb->peak[(int64_t)n * D + d] <= pb->cap[d] && r-- == 0)", "if (r-- == 0)"),
+    "child_of_wrong_parent": ("const int64_t p = c % n_parents;", "const int64_t p = (c / 2) % n_parents;"),
 }
 
 PIN_FILES = ["tests/test_oracle_golden.py", "tests/test_oracle_properties.py",
-             "tests/test_oracle_stochastic.py"]
+             "tests/test_oracle_stochastic.py", "tests/test_oracle_search.py"]
 
 
 def _run_mutant(name, tmp):
