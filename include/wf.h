@@ -14,6 +14,9 @@
  *   wf_eval_plans           play every plan forward (Eq. 2-11) -> metrics
  *   wf_topk                 the k best plans by the ranking key
  *   wf_eval_plans_static    wf_eval_plans without a context or any allocation
+ *   wf_mutate_plans         children of plans with a few point changes each
+ *   wf_merge_elite          keep the k best of an elite and its children
+ *   wf_local_search         rounds of mutate -> evaluate -> merge
  *   wf_ctx_destroy, wf_strerror
  *
  * Conventions.
@@ -207,6 +210,49 @@ int wf_topk(wf_ctx *ctx, const wf_eval_out *res, int64_t P, int32_t k,
  */
 int wf_eval_plans_static(const wf_problem *prob, const wf_plans *plans, const wf_eval_out *out,
                          void *stream);
+
+/*
+ * Local search around the best plans.  The paper's scheduler re-ranks its
+ * uncommitted decisions whenever arrivals, completions or model transitions
+ * change the picture (Section 3.5); these calls search the neighbourhood of
+ * the k best evaluated plans (the elite) for better ones.  All plan and
+ * result pointers are DEVICE pointers owned by the caller; parents and
+ * children are separate buffers that must not overlap, and either both or
+ * neither carry retain rows.  Asynchronous on `stream`; no allocation.
+ *
+ * wf_mutate_plans: children->P children.  Child c copies parent
+ * c mod parents->P and then takes n_ops (0..4096) changes in turn; change s
+ * is decoded from h = mix(mix(mix(seed ^ round) ^ c) ^ s) (mix = SplitMix64
+ * output), x = bits 8..39 of h, y = bits 40..63:
+ *   h mod 4 = 0  place[n] for n = x mod N becomes the (y mod f)-th, in
+ *               ascending order, of the f devices whose capacity holds
+ *               peak[n][d] (Eq. 8);
+ *             1  flip fuse bit n = x mod N (Eq. 3);
+ *             2  flip prefetch bit n = x mod N (Eq. 5);
+ *             3  swap dispatch positions i = x mod (N - 1) and i + 1 unless
+ *               the node at i is a graph predecessor of the node at i + 1
+ *               (Eq. 10); no change when N = 1 or order[i + 1] >= N.
+ * Retain rows are copied.  Children of valid plans are valid.  Returns
+ * WF_EINVAL for bad sizes, strides, alignment or n_ops.
+ *
+ * wf_merge_elite: elite->P = k (1..1024) evaluated plans and
+ * children->P evaluated children, k + children->P <= max_P.  The union is
+ * ranked by the wf_topk key with the elite at indices 0..k-1 and child c at
+ * k + c (so ties keep elite plans); the k best stay.  An elite slot whose
+ * plan stays is untouched; the slots whose plans left, in ascending order,
+ * receive the entering children in key order (rows and results).
+ *
+ * wf_local_search: `rounds` times: wf_mutate_plans(elite -> children, round
+ * = round0 + r), wf_eval_plans(children), wf_merge_elite.  The elite's
+ * results must be those of its plans on entry.
+ */
+int wf_mutate_plans(wf_ctx *ctx, const wf_plans *parents, const wf_plans *children, uint64_t seed,
+                    int64_t round, int32_t n_ops, void *stream);
+int wf_merge_elite(wf_ctx *ctx, const wf_plans *elite, const wf_eval_out *elite_res,
+                   const wf_plans *children, const wf_eval_out *child_res, void *stream);
+int wf_local_search(wf_ctx *ctx, const wf_plans *elite, const wf_eval_out *elite_res,
+                    const wf_plans *children, const wf_eval_out *child_res, uint64_t seed,
+                    int64_t round0, int32_t rounds, int32_t n_ops, void *stream);
 
 /*
  * Synchronize `stream` and report device-side failures of earlier calls on

@@ -321,6 +321,8 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
         c->topk_scratch_bytes = wf_topk_scratch_bytes(max_P);
         rc = wf_cuda_check(cudaMalloc(&c->topk_scratch, c->topk_scratch_bytes), "cudaMalloc(topk scratch)");
     }
+    if (!rc) rc = wf_cuda_check(cudaMalloc(&c->search_scratch, wf_search_scratch_bytes(max_P)),
+                                "cudaMalloc(search scratch)");
     if (!rc) rc = wf_cuda_check(cudaMallocHost(&c->h_ovf, sizeof(int32_t)), "cudaMallocHost(overflow count)");
     if (!rc) rc = wf_cuda_check(cudaEventCreateWithFlags(&c->ovf_event, cudaEventDisableTiming), "cudaEventCreate");
     if (!rc) rc = wf_cuda_check(cudaEventCreateWithFlags(&c->sweep_done, cudaEventDisableTiming), "cudaEventCreate");
@@ -339,6 +341,7 @@ extern "C" void wf_ctx_destroy(wf_ctx *c)
     if (c->tables) cudaFree(c->tables);
     if (c->eval_scratch) cudaFree(c->eval_scratch);
     if (c->topk_scratch) cudaFree(c->topk_scratch);
+    if (c->search_scratch) cudaFree(c->search_scratch);
     if (c->side) cudaStreamSynchronize(c->side);
     if (c->side) cudaStreamDestroy(c->side);
     if (c->ovf_event) cudaEventDestroy(c->ovf_event);
@@ -363,23 +366,42 @@ extern "C" int wf_forecast_readiness(wf_ctx *c, int64_t *rel, int64_t *comp, voi
 
 static bool aligned16(const void *p) { return ((uintptr_t)p & 15u) == 0; }
 
+int wf_check_plans(const wf_ctx *c, const wf_plans *pl, const char *what)
+{
+    REQUIRE(pl, "%s: NULL plans", what);
+    REQUIRE(pl->P >= 1 && pl->P <= c->max_P, "%s: P=%lld outside 1..max_P=%lld", what,
+            (long long)pl->P, (long long)c->max_P);
+    REQUIRE(pl->place && pl->order && pl->fuse && pl->prefetch, "%s: NULL plan array", what);
+    const int64_t N = c->dp.N;
+    const int64_t words = (N + 31) / 32;
+    REQUIRE(pl->place_stride >= N && pl->place_stride % 16 == 0, "%s: place_stride", what);
+    REQUIRE(pl->order_stride >= 2 * N && pl->order_stride % 16 == 0, "%s: order_stride", what);
+    REQUIRE(pl->bits_stride >= 4 * words && pl->bits_stride % 16 == 0, "%s: bits_stride", what);
+    REQUIRE(pl->plan_base >= 0, "%s: plan_base < 0", what);
+    REQUIRE(aligned16(pl->place) && aligned16(pl->order) && aligned16(pl->fuse) &&
+                aligned16(pl->prefetch) && (pl->retain == nullptr || aligned16(pl->retain)),
+            "%s: plan arrays must be 16-byte aligned", what);
+    return WF_OK;
+}
+
+int wf_check_out(const wf_eval_out *out, const char *what)
+{
+    REQUIRE(out, "%s: NULL results", what);
+    REQUIRE(out->makespan_us && out->p95_us && out->gpu_us && out->status, "%s: NULL result array", what);
+    return WF_OK;
+}
+
+int wf_select_device(const wf_ctx *c)
+{
+    return wf_cuda_check(cudaSetDevice(c->device), "cudaSetDevice");
+}
+
 extern "C" int wf_eval_plans(wf_ctx *c, const wf_plans *pl, const wf_eval_out *out, void *stream)
 {
     REQUIRE(c && pl && out, "NULL argument");
-    REQUIRE(pl->P >= 1 && pl->P <= c->max_P, "P=%lld outside 1..max_P=%lld",
-            (long long)pl->P, (long long)c->max_P);
-    REQUIRE(pl->place && pl->order && pl->fuse && pl->prefetch, "NULL plan array");
-    REQUIRE(out->makespan_us && out->p95_us && out->gpu_us && out->status, "NULL output array");
-    const int64_t N = c->dp.N;
-    const int64_t words = (N + 31) / 32;
-    REQUIRE(pl->place_stride >= N && pl->place_stride % 16 == 0, "place_stride");
-    REQUIRE(pl->order_stride >= 2 * N && pl->order_stride % 16 == 0, "order_stride");
-    REQUIRE(pl->bits_stride >= 4 * words && pl->bits_stride % 16 == 0, "bits_stride");
-    REQUIRE(pl->plan_base >= 0, "plan_base < 0");
-    REQUIRE(aligned16(pl->place) && aligned16(pl->order) && aligned16(pl->fuse) &&
-                aligned16(pl->prefetch) && (pl->retain == nullptr || aligned16(pl->retain)),
-            "plan arrays must be 16-byte aligned");
-    int rc = select_device(c);
+    int rc = wf_check_plans(c, pl, "plans");
+    if (!rc) rc = wf_check_out(out, "results");
+    if (!rc) rc = select_device(c);
     if (rc) return rc;
     return wf_launch_eval(c, pl, out, (cudaStream_t)stream);
 }

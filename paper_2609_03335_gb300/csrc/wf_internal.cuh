@@ -79,6 +79,7 @@ struct wf_ctx {
     bool prefer_wide;
     bool wide_pending;
     int64_t wide_P;
+    void *search_scratch;       // local search: the union's results [max_P], top-k ids, slot pairs
     int32_t *h_ovf;             // pinned host copy of ovf_count[0]
     cudaEvent_t sweep_done;     // recorded on the caller's stream after the sweeps
     cudaEvent_t ovf_event;      // recorded on side after the read-back
@@ -91,9 +92,12 @@ int32_t wf_assign_slots(int32_t N, int32_t W, const int32_t *pred_off, const int
                         const int32_t *session, const int32_t *fprev, const int32_t *fnext,
                         int32_t *rslot, std::vector<int32_t> &wl_off, std::vector<uint16_t> &wl);
 
-// Error plumbing (wf_ctx.cu).
+// Error plumbing and argument checks (wf_ctx.cu).
 int wf_set_error(int code, const char *fmt, ...);
 int wf_cuda_check(cudaError_t e, const char *what);
+int wf_check_plans(const wf_ctx *c, const wf_plans *pl, const char *what);
+int wf_check_out(const wf_eval_out *out, const char *what);
+int wf_select_device(const wf_ctx *c);
 
 // Launchers (one per translation unit).
 int wf_launch_forecast(wf_ctx *ctx, int64_t *rel, int64_t *comp, cudaStream_t st);
@@ -103,6 +107,7 @@ int wf_launch_topk(wf_ctx *ctx, const wf_eval_out *res, int64_t P, int32_t k, in
 size_t wf_eval_row_bytes(const wf_dev_problem &dp);
 size_t wf_eval_scratch_bytes(const wf_dev_problem &dp, int64_t max_P, int64_t *units);
 size_t wf_topk_scratch_bytes(int64_t max_P);
+size_t wf_search_scratch_bytes(int64_t max_P);
 // The shared-memory sweeps that apply to a problem: u32 times with 16 plans
 // per CTA, and u64 times with plans64 plans per CTA (0 bytes = not usable).
 struct wf_sweep_cfg {

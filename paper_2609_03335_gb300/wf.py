@@ -23,7 +23,7 @@ INT64_MAX = np.iinfo(np.int64).max
 # Every entry point declared in include/wf.h.
 EXPORTS = ("wf_problem_check", "wf_ctx_create", "wf_forecast_readiness", "wf_eval_plans",
            "wf_topk", "wf_ctx_status", "wf_ctx_destroy", "wf_strerror", "wf_last_error",
-           "wf_eval_plans_static")
+           "wf_eval_plans_static", "wf_mutate_plans", "wf_merge_elite", "wf_local_search")
 
 
 class WfError(RuntimeError):
@@ -76,6 +76,9 @@ def load_library():
         "wf_forecast_readiness": ([p, p, p, p], ctypes.c_int),
         "wf_eval_plans": ([p, p, p, p], ctypes.c_int),
         "wf_topk": ([p, p, i64, i32, p, p, p], ctypes.c_int),
+        "wf_mutate_plans": ([p, p, p, ctypes.c_uint64, i64, i32, p], ctypes.c_int),
+        "wf_merge_elite": ([p, p, p, p, p, p], ctypes.c_int),
+        "wf_local_search": ([p, p, p, p, p, ctypes.c_uint64, i64, i32, i32, p], ctypes.c_int),
         "wf_ctx_status": ([p, p], ctypes.c_int),
         "wf_ctx_destroy": ([p], None),
         "wf_strerror": ([ctypes.c_int], ctypes.c_char_p),
@@ -207,6 +210,26 @@ class DevicePlans:
         self.plan_base = int(plan_base)
 
     @staticmethod
+    def empty(P: int, N: int, with_retain: bool = False, device="cuda", plan_base: int = 0):
+        """Uninitialised rows padded to 16 bytes."""
+        import torch
+        pad = lambda b: (b + 15) // 16 * 16
+        words = pad(4 * ((N + 31) // 32)) // 4
+        mk = lambda cols, dt: torch.empty((P, cols), dtype=dt, device=device)
+        return DevicePlans(mk(pad(N), torch.uint8), mk(pad(2 * N) // 2, torch.int16), mk(words, torch.int32),
+                           mk(words, torch.int32), mk(words, torch.int32) if with_retain else None,
+                           plan_base=plan_base)
+
+    def numpy(self, N: int):
+        """Host copies of rows 0..P-1 without padding: place, order, fuse, prefetch, retain."""
+        words = (N + 31) // 32
+        out = [self.place[:, :N].cpu().numpy(), self.order[:, :N].cpu().numpy().view(np.uint16),
+               self.fuse[:, :words].cpu().numpy().view(np.uint32),
+               self.prefetch[:, :words].cpu().numpy().view(np.uint32)]
+        out.append(None if self.retain is None else self.retain[:, :words].cpu().numpy().view(np.uint32))
+        return out
+
+    @staticmethod
     def from_host(plans, device="cuda", non_blocking=False):
         import torch
 
@@ -265,6 +288,28 @@ def wf_topk(ctx: Ctx, res: Results, P: int, k: int, ids, keys=None, stream=None)
     _check(load_library().wf_topk(ctx.ptr, ctypes.byref(oc), int(P), int(k), ids.data_ptr(),
                                   None if keys is None else keys.data_ptr(), _stream_handle(stream)),
            "wf_topk")
+
+
+def wf_mutate_plans(ctx: Ctx, parents: DevicePlans, children: DevicePlans, seed: int, round_: int,
+                    n_ops: int, stream=None):
+    pa, ch = parents.c(), children.c()
+    _check(load_library().wf_mutate_plans(ctx.ptr, ctypes.byref(pa), ctypes.byref(ch), seed & ((1 << 64) - 1),
+                                          int(round_), int(n_ops), _stream_handle(stream)), "wf_mutate_plans")
+
+
+def wf_merge_elite(ctx: Ctx, elite: DevicePlans, elite_res: Results, children: DevicePlans,
+                   child_res: Results, stream=None):
+    el, er, ch, cr = elite.c(), elite_res.c(), children.c(), child_res.c()
+    _check(load_library().wf_merge_elite(ctx.ptr, ctypes.byref(el), ctypes.byref(er), ctypes.byref(ch),
+                                         ctypes.byref(cr), _stream_handle(stream)), "wf_merge_elite")
+
+
+def wf_local_search(ctx: Ctx, elite: DevicePlans, elite_res: Results, children: DevicePlans,
+                    child_res: Results, seed: int, round0: int, rounds: int, n_ops: int, stream=None):
+    el, er, ch, cr = elite.c(), elite_res.c(), children.c(), child_res.c()
+    _check(load_library().wf_local_search(ctx.ptr, ctypes.byref(el), ctypes.byref(er), ctypes.byref(ch),
+                                          ctypes.byref(cr), seed & ((1 << 64) - 1), int(round0), int(rounds),
+                                          int(n_ops), _stream_handle(stream)), "wf_local_search")
 
 
 def evaluate(ctx: Ctx, plans, k: int, stream=None):
