@@ -185,6 +185,41 @@ def run_reference(args, rank, world):
     print(json.dumps(line), flush=True)
 
 
+def local_search_timing(wf, ctx, dp, prob, P, stream, flush, peak_gbs, k=32, rounds=3):
+    """Local search around the batch's first k plans: P - k children per
+    round (mutate -> evaluate -> merge; the context holds P plans).  The
+    mutation kernel alone is timed too; it writes the child rows and reads
+    the k parent rows (from L2)."""
+    import torch
+    N = prob.N
+    P = P - k
+    elite = wf.DevicePlans(dp.place[:k], dp.order[:k], dp.fuse[:k], dp.prefetch[:k], None, plan_base=0)
+    er = wf.Results(k, dp.place.device)
+    kids = wf.DevicePlans.empty(P, N, device=dp.place.device, plan_base=k)
+    kr = wf.Results(P, dp.place.device)
+    with torch.cuda.stream(stream):
+        wf.wf_eval_plans(ctx, elite, er, stream)
+        wf.wf_local_search(ctx, elite, er, kids, kr, seed=7, round0=0, rounds=1, n_ops=3, stream=stream)
+        e = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        flush.zero_()
+        e[0].record(stream)
+        wf.wf_mutate_plans(ctx, elite, kids, seed=7, round_=1, n_ops=3, stream=stream)
+        e[1].record(stream)
+        flush.zero_()
+        e[2].record(stream)
+        wf.wf_local_search(ctx, elite, er, kids, kr, seed=7, round0=2, rounds=rounds, n_ops=3, stream=stream)
+        e[3].record(stream)
+    torch.cuda.synchronize()
+    mut_ms = e[0].elapsed_time(e[1])
+    ls_ms = e[2].elapsed_time(e[3])
+    row = N + 2 * N + 2 * 4 * ((N + 31) // 32)
+    gbs = 2 * row * P / (mut_ms * 1e-3) / 1e9
+    return {"k": k, "children_per_round": P, "rounds": rounds, "n_ops": 3,
+            "ms_per_round": ls_ms / rounds, "children_per_s": P * rounds / (ls_ms * 1e-3),
+            "mutate_kernel": {"ms": mut_ms, "bytes_per_child": 2 * row, "achieved_gbs": gbs,
+                              "frac": gbs / peak_gbs if peak_gbs else None, "bound": "hbm"}}
+
+
 def run_gpu(args, rank, world, local):
     import torch
 
@@ -286,6 +321,7 @@ def run_gpu(args, rank, world, local):
         e1.record(stream)
     torch.cuda.synchronize()
     barrier(world)
+    search = local_search_timing(wf, ctx, dp, prob, P, stream, flush, peak_gbs=read_peaks().get("hbm_gbs"))
     clk = clocks.stop()
     e2e_ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, world)
     # the host reads the top-k it copied back
@@ -296,9 +332,10 @@ def run_gpu(args, rank, world, local):
     peaks = read_peaks()
     peak = peaks.get("hbm_gbs")
     traffic, _ = read_traffic(WORKLOAD)
-    # forecast, status, sweep, overflow pass, top-k passes (the overflow-count
-    # reset is a memset, not a kernel)
-    launches = args.steps * (4 + topk_launches(P, k))
+    # forecast, status, 32-bit sweep, 64-bit sweep over its hand-offs, int64
+    # pass over what is left, top-k passes (the count reset is a memset and
+    # the count read-back a copy, not kernels)
+    launches = args.steps * (5 + topk_launches(P, k))
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -334,6 +371,7 @@ def run_gpu(args, rank, world, local):
             "cpu_baseline": cpu,
             "clocks": clk,
             "gpu_launches": launches,
+            "local_search": search,
         }
         print(json.dumps(line), flush=True)
     ctx.close()
