@@ -201,22 +201,24 @@ def local_search_timing(wf, ctx, dp, prob, P, stream, flush, peak_gbs, k=32, rou
         wf.wf_eval_plans(ctx, elite, er, stream)
         wf.wf_local_search(ctx, elite, er, kids, kr, seed=7, round0=0, rounds=1, n_ops=3, stream=stream)
         e = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
-        flush.zero_()
-        e[0].record(stream)
-        wf.wf_mutate_plans(ctx, elite, kids, seed=7, round_=1, n_ops=3, stream=stream)
-        e[1].record(stream)
+        mut = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(5)]
+        for r, (a, b) in enumerate(mut):
+            flush.zero_()
+            a.record(stream)
+            wf.wf_mutate_plans(ctx, elite, kids, seed=7, round_=1 + r, n_ops=3, stream=stream)
+            b.record(stream)
         flush.zero_()
         e[2].record(stream)
         wf.wf_local_search(ctx, elite, er, kids, kr, seed=7, round0=2, rounds=rounds, n_ops=3, stream=stream)
         e[3].record(stream)
     torch.cuda.synchronize()
-    mut_ms = e[0].elapsed_time(e[1])
+    mut_ms = float(np.median([a.elapsed_time(b) for a, b in mut]))
     ls_ms = e[2].elapsed_time(e[3])
     row = N + 2 * N + 2 * 4 * ((N + 31) // 32)
     gbs = 2 * row * P / (mut_ms * 1e-3) / 1e9
     return {"k": k, "children_per_round": P, "rounds": rounds, "n_ops": 3,
             "ms_per_round": ls_ms / rounds, "children_per_s": P * rounds / (ls_ms * 1e-3),
-            "mutate_kernel": {"ms": mut_ms, "bytes_per_child": 2 * row, "achieved_gbs": gbs,
+            "mutate_kernel": {"ms": mut_ms, "timing": "median of 5 launches, L2 flushed before each", "bytes_per_child": 2 * row, "achieved_gbs": gbs,
                               "frac": gbs / peak_gbs if peak_gbs else None, "bound": "hbm"}}
 
 
@@ -365,7 +367,8 @@ def run_gpu(args, rank, world, local):
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak if peak else None,
                          "traffic": traffic,
-                         "kernel": "wf_eval_plans = status_kernel + pc_kernel<uint32_t> + eval_list_kernel",
+                         "kernel": "wf_eval_plans = status_kernel + pc_kernel (u32 times) + pc_kernel (u64 "
+                                   "times, hand-offs) + eval_list_kernel",
                          "algorithmic_bytes_per_plan": bpp, "kernel_ms": eval_ms_mean,
                          "peak_source": "MEASURED_PEAKS.json hbm_gbs (measured copy)" if peak else None},
             "cpu_baseline": cpu,
