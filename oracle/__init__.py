@@ -75,7 +75,9 @@ def _setup(lib):
     lib.orc_multiplier.restype = ctypes.c_int64
     lib.orc_mutate.argtypes = [p, p, i64, p, i64, p, p, p, i64, i64, p, i64, p, i64, p, p, p, i64, i64,
                                ctypes.c_uint64, i64, ctypes.c_int32]
-    for f in ("orc_fusible_next", "orc_forecast", "orc_status", "orc_eval_plan", "orc_eval_batch", "orc_mutate"):
+    lib.orc_construct.argtypes = [p, p, ctypes.c_uint64, ctypes.c_uint64, i64, p, p, p, p, p]
+    for f in ("orc_fusible_next", "orc_forecast", "orc_status", "orc_eval_plan", "orc_eval_batch", "orc_mutate",
+              "orc_construct"):
         getattr(lib, f).restype = ctypes.c_int
     return lib
 
@@ -336,3 +338,22 @@ def local_search(prob, elite, elite_metrics, n_children: int, seed: int, round0:
                 if getattr(cur, a) is not None:
                     getattr(cur, a)[s] = getattr(ch, a)[c]
     return cur, met
+
+
+def construct(prob, P: int, seed: int, jitter: int, plan_base: int = 0):
+    """P plans from the list-scheduling constructor (plan index plan_base + p
+    seeds the jitter).  Returns (PlanRows, end times int64 [P])."""
+    op = OracleProblem(prob)
+    N = op.N
+    out = PlanRows(P, N, False, plan_base)
+    ends = np.zeros(P, np.int64)
+    end = ctypes.c_int64(0)
+    for p in range(P):
+        rc = op.lib.orc_construct(ctypes.byref(op.c), op.fnext.ctypes.data, seed & ((1 << 64) - 1),
+                                  (plan_base + p) & ((1 << 64) - 1), int(jitter),
+                                  out.place[p].ctypes.data, out.order[p].ctypes.data,
+                                  out.fuse[p].ctypes.data, out.prefetch[p].ctypes.data, ctypes.byref(end))
+        if rc != 0:
+            raise RuntimeError(f"oracle construct failed ({rc})")
+        ends[p] = end.value
+    return out, ends

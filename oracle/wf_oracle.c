@@ -566,3 +566,177 @@ int orc_mutate(const orc_problem *pb,
     }
     return 0;
 }
+
+/*
+ * Plan construction (Algorithm 1 read for a whole window, one plan per
+ * call).  The constructor is a list scheduler that plays each decision
+ * forward with the evaluation rules above, so the finish times it sees are
+ * the ones the evaluator will report for its plan:
+ *
+ *   RankReady: a unit is ready once every graph predecessor is dispatched;
+ *     its rank is its release (Eq. 2: session arrival and predecessor
+ *     finishes) plus a jitter drawn per (plan, node); the ready unit with
+ *     the smallest (rank, node id) goes next -- the one that has waited
+ *     longest (aging).
+ *   BestFeasibleBinding: among the devices whose capacity holds the node
+ *     (Eq. 8), the one with the smallest predicted finish of the node
+ *     (a resident model costs no load; a missing one is loaded on the
+ *     device, prefetched when the device would otherwise idle before the
+ *     release) plus a jitter drawn per (plan, node, device); ties go to
+ *     the lower device.
+ *   Units: the node's fusible chain (Eq. 3) follows it on the same device
+ *     while each next member fits there (fuse bit 1), dispatched at once.
+ *   PlanPrefetch: the head's prefetch bit is set when its model is not
+ *     resident on the device and the device is free before the release.
+ *   Retain: every model stays resident (no retain row).
+ *
+ * Jitter: h = mix(mix(seed ^ plan) ^ node); rank jitter h mod (J + 1),
+ * device jitter mix(h ^ (d + 1)) mod (J + 1); J = 0 gives the plain greedy.
+ * Outputs the plan rows (fuse / prefetch rows of ceil(N/32) words) and the
+ * largest finish.  Returns 0, or -1 when memory runs out.
+ */
+int orc_construct(const orc_problem *pb, const int32_t *fnext, uint64_t seed, uint64_t plan, int64_t jitter,
+                  uint8_t *place, uint16_t *order, uint32_t *fuse, uint32_t *prefetch, int64_t *end_out)
+{
+    const int32_t N = pb->N, D = pb->D, M = pb->M;
+    const int32_t E = pb->pred_off[N];
+    const int32_t words = (N + 31) / 32;
+    int64_t *c = (int64_t *)malloc(sizeof(int64_t) * (size_t)N);
+    int64_t *rel = (int64_t *)malloc(sizeof(int64_t) * (size_t)N);
+    int64_t *rank = (int64_t *)malloc(sizeof(int64_t) * (size_t)N);
+    int32_t *pending = (int32_t *)malloc(sizeof(int32_t) * (size_t)N);
+    int32_t *ready = (int32_t *)malloc(sizeof(int32_t) * (size_t)N);
+    int32_t *succ_off = (int32_t *)calloc((size_t)N + 1, sizeof(int32_t));
+    int32_t *succ = (int32_t *)malloc(sizeof(int32_t) * (size_t)(E > 0 ? E : 1));
+    int32_t *chain = (int32_t *)malloc(sizeof(int32_t) * (size_t)N);
+    int64_t *t_free = (int64_t *)calloc((size_t)D, sizeof(int64_t));
+    int64_t *used = (int64_t *)calloc((size_t)D, sizeof(int64_t));
+    int64_t *stamp = (int64_t *)calloc((size_t)D * (size_t)M, sizeof(int64_t));
+    int rc = 0;
+    if (!c || !rel || !rank || !pending || !ready || !succ_off || !succ || !chain || !t_free || !used || !stamp) {
+        rc = -1;
+        goto out;
+    }
+    /* Successor lists (the transpose of the predecessor CSR). */
+    for (int32_t e = 0; e < E; ++e) succ_off[pb->pred_idx[e] + 1] += 1;
+    for (int32_t v = 0; v < N; ++v) succ_off[v + 1] += succ_off[v];
+    {
+        int32_t *fill = pending;  /* scratch, reset below */
+        for (int32_t v = 0; v < N; ++v) fill[v] = succ_off[v];
+        for (int32_t v = 0; v < N; ++v)
+            for (int32_t e = pb->pred_off[v]; e < pb->pred_off[v + 1]; ++e) succ[fill[pb->pred_idx[e]]++] = v;
+    }
+    memset(fuse, 0, sizeof(uint32_t) * (size_t)words);
+    memset(prefetch, 0, sizeof(uint32_t) * (size_t)words);
+
+    int32_t nready = 0, pos = 0;
+    int64_t end = 0, seq = 0;
+    for (int32_t v = 0; v < N; ++v) {
+        pending[v] = pb->pred_off[v + 1] - pb->pred_off[v];
+        if (pending[v] == 0) {
+            const uint64_t h = orc_splitmix64(orc_splitmix64(seed ^ plan) ^ (uint64_t)v);
+            rel[v] = pb->arrival[pb->session[v]];
+            rank[v] = rel[v] + (jitter > 0 ? (int64_t)(h % (uint64_t)(jitter + 1)) : 0);
+            ready[nready++] = v;
+        }
+    }
+    while (nready > 0) {
+        /* RankReady: smallest (rank, node id). */
+        int32_t j = 0;
+        for (int32_t k = 1; k < nready; ++k) {
+            const int32_t a = ready[k], b = ready[j];
+            if (rank[a] < rank[b] || (rank[a] == rank[b] && a < b)) j = k;
+        }
+        const int32_t u = ready[j];
+        ready[j] = ready[--nready];
+        const int32_t m = pb->model[u];
+        const int64_t arr = pb->arrival[pb->session[u]];
+        const uint64_t hu = orc_splitmix64(orc_splitmix64(seed ^ plan) ^ (uint64_t)u);
+
+        /* BestFeasibleBinding: smallest predicted finish (+ jitter). */
+        int32_t d = -1;
+        int64_t best = 0;
+        for (int32_t dd = 0; dd < D; ++dd) {
+            if (pb->peak[(int64_t)u * D + dd] > pb->cap[dd]) continue;
+            int64_t start;
+            if (stamp[(int64_t)dd * M + m] != 0) {
+                start = imax64(t_free[dd], rel[u]);
+            } else {
+                const int64_t ls = t_free[dd] < rel[u] ? imax64(t_free[dd], arr) : imax64(t_free[dd], rel[u]);
+                start = imax64(ls + pb->load[(int64_t)m * D + dd], rel[u]);
+            }
+            const int64_t fin = start + pb->grant + pb->lat[(int64_t)u * D + dd];
+            const int64_t score =
+                fin + (jitter > 0 ? (int64_t)(orc_splitmix64(hu ^ (uint64_t)(dd + 1)) % (uint64_t)(jitter + 1)) : 0);
+            if (d < 0 || score < best) { d = dd; best = score; }
+        }
+        if (d < 0) { rc = -2; goto out; }  /* no device holds u: the problem is invalid */
+
+        /* The unit: u and the members of its fusible chain that fit on d. */
+        int32_t len = 0;
+        chain[len++] = u;
+        for (int32_t s = fnext[u]; s >= 0 && pb->peak[(int64_t)s * D + d] <= pb->cap[d]; s = fnext[s])
+            chain[len++] = s;
+        const int hit = stamp[(int64_t)d * M + m] != 0;
+        const int pf = !hit && t_free[d] < rel[u];
+        for (int32_t k = 0; k < len; ++k) {
+            const int32_t x = chain[k];
+            place[x] = (uint8_t)d;
+            order[pos++] = (uint16_t)x;
+            if (k > 0) fuse[x >> 5] |= 1u << (x & 31);
+        }
+        if (pf) prefetch[u >> 5] |= 1u << (u & 31);
+
+        /* Play the unit forward exactly as the evaluation does. */
+        int64_t kv_adm = 0;
+        for (int32_t k = 0; k < len; ++k)
+            kv_adm = imax64(kv_adm, (int64_t)pb->peak[(int64_t)chain[k] * D + d] - pb->weight[m]);
+        const int64_t admit = hit ? kv_adm : pb->weight[m] + kv_adm;
+        int64_t *lru = &stamp[(int64_t)d * M];
+        while (used[d] + admit > pb->cap[d]) {  /* Eq. 11, least recently used first */
+            int32_t victim = -1;
+            for (int32_t k = 0; k < M; ++k)
+                if (k != m && lru[k] != 0 && (victim < 0 || lru[k] < lru[victim])) victim = k;
+            if (victim < 0) { rc = -3; goto out; }
+            used[d] -= pb->weight[victim];
+            lru[victim] = 0;
+        }
+        int64_t start;
+        if (hit) {
+            start = imax64(t_free[d], rel[u]);
+        } else {
+            const int64_t ls = pf ? imax64(t_free[d], arr) : imax64(t_free[d], rel[u]);
+            start = imax64(ls + pb->load[(int64_t)m * D + d], rel[u]);
+            used[d] += pb->weight[m];
+        }
+        int64_t t = start + pb->grant;
+        for (int32_t k = 0; k < len; ++k) {
+            t += pb->lat[(int64_t)chain[k] * D + d];
+            c[chain[k]] = t;
+        }
+        t_free[d] = t;
+        lru[m] = ++seq;
+        end = imax64(end, t);
+
+        /* Successors of the unit's last member become ready when their
+         * last predecessor is dispatched (the other members' only
+         * successors are inside the unit). */
+        const int32_t tail = chain[len - 1];
+        for (int32_t e = succ_off[tail]; e < succ_off[tail + 1]; ++e) {
+            const int32_t y = succ[e];
+            if (--pending[y] > 0) continue;
+            int64_t r = pb->arrival[pb->session[y]];
+            for (int32_t f = pb->pred_off[y]; f < pb->pred_off[y + 1]; ++f) r = imax64(r, c[pb->pred_idx[f]]);
+            const uint64_t h = orc_splitmix64(orc_splitmix64(seed ^ plan) ^ (uint64_t)y);
+            rel[y] = r;
+            rank[y] = r + (jitter > 0 ? (int64_t)(h % (uint64_t)(jitter + 1)) : 0);
+            ready[nready++] = y;
+        }
+    }
+    if (pos != N) rc = -4;  /* unreachable for an acyclic window */
+    *end_out = end;
+out:
+    free(c); free(rel); free(rank); free(pending); free(ready); free(succ_off); free(succ); free(chain);
+    free(t_free); free(used); free(stamp);
+    return rc;
+}

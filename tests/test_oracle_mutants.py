@@ -53,10 +53,15 @@ MUTANTS = {
     "swap_crosses_edges": ("if (v < N && !(u < N && is_pred(pb, u, v)))", "if (v < N)"),
     "move_ignores_capacity": ("if (pb->peak[(int64_t)n * D + d] <= pb->cap[d] && r-- == 0)", "if (r-- == 0)"),
     "child_of_wrong_parent": ("const int64_t p = c % n_parents;", "const int64_t p = (c / 2) % n_parents;"),
+    "construct_rank_ignores_release": ("rank[y] = r + (jitter", "rank[y] = 0 + (jitter"),
+    "construct_binding_ignores_residency": ("if (stamp[(int64_t)dd * M + m] != 0) {", "if (0) {"),
+    "construct_prefetch_always": ("const int pf = !hit && t_free[d] < rel[u];", "const int pf = !hit;"),
+    "construct_no_fusion": ("s >= 0 && pb->peak[(int64_t)s * D + d] <= pb->cap[d]; s = fnext[s])",
+                            "s >= 0 && 0; s = fnext[s])"),
 }
 
 PIN_FILES = ["tests/test_oracle_golden.py", "tests/test_oracle_properties.py",
-             "tests/test_oracle_stochastic.py", "tests/test_oracle_search.py"]
+             "tests/test_oracle_stochastic.py", "tests/test_oracle_search.py", "tests/test_oracle_construct.py"]
 
 
 def _run_mutant(name, tmp):
