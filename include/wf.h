@@ -17,6 +17,7 @@
  *   wf_mutate_plans         children of plans with a few point changes each
  *   wf_merge_elite          keep the k best of an elite and its children
  *   wf_local_search         rounds of mutate -> evaluate -> merge
+ *   wf_construct_plans      plans built by a list scheduler (Algorithm 1)
  *   wf_ctx_destroy, wf_strerror
  *
  * Conventions.
@@ -253,6 +254,35 @@ int wf_merge_elite(wf_ctx *ctx, const wf_plans *elite, const wf_eval_out *elite_
 int wf_local_search(wf_ctx *ctx, const wf_plans *elite, const wf_eval_out *elite_res,
                     const wf_plans *children, const wf_eval_out *child_res, uint64_t seed,
                     int64_t round0, int32_t rounds, int32_t n_ops, void *stream);
+
+/*
+ * Plan construction: Algorithm 1 (rank the ready units, bind each to one
+ * feasible device, load / prefetch, Section 3.5) read as a list scheduler
+ * over the whole window, one plan per row of *out (DEVICE pointers, the
+ * layout of wf_plans; out->P plans).  Repeatedly:
+ *   - the ready node (every graph predecessor dispatched) with the smallest
+ *     (release + jitter, node id) goes next; release = max(session arrival,
+ *     predecessor finishes) (Eq. 2);
+ *   - its device is the one, among those whose capacity holds it (Eq. 8),
+ *     with the smallest predicted finish + jitter (ties: lower device): a
+ *     resident model starts at max(device free, release); a missing one is
+ *     loaded first, from max(device free, arrival) when the device is free
+ *     before the release (the prefetch bit is then set), else from
+ *     max(device free, release);
+ *   - its fusible chain (Eq. 3) follows it on that device while each next
+ *     member fits there (fuse bits 1), and the unit is played forward with
+ *     the rules of wf_eval_plans (reclamation, Eq. 11), so evaluating the
+ *     plan reproduces the constructor's timeline.
+ * Jitter of plan index g = out->plan_base + p: h = mix(mix(seed ^ g) ^ node),
+ * rank jitter h mod (jitter_us + 1), device jitter mix(h ^ (d + 1)) mod
+ * (jitter_us + 1); jitter_us = 0 makes every plan the plain greedy one.
+ * Retain rows, if given, are set to all ones.  WF_EINVAL when the window's
+ * horizon (latest arrival + every node's worst load + run + grant) plus
+ * jitter_us reaches 2^47 us.  The first call on a context allocates the
+ * constructor's state (about 20 N bytes per plan built at once, at most
+ * 128 plans per SM); later calls allocate nothing.  Asynchronous on stream.
+ */
+int wf_construct_plans(wf_ctx *ctx, const wf_plans *out, uint64_t seed, int64_t jitter_us, void *stream);
 
 /*
  * Synchronize `stream` and report device-side failures of earlier calls on

@@ -250,6 +250,27 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
         for (int32_t e = pb->pred_off[v]; e < pb->pred_off[v + 1]; ++e)
             edges[e] = (uint32_t)pb->pred_idx[e] | ((uint32_t)v << 16);
     size_t o_edges = img.add(edges.data(), sizeof(uint32_t) * E);
+    // Successor lists (the transpose of pred CSR) for the plan constructor,
+    // and a bound on any time a plan of the window can reach.
+    std::vector<int32_t> succ_off(N + 1, 0), succ_idx(E > 0 ? E : 1);
+    for (int32_t e = 0; e < E; ++e) succ_off[pb->pred_idx[e] + 1] += 1;
+    for (int32_t v = 0; v < N; ++v) succ_off[v + 1] += succ_off[v];
+    {
+        std::vector<int32_t> fill(succ_off.begin(), succ_off.end() - 1);
+        for (int32_t v = 0; v < N; ++v)
+            for (int32_t e = pb->pred_off[v]; e < pb->pred_off[v + 1]; ++e) succ_idx[fill[pb->pred_idx[e]]++] = v;
+    }
+    size_t o_soff = img.add(succ_off.data(), sizeof(int32_t) * (N + 1));
+    size_t o_sidx = img.add(succ_idx.data(), sizeof(int32_t) * succ_idx.size());
+    int64_t horizon = 0;
+    for (int32_t w = 0; w < W; ++w) horizon = std::max(horizon, pb->arrival_us[w]);
+    for (int32_t n = 0; n < N; ++n) {
+        int64_t worst = 0;
+        for (int32_t d = 0; d < D; ++d)
+            worst = std::max(worst, (int64_t)pb->lat_us[(int64_t)n * D + d] +
+                                        pb->load_us[(int64_t)pb->model[n] * D + d]);
+        horizon += worst + pb->grant_us;
+    }
     size_t o_ovf = img.add(nullptr, sizeof(int32_t) * (2 * (size_t)max_P + 64));
 
     wf_ctx *c = (wf_ctx *)calloc(1, sizeof(wf_ctx));
@@ -303,6 +324,9 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
     dp.links = (const uint32_t *)(base + o_links);
     dp.fitmask = (const uint32_t *)(base + o_fit);
     dp.edges = (const uint32_t *)(base + o_edges);
+    dp.succ_off = (const int32_t *)(base + o_soff);
+    dp.succ_idx = (const int32_t *)(base + o_sidx);
+    dp.horizon = horizon;
     int64_t amax = 0;
     for (int32_t w = 0; w < W; ++w) amax = std::max(amax, pb->arrival_us[w]);
     dp.max_arrival = amax;
@@ -342,6 +366,7 @@ extern "C" void wf_ctx_destroy(wf_ctx *c)
     if (c->eval_scratch) cudaFree(c->eval_scratch);
     if (c->topk_scratch) cudaFree(c->topk_scratch);
     if (c->search_scratch) cudaFree(c->search_scratch);
+    if (c->construct_scratch) cudaFree(c->construct_scratch);
     if (c->side) cudaStreamSynchronize(c->side);
     if (c->side) cudaStreamDestroy(c->side);
     if (c->ovf_event) cudaEventDestroy(c->ovf_event);

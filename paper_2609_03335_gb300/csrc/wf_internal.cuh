@@ -47,6 +47,9 @@ struct wf_dev_problem {
     const uint32_t *links;      // [N] fusible predecessor | fusible successor << 16 (0xFFFF = none)
     const uint32_t *fitmask;    // [N rounded up to 4] bit d: peak[n][d] <= cap[d]
     const uint32_t *edges;      // [E] predecessor | successor << 16
+    const int32_t *succ_off;    // [N+1] successor lists (CSR)
+    const int32_t *succ_idx;    // [E]
+    int64_t horizon;            // no finish of any plan exceeds this (latest arrival + every node's worst load + run + grant)
     int64_t max_arrival;
 };
 
@@ -80,6 +83,8 @@ struct wf_ctx {
     bool wide_pending;
     int64_t wide_P;
     void *search_scratch;       // local search: the union's results [max_P], top-k ids, slot pairs
+    void *construct_scratch;    // plan constructor: per-thread state, allocated by its first call
+    int64_t construct_threads;
     int32_t *h_ovf;             // pinned host copy of ovf_count[0]
     cudaEvent_t sweep_done;     // recorded on the caller's stream after the sweeps
     cudaEvent_t ovf_event;      // recorded on side after the read-back

@@ -23,7 +23,8 @@ INT64_MAX = np.iinfo(np.int64).max
 # Every entry point declared in include/wf.h.
 EXPORTS = ("wf_problem_check", "wf_ctx_create", "wf_forecast_readiness", "wf_eval_plans",
            "wf_topk", "wf_ctx_status", "wf_ctx_destroy", "wf_strerror", "wf_last_error",
-           "wf_eval_plans_static", "wf_mutate_plans", "wf_merge_elite", "wf_local_search")
+           "wf_eval_plans_static", "wf_mutate_plans", "wf_merge_elite", "wf_local_search",
+           "wf_construct_plans")
 
 
 class WfError(RuntimeError):
@@ -79,6 +80,7 @@ def load_library():
         "wf_mutate_plans": ([p, p, p, ctypes.c_uint64, i64, i32, p], ctypes.c_int),
         "wf_merge_elite": ([p, p, p, p, p, p], ctypes.c_int),
         "wf_local_search": ([p, p, p, p, p, ctypes.c_uint64, i64, i32, i32, p], ctypes.c_int),
+        "wf_construct_plans": ([p, p, ctypes.c_uint64, i64, p], ctypes.c_int),
         "wf_ctx_status": ([p, p], ctypes.c_int),
         "wf_ctx_destroy": ([p], None),
         "wf_strerror": ([ctypes.c_int], ctypes.c_char_p),
@@ -310,6 +312,12 @@ def wf_local_search(ctx: Ctx, elite: DevicePlans, elite_res: Results, children: 
     _check(load_library().wf_local_search(ctx.ptr, ctypes.byref(el), ctypes.byref(er), ctypes.byref(ch),
                                           ctypes.byref(cr), seed & ((1 << 64) - 1), int(round0), int(rounds),
                                           int(n_ops), _stream_handle(stream)), "wf_local_search")
+
+
+def wf_construct_plans(ctx: Ctx, out: DevicePlans, seed: int, jitter_us: int, stream=None):
+    pl = out.c()
+    _check(load_library().wf_construct_plans(ctx.ptr, ctypes.byref(pl), seed & ((1 << 64) - 1), int(jitter_us),
+                                             _stream_handle(stream)), "wf_construct_plans")
 
 
 def evaluate(ctx: Ctx, plans, k: int, stream=None):
