@@ -222,6 +222,31 @@ def local_search_timing(wf, ctx, dp, prob, P, stream, flush, peak_gbs, k=32, rou
                               "frac": gbs / peak_gbs if peak_gbs else None, "bound": "hbm"}}
 
 
+def construct_timing(wf, ctx, prob, P, k, stream, flush, random_best, jitter=200000):
+    """The plan constructor over a batch of P plans (jittered list schedules),
+    timed on the device, then evaluated: its best makespan against the best
+    of the random batch."""
+    import torch
+    dev = torch.device("cuda", torch.cuda.current_device())
+    out = wf.DevicePlans.empty(P, prob.N, device=dev)
+    res = wf.Results(P, dev)
+    ids = torch.empty(k, dtype=torch.int32, device=dev)
+    keys = torch.empty((k, 3), dtype=torch.int64, device=dev)
+    e = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    with torch.cuda.stream(stream):
+        wf.wf_construct_plans(ctx, out, seed=11, jitter_us=jitter, stream=stream)  # first call allocates
+        flush.zero_()
+        e[0].record(stream)
+        wf.wf_construct_plans(ctx, out, seed=12, jitter_us=jitter, stream=stream)
+        e[1].record(stream)
+        wf.wf_eval_plans(ctx, out, res, stream)
+        wf.wf_topk(ctx, res, P, k, ids, keys, stream)
+    torch.cuda.synchronize()
+    ms = e[0].elapsed_time(e[1])
+    return {"plans": P, "jitter_us": jitter, "ms": ms, "plans_per_s": P / (ms * 1e-3),
+            "best_makespan_us": int(keys[0, 0].item()), "random_batch_best_makespan_us": random_best}
+
+
 def run_gpu(args, rank, world, local):
     import torch
 
@@ -324,6 +349,7 @@ def run_gpu(args, rank, world, local):
     torch.cuda.synchronize()
     barrier(world)
     search = local_search_timing(wf, ctx, dp, prob, P, stream, flush, peak_gbs=read_peaks().get("hbm_gbs"))
+    built = construct_timing(wf, ctx, prob, P, k, stream, flush, random_best=int(keys[0, 0].item()))
     clk = clocks.stop()
     e2e_ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, world)
     # the host reads the top-k it copied back
@@ -375,6 +401,7 @@ def run_gpu(args, rank, world, local):
             "clocks": clk,
             "gpu_launches": launches,
             "local_search": search,
+            "construct": built,
         }
         print(json.dumps(line), flush=True)
     ctx.close()
