@@ -78,6 +78,19 @@ def read_traffic(workload: str):
     return d["per_launch"][workload], d.get("kernel_hash")
 
 
+def read_instructions(workload: str):
+    """Warp instructions of one evaluation call from the same ncu summary (same
+    kernel-source condition as the traffic)."""
+    try:
+        with open(os.path.join(ROOT, "profiles", "eval_traffic.json")) as f:
+            d = json.load(f)
+    except OSError:
+        return None
+    if d.get("kernel_hash") != kernel_source_hash():
+        return None
+    return d.get("warp_instructions", {}).get(workload)
+
+
 class ClockSampler:
     """nvidia-smi clocks and throttle reasons sampled every 50 ms."""
 
@@ -247,6 +260,21 @@ def construct_timing(wf, ctx, prob, P, k, stream, flush, random_best, jitter=200
             "best_makespan_us": int(keys[0, 0].item()), "random_batch_best_makespan_us": random_best}
 
 
+def issue_roofline(eval_ms, clk, sms):
+    """The integer-issue roofline of the evaluation call: its warp
+    instructions (ncu, same kernel source) over its CUDA-event time, against
+    4 warp instructions per clock per SM at the median SM clock sampled
+    during the run."""
+    inst = read_instructions(WORKLOAD)
+    mhz = (clk or {}).get("sm_mhz")
+    if not inst or not mhz:
+        return None
+    achieved = inst / (eval_ms * 1e-3)
+    peak = 4.0 * sms * mhz * 1e6
+    return {"bound": "issue", "achieved": achieved, "peak": peak, "unit": "warp instructions/s",
+            "frac": achieved / peak, "warp_instructions": inst, "sms": sms, "sm_mhz": mhz}
+
+
 def run_gpu(args, rank, world, local):
     import torch
 
@@ -397,6 +425,7 @@ def run_gpu(args, rank, world, local):
                                    "times, hand-offs) + eval_list_kernel",
                          "algorithmic_bytes_per_plan": bpp, "kernel_ms": eval_ms_mean,
                          "peak_source": "MEASURED_PEAKS.json hbm_gbs (measured copy)" if peak else None},
+            "roofline_issue": issue_roofline(eval_ms_mean, clk, torch.cuda.get_device_properties(dev).multi_processor_count),
             "cpu_baseline": cpu,
             "clocks": clk,
             "gpu_launches": launches,
