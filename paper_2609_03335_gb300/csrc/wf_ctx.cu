@@ -235,6 +235,24 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
     for (int32_t n = 0; n < N; ++n)
         links[n] = ((uint32_t)dv.fprev[n] & 0xFFFFu) | ((uint32_t)dv.fnext[n] << 16);  // -1 -> 0xFFFF
     size_t o_links = img.add(links.data(), sizeof(uint32_t) * N);
+    // Per-node record of the sweep's producers: links; release slot code
+    // (slot | accumulator << 15; the zero slot nslots + 1 without
+    // predecessors) | model << 16 | write-list length (max 7) << 20; session
+    // arrival (u32: the sweep runs only with arrivals below 2^32); the first
+    // two write codes, the sink slot nslots standing in for absent ones.
+    std::vector<uint4> hrec(N);
+    if (nslots > 0) {
+        const uint32_t trash = (uint32_t)nslots, zero = trash + 1;
+        for (int32_t n = 0; n < N; ++n) {
+            const uint32_t rs = rslot[n] < 0 ? zero
+                                             : (((uint32_t)rslot[n] & 0x7FFFu) | ((rslot[n] & WF_RSLOT_ACC) ? 0x8000u : 0u));
+            const int32_t a = wl_off[n], len = wl_off[n + 1] - wl_off[n];
+            const uint32_t c0 = len > 0 ? wl[a] : trash, c1 = len > 1 ? wl[a + 1] : trash;
+            hrec[n] = make_uint4(links[n], rs | ((uint32_t)pb->model[n] << 16) | ((uint32_t)std::min(len, 7) << 20),
+                                 (uint32_t)pb->arrival_us[pb->session[n]], c0 | (c1 << 16));
+        }
+    }
+    size_t o_hrec = img.add(hrec.data(), sizeof(uint4) * N);
     size_t o_wloff = img.add(wl_off.data(), sizeof(int32_t) * (N + 1));
     size_t o_wl = img.add(wl.data(), sizeof(uint16_t) * wl.size());
     size_t o_lk = img.add(lk.data(), sizeof(int2) * lk.size());
@@ -322,6 +340,7 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
     dp.wl = (const uint16_t *)(base + o_wl);
     dp.lk = (const int2 *)(base + o_lk);
     dp.links = (const uint32_t *)(base + o_links);
+    dp.hrec = (const uint4 *)(base + o_hrec);
     dp.fitmask = (const uint32_t *)(base + o_fit);
     dp.edges = (const uint32_t *)(base + o_edges);
     dp.succ_off = (const int32_t *)(base + o_soff);

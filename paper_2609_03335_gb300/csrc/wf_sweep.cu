@@ -182,11 +182,8 @@ __device__ TT select_strided(TT *v, int32_t n, int32_t r)
 // Two extra slots follow a plan's nslots slots: a sink that absorbs writes
 // with no reader (index nslots) and a slot that always holds 0 (nslots + 1),
 // the release slot of a node without predecessors.  With them every unit
-// reads one release slot and writes its first two codes without branching.
-__device__ __forceinline__ uint32_t rslot16(int32_t code, uint32_t zero)
-{
-    return code < 0 ? zero : (((uint32_t)code & 0x7FFFu) | ((code & WF_RSLOT_ACC) ? 0x8000u : 0u));
-}
+// reads one release slot and writes its first two codes without branching;
+// the host encodes both into the per-node records (hrec).
 
 // Row pointers of one plan.
 struct PlanPtrs {
@@ -195,7 +192,10 @@ struct PlanPtrs {
     const uint32_t *fuse, *prefetch, *retain;
 };
 
-// Producer: the unit record of dispatch position i of a plan.
+// Producer: the unit record of dispatch position i of a plan.  One 16-byte
+// gather (hrec) gives a node's links, release slot, model, write codes and
+// arrival; the chain walk reads the members' records, whose last one holds
+// the unit's write codes.
 __device__ __forceinline__ void produce(const wf_dev_problem &dp, const PlanPtrs &r, int32_t i,
                                         uint32_t rec[kRecWords], int32_t *head = nullptr)
 {
@@ -204,12 +204,10 @@ __device__ __forceinline__ void produce(const wf_dev_problem &dp, const PlanPtrs
     if (head) *head = h;
     // Loads that depend on h alone go out together, ahead of any branch.
     const int32_t d = __ldg(r.place + h);
-    const uint32_t lh = __ldg(dp.links + h);
+    const uint4 hr = __ldg(dp.hrec + h);
     const uint32_t fw = __ldg(r.fuse + (h >> 5));
     const uint32_t pw = __ldg(r.prefetch + (h >> 5));
-    const int4 nr = __ldg(dp.noderec + 2 * h);
-    int4 wr = __ldg(dp.noderec + 2 * h + 1);
-    const uint32_t fp = lh & 0xFFFFu;
+    const uint32_t fp = hr.x & 0xFFFFu;
     if (fp != 0xFFFFu && ((fw >> (h & 31)) & 1u) && __ldg(r.place + fp) == d) {  // runs inside its head's unit
         rec[3] = kSkip;
         return;
@@ -217,30 +215,31 @@ __device__ __forceinline__ void produce(const wf_dev_problem &dp, const PlanPtrs
     const int2 lk0 = __ldg(dp.lk + h * D + d);
     uint32_t run = (uint32_t)lk0.x + (uint32_t)dp.grant, ovf = 0;  // both < 2^31: no wrap
     int32_t kv = lk0.y, tail = h;
-    for (uint32_t s = lh >> 16; s != 0xFFFFu; s = __ldg(dp.links + s) >> 16) {  // Eq. 3 chain
+    uint32_t ty = hr.y, tw = hr.w;  // the tail's write codes
+    for (uint32_t s = hr.x >> 16; s != 0xFFFFu;) {  // Eq. 3 chain
         if (!bit_of_g(r.fuse, s) || __ldg(r.place + s) != d) break;
         const int2 lk = __ldg(dp.lk + s * D + d);
+        const uint4 sr = __ldg(dp.hrec + s);
         const uint32_t r2 = run + (uint32_t)lk.x;
         ovf |= r2 < run;
         run = r2;
         kv = max(kv, lk.y);
         tail = (int32_t)s;
+        ty = sr.y;
+        tw = sr.w;
+        s = sr.x >> 16;
     }
-    if (tail != h) wr = __ldg(dp.noderec + 2 * tail + 1);
-    const uint32_t nwl = (uint32_t)min(wr.y, 7);
-    const uint32_t trash = (uint32_t)dp.nslots;
-    const uint32_t c0 = nwl > 0 ? (uint32_t)wr.z & 0xFFFFu : trash;
-    const uint32_t c1 = nwl > 1 ? (uint32_t)wr.z >> 16 : trash;
-    const uint32_t c2 = nwl > 2 ? (uint32_t)__ldg(dp.wl + wr.x + 2) : 0u;
+    const uint32_t nwl = (ty >> 20) & 7u;
+    const uint32_t c2 = nwl > 2 ? (uint32_t)__ldg(dp.wl + __ldg(dp.wl_off + tail) + 2) : 0u;
     const uint32_t pf = (pw >> (h & 31)) & 1u;
     const uint32_t reclaim = r.retain ? !bit_of_g(r.retain, tail) : 0u;
     rec[0] = ovf ? kRunCap : run;
     rec[1] = (uint32_t)kv;
-    rec[2] = (uint32_t)__ldg(dp.arrival + (nr.w >> 8));
-    rec[3] = (uint32_t)d | (((uint32_t)nr.w & 15u) << 5) | (pf << 9) | (reclaim << 10) | (nwl << 11) |
-             (c0 << 16);
-    rec[4] = c1 | (c2 << 16);
-    rec[5] = (uint32_t)tail | (rslot16(nr.z, trash + 1) << 16);
+    rec[2] = hr.z;
+    rec[3] = (uint32_t)d | (((hr.y >> 16) & 15u) << 5) | (pf << 9) | (reclaim << 10) | (nwl << 11) |
+             (tw << 16);
+    rec[4] = (tw >> 16) | (c2 << 16);
+    rec[5] = (uint32_t)tail | (hr.y << 16);
 }
 
 template <typename TT, int kS>
@@ -298,29 +297,39 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
         // ---------------- producers: lane = dispatch position ----------------
         __syncthreads();
         const int pos = lane % kChunk, sub = lane / kChunk;
+        // The plans this lane serves, fixed for the whole sweep: row pointers
+        // and whether the plan is live, resolved once.
+        constexpr int kStep = S::kProducers * kPlansPerIter;
+        constexpr int kIters = (kP + kStep - 1) / kStep;
+        PlanPtrs rp[kIters];
+        bool okq[kIters];
+#pragma unroll
+        for (int j = 0; j < kIters; ++j) {
+            const int q = (warp - 2) * kPlansPerIter + j * kStep + sub;
+            okq[j] = q < kP && q < ng;
+            if (okq[j]) {
+                const int64_t pq = in_list ? (int64_t)__ldg(in_list + j0 + q) : j0 + q;
+                okq[j] = __ldg(out.status + pq) == 0;
+                rp[j].place = pl.place + pq * pl.place_stride;
+                rp[j].order = (const uint16_t *)((const uint8_t *)pl.order + pq * pl.order_stride);
+                rp[j].fuse = (const uint32_t *)((const uint8_t *)pl.fuse + pq * pl.bits_stride);
+                rp[j].prefetch = (const uint32_t *)((const uint8_t *)pl.prefetch + pq * pl.bits_stride);
+                rp[j].retain = pl.retain ? (const uint32_t *)((const uint8_t *)pl.retain + pq * pl.bits_stride)
+                                         : nullptr;
+            }
+        }
         for (int32_t c = 0; c < chunks; ++c) {
             const int b = c % kBuffers;
             if (c >= kBuffers) named_sync(kEmpty + b, kProdThreads + 32);  // timing released buffer b
             const bool quit = kNarrow && *gave_up;
             uint32_t *rb = ring + b * kRecWords * kChunk * kPitch;
             const int32_t i = c * kChunk + pos;
-            for (int q0 = (warp - 2) * kPlansPerIter; q0 < kP; q0 += S::kProducers * kPlansPerIter) {
-                const int q = q0 + sub;
+#pragma unroll
+            for (int j = 0; j < kIters; ++j) {
+                const int q = (warp - 2) * kPlansPerIter + j * kStep + sub;
                 if (q >= kP) continue;
                 uint32_t rec[kRecWords] = {0, 0, 0, kSkip, 0, 0};
-                if (q < ng && i < N && !quit) {
-                    const int64_t pq = in_list ? (int64_t)__ldg(in_list + j0 + q) : j0 + q;
-                    if (__ldg(out.status + pq) == 0) {
-                        PlanPtrs r;
-                        r.place = pl.place + pq * pl.place_stride;
-                        r.order = (const uint16_t *)((const uint8_t *)pl.order + pq * pl.order_stride);
-                        r.fuse = (const uint32_t *)((const uint8_t *)pl.fuse + pq * pl.bits_stride);
-                        r.prefetch = (const uint32_t *)((const uint8_t *)pl.prefetch + pq * pl.bits_stride);
-                        r.retain = pl.retain ? (const uint32_t *)((const uint8_t *)pl.retain + pq * pl.bits_stride)
-                                             : nullptr;
-                        produce(dp, r, i, rec);
-                    }
-                }
+                if (okq[j] && i < N && !quit) produce(dp, rp[j], i, rec);
 #pragma unroll
                 for (int w = 0; w < kRecWords; ++w) rb[(w * kChunk + pos) * kPitch + q] = rec[w];
             }
