@@ -52,7 +52,8 @@ class _Problem(ctypes.Structure):
                 ("weight", ctypes.c_void_p), ("load", ctypes.c_void_p), ("cap", ctypes.c_void_p),
                 ("grant", ctypes.c_int32), ("S", ctypes.c_int32), ("seed", ctypes.c_uint64),
                 ("bm_r", ctypes.c_void_p), ("bm_c", ctypes.c_void_p), ("bm_e", ctypes.c_void_p),
-                ("bm_rn", ctypes.c_int32), ("bm_cn", ctypes.c_int32), ("bm_en", ctypes.c_int32)]
+                ("bm_rn", ctypes.c_int32), ("bm_cn", ctypes.c_int32), ("bm_en", ctypes.c_int32),
+                ("reclaim", ctypes.c_int32)]
 
 
 class _Trace(ctypes.Structure):
@@ -123,7 +124,7 @@ class OracleProblem:
                           int(prob.grant_us), self.S, int(prob.seed) & ((1 << 64) - 1),
                           ar["bm_r"].ctypes.data, ar["bm_c"].ctypes.data, ar["bm_e"].ctypes.data,
                           int(np.asarray(prob.bm_r).size), int(np.asarray(prob.bm_c).size),
-                          int(np.asarray(prob.bm_e).size))
+                          int(np.asarray(prob.bm_e).size), int(getattr(prob, "reclaim", 0)))
         self.fnext = np.empty(self.N, np.int32)
         if self.lib.orc_fusible_next(ctypes.byref(self.c), self.fnext.ctypes.data) != 0:
             raise MemoryError("oracle allocation failed")

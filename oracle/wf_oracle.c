@@ -67,6 +67,7 @@ typedef struct {
     uint64_t seed;
     const int32_t *bm_r, *bm_c, *bm_e;
     int32_t bm_rn, bm_cn, bm_en;
+    int32_t reclaim;           /* 0: least recently used first; 1: by next use (see next_use_victim) */
 } orc_problem;
 
 /* Optional record of one deterministic run, for the invariant checker. */
@@ -228,6 +229,47 @@ int orc_status(const orc_problem *pb, const uint8_t *place, const uint16_t *orde
  * *makespan and *gpu.  Returns 0, -1 on allocation failure, -2 if a unit
  * cannot be admitted even on an empty device (never for a valid plan).
  */
+/*
+ * Reclamation by next use (the paper's preference order when it reclaims,
+ * Section 3.5: redundant copies first, then the model whose next use is
+ * farthest relative to its reload cost, least recently used for the rest).
+ * Among the models resident on device d other than m, the victim is the
+ * first by:
+ *   1. resident on another device too (a redundant copy);
+ *   2. larger (next use - i) / load[k][d], where next use is the dispatch
+ *      position of the next unit on d with model k after position i (none:
+ *      infinitely far) and a zero load cost makes the ratio infinite; two
+ *      infinite ratios tie;
+ *   3. smaller last-use stamp (least recently used).
+ * is_head[j] marks the dispatch positions that start a unit.
+ */
+static int32_t next_use_victim(const orc_problem *pb, const uint8_t *place, const uint16_t *order,
+                               const uint8_t *is_head, int32_t i, int32_t d, int32_t m, const int64_t *stamp)
+{
+    const int32_t N = pb->N, D = pb->D, M = pb->M;
+    int32_t best = -1, best_red = 0, best_inf = 0;
+    int64_t best_dist = 0, best_cost = 0;
+    for (int32_t k = 0; k < M; ++k) {
+        if (k == m || stamp[(int64_t)d * M + k] == 0) continue;
+        int32_t red = 0;
+        for (int32_t e = 0; e < D; ++e)
+            if (e != d && stamp[(int64_t)e * M + k] != 0) red = 1;
+        int64_t dist = -1;
+        for (int32_t j = i + 1; j < N && dist < 0; ++j)
+            if (is_head[j] && place[order[j]] == d && pb->model[order[j]] == k) dist = j - i;
+        const int64_t cost = pb->load[(int64_t)k * D + d];
+        const int inf = dist < 0 || cost == 0;
+        int better;
+        if (best < 0) better = 1;
+        else if (red != best_red) better = red > best_red;
+        else if (inf != best_inf) better = inf > best_inf;
+        else if (!inf && dist * best_cost != best_dist * cost) better = dist * best_cost > best_dist * cost;
+        else better = stamp[(int64_t)d * M + k] < stamp[(int64_t)d * M + best];
+        if (better) { best = k; best_red = red; best_inf = inf; best_dist = dist; best_cost = cost; }
+    }
+    return best;
+}
+
 static int simulate(const orc_problem *pb, const int32_t *fnext,
                     const uint8_t *place, const uint16_t *order,
                     const uint32_t *fuse, const uint32_t *prefetch, const uint32_t *retain,
@@ -243,8 +285,22 @@ static int simulate(const orc_problem *pb, const int32_t *fnext,
     int64_t *stamp = (int64_t *)malloc(sizeof(int64_t) * (size_t)D * (size_t)M);
     uint8_t *done = (uint8_t *)malloc((size_t)N);
     int32_t *chain = (int32_t *)malloc(sizeof(int32_t) * (size_t)N);
+    uint8_t *is_head = (uint8_t *)malloc((size_t)N);
+    int32_t *fprev = (int32_t *)malloc(sizeof(int32_t) * (size_t)N);
     int rc = 0;
-    if (!t_free || !occ_since || !gpu || !used || !nres || !stamp || !done || !chain) { rc = -1; goto out; }
+    if (!t_free || !occ_since || !gpu || !used || !nres || !stamp || !done || !chain || !is_head || !fprev) {
+        rc = -1;
+        goto out;
+    }
+    /* Dispatch positions that start a unit: every node but those that run
+     * inside their fusible predecessor's unit (fuse bit set, same device). */
+    for (int32_t v = 0; v < N; ++v) fprev[v] = -1;
+    for (int32_t u = 0; u < N; ++u)
+        if (fnext[u] >= 0) fprev[fnext[u]] = u;
+    for (int32_t j = 0; j < N; ++j) {
+        const int32_t x = order[j];
+        is_head[j] = !(fprev[x] >= 0 && bit_of(fuse, x) && place[x] == place[fprev[x]]);
+    }
 
     /* Initial snapshot: every device idle and empty at t = 0. */
     for (int32_t d = 0; d < D; ++d) {
@@ -291,8 +347,12 @@ static int simulate(const orc_problem *pb, const int32_t *fnext,
          * until resident weights plus the incoming demand fit the device. */
         while (used[d] + need > pb->cap[d]) {
             int32_t victim = -1;
-            for (int32_t k = 0; k < M; ++k)
-                if (k != m && st[k] != 0 && (victim < 0 || st[k] < st[victim])) victim = k;
+            if (pb->reclaim) {
+                victim = next_use_victim(pb, place, order, is_head, i, d, m, stamp);
+            } else {
+                for (int32_t k = 0; k < M; ++k)
+                    if (k != m && st[k] != 0 && (victim < 0 || st[k] < st[victim])) victim = k;
+            }
             if (victim < 0) { rc = -2; goto out; }
             used[d] -= pb->weight[victim];
             st[victim] = 0;
@@ -378,6 +438,7 @@ static int simulate(const orc_problem *pb, const int32_t *fnext,
     if (tr) for (int32_t n = 0; n < N; ++n) tr->finish[n] = c[n];
 out:
     free(t_free); free(occ_since); free(gpu); free(used); free(nres); free(stamp); free(done); free(chain);
+    free(is_head); free(fprev);
     return rc;
 }
 

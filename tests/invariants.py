@@ -3,6 +3,8 @@
 It re-derives nothing from the oracle's code: it checks the equations the
 paper states as constraints on any feasible graph-schedule plan.
 """
+from fractions import Fraction
+
 import numpy as np
 
 from randprob import preds_of
@@ -98,15 +100,28 @@ def check_trace(prob, plans, p, res, fnext, forecast=None):
         assert (tr["load_start"][h] < 0) == hit
         need = kv if hit else W[m] + kv
         used = sum(W[k] for k in resident[d])
-        # evictions are exactly the least recent others, taken until it fits
-        others = sorted((t, k) for k, t in resident[d].items() if k != m)
+        # evictions are exactly the first others in reclamation order, taken
+        # until it fits: least recent first, or (next-use reclamation)
+        # redundant copies, then farthest next use per unit of reload cost,
+        # then least recent
+        if getattr(prob, "reclaim", 0):
+            def order_key(k):
+                red = any(k in resident[e] for e in range(D) if e != d)
+                later = [pos[x] for x in heads if pos[x] > pos[h] and place[x] == d and int(prob.model[x]) == k]
+                cost = int(prob.load_us[k * D + d])
+                if not later or cost == 0:
+                    return (not red, 0, 0, resident[d][k])
+                return (not red, 1, Fraction(-(min(later) - pos[h]), cost), resident[d][k])
+            others = sorted((order_key(k), k) for k in resident[d] if k != m)
+        else:
+            others = sorted((t, k) for k, t in resident[d].items() if k != m)
         taken = 0
         expect_ev = []
         while used - taken + need > prob.cap_mib[d]:
-            t, k = others[len(expect_ev)]
+            _, k = others[len(expect_ev)]
             expect_ev.append(k)
             taken += W[k]
-        assert sorted(ev) == sorted(expect_ev), ("LRU victims", h, ev, expect_ev)
+        assert sorted(ev) == sorted(expect_ev), ("reclamation victims", h, ev, expect_ev)
         for k in ev:
             del resident[d][k]
         resident[d][m] = pos[h]

@@ -56,12 +56,17 @@ MUTANTS = {
     "construct_rank_ignores_release": ("rank[y] = r + (jitter", "rank[y] = 0 + (jitter"),
     "construct_binding_ignores_residency": ("if (stamp[(int64_t)dd * M + m] != 0) {", "if (0) {"),
     "construct_prefetch_always": ("const int pf = !hit && t_free[d] < rel[u];", "const int pf = !hit;"),
+    "next_use_ignores_redundancy": ("else if (red != best_red) better = red > best_red;", "else if (0) better = 0;"),
+    "next_use_ignores_cost": ("else if (!inf && dist * best_cost != best_dist * cost) better = dist * best_cost > best_dist * cost;",
+                              "else if (!inf && dist != best_dist) better = dist > best_dist;"),
+    "next_use_nearest_first": ("better = dist * best_cost > best_dist * cost;", "better = dist * best_cost < best_dist * cost;"),
     "construct_no_fusion": ("s >= 0 && pb->peak[(int64_t)s * D + d] <= pb->cap[d]; s = fnext[s])",
                             "s >= 0 && 0; s = fnext[s])"),
 }
 
 PIN_FILES = ["tests/test_oracle_golden.py", "tests/test_oracle_properties.py",
-             "tests/test_oracle_stochastic.py", "tests/test_oracle_search.py", "tests/test_oracle_construct.py"]
+             "tests/test_oracle_stochastic.py", "tests/test_oracle_search.py", "tests/test_oracle_construct.py",
+             "tests/test_oracle_reclaim.py"]
 
 
 def _run_mutant(name, tmp):

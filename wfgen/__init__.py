@@ -99,6 +99,7 @@ class Problem:
     bm_c: np.ndarray = field(default_factory=lambda: np.zeros(0, np.int32))
     bm_e: np.ndarray = field(default_factory=lambda: np.zeros(0, np.int32))
     name: str = ""
+    reclaim: int = 0          # reclamation order: 0 least recently used, 1 by next use
 
     @property
     def E(self) -> int:
