@@ -18,6 +18,7 @@
  *   wf_merge_elite          keep the k best of an elite and its children
  *   wf_local_search         rounds of mutate -> evaluate -> merge
  *   wf_construct_plans      plans built by a list scheduler (Algorithm 1)
+ *   wf_ctx_set_reclaim      reclamation order: LRU or by next use
  *   wf_ctx_destroy, wf_strerror
  *
  * Conventions.
@@ -50,6 +51,12 @@ enum {
     WF_ENOMEM = 2,    /* device or host allocation failed */
     WF_ECUDA = 3,     /* a CUDA launch or runtime error (see wf_strerror) */
     WF_ETIMEOUT = 4   /* a bounded device-side wait expired; results are invalid */
+};
+
+/* Reclamation order (wf_ctx_set_reclaim). */
+enum {
+    WF_RECLAIM_LRU = 0,      /* least recently used first (the default) */
+    WF_RECLAIM_NEXT_USE = 1  /* redundant copies, then farthest next use per reload cost, then LRU */
 };
 
 /* Plan status bits (wf_eval_out.status). */
@@ -283,6 +290,24 @@ int wf_local_search(wf_ctx *ctx, const wf_plans *elite, const wf_eval_out *elite
  * 128 plans per SM); later calls allocate nothing.  Asynchronous on stream.
  */
 int wf_construct_plans(wf_ctx *ctx, const wf_plans *out, uint64_t seed, int64_t jitter_us, void *stream);
+
+/*
+ * Reclamation order of the context's evaluations (Eq. 11 admission).  The
+ * paper reclaims idle replicas preferring redundant copies, then distant next
+ * use relative to reload cost, with least-recently-used order as the fallback
+ * (Section 3.5).  WF_RECLAIM_LRU (the default) evicts least recently used
+ * first.  WF_RECLAIM_NEXT_USE evicts, one at a time until the unit fits:
+ * first a model also resident on another device; among equals the one whose
+ * next use on this device (the next dispatch position whose unit runs that
+ * model there; none = infinitely far) lies farthest from the current position
+ * per microsecond of its reload cost (a zero cost counts as infinitely far);
+ * among equals the least recently used.  The next-use policy needs S = 0, a
+ * window the shared-memory sweep holds, and fusible chains whose run time
+ * stays below 2^32 us; otherwise WF_EINVAL.  The first switch to it allocates
+ * a [max_P][N] u16 table.  Not thread-safe with calls in flight on the
+ * context.  wf_eval_plans_static always uses WF_RECLAIM_LRU.
+ */
+int wf_ctx_set_reclaim(wf_ctx *ctx, int32_t policy);
 
 /*
  * Synchronize `stream` and report device-side failures of earlier calls on

@@ -280,6 +280,17 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
     }
     size_t o_soff = img.add(succ_off.data(), sizeof(int32_t) * (N + 1));
     size_t o_sidx = img.add(succ_idx.data(), sizeof(int32_t) * succ_idx.size());
+    int64_t max_chain = 0;
+    for (int32_t h = 0; h < N; ++h) {
+        if (dv.fprev[h] >= 0) continue;
+        int64_t sum = pb->grant_us;
+        for (int32_t x = h; x >= 0; x = dv.fnext[x]) {
+            int64_t worst = 0;
+            for (int32_t d = 0; d < D; ++d) worst = std::max(worst, (int64_t)pb->lat_us[(int64_t)x * D + d]);
+            sum += worst;
+        }
+        max_chain = std::max(max_chain, sum);
+    }
     int64_t horizon = 0;
     for (int32_t w = 0; w < W; ++w) horizon = std::max(horizon, pb->arrival_us[w]);
     for (int32_t n = 0; n < N; ++n) {
@@ -346,6 +357,9 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
     dp.succ_off = (const int32_t *)(base + o_soff);
     dp.succ_idx = (const int32_t *)(base + o_sidx);
     dp.horizon = horizon;
+    dp.max_chain_run = max_chain;
+    dp.reclaim = 0;
+    dp.nextuse = nullptr;
     int64_t amax = 0;
     for (int32_t w = 0; w < W; ++w) amax = std::max(amax, pb->arrival_us[w]);
     dp.max_arrival = amax;
@@ -386,6 +400,7 @@ extern "C" void wf_ctx_destroy(wf_ctx *c)
     if (c->topk_scratch) cudaFree(c->topk_scratch);
     if (c->search_scratch) cudaFree(c->search_scratch);
     if (c->construct_scratch) cudaFree(c->construct_scratch);
+    if (c->dp.nextuse) cudaFree(c->dp.nextuse);
     if (c->side) cudaStreamSynchronize(c->side);
     if (c->side) cudaStreamDestroy(c->side);
     if (c->ovf_event) cudaEventDestroy(c->ovf_event);
@@ -460,6 +475,33 @@ extern "C" int wf_topk(wf_ctx *c, const wf_eval_out *res, int64_t P, int32_t k, 
     int rc = select_device(c);
     if (rc) return rc;
     return wf_launch_topk(c, res, P, k, ids, keys, (cudaStream_t)stream);
+}
+
+extern "C" int wf_ctx_set_reclaim(wf_ctx *c, int32_t policy)
+{
+    REQUIRE(c, "NULL context");
+    REQUIRE(policy == WF_RECLAIM_LRU || policy == WF_RECLAIM_NEXT_USE, "unknown reclamation policy %d", policy);
+    if (policy == WF_RECLAIM_LRU) {
+        c->dp.reclaim = 0;
+        return WF_OK;
+    }
+    REQUIRE(c->dp.S == 0, "reclamation by next use needs deterministic latencies (S = 0)");
+    REQUIRE(c->dp.max_chain_run < (int64_t)UINT32_MAX,
+            "a fusible chain may run %lld us, beyond the shared-memory sweep", (long long)c->dp.max_chain_run);
+    wf_dev_problem probe = c->dp;
+    probe.reclaim = 1;
+    const wf_sweep_cfg cfg = wf_sweep_config(probe);
+    REQUIRE(cfg.smem64, "reclamation by next use needs the 64-bit shared-memory sweep, "
+                        "which this window does not fit");
+    int rc = select_device(c);
+    if (rc) return rc;
+    if (!c->dp.nextuse) {
+        rc = wf_cuda_check(cudaMalloc(&c->dp.nextuse, sizeof(uint16_t) * (size_t)c->max_P * (size_t)c->dp.N),
+                           "cudaMalloc(next-use table)");
+        if (rc) { c->dp.nextuse = nullptr; return rc; }
+    }
+    c->dp.reclaim = 1;
+    return WF_OK;
 }
 
 extern "C" int wf_ctx_status(wf_ctx *c, void *stream)

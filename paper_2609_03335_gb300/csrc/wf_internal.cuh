@@ -51,6 +51,12 @@ struct wf_dev_problem {
     const int32_t *succ_off;    // [N+1] successor lists (CSR)
     const int32_t *succ_idx;    // [E]
     int64_t horizon;            // no finish of any plan exceeds this (latest arrival + every node's worst load + run + grant)
+    // Reclamation order (0: least recently used; 1: by next use) and, for 1,
+    // the next use of each unit's model on its device: [max_P][N] dispatch
+    // positions (0xFFFF = none), filled per call.
+    int32_t reclaim;
+    uint16_t *nextuse;
+    int64_t max_chain_run;      // the longest fusible chain's run time on its slowest devices, plus the grant
     int64_t max_arrival;
 };
 
@@ -122,6 +128,7 @@ struct wf_sweep_cfg {
     int plans64;
 };
 wf_sweep_cfg wf_sweep_config(const wf_dev_problem &dp);
+int wf_launch_nextuse(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, cudaStream_t st);
 size_t wf_stoch_smem(const wf_dev_problem &dp);
 int wf_launch_stoch(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, size_t smem,
                     int32_t *ovf_list, int32_t *ovf_count, cudaStream_t st);

@@ -118,11 +118,14 @@ constexpr uint32_t kEmptied = 1u << 15;    // after residency: the unit's reclai
 constexpr uint32_t kRunCap = 0xFFFFFFFFu;  // saturation of w0
 
 struct PcLayout {
-    uint32_t weight, cap, load, arr, ring, slots, tfree, used, queue, nres, open, flag, total;
+    uint32_t weight, cap, load, arr, ring, slots, tfree, used, queue, nres, open, flag, nuse, rcnt, total;
 };
 
-// Shared memory of a CTA of kP plans with TT times and NS slots per plan.
-template <int kP, typename TT>
+// Shared memory of a CTA of kP plans with TT times and NS slots per plan;
+// with reclamation by next use (kReclaim) the ring carries a seventh record
+// word and each plan keeps per (device, model) the next use of the resident
+// copy and per model the number of devices holding it.
+template <int kP, typename TT, int kReclaim = 0>
 __host__ __device__ inline PcLayout pc_layout(int32_t D, int32_t M, int32_t W, int32_t NS)
 {
     constexpr uint32_t t = sizeof(TT);
@@ -132,7 +135,7 @@ __host__ __device__ inline PcLayout pc_layout(int32_t D, int32_t M, int32_t W, i
     l.cap = o; o += round16(4u * D);
     l.load = o; o += round16(4u * M * D);
     l.arr = o; o += round16(4u * W);
-    l.ring = o; o += round16(4u * kBuffers * kRecWords * kChunk * PcShape<kP>::kPitch);
+    l.ring = o; o += round16(4u * kBuffers * (kRecWords + kReclaim) * kChunk * PcShape<kP>::kPitch);
     l.slots = o; o += round16(t * (uint32_t)NS * kP);
     l.tfree = o; o += round16(t * D * kP);
     l.used = o; o += round16(4u * D * kP);
@@ -140,6 +143,8 @@ __host__ __device__ inline PcLayout pc_layout(int32_t D, int32_t M, int32_t W, i
     l.nres = o; o += round16((uint32_t)D * kP);
     l.open = o; o += round16(4u * kP);
     l.flag = o; o += 16;
+    l.nuse = o; o += kReclaim ? round16(2u * D * M * kP) : 0u;
+    l.rcnt = o; o += kReclaim ? round16((uint32_t)M * kP) : 0u;
     l.total = o;
     return l;
 }
@@ -255,11 +260,12 @@ __device__ __forceinline__ void publish(TT *slots, uint32_t code, TT c)
 // ovf_list; once every plan of a CTA has, its stages run on without loads.
 // TT = uint64_t: only a unit whose summed run time reaches 2^32 - 1 sends its
 // plan to ovf_list.
-template <typename Q, typename TT, int kP>
+template <typename Q, typename TT, int kP, int kReclaim>
 __global__ void __launch_bounds__(32 * PcShape<kP>::kWarps)
 pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_list, const int32_t *in_count,
           int32_t *ovf_list, int32_t *ovf_count)
 {
+    constexpr int kRW = kRecWords + kReclaim;  // words per record in the ring
     using S = PcShape<kP>;
     constexpr int kPitch = S::kPitch;
     constexpr int kProdThreads = 32 * S::kProducers;
@@ -267,7 +273,7 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
     extern __shared__ __align__(128) uint8_t sm[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int32_t N = dp.N, D = dp.D, M = dp.M, W = dp.W;
-    const PcLayout L = pc_layout<kP, TT>(D, M, W, dp.nslots + 2);
+    const PcLayout L = pc_layout<kP, TT, kReclaim>(D, M, W, dp.nslots + 2);
     const int64_t total = in_list ? (int64_t)*in_count : pl.P;
     if ((int64_t)blockIdx.x * kP >= total) return;  // the whole CTA: no plan
     uint32_t *ring = (uint32_t *)(sm + L.ring);
@@ -303,12 +309,15 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
         constexpr int kIters = (kP + kStep - 1) / kStep;
         PlanPtrs rp[kIters];
         bool okq[kIters];
+        int64_t qplan[kIters];
 #pragma unroll
         for (int j = 0; j < kIters; ++j) {
             const int q = (warp - 2) * kPlansPerIter + j * kStep + sub;
             okq[j] = q < kP && q < ng;
+            qplan[j] = 0;
             if (okq[j]) {
                 const int64_t pq = in_list ? (int64_t)__ldg(in_list + j0 + q) : j0 + q;
+                qplan[j] = pq;
                 okq[j] = __ldg(out.status + pq) == 0;
                 rp[j].place = pl.place + pq * pl.place_stride;
                 rp[j].order = (const uint16_t *)((const uint8_t *)pl.order + pq * pl.order_stride);
@@ -322,7 +331,7 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
             const int b = c % kBuffers;
             if (c >= kBuffers) named_sync(kEmpty + b, kProdThreads + 32);  // timing released buffer b
             const bool quit = kNarrow && *gave_up;
-            uint32_t *rb = ring + b * kRecWords * kChunk * kPitch;
+            uint32_t *rb = ring + b * kRW * kChunk * kPitch;
             const int32_t i = c * kChunk + pos;
 #pragma unroll
             for (int j = 0; j < kIters; ++j) {
@@ -332,6 +341,10 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
                 if (okq[j] && i < N && !quit) produce(dp, rp[j], i, rec);
 #pragma unroll
                 for (int w = 0; w < kRecWords; ++w) rb[(w * kChunk + pos) * kPitch + q] = rec[w];
+                if (kReclaim)  // the next use of this unit's model on its device
+                    rb[(kRecWords * kChunk + pos) * kPitch + q] =
+                        (okq[j] && i < N && !quit) ? (uint32_t)__ldg(dp.nextuse + qplan[j] * (int64_t)N + i)
+                                                   : 0xFFFFu;
             }
             named_arrive(kFullP + b, kProdThreads + 32);  // buffer b is full
         }
@@ -343,13 +356,18 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
         uint32_t *used = (uint32_t *)(sm + L.used) + lane;
         Q *queue = (Q *)(sm + L.queue) + lane;
         uint8_t *nres = sm + L.nres + lane;
-        if (mine)
+        uint16_t *nuse = (uint16_t *)(sm + L.nuse) + lane;  // [device][model][plan]
+        uint8_t *rcnt = sm + L.rcnt + lane;                 // [model][plan]
+        if (mine) {
             for (int32_t d = 0; d < D; ++d) { used[d * kP] = 0; queue[d * kP] = 0; nres[d * kP] = 0; }
+            if (kReclaim)
+                for (int32_t k = 0; k < M; ++k) rcnt[k * kP] = 0;
+        }
         __syncthreads();
         for (int32_t c = 0; c < chunks; ++c) {
             const int b = c % kBuffers;
             named_sync(kFullP + b, kProdThreads + 32);
-            uint32_t *rb = ring + b * kRecWords * kChunk * kPitch + lane;
+            uint32_t *rb = ring + b * kRW * kChunk * kPitch + lane;
             const int32_t kmax = min(kChunk, N - c * kChunk);
             for (int32_t k = 0; k < kmax && live; ++k) {
                 const uint32_t r3 = rb[(3 * kChunk + k) * kPitch];
@@ -371,14 +389,49 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
                 q = hit ? Lru<Q>::remove(q, hit ? kq : 0) : q;  // (an index below the queue length)
                 n -= hit ? 1u : 0u;
                 const uint32_t need = hit ? r1 : wm + r1;
-                uint32_t e = 0;
-                while (u_d + need > capd && e < n) {
-                    u_d -= (uint32_t)weight[(uint32_t)(q >> (4 * e)) & 15u];
-                    ++e;
+                if (kReclaim) {
+                    // Victims one at a time: a copy also resident elsewhere,
+                    // then the largest (next use - position) / reload cost
+                    // (no next use or a free reload: infinite), then the
+                    // least recently used (the earlier queue entry).
+                    const int64_t here = c * kChunk + k;
+                    while (u_d + need > capd && n > 0) {
+                        int32_t best = 0;
+                        uint32_t bred = 0, binf = 0;
+                        int64_t bdist = 0, bcost = 0;
+                        for (int32_t e = 0; e < (int32_t)n; ++e) {
+                            const uint32_t kk = (uint32_t)(q >> (4 * e)) & 15u;
+                            const uint32_t red = rcnt[kk * kP] > 1;
+                            const uint32_t nu = nuse[(d * M + kk) * kP];
+                            const int64_t cost = load[kk * D + d];
+                            const uint32_t inf = nu == 0xFFFFu || cost == 0;
+                            const int64_t dist = (int64_t)nu - here;
+                            bool better;
+                            if (e == 0) better = true;
+                            else if (red != bred) better = red > bred;
+                            else if (inf != binf) better = inf > binf;
+                            else better = !inf && dist * bcost > bdist * cost;
+                            if (better) { best = e; bred = red; binf = inf; bdist = dist; bcost = cost; }
+                        }
+                        const uint32_t victim = (uint32_t)(q >> (4 * best)) & 15u;
+                        u_d -= (uint32_t)weight[victim];
+                        rcnt[victim * kP] -= 1;
+                        q = Lru<Q>::remove(q, best);
+                        n -= 1;
+                    }
+                    if (u_d + need > capd) atomicExch(dp.err, 2);  // unreachable for a valid plan
+                    if (!hit) rcnt[m * kP] += 1;
+                    nuse[(d * M + m) * kP] = (uint16_t)rb[(kRecWords * kChunk + k) * kPitch];
+                } else {
+                    uint32_t e = 0;
+                    while (u_d + need > capd && e < n) {
+                        u_d -= (uint32_t)weight[(uint32_t)(q >> (4 * e)) & 15u];
+                        ++e;
+                    }
+                    if (u_d + need > capd) atomicExch(dp.err, 2);  // unreachable for a valid plan
+                    q = e < (uint32_t)Lru<Q>::kSlots ? (q >> (4 * e)) : (Q)0;
+                    n -= e;
                 }
-                if (u_d + need > capd) atomicExch(dp.err, 2);  // unreachable for a valid plan
-                q = e < (uint32_t)Lru<Q>::kSlots ? (q >> (4 * e)) : (Q)0;
-                n -= e;
                 q |= (Q)m << (4 * n);  // the unit's model is now the most recently used
                 n += 1;
                 u_d += hit ? 0u : wm;
@@ -388,6 +441,7 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
                     n -= 1;
                     u_d -= wm;
                     emptied = n == 0;
+                    if (kReclaim) rcnt[m * kP] -= 1;
                 }
                 queue[d * kP] = q;
                 nres[d * kP] = (uint8_t)n;
@@ -426,7 +480,7 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
     for (int32_t c = 0; c < chunks; ++c) {
         const int b = c % kBuffers;
         named_sync(kFullR + b, 64);
-        const uint32_t *rb = ring + b * kRecWords * kChunk * kPitch + lane;
+        const uint32_t *rb = ring + b * kRW * kChunk * kPitch + lane;
         const int32_t kmax = min(kChunk, N - c * kChunk);
         for (int32_t k = 0; k < kmax && live; ++k) {
             const uint32_t r3 = rb[(3 * kChunk + k) * kPitch];
@@ -777,6 +831,51 @@ stoch_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list,
     }
 }
 
+// Next use, for reclamation by next use: for every dispatch position i that
+// starts a unit, the next position that starts a unit on the same device with
+// the same model (0xFFFF: none).  A warp per plan walks its positions from the
+// end, 32 at a time; lanes with equal (device, model) keys find each other
+// with __match_any_sync, and a shared table carries the first occurrence of
+// each key to the chunk before.
+constexpr int kNuWarps = 4;
+
+__global__ void __launch_bounds__(32 * kNuWarps)
+nextuse_kernel(wf_dev_problem dp, wf_plans pl, const uint32_t *status, uint16_t *table)
+{
+    extern __shared__ __align__(16) uint8_t nsm[];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int32_t N = dp.N, D = dp.D, M = dp.M;
+    uint16_t *last = (uint16_t *)nsm + warp * D * M;
+    for (int64_t p = (int64_t)blockIdx.x * kNuWarps + warp; p < pl.P; p += (int64_t)gridDim.x * kNuWarps) {
+        if (__ldg(status + p) != 0) continue;  // uniform over the warp
+        const uint8_t *place = pl.place + p * pl.place_stride;
+        const uint16_t *order = (const uint16_t *)((const uint8_t *)pl.order + p * pl.order_stride);
+        const uint32_t *fuse = (const uint32_t *)((const uint8_t *)pl.fuse + p * pl.bits_stride);
+        uint16_t *out = table + p * (int64_t)N;
+        for (int32_t k = lane; k < D * M; k += 32) last[k] = 0xFFFFu;
+        __syncwarp();
+        for (int32_t base = ((N - 1) / 32) * 32; base >= 0; base -= 32) {
+            const int32_t j = base + lane;
+            uint32_t key = 0xFFFFFFFFu;  // not the start of a unit
+            if (j < N) {
+                const int32_t x = __ldg(order + j);
+                const int32_t d = __ldg(place + x);
+                const uint4 hr = __ldg(dp.hrec + x);
+                const uint32_t fp = hr.x & 0xFFFFu;
+                const bool member = fp != 0xFFFFu && ((__ldg(fuse + (x >> 5)) >> (x & 31)) & 1u) &&
+                                    __ldg(place + fp) == d;
+                if (!member) key = (uint32_t)d * M + ((hr.y >> 16) & 15u);
+            }
+            const uint32_t same = __match_any_sync(0xFFFFFFFFu, key);
+            const uint32_t above = lane == 31 ? 0u : (same & (0xFFFFFFFFu << (lane + 1)));
+            if (key != 0xFFFFFFFFu) out[j] = above ? (uint16_t)(base + __ffs((int)above) - 1) : last[key];
+            __syncwarp();
+            if (key != 0xFFFFFFFFu && lane == __ffs((int)same) - 1) last[key] = (uint16_t)j;
+            __syncwarp();
+        }
+    }
+}
+
 // Status bits of every plan (Eq. 8-10), one warp per plan.  Four nodes per
 // lane check placement and fit (one fit mask per node); the warp scatters the
 // inverse of the dispatch sequence (u16 positions) into shared memory and
@@ -910,12 +1009,13 @@ int plans_per_sm(size_t smem, int kp)
     return smem <= 227 * 1024 ? kp * (int)((228 * 1024) / (smem + 1024)) : 0;
 }
 
-template <typename Q, typename TT, int kP>
+template <typename Q, typename TT, int kP, int kR>
 int launch_pc(const wf_dev_problem &dp, int sms, const wf_plans *pl, const wf_eval_out *out, size_t smem,
               const int32_t *in_list, const int32_t *in_count, int32_t *list, int32_t *count, cudaStream_t st)
 {
-    int rc = wf_cuda_check(cudaFuncSetAttribute(pc_kernel<Q, TT, kP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                (int)smem), "sweep smem attribute");
+    int rc = wf_cuda_check(cudaFuncSetAttribute(pc_kernel<Q, TT, kP, kR>,
+                                                cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
+                           "sweep smem attribute");
     if (rc) return rc;
     // Every plan: a CTA per group.  A list (of unknown length): at most as
     // many CTAs as are resident at once, each walking over groups.
@@ -924,36 +1024,58 @@ int launch_pc(const wf_dev_problem &dp, int sms, const wf_plans *pl, const wf_ev
         const int64_t per_sm = std::max<int64_t>(1, std::min<int64_t>(8, (228 * 1024) / (int64_t)(smem + 1024)));
         blocks = std::min<int64_t>(blocks, per_sm * sms);
     }
-    pc_kernel<Q, TT, kP><<<(unsigned)blocks, 32 * PcShape<kP>::kWarps, smem, st>>>(dp, *pl, *out, in_list, in_count, list,
+    pc_kernel<Q, TT, kP, kR><<<(unsigned)blocks, 32 * PcShape<kP>::kWarps, smem, st>>>(dp, *pl, *out, in_list, in_count, list,
                                                                           count);
     return wf_cuda_check(cudaGetLastError(), "sweep launch");
+}
+
+template <typename TT, int kR>
+int launch_pc_r(const wf_ctx *ctx, int kp, const wf_plans *pl, const wf_eval_out *out, size_t smem,
+                const int32_t *in_list, const int32_t *in_count, int32_t *list, int32_t *count, cudaStream_t st)
+{
+    const wf_dev_problem &dp = ctx->dp;
+    const int sms = ctx->sms;
+    if (kp == 16)
+        return dp.M <= 8
+                   ? launch_pc<uint32_t, TT, 16, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
+                   : launch_pc<uint64_t, TT, 16, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
+    return dp.M <= 8 ? launch_pc<uint32_t, TT, 6, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
+                     : launch_pc<uint64_t, TT, 6, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
 }
 
 template <typename TT>
 int launch_pc_q(const wf_ctx *ctx, int kp, const wf_plans *pl, const wf_eval_out *out, size_t smem,
                 const int32_t *in_list, const int32_t *in_count, int32_t *list, int32_t *count, cudaStream_t st)
 {
-    const wf_dev_problem &dp = ctx->dp;
-    const int sms = ctx->sms;
-    if (kp == 16)
-        return dp.M <= 8 ? launch_pc<uint32_t, TT, 16>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
-                         : launch_pc<uint64_t, TT, 16>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
-    return dp.M <= 8 ? launch_pc<uint32_t, TT, 6>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
-                     : launch_pc<uint64_t, TT, 6>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
+    return ctx->dp.reclaim ? launch_pc_r<TT, 1>(ctx, kp, pl, out, smem, in_list, in_count, list, count, st)
+                           : launch_pc_r<TT, 0>(ctx, kp, pl, out, smem, in_list, in_count, list, count, st);
 }
 
 }  // namespace
+
+int wf_launch_nextuse(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, cudaStream_t st)
+{
+    const wf_dev_problem &dp = ctx->dp;
+    const size_t smem = (size_t)kNuWarps * dp.D * dp.M * sizeof(uint16_t);
+    const int64_t blocks = std::min<int64_t>((pl->P + kNuWarps - 1) / kNuWarps, (int64_t)ctx->sms * 16);
+    nextuse_kernel<<<(unsigned)blocks, 32 * kNuWarps, smem, st>>>(dp, *pl, out->status, dp.nextuse);
+    return wf_cuda_check(cudaGetLastError(), "next-use launch");
+}
 
 wf_sweep_cfg wf_sweep_config(const wf_dev_problem &dp)
 {
     wf_sweep_cfg c = {0, 0, 0};
     if (!sweep_usable(dp)) return c;
     const int32_t NS = dp.nslots + 2;
-    const size_t s32 = pc_layout<16, uint32_t>(dp.D, dp.M, dp.W, NS).total;
+    const bool r = dp.reclaim != 0;
+    const size_t s32 = r ? pc_layout<16, uint32_t, 1>(dp.D, dp.M, dp.W, NS).total
+                         : pc_layout<16, uint32_t, 0>(dp.D, dp.M, dp.W, NS).total;
     if (s32 <= 227 * 1024) c.smem32 = s32;
     // The u64 sweep: 16 plans per CTA, or 6 where that keeps more plans per SM.
-    const size_t s16 = pc_layout<16, uint64_t>(dp.D, dp.M, dp.W, NS).total;
-    const size_t s6 = pc_layout<6, uint64_t>(dp.D, dp.M, dp.W, NS).total;
+    const size_t s16 = r ? pc_layout<16, uint64_t, 1>(dp.D, dp.M, dp.W, NS).total
+                         : pc_layout<16, uint64_t, 0>(dp.D, dp.M, dp.W, NS).total;
+    const size_t s6 = r ? pc_layout<6, uint64_t, 1>(dp.D, dp.M, dp.W, NS).total
+                        : pc_layout<6, uint64_t, 0>(dp.D, dp.M, dp.W, NS).total;
     const int a = plans_per_sm(s16, 16), b = plans_per_sm(s6, 6);
     if (a > 0 && a >= b) { c.smem64 = s16; c.plans64 = 16; }
     else if (b > 0) { c.smem64 = s6; c.plans64 = 6; }
@@ -965,6 +1087,7 @@ int wf_launch_sweep(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, con
                     const int32_t **rest_list, const int32_t **rest_count)
 {
     int rc = launch_status(ctx, pl, out, st);
+    if (!rc && ctx->dp.reclaim) rc = wf_launch_nextuse(ctx, pl, out, st);
     if (rc) return rc;
     if (cfg.smem32 && !(wide_first && cfg.smem64)) {
         // u32 times for every plan; the plans that leave 32 bits go on to the

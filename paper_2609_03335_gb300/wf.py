@@ -24,7 +24,7 @@ INT64_MAX = np.iinfo(np.int64).max
 EXPORTS = ("wf_problem_check", "wf_ctx_create", "wf_forecast_readiness", "wf_eval_plans",
            "wf_topk", "wf_ctx_status", "wf_ctx_destroy", "wf_strerror", "wf_last_error",
            "wf_eval_plans_static", "wf_mutate_plans", "wf_merge_elite", "wf_local_search",
-           "wf_construct_plans")
+           "wf_construct_plans", "wf_ctx_set_reclaim")
 
 
 class WfError(RuntimeError):
@@ -81,6 +81,7 @@ def load_library():
         "wf_merge_elite": ([p, p, p, p, p, p], ctypes.c_int),
         "wf_local_search": ([p, p, p, p, p, ctypes.c_uint64, i64, i32, i32, p], ctypes.c_int),
         "wf_construct_plans": ([p, p, ctypes.c_uint64, i64, p], ctypes.c_int),
+        "wf_ctx_set_reclaim": ([p, i32], ctypes.c_int),
         "wf_ctx_status": ([p, p], ctypes.c_int),
         "wf_ctx_destroy": ([p], None),
         "wf_strerror": ([ctypes.c_int], ctypes.c_char_p),
@@ -168,6 +169,9 @@ class Ctx:
         self.ptr = ctypes.c_void_p()
         _check(load_library().wf_ctx_create(ctypes.byref(self.host.c), self.device, self.max_P,
                                             ctypes.byref(self.ptr)), "wf_ctx_create")
+        reclaim = int(getattr(prob, "reclaim", 0))
+        if reclaim:
+            wf_ctx_set_reclaim(self, reclaim)
 
     @property
     def N(self):
@@ -183,6 +187,13 @@ class Ctx:
             self.close()
         except Exception:
             pass
+
+
+RECLAIM_LRU, RECLAIM_NEXT_USE = 0, 1
+
+
+def wf_ctx_set_reclaim(ctx: Ctx, policy: int):
+    _check(load_library().wf_ctx_set_reclaim(ctx.ptr, int(policy)), "wf_ctx_set_reclaim")
 
 
 def wf_ctx_create(prob, device: int = 0, max_P: int = 1) -> Ctx:
