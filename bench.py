@@ -275,6 +275,29 @@ def issue_roofline(eval_ms, clk, sms):
             "frac": achieved / peak, "warp_instructions": inst, "sms": sms, "sm_mhz": mhz}
 
 
+def reclaim_timing(wf, ctx, dp, res_lru, P, stream, flush):
+    """The same batch under reclamation by next use: eval time (next-use pass
+    included) and the batch's mean makespan and GPU time against LRU."""
+    import torch
+    lru = [t.clone() for t in (res_lru.makespan, res_lru.gpu, res_lru.status)]
+    wf.wf_ctx_set_reclaim(ctx, wf.RECLAIM_NEXT_USE)
+    res = wf.Results(P, dp.place.device)
+    e = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    with torch.cuda.stream(stream):
+        wf.wf_eval_plans(ctx, dp, res, stream)
+        flush.zero_()
+        e[0].record(stream)
+        wf.wf_eval_plans(ctx, dp, res, stream)
+        e[1].record(stream)
+    torch.cuda.synchronize()
+    wf.wf_ctx_set_reclaim(ctx, wf.RECLAIM_LRU)
+    ok = (res.status == 0) & (lru[2] == 0)
+    mean = lambda t: float(t[ok].double().mean().item())
+    return {"eval_ms": e[0].elapsed_time(e[1]), "plans": P,
+            "mean_makespan_us": {"lru": mean(lru[0]), "next_use": mean(res.makespan)},
+            "mean_gpu_us": {"lru": mean(lru[1]), "next_use": mean(res.gpu)}}
+
+
 def run_gpu(args, rank, world, local):
     import torch
 
@@ -376,6 +399,7 @@ def run_gpu(args, rank, world, local):
         e1.record(stream)
     torch.cuda.synchronize()
     barrier(world)
+    nextuse = reclaim_timing(wf, ctx, dp, res, P, stream, flush)  # before the search rewrites rows 0..31
     search = local_search_timing(wf, ctx, dp, prob, P, stream, flush, peak_gbs=read_peaks().get("hbm_gbs"))
     built = construct_timing(wf, ctx, prob, P, k, stream, flush, random_best=int(keys[0, 0].item()))
     clk = clocks.stop()
@@ -431,6 +455,7 @@ def run_gpu(args, rank, world, local):
             "gpu_launches": launches,
             "local_search": search,
             "construct": built,
+            "reclaim_next_use": nextuse,
         }
         print(json.dumps(line), flush=True)
     ctx.close()
