@@ -185,14 +185,14 @@ def run_reference(args, rank, world):
     dt = (time.perf_counter() - t0) / args.steps
     value = sample / dt
     line = {
-        "impl": "reference", "metric": METRIC, "value": value, "unit": "plans/s",
+        "impl": "reference", "metric": metric_of(w.problem), "value": value, "unit": "plans/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64",
         "data": "synthetic",
-        "config": {"workload": f"{WORKLOAD}: 64 sessions, N=2000, D=8, M=8; oracle step = first "
-                               f"{sample} plans of the batch", "P": sample, "N": w.problem.N},
+        "config": {"workload": f"{WORKLOAD}: {w.description}; oracle step = first {sample} plans of the batch",
+                   "P": sample, "N": w.problem.N},
         "cpu_baseline": {"value": value, "unit": "plans/s", "cores": 1, "kind": "oracle",
-                         "sample": f"first {sample} plans of the burst batch per step, one thread"},
+                         "sample": f"first {sample} plans of the {WORKLOAD} batch per step, one thread"},
         "e2e": {"value": value, "unit": "plans/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -260,6 +260,13 @@ def construct_timing(wf, ctx, prob, P, k, stream, flush, random_best, jitter=200
             "best_makespan_us": int(keys[0, 0].item()), "random_batch_best_makespan_us": random_best}
 
 
+def metric_of(prob):
+    """The headline metric for the burst workload; the same form for others."""
+    if WORKLOAD == "burst":
+        return METRIC
+    return f"candidate plans evaluated/sec (N={prob.N},D={prob.D}" + (f",S={prob.S})" if prob.S else ")")
+
+
 def issue_roofline(eval_ms, clk, sms):
     """The integer-issue roofline of the evaluation call: its warp
     instructions (ncu, same kernel source) over its CUDA-event time, against
@@ -308,7 +315,7 @@ def run_gpu(args, rank, world, local):
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     w = wfgen.config(WORKLOAD)
-    prob, P, k = w.problem, w.P, w.k
+    prob, P, k = w.problem, (args.plans or w.P), w.k
     plans = wfgen.make_plans(prob, P, w.plan_seed, plan_base=rank * P)
     t0 = time.perf_counter()
     ctx = wf.Ctx(prob, max_P=P, device=local)
@@ -399,7 +406,8 @@ def run_gpu(args, rank, world, local):
         e1.record(stream)
     torch.cuda.synchronize()
     barrier(world)
-    nextuse = reclaim_timing(wf, ctx, dp, res, P, stream, flush)  # before the search rewrites rows 0..31
+    # before the search rewrites rows 0..31; the policy needs deterministic latencies
+    nextuse = reclaim_timing(wf, ctx, dp, res, P, stream, flush) if prob.S == 0 else None
     search = local_search_timing(wf, ctx, dp, prob, P, stream, flush, peak_gbs=read_peaks().get("hbm_gbs"))
     built = construct_timing(wf, ctx, prob, P, k, stream, flush, random_best=int(keys[0, 0].item()))
     clk = clocks.stop()
@@ -415,27 +423,29 @@ def run_gpu(args, rank, world, local):
     # forecast, status, 32-bit sweep, 64-bit sweep over its hand-offs, int64
     # pass over what is left, top-k passes (the count reset is a memset and
     # the count read-back a copy, not kernels)
-    launches = args.steps * (5 + topk_launches(P, k))
+    # (stochastic latencies: forecast, status, sample sweep, int64 pass over
+    # its hand-offs, top-k passes)
+    launches = args.steps * ((5 if prob.S == 0 else 4) + topk_launches(P, k))
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         import oracle
         oracle.build()
-        sample = P
+        sample = P if WORKLOAD == "burst" else min(P, 1024)
         t0 = time.perf_counter()
         oracle.eval_plans(prob, plans, 0, sample)
         dt = time.perf_counter() - t0
         cpu = {"value": sample / dt, "unit": "plans/s", "cores": 1, "kind": "oracle",
-               "sample": f"all {sample} plans of the burst batch, one thread, {dt:.2f} s"}
+               "sample": f"{'all' if sample == P else 'the first'} {sample} plans of the {WORKLOAD} batch, "
+                         f"one thread, {dt:.2f} s"}
 
     if rank == 0:
         line = {
-            "metric": METRIC, "value": P * world / (ms_per_step * 1e-3), "unit": "plans/s",
+            "metric": metric_of(prob), "value": P * world / (ms_per_step * 1e-3), "unit": "plans/s",
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64",
             "data": "synthetic",
-            "config": {"workload": "burst: 64 sessions (Poisson arrivals, mean gap 0.5 s), N=2000, "
-                                   "D=8, M=8, P=16384 plans per GPU, k=32",
+            "config": {"workload": f"{WORKLOAD}: {w.description} plans per GPU (here {P}), k={k}",
                        "P_per_gpu": P, "N": prob.N, "k": k,
                        "l2": "flushed between timed steps (256 MiB write)",
                        "ctx_create_ms": ctx_ms,
@@ -445,8 +455,9 @@ def run_gpu(args, rank, world, local):
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak if peak else None,
                          "traffic": traffic,
-                         "kernel": "wf_eval_plans = status_kernel + pc_kernel (u32 times) + pc_kernel (u64 "
-                                   "times, hand-offs) + eval_list_kernel",
+                         "kernel": ("wf_eval_plans = status_kernel + pc_kernel (u32 times) + pc_kernel (u64 "
+                                    "times, hand-offs) + eval_list_kernel") if prob.S == 0 else
+                                   "wf_eval_plans = status_kernel + stoch_kernel + eval_stoch_kernel (hand-offs)",
                          "algorithmic_bytes_per_plan": bpp, "kernel_ms": eval_ms_mean,
                          "peak_source": "MEASURED_PEAKS.json hbm_gbs (measured copy)" if peak else None},
             "roofline_issue": issue_roofline(eval_ms_mean, clk, torch.cuda.get_device_properties(dev).multi_processor_count),
@@ -468,7 +479,12 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=("gpu", "reference"), default="gpu")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--workload", default="burst", choices=("tiny", "mix", "burst", "stochastic", "large"),
+                    help="the synthetic window (burst is the headline configuration)")
+    ap.add_argument("--plans", type=int, default=0, help="plans per GPU (default: the workload's)")
     args = ap.parse_args()
+    global WORKLOAD
+    WORKLOAD = args.workload
     rank, world, local = dist_setup()
     if args.impl == "reference":
         run_reference(args, rank, world)
