@@ -640,66 +640,68 @@ stoch_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list,
     }
 
     if (warp == tw) {
-        // ---------------- residency, once for all samples (lane 0) ----------------
-        uint32_t *usedp = (uint32_t *)(sm + L.used);
-        Q *queuep = (Q *)(sm + L.queue);
-        uint8_t *nresp = sm + L.nres;
+        // ---------------- residency, once for all samples: lane = device ----------------
+        // Residency is per device, so lane d owns device d's queue, weight
+        // and count in registers and plays the chunk's units on d in
+        // dispatch order; lanes of different devices run side by side.
         __syncthreads();
-        Q q[1];
-        if (lane == 0)
-            for (int32_t d = 0; d < D; ++d) { usedp[d] = 0; queuep[d] = 0; nresp[d] = 0; }
+        Q q = 0;
+        uint32_t n = 0, u_d = 0;
+        const bool dev = lane < D;
+        const uint32_t capd = dev ? (uint32_t)cap[lane] : 0u;
         for (int32_t c = 0; c < chunks; ++c) {
             const int b = c % kBuffers;
             named_sync(kSFullP + b, 64);
             uint32_t *rb = ring + b * kSRec * kSChunk;
             const int32_t kmax = min(kSChunk, N - c * kSChunk);
-            for (int32_t k = 0; k < kmax && lane == 0; ++k) {
+            // The chunk's positions on each device: one ballot per device.
+            const uint32_t r3l = lane < kmax ? rb[3 * kSChunk + lane] : kSkip;
+            const int32_t dl = (r3l & kSkip) ? -1 : (int32_t)(r3l & 31u);
+            uint32_t mine = 0;
+            for (int32_t dd = 0; dd < D; ++dd) {
+                const uint32_t bal = __ballot_sync(0xFFFFFFFFu, dl == dd);
+                if (lane == dd) mine = bal;
+            }
+            while (mine) {
+                const int32_t k = __ffs((int)mine) - 1;
+                mine &= mine - 1;
                 const uint32_t r3 = rb[3 * kSChunk + k];
-                if (r3 & kSkip) continue;
                 uint32_t &r1 = rb[1 * kSChunk + k];
-                const int32_t d = (int32_t)(r3 & 31u);
                 const uint32_t m = (r3 >> 5) & 15u;
-                q[0] = queuep[d];
-                uint32_t n = nresp[d];
-                uint32_t u_d = usedp[d];
                 const uint32_t wm = (uint32_t)weight[m];
-                const uint32_t capd = (uint32_t)cap[d];
                 const bool was_empty = n == 0;
-                const int32_t kq = Lru<Q>::find(q[0], n, m);
+                const int32_t kq = Lru<Q>::find(q, n, m);
                 const bool hit = kq < (int32_t)n;
-                if (hit) { q[0] = Lru<Q>::remove(q[0], kq); n -= 1; }
+                q = hit ? Lru<Q>::remove(q, hit ? kq : 0) : q;  // (an index below the queue length)
+                n -= hit ? 1u : 0u;
                 const uint32_t need = hit ? r1 : wm + r1;
                 uint32_t e = 0;
                 while (u_d + need > capd && e < n) {
-                    u_d -= (uint32_t)weight[(uint32_t)(q[0] >> (4 * e)) & 15u];
+                    u_d -= (uint32_t)weight[(uint32_t)(q >> (4 * e)) & 15u];
                     ++e;
                 }
                 if (u_d + need > capd) atomicExch(dp.err, 2);  // unreachable for a valid plan
-                q[0] = e < (uint32_t)Lru<Q>::kSlots ? (q[0] >> (4 * e)) : (Q)0;
+                q = e < (uint32_t)Lru<Q>::kSlots ? (q >> (4 * e)) : (Q)0;
                 n -= e;
-                q[0] |= (Q)m << (4 * n);
+                q |= (Q)m << (4 * n);
                 n += 1;
                 u_d += hit ? 0u : wm;
                 uint32_t emptied = 0;
                 if ((r3 >> 10) & 1u) {
-                    q[0] &= ~((Q)0xF << (4 * (n - 1)));
+                    q &= ~((Q)0xF << (4 * (n - 1)));
                     n -= 1;
                     u_d -= wm;
                     emptied = n == 0;
                 }
-                queuep[d] = q[0];
-                nresp[d] = (uint8_t)n;
-                usedp[d] = u_d;
                 r1 = (hit ? 1u : 0u) | (was_empty ? 2u : 0u) | (emptied << 2);
             }
+            __syncwarp();
             named_arrive(kSFullR + b, kSTiming + 32);
         }
         uint32_t *hist = (uint32_t *)(sm + L.hist);
-        if (lane == 0) {
-            uint32_t o = 0;
-            for (int32_t d = 0; d < D; ++d) o += nresp[d] != 0;
-            hist[256] = o;  // devices still occupied at the end (same for every sample)
-        }
+        // devices still occupied at the end (the same for every sample)
+        const uint32_t open = __popc(__ballot_sync(0xFFFFFFFFu, dev && n != 0));
+        if (lane == 0) hist[256] = open;
         named_arrive(kSOpen, kSTiming + 32);
         return;
     }
