@@ -27,7 +27,8 @@
 
 namespace {
 
-constexpr int kThreads = 128;
+constexpr int kThreads = 32;     // one warp per CTA, so the plans spread over every SM
+constexpr int kPlansPerSm = 128;  // plans built at once per SM (the scratch is sized for them)
 
 __device__ __forceinline__ uint64_t mix64(uint64_t x)  // SplitMix64 output function
 {
@@ -236,8 +237,8 @@ extern "C" int wf_construct_plans(wf_ctx *c, const wf_plans *out, uint64_t seed,
     if (rc) return rc;
     const wf_dev_problem &dp = c->dp;
     if (!c->construct_scratch) {
-        // First call: per-thread state for up to 128 plans per SM at once.
-        c->construct_threads = std::min<int64_t>(c->max_P, (int64_t)c->sms * kThreads);
+        // First call: per-thread state for up to kPlansPerSm plans per SM at once.
+        c->construct_threads = std::min<int64_t>(c->max_P, (int64_t)c->sms * kPlansPerSm);
         rc = wf_cuda_check(cudaMalloc(&c->construct_scratch, scratch_bytes(dp.N, dp.D, dp.M) * c->construct_threads),
                            "cudaMalloc(constructor scratch)");
         if (rc) { c->construct_scratch = nullptr; return rc; }
