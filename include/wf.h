@@ -92,6 +92,10 @@ typedef struct wf_ctx wf_ctx;
  *     zq = floor(bm_r[h & (bm_rn-1)] * bm_c[(h >> 32) & (bm_cn-1)] / 2^18);
  *     bm_rn and bm_cn must be powers of two, bm_en odd and large enough
  *     for every zq, bm_e >= 0.  Ignored when S == 0.
+ *   margin_mib >= 0: the admission margin epsilon_M of Section 3.3 (memory
+ *     reserved for admission = predicted peak + margin).  Every capacity
+ *     check -- a node fitting a device (Eq. 8) and the admission of a unit
+ *     (Eq. 11) -- uses peak + margin_mib in place of peak.
  */
 typedef struct {
     int32_t N, D, M, W;
@@ -110,6 +114,7 @@ typedef struct {
     uint64_t seed;
     const int32_t *bm_r, *bm_c, *bm_e;
     int32_t bm_rn, bm_cn, bm_en;
+    int32_t margin_mib;
 } wf_problem;
 
 /*

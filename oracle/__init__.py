@@ -111,7 +111,9 @@ class OracleProblem:
             pred_off=_a(prob.pred_off, np.int32), pred_idx=_a(prob.pred_idx, np.int32),
             model=_a(prob.model, np.uint8), session=_a(prob.session, np.int32),
             arrival=_a(prob.arrival_us, np.int64), lat=_a(prob.lat_us, np.int32),
-            peak=_a(prob.peak_mib, np.int32), weight=_a(prob.weight_mib, np.int32),
+            # admission memory (Section 3.3): predicted peak + margin, in every capacity check
+            peak=_a(np.asarray(prob.peak_mib, np.int64) + int(getattr(prob, "margin_mib", 0)), np.int32),
+            weight=_a(prob.weight_mib, np.int32),
             load=_a(prob.load_us, np.int32), cap=_a(prob.cap_mib, np.int32),
             bm_r=_a(prob.bm_r, np.int32), bm_c=_a(prob.bm_c, np.int32), bm_e=_a(prob.bm_e, np.int32))
         if self.arrays["pred_idx"].size == 0:

@@ -74,6 +74,7 @@ static int validate(const wf_problem *pb, wf_derived *dv)
     const int32_t E = pb->pred_off[N];
     REQUIRE(E == 0 || pb->pred_idx, "pred_idx is NULL with E=%d", E);
     REQUIRE(pb->grant_us >= 0, "grant_us < 0");
+    REQUIRE(pb->margin_mib >= 0, "margin_mib < 0");
     for (int32_t m = 0; m < M; ++m) REQUIRE(pb->weight_mib[m] >= 1, "weight_mib[%d] < 1", m);
     for (int32_t d = 0; d < D; ++d) REQUIRE(pb->cap_mib[d] >= 1, "cap_mib[%d] < 1", d);
     for (int64_t i = 0; i < (int64_t)M * D; ++i) REQUIRE(pb->load_us[i] >= 0, "load_us < 0");
@@ -90,7 +91,8 @@ static int validate(const wf_problem *pb, wf_derived *dv)
             REQUIRE(pb->lat_us[i] >= 0, "lat_us[%d][%d] < 0", v, d);
             REQUIRE(pb->peak_mib[i] >= pb->weight_mib[pb->model[v]],
                     "peak_mib[%d][%d] below the model weight", v, d);
-            fits |= pb->peak_mib[i] <= pb->cap_mib[d];
+            REQUIRE((int64_t)pb->peak_mib[i] + pb->margin_mib <= INT32_MAX, "peak_mib + margin_mib overflows");
+            fits |= (int64_t)pb->peak_mib[i] + pb->margin_mib <= pb->cap_mib[d];
         }
         REQUIRE(fits, "activation %d fits on no device", v);
         for (int32_t e = pb->pred_off[v]; e < pb->pred_off[v + 1]; ++e) {
@@ -201,7 +203,11 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
     size_t o_sess = img.add(pb->session, sizeof(int32_t) * N);
     size_t o_arr = img.add(pb->arrival_us, sizeof(int64_t) * W);
     size_t o_lat = img.add(pb->lat_us, sizeof(int32_t) * (size_t)N * D);
-    size_t o_peak = img.add(pb->peak_mib, sizeof(int32_t) * (size_t)N * D);
+    // Admission memory (Section 3.3): predicted peak + margin, used wherever a
+    // capacity is checked.
+    std::vector<int32_t> adm((size_t)N * D);
+    for (size_t i = 0; i < adm.size(); ++i) adm[i] = pb->peak_mib[i] + pb->margin_mib;
+    size_t o_peak = img.add(adm.data(), sizeof(int32_t) * (size_t)N * D);
     size_t o_w = img.add(pb->weight_mib, sizeof(int32_t) * M);
     size_t o_load = img.add(pb->load_us, sizeof(int32_t) * (size_t)M * D);
     size_t o_cap = img.add(pb->cap_mib, sizeof(int32_t) * D);
@@ -227,7 +233,7 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
         noderec[2 * n + 1] = make_int4(a, len, (int32_t)(c0 | (c1 << 16)), 0);
         for (int32_t d = 0; d < D; ++d) {
             const int64_t i = (int64_t)n * D + d;
-            lk[i] = make_int2(pb->lat_us[i], pb->peak_mib[i] - pb->weight_mib[pb->model[n]]);
+            lk[i] = make_int2(pb->lat_us[i], adm[i] - pb->weight_mib[pb->model[n]]);
         }
     }
     size_t o_rec = img.add(noderec.data(), sizeof(int4) * noderec.size());
@@ -261,7 +267,7 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
     std::vector<uint32_t> fitmask(((size_t)N + 3) & ~(size_t)3, 0u);
     for (int32_t n = 0; n < N; ++n)
         for (int32_t d = 0; d < D; ++d)
-            if (pb->peak_mib[(int64_t)n * D + d] <= pb->cap_mib[d]) fitmask[n] |= 1u << d;
+            if (adm[(int64_t)n * D + d] <= pb->cap_mib[d]) fitmask[n] |= 1u << d;
     size_t o_fit = img.add(fitmask.data(), sizeof(uint32_t) * fitmask.size());
     std::vector<uint32_t> edges(E);
     for (int32_t v = 0; v < N; ++v)

@@ -575,6 +575,8 @@ extern "C" int wf_eval_plans_static(const wf_problem *pb, const wf_plans *pl, co
     if (N < 1 || N > 65535 || D < 1 || D > 32 || M < 1 || M > 16 || W < 1)
         return wf_set_error(WF_EINVAL, "sizes outside N 1..65535, D 1..32, M 1..16, W >= 1");
     if (pb->S != 0) return wf_set_error(WF_EINVAL, "wf_eval_plans_static evaluates deterministic problems (S = 0) only");
+    if (pb->margin_mib != 0)
+        return wf_set_error(WF_EINVAL, "wf_eval_plans_static takes no admission margin (fold it into peak_mib)");
     if (!pb->pred_off || !pb->model || !pb->session || !pb->arrival_us || !pb->lat_us || !pb->peak_mib ||
         !pb->weight_mib || !pb->load_us || !pb->cap_mib || pb->grant_us < 0)
         return wf_set_error(WF_EINVAL, "a problem table pointer is NULL or grant_us < 0");

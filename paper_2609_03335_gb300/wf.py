@@ -43,7 +43,8 @@ class wf_problem(ctypes.Structure):
                 ("load_us", ctypes.c_void_p), ("cap_mib", ctypes.c_void_p),
                 ("grant_us", ctypes.c_int32), ("S", ctypes.c_int32), ("seed", ctypes.c_uint64),
                 ("bm_r", ctypes.c_void_p), ("bm_c", ctypes.c_void_p), ("bm_e", ctypes.c_void_p),
-                ("bm_rn", ctypes.c_int32), ("bm_cn", ctypes.c_int32), ("bm_en", ctypes.c_int32)]
+                ("bm_rn", ctypes.c_int32), ("bm_cn", ctypes.c_int32), ("bm_en", ctypes.c_int32),
+                ("margin_mib", ctypes.c_int32)]
 
 
 class wf_plans(ctypes.Structure):
@@ -140,7 +141,8 @@ class HostProblem:
                             ptr["arrival_us"], ptr["lat_us"], ptr["peak_mib"], ptr["weight_mib"],
                             ptr["load_us"], ptr["cap_mib"], int(prob.grant_us), int(prob.S),
                             int(prob.seed) & ((1 << 64) - 1), ptr["bm_r"], ptr["bm_c"], ptr["bm_e"],
-                            int(k["bm_r"].size), int(k["bm_c"].size), int(k["bm_e"].size))
+                            int(k["bm_r"].size), int(k["bm_c"].size), int(k["bm_e"].size),
+                            int(getattr(prob, "margin_mib", 0)))
         self.N, self.D, self.M, self.W, self.S = (int(prob.N), int(prob.D), int(prob.M),
                                                   int(prob.W), int(prob.S))
 
@@ -361,7 +363,8 @@ class DeviceProblem:
         self.c = wf_problem(hp.N, hp.D, hp.M, hp.W, ptr["pred_off"], ptr["pred_idx"], ptr["model"],
                             ptr["session"], ptr["arrival_us"], ptr["lat_us"], ptr["peak_mib"],
                             ptr["weight_mib"], ptr["load_us"], ptr["cap_mib"], int(prob.grant_us),
-                            int(prob.S), int(prob.seed) & ((1 << 64) - 1), None, None, None, 0, 0, 0)
+                            int(prob.S), int(prob.seed) & ((1 << 64) - 1), None, None, None, 0, 0, 0,
+                            int(getattr(prob, "margin_mib", 0)))
 
 
 def wf_eval_plans_static(prob: DeviceProblem, plans: DevicePlans, out: Results, stream=None):

@@ -372,3 +372,26 @@ def test_topk_with_massive_ties():
         want = oracle_eval(w.problem, plans)
         ids, keys = oracle.topk(want["makespan"], want["p95"], want["gpu"], want["status"], k)
         assert np.array_equal(got["ids"], ids) and np.array_equal(got["keys"], keys)
+
+
+@pytest.mark.parametrize("seed", range(3))
+def test_admission_margin(seed):
+    """The admission margin (peak + margin in every capacity check) on random
+    windows and the burst window."""
+    rng = np.random.default_rng(5100 + seed)
+    prob = random_problem(rng, n_sessions=int(rng.integers(1, 6)), D=int(rng.integers(1, 5)))
+    margin = int(rng.integers(1, 400))
+    fits = prob.with_(margin_mib=margin).fits().any(axis=1).all()
+    prob = prob.with_(margin_mib=margin if fits else 0)
+    plans = wfgen.make_plans(prob, int(rng.integers(1, 300)), seed, p_retain=0.5 if seed % 2 else None)
+    if plans.P >= 8:
+        inject_invalid(plans, prob, rng)
+    assert_same(gpu_eval(prob, plans, forecast=True), oracle_eval(prob, plans))
+    w = wfgen.config("burst")
+    prob = w.problem.with_(margin_mib=512)
+    plans = wfgen.make_plans(prob, 1024, seed)
+    got = gpu_eval(prob, plans, k=8, forecast=True)
+    want = oracle_eval(prob, plans)
+    assert_same(got, want)
+    rel, comp = oracle.forecast(prob)
+    assert np.array_equal(got["rel"], rel) and np.array_equal(got["comp"], comp)

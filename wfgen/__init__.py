@@ -100,6 +100,7 @@ class Problem:
     bm_e: np.ndarray = field(default_factory=lambda: np.zeros(0, np.int32))
     name: str = ""
     reclaim: int = 0          # reclamation order: 0 least recently used, 1 by next use
+    margin_mib: int = 0       # admission margin: capacity checks use peak + margin
 
     @property
     def E(self) -> int:
@@ -121,7 +122,7 @@ class Problem:
 
     def fits(self) -> np.ndarray:
         """bool [N][D]: peak memory within device capacity (placement sampling)."""
-        return self.peak_mib.reshape(self.N, self.D) <= self.cap_mib[None, :]
+        return self.peak_mib.reshape(self.N, self.D) + int(self.margin_mib) <= self.cap_mib[None, :]
 
     def with_(self, **kw) -> "Problem":
         d = dict(self.__dict__)
