@@ -393,9 +393,15 @@ int wf_launch_eval(wf_ctx *ctx, const wf_plans *plans, const wf_eval_out *out, c
         if (dp.reclaim && !cfg.smem64)
             return wf_set_error(WF_EINVAL, "reclamation by next use runs only in the shared-memory sweep");
         if (cfg.smem32 || cfg.smem64) {
+            // Under stream capture (a CUDA graph) nothing but launches on the
+            // stream may happen: the path choice stays as it is.
+            cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+            int rc0 = wf_cuda_check(cudaStreamIsCapturing(st, &cs), "stream capture status");
+            if (rc0) return rc0;
+            const bool capturing = cs != cudaStreamCaptureStatusNone;
             // Path choice: the u32 sweep's hand-off count of an earlier call,
             // if it has arrived (never waited for).
-            if (ctx->wide_pending) {
+            if (ctx->wide_pending && !capturing) {
                 const cudaError_t q = cudaEventQuery(ctx->ovf_event);
                 if (q == cudaSuccess) {
                     ctx->prefer_wide = 2 * (int64_t)*ctx->h_ovf > ctx->wide_P;
@@ -412,10 +418,7 @@ int wf_launch_eval(wf_ctx *ctx, const wf_plans *plans, const wf_eval_out *out, c
             if (!rc) rc = wf_launch_sweep(ctx, plans, out, cfg, wide_first, ctx->ovf_count, ctx->ovf_list,
                                           ctx->ovf_list2, st, &rest, &rest_count);
             if (rc) return rc;
-            cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
-            rc = wf_cuda_check(cudaStreamIsCapturing(st, &cs), "stream capture status");
-            if (rc) return rc;
-            if (cfg.smem32 && !wide_first && !ctx->wide_pending && cs == cudaStreamCaptureStatusNone) {
+            if (cfg.smem32 && !wide_first && !ctx->wide_pending && !capturing) {
                 // The read-back runs on the context's side stream after the
                 // sweeps, so the caller's stream never waits for it.  A later
                 // call may reset the count before the copy runs; the value
