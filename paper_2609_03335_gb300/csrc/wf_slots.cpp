@@ -155,7 +155,12 @@ int32_t wf_assign_slots(int32_t N, int32_t W, const int32_t *pred_off, const int
         }
         for (int32_t v : nodes)
             if (soff[v + 1] == soff[v]) writes[v].push_back({w, 1});
-        if (next > 32767) return -1;
+        if (next > 32767) {  // too many slots: the sweep does not apply (empty write lists)
+            wl_off.assign(N + 1, 0);
+            wl.clear();
+            for (int32_t v = 0; v < N; ++v) rslot[v] = -1;
+            return -1;
+        }
     }
     wl_off.assign(N + 1, 0);
     wl.clear();

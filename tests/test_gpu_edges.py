@@ -1,0 +1,138 @@
+"""Edge cases through the C ABI: the largest window, argument errors, padded
+rows, and two contexts working on two streams at once."""
+import numpy as np
+import pytest
+
+import oracle
+import wfgen
+from gpu_util import assert_same, gpu_eval, lib, oracle_eval
+from randprob import random_problem
+
+pytestmark = pytest.mark.gpu
+
+
+def chains_window(lengths, D=2, M=2, seed=0):
+    """Independent chains of the given lengths, one session each (alternating
+    models, so nothing is fusible)."""
+    rng = np.random.default_rng(seed)
+    N = int(sum(lengths))
+    n_sessions = len(lengths)
+    session = np.repeat(np.arange(n_sessions), lengths).astype(np.int32)
+    first = np.r_[0, np.cumsum(lengths)[:-1]]
+    pred_off = np.zeros(N + 1, np.int32)
+    pred_idx = []
+    for v in range(N):
+        if v != first[session[v]]:
+            pred_idx.append(v - 1)
+        pred_off[v + 1] = len(pred_idx)
+    model = (np.arange(N) % M).astype(np.uint8)
+    lat = rng.integers(1, 1000, N * D).astype(np.int32)
+    weight = np.array([2 + m for m in range(M)], np.int32)
+    peak = (weight[model].repeat(D) + rng.integers(0, 3, N * D)).astype(np.int32)
+    return wfgen.Problem(N=N, D=D, M=M, W=n_sessions, pred_off=pred_off, pred_idx=np.array(pred_idx, np.int32),
+                         model=model, session=session,
+                         arrival_us=rng.integers(0, 10000, n_sessions).astype(np.int64), lat_us=lat,
+                         peak_mib=peak, weight_mib=weight, load_us=rng.integers(1, 100, M * D).astype(np.int32),
+                         cap_mib=np.full(D, 12, np.int32))
+
+
+def test_largest_window():
+    """N = 65535, the ABI's limit (beyond the shared-memory sweep, which
+    takes N <= 65534; five sessions of 13,107 activations would also need
+    more finish-time slots than the sweep holds: the exact int64 path runs)."""
+    prob = chains_window([13107] * 5)
+    assert prob.N == 65535
+    plans = wfgen.make_plans(prob, 3, 1)
+    got = gpu_eval(prob, plans, k=2, forecast=True)
+    assert_same(got, oracle_eval(prob, plans))
+    rel, comp = oracle.forecast(prob)
+    assert np.array_equal(got["rel"], rel) and np.array_equal(got["comp"], comp)
+
+
+def test_largest_sweep_window_and_constructor():
+    """N = 65534 in 33 sessions still fits the sweep's 16-bit positions and
+    its slots; the constructor's 16-bit node ids cover it too."""
+    import torch
+    wf = lib()
+    prob = chains_window([2047] * 32 + [30], seed=2)
+    assert prob.N == 65534
+    plans = wfgen.make_plans(prob, 2, 3)
+    assert_same(gpu_eval(prob, plans), oracle_eval(prob, plans))
+    ctx = wf.Ctx(prob, max_P=2)
+    out = wf.DevicePlans.empty(2, prob.N)
+    wf.wf_construct_plans(ctx, out, seed=4, jitter_us=100)
+    torch.cuda.synchronize()
+    want, _ = oracle.construct(prob, 2, seed=4, jitter=100)
+    got = out.numpy(prob.N)
+    assert np.array_equal(got[0], want.place) and np.array_equal(got[1], want.order)
+
+
+def test_argument_errors():
+    import torch
+    wf = lib()
+    w = wfgen.config("tiny")
+    ctx = wf.Ctx(w.problem, max_P=16)
+    plans = wf.DevicePlans.from_host(wfgen.make_plans(w.problem, 16, 0), "cuda")
+    res = wf.Results(16)
+    with pytest.raises(wf.WfError):
+        wf.wf_eval_plans(ctx, plans, res, P=0)
+    big = wf.DevicePlans.from_host(wfgen.make_plans(w.problem, 17, 0), "cuda")
+    with pytest.raises(wf.WfError):
+        wf.wf_eval_plans(ctx, big, wf.Results(17))
+    ids = torch.empty(17, dtype=torch.int32, device="cuda")
+    wf.wf_eval_plans(ctx, plans, res)
+    with pytest.raises(wf.WfError):
+        wf.wf_topk(ctx, res, 16, 17, ids)
+    odd = wf.DevicePlans(plans.place[:, :12], plans.order, plans.fuse, plans.prefetch)  # stride 16 ok
+    wf.wf_eval_plans(ctx, odd, res)
+    bad = wf.DevicePlans(plans.place.reshape(-1)[4:4 + 16 * 12].reshape(16, 12), plans.order, plans.fuse,
+                         plans.prefetch)  # 12-byte rows: stride not a multiple of 16
+    with pytest.raises(wf.WfError):
+        wf.wf_eval_plans(ctx, bad, res)
+    torch.cuda.synchronize()
+    wf.wf_ctx_status(ctx)
+
+
+def test_padded_rows():
+    """Rows with twice the minimal stride give the same results."""
+    import torch
+    wf = lib()
+    w = wfgen.config("mix")
+    host = wfgen.make_plans(w.problem, 300, 8)
+    dense = wf.DevicePlans.from_host(host, "cuda")
+
+    def widen(t):
+        wide = torch.zeros((t.shape[0], 2 * t.shape[1]), dtype=t.dtype, device=t.device)
+        wide[:, :t.shape[1]] = t
+        return wide[:, :t.shape[1]]
+    wide = wf.DevicePlans(widen(dense.place), widen(dense.order), widen(dense.fuse), widen(dense.prefetch))
+    assert wide.place.stride(0) == 2 * dense.place.stride(0)
+    got = gpu_eval(w.problem, host)
+    ctx = wf.Ctx(w.problem, max_P=300)
+    res = wf.Results(300)
+    wf.wf_eval_plans(ctx, wide, res)
+    torch.cuda.synchronize()
+    for a, b in zip(res.numpy(), (got["makespan"], got["p95"], got["gpu"], got["status"])):
+        assert np.array_equal(a, b)
+
+
+def test_two_contexts_on_two_streams():
+    import torch
+    wf = lib()
+    jobs = []
+    for name, seed in (("burst", 1), ("mix", 2)):
+        w = wfgen.config(name)
+        host = wfgen.make_plans(w.problem, 2048, seed)
+        ctx = wf.Ctx(w.problem, max_P=2048)
+        dp = wf.DevicePlans.from_host(host, "cuda")
+        jobs.append((w.problem, host, ctx, dp, wf.Results(2048), torch.cuda.Stream()))
+    torch.cuda.synchronize()
+    for _ in range(3):
+        for prob, host, ctx, dp, res, s in jobs:
+            with torch.cuda.stream(s):
+                wf.wf_eval_plans(ctx, dp, res, s)
+    torch.cuda.synchronize()
+    for prob, host, ctx, dp, res, s in jobs:
+        want = oracle.eval_plans(prob, host, threads=8)
+        for a, b in zip(res.numpy(), want):
+            assert np.array_equal(a, b)
