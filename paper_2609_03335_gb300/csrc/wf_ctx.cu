@@ -247,6 +247,7 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
     // arrival (u32: the sweep runs only with arrivals below 2^32); the first
     // two write codes, the sink slot nslots standing in for absent ones.
     std::vector<uint4> hrec(N);
+    std::vector<uint32_t> wc23(N, 0);
     if (nslots > 0) {
         const uint32_t trash = (uint32_t)nslots, zero = trash + 1;
         for (int32_t n = 0; n < N; ++n) {
@@ -256,9 +257,11 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
             const uint32_t c0 = len > 0 ? wl[a] : trash, c1 = len > 1 ? wl[a + 1] : trash;
             hrec[n] = make_uint4(links[n], rs | ((uint32_t)pb->model[n] << 16) | ((uint32_t)std::min(len, 7) << 20),
                                  (uint32_t)pb->arrival_us[pb->session[n]], c0 | (c1 << 16));
+            wc23[n] = (len > 2 ? wl[a + 2] : trash) | ((uint32_t)(len > 3 ? wl[a + 3] : trash) << 16);
         }
     }
     size_t o_hrec = img.add(hrec.data(), sizeof(uint4) * N);
+    size_t o_wc23 = img.add(wc23.data(), sizeof(uint32_t) * N);
     size_t o_wloff = img.add(wl_off.data(), sizeof(int32_t) * (N + 1));
     size_t o_wl = img.add(wl.data(), sizeof(uint16_t) * wl.size());
     size_t o_lk = img.add(lk.data(), sizeof(int2) * lk.size());
@@ -358,6 +361,7 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
     dp.lk = (const int2 *)(base + o_lk);
     dp.links = (const uint32_t *)(base + o_links);
     dp.hrec = (const uint4 *)(base + o_hrec);
+    dp.wc23 = (const uint32_t *)(base + o_wc23);
     dp.fitmask = (const uint32_t *)(base + o_fit);
     dp.edges = (const uint32_t *)(base + o_edges);
     dp.succ_off = (const int32_t *)(base + o_soff);

@@ -3,14 +3,15 @@
 // Deterministic plans (pc_kernel): a CTA plays 16 plans as a three-stage warp
 // pipeline over 16 dispatch positions at a time.  Producer warps turn each
 // (plan, position) into a unit record (Eq. 3-4 chain, write list, release
-// slot); one residency warp settles LRU model residency under capacity
-// (Eq. 11) with lane = plan; one timing warp plays releases, loads, starts and
-// finishes (Eq. 2, 5, 7, 10) with lane = plan.  Records pass through a ring of
-// three buffers guarded by named barriers.  Per-plan state lives in shared
-// memory, interleaved [index][plan]:
+// slot); two residency warps settle LRU model residency under capacity
+// (Eq. 11) with four lanes per plan, each playing its own devices' units;
+// one timing warp plays releases, loads, starts and finishes (Eq. 2, 5, 7,
+// 10) with lane = plan.  Records pass through a ring of four buffers guarded
+// by named barriers.  Per-plan state lives in shared memory:
 //   - finish-time slots (u32 microseconds) assigned statically from the DAG
-//     (wf_slots.cpp) instead of one word per activation;
-//   - per device: free time, resident weights, resident count, LRU queue.
+//     (wf_slots.cpp) instead of one word per activation, [slot][plan];
+//   - per device: free time [device][plan]; resident weights, count and LRU
+//     queue [device row][residency lane].
 // Status bits (Eq. 8-10) come first from status_kernel, a warp per plan.
 //
 // Stochastic latencies (stoch_kernel): one plan per CTA, the same pipeline
@@ -77,21 +78,37 @@ __device__ __forceinline__ uint32_t bit_of_g(const uint32_t *row, int32_t n)
 }
 
 // CTA shape, a three-stage pipeline over kChunk dispatch positions at a time:
-// warps 2..kProducers+1 prepare the unit records of kP plans (lane =
-// position) into a ring of kBuffers buffers; warp 1 settles model residency
-// (lane = plan: hits, reclamations, occupancy changes); warp 0 plays the
-// timing (lane = plan: releases, starts, finishes, slots).  With u32 times
-// and 16 plans per CTA, four CTAs share an SM at 2,000 activations; the u64
-// variant holds fewer plans per CTA when its slots need the room.
+// the last kProducers warps prepare the unit records of kP plans (lane =
+// position) into a ring of kBuffers buffers; warps 1..kRes settle model
+// residency (lane = plan and device group: hits, reclamations, occupancy
+// changes); warp 0 plays the timing (lane = plan: releases, starts,
+// finishes, slots).  With u32 times and 16 plans per CTA, four CTAs share an
+// SM at 2,000 activations; the u64 variant holds fewer plans per CTA when its
+// slots need the room.
 constexpr int kChunk = 16;
 constexpr int kPlansPerIter = 32 / kChunk;  // plans a producer warp covers per iteration
-constexpr int kBuffers = 3;
+constexpr int kPlans32 = 16;                // plans per CTA of the u32 sweep
+// Record buffers of the ring: four, or three under reclamation by next use,
+// whose seventh record word would otherwise cost a CTA per SM at 2,000
+// activations.  Named barriers: kFullP + b (producers -> residency), kFullR +
+// b (residency -> timing), kEmpty + b (timing -> producers) for buffer b;
+// kOpen (residency -> timing, once at the end).
+template <int kReclaim>
+struct Ring {
+    static constexpr int kBuffers = kReclaim ? 3 : 4;
+    static constexpr int kFullP = 1, kFullR = kFullP + kBuffers, kEmpty = kFullR + kBuffers, kOpen = kEmpty + kBuffers;
+    static_assert(kOpen < 16, "named barriers");
+};
 constexpr int kRecWords = 6;
 
 template <int kP>
 struct PcShape {
-    static constexpr int kProducers = kP >= 6 ? 3 : 2;
-    static constexpr int kWarps = 2 + kProducers;
+    static constexpr int kProducers = kP >= 32 ? 8 : kP >= 16 ? 4 : kP >= 6 ? 3 : 2;
+    static constexpr int kRes = kP >= 32 ? 4 : kP >= 16 ? 2 : 1;  // residency warps
+    static constexpr int kWarps = 1 + kRes + kProducers;
+    // Four 16-plan CTAs share an SM (shared memory allows it at 2,000
+    // activations), which bounds the registers per thread.
+    static constexpr int kMinBlocks = kP >= 32 ? 2 : kP >= 16 ? 4 : 1;
     // Words per (word, position) row of the ring.  A producer store covers 16
     // positions x 2 plans; a pitch of 2 (mod 4) puts those 32 words in 32
     // distinct banks, and the consumers' plan-major loads are contiguous.
@@ -109,16 +126,30 @@ struct PcShape {
 //      | first write code << 16; the residency stage clears the prefetch bit
 //      on a hit and sets kWasEmpty (bit 10) and kEmptied (bit 15) for timing
 //   w4 second write code | third write code << 16
-//   w5 the unit's last member (its full write list when it has more than
-//      three codes) | release slot code << 16 (bit 31: accumulator; 0xFFFF: none)
+//   w5 the unit's last member | release slot code << 16 (bit 31: accumulator;
+//      0xFFFF: none); in the batched producer's records the low half holds
+//      the fourth write code instead when the unit writes exactly four (with
+//      five or more, the timing stage reads the last member's list)
 constexpr uint32_t kSkip = 1u << 14;
 constexpr uint32_t kPrefetch = 1u << 9;
 constexpr uint32_t kWasEmpty = 1u << 10;   // after residency: a miss on an empty device
 constexpr uint32_t kEmptied = 1u << 15;    // after residency: the unit's reclaim empties the device
 constexpr uint32_t kRunCap = 0xFFFFFFFFu;  // saturation of w0
 
+// Residency lanes per plan: a device group each (d = g mod kG), or one lane
+// for every device under reclamation by next use.
+// A lane's state for its t-th device (d = g + t kG) sits at [t][lane]: the
+// lanes of a warp touch consecutive words.
+template <int kP, int kReclaim>
+struct PcGroups {
+    static constexpr int kG = kReclaim ? 1 : (32 * PcShape<kP>::kRes) / kP;
+    static constexpr int kLanes = kG == 1 ? kP : 32 * PcShape<kP>::kRes;  // row length of the state
+    static_assert(kG >= 1 && kG * kP <= 32 * PcShape<kP>::kRes, "residency lanes");
+    __host__ __device__ static int32_t rows(int32_t D) { return (D + kG - 1) / kG; }
+};
+
 struct PcLayout {
-    uint32_t weight, cap, load, arr, ring, slots, tfree, used, queue, nres, open, flag, nuse, rcnt, total;
+    uint32_t weight, cap, load, arr, ring, slots, tfree, used, queue, nres, open, flag, nuse, rcnt, gmask, total;
 };
 
 // Shared memory of a CTA of kP plans with TT times and NS slots per plan;
@@ -135,24 +166,22 @@ __host__ __device__ inline PcLayout pc_layout(int32_t D, int32_t M, int32_t W, i
     l.cap = o; o += round16(4u * D);
     l.load = o; o += round16(4u * M * D);
     l.arr = o; o += round16(4u * W);
-    l.ring = o; o += round16(4u * kBuffers * (kRecWords + kReclaim) * kChunk * PcShape<kP>::kPitch);
+    l.ring = o; o += round16(4u * Ring<kReclaim>::kBuffers * (kRecWords + kReclaim) * kChunk * PcShape<kP>::kPitch);
     l.slots = o; o += round16(t * (uint32_t)NS * kP);
     l.tfree = o; o += round16(t * D * kP);
-    l.used = o; o += round16(4u * D * kP);
-    l.queue = o; o += round16((M <= 8 ? 4u : 8u) * D * kP);  // Lru<uint32_t> or Lru<uint64_t>
-    l.nres = o; o += round16((uint32_t)D * kP);
+    const uint32_t rs = (uint32_t)(PcGroups<kP, kReclaim>::rows(D) * PcGroups<kP, kReclaim>::kLanes);
+    l.used = o; o += round16(4u * rs);
+    l.queue = o; o += round16((M <= 8 ? 4u : 8u) * rs);  // Lru<uint32_t> or Lru<uint64_t>
+    l.nres = o; o += round16(rs);
     l.open = o; o += round16(4u * kP);
     l.flag = o; o += 16;
     l.nuse = o; o += kReclaim ? round16(2u * D * M * kP) : 0u;
     l.rcnt = o; o += kReclaim ? round16((uint32_t)M * kP) : 0u;
+    l.gmask = o; o += round16(4u * Ring<kReclaim>::kBuffers * PcGroups<kP, kReclaim>::kG * kP);
     l.total = o;
     return l;
 }
 
-// Named barriers: kFullP + b (producers -> residency), kFullR + b (residency
-// -> timing), kEmpty + b (timing -> producers) for ring buffer b; kOpen
-// (residency -> timing, once at the end).
-constexpr int kFullP = 1, kFullR = kFullP + kBuffers, kEmpty = kFullR + kBuffers, kOpen = kEmpty + kBuffers;
 
 __device__ __forceinline__ void named_sync(int id, int threads)
 {
@@ -235,7 +264,7 @@ __device__ __forceinline__ void produce(const wf_dev_problem &dp, const PlanPtrs
         s = sr.x >> 16;
     }
     const uint32_t nwl = (ty >> 20) & 7u;
-    const uint32_t c2 = nwl > 2 ? (uint32_t)__ldg(dp.wl + __ldg(dp.wl_off + tail) + 2) : 0u;
+    const uint32_t c2 = __ldg(dp.wc23 + tail) & 0xFFFFu;
     const uint32_t pf = (pw >> (h & 31)) & 1u;
     const uint32_t reclaim = r.retain ? !bit_of_g(r.retain, tail) : 0u;
     rec[0] = ovf ? kRunCap : run;
@@ -247,6 +276,104 @@ __device__ __forceinline__ void produce(const wf_dev_problem &dp, const PlanPtrs
     rec[5] = (uint32_t)tail | (hr.y << 16);
 }
 
+// Row of one plan for the batched producer: placement and dispatch rows, and
+// the byte offset of its fusion / prefetch / retain bit rows.
+struct RowPtrs {
+    const uint8_t *place;
+    const uint16_t *order;
+    int64_t boff;
+};
+
+__device__ __forceinline__ const uint32_t *bits_row(const uint32_t *base, int64_t boff)
+{
+    return (const uint32_t *)((const uint8_t *)base + boff);
+}
+
+// The records of kI (plan, position) pairs at once, with the gathers of all
+// pairs issued together in three dependent rounds: the head's own tables
+// (placement, node record, fusion / prefetch / retain words, third and
+// fourth write codes); then its run time and KV on its device and the placement and fusion
+// bit of its fusible neighbours; then the rare fused chain, walked as in
+// produce().  Each record goes to the ring as soon as it is complete; act[j]
+// false leaves a skip record.  dev[j] is the unit's device (all ones for a
+// skip record).
+template <int kI, int kPitch>
+__device__ __forceinline__ void produce_batch(const wf_dev_problem &dp, const wf_plans &pl, const RowPtrs *rp,
+                                              const bool *act, const int32_t *hh, uint32_t *rb, int pos,
+                                              const int *qq, uint32_t *dev)
+{
+    const int32_t D = dp.D;
+    uint32_t d[kI], fw[kI], pw[kI], rw[kI], c2[kI];
+    uint4 hr[kI];
+#pragma unroll
+    for (int j = 0; j < kI; ++j) {
+        const int32_t h = hh[j];
+        d[j] = act[j] ? __ldg(rp[j].place + h) : 0u;
+        hr[j] = act[j] ? __ldg(dp.hrec + h) : make_uint4(0xFFFFFFFFu, 0, 0, 0);
+        fw[j] = act[j] ? __ldg(bits_row(pl.fuse, rp[j].boff) + (h >> 5)) : 0u;
+        pw[j] = act[j] ? __ldg(bits_row(pl.prefetch, rp[j].boff) + (h >> 5)) : 0u;
+        rw[j] = act[j] && pl.retain ? __ldg(bits_row(pl.retain, rp[j].boff) + (h >> 5)) : 0xFFFFFFFFu;
+        c2[j] = act[j] ? __ldg(dp.wc23 + h) : 0u;
+    }
+    int2 lk0[kI];
+    uint32_t pprev[kI], fnx[kI], pnx[kI];
+#pragma unroll
+    for (int j = 0; j < kI; ++j) {
+        const uint32_t fp = hr[j].x & 0xFFFFu, s = hr[j].x >> 16;
+        lk0[j] = act[j] ? __ldg(dp.lk + hh[j] * D + (int32_t)d[j]) : make_int2(0, 0);
+        pprev[j] = act[j] && fp != 0xFFFFu ? __ldg(rp[j].place + fp) : 0xFFFFFFFFu;  // never a device
+        fnx[j] = act[j] && s != 0xFFFFu ? __ldg(bits_row(pl.fuse, rp[j].boff) + (s >> 5)) : 0u;
+        pnx[j] = act[j] && s != 0xFFFFu ? __ldg(rp[j].place + s) : 0xFFFFFFFFu;
+    }
+#pragma unroll
+    for (int j = 0; j < kI; ++j) {
+        dev[j] = 0xFFFFFFFFu;
+        if (qq[j] < 0) continue;  // a lane beyond the CTA's plans
+        uint32_t *dst = rb + pos * kPitch + qq[j];
+        const int32_t h = hh[j];
+        const uint32_t s0 = hr[j].x >> 16;
+        if (!act[j] || (((fw[j] >> (h & 31)) & 1u) && pprev[j] == d[j])) {  // no unit, or inside its head's
+#pragma unroll
+            for (int w = 0; w < kRecWords; ++w) dst[w * kChunk * kPitch] = w == 3 ? kSkip : 0u;
+            continue;
+        }
+        uint32_t run = (uint32_t)lk0[j].x + (uint32_t)dp.grant, ovf = 0;  // both < 2^31: no wrap
+        int32_t kv = lk0[j].y, tail = h;
+        uint32_t ty = hr[j].y, tw = hr[j].w, c2t = c2[j], rwt = rw[j];
+        if (s0 != 0xFFFFu && ((fnx[j] >> (s0 & 31)) & 1u) && pnx[j] == d[j]) {  // Eq. 3 chain
+            const uint32_t *fuse = bits_row(pl.fuse, rp[j].boff);
+            for (uint32_t s = s0; s != 0xFFFFu;) {
+                if (s != s0 && (!bit_of_g(fuse, s) || __ldg(rp[j].place + s) != d[j])) break;
+                const int2 lk = __ldg(dp.lk + s * D + d[j]);
+                const uint4 sr = __ldg(dp.hrec + s);
+                const uint32_t r2 = run + (uint32_t)lk.x;
+                ovf |= r2 < run;
+                run = r2;
+                kv = max(kv, lk.y);
+                tail = (int32_t)s;
+                ty = sr.y;
+                tw = sr.w;
+                s = sr.x >> 16;
+            }
+            c2t = __ldg(dp.wc23 + tail);
+            rwt = pl.retain ? __ldg(bits_row(pl.retain, rp[j].boff) + (tail >> 5)) : 0xFFFFFFFFu;
+        }
+        const uint32_t nwl = (ty >> 20) & 7u;
+        const uint32_t pf = (pw[j] >> (h & 31)) & 1u;
+        const uint32_t reclaim = ((rwt >> (tail & 31)) & 1u) ^ 1u;
+        dst[0 * kChunk * kPitch] = ovf ? kRunCap : run;
+        dst[1 * kChunk * kPitch] = (uint32_t)kv;
+        dst[2 * kChunk * kPitch] = hr[j].z;
+        dst[3 * kChunk * kPitch] =
+            d[j] | (((hr[j].y >> 16) & 15u) << 5) | (pf << 9) | (reclaim << 10) | (nwl << 11) | (tw << 16);
+        dev[j] = d[j];
+        dst[4 * kChunk * kPitch] = (tw >> 16) | (c2t << 16);
+        dst[5 * kChunk * kPitch] = (nwl == 4 ? c2t >> 16 : (uint32_t)tail) | (hr[j].y << 16);
+    }
+}
+
+// A finish time into a slot: an accumulator keeps the latest of its
+// writers, any other slot takes the value.
 template <typename TT, int kS>
 __device__ __forceinline__ void publish(TT *slots, uint32_t code, TT c)
 {
@@ -261,7 +388,7 @@ __device__ __forceinline__ void publish(TT *slots, uint32_t code, TT c)
 // TT = uint64_t: only a unit whose summed run time reaches 2^32 - 1 sends its
 // plan to ovf_list.
 template <typename Q, typename TT, int kP, int kReclaim>
-__global__ void __launch_bounds__(32 * PcShape<kP>::kWarps)
+__global__ void __launch_bounds__(32 * PcShape<kP>::kWarps, PcShape<kP>::kMinBlocks)
 pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_list, const int32_t *in_count,
           int32_t *ovf_list, int32_t *ovf_count)
 {
@@ -269,7 +396,12 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
     using S = PcShape<kP>;
     constexpr int kPitch = S::kPitch;
     constexpr int kProdThreads = 32 * S::kProducers;
+    constexpr int kResThreads = 32 * S::kRes;
     constexpr bool kNarrow = sizeof(TT) == 4;
+    constexpr int kG = PcGroups<kP, kReclaim>::kG;  // residency lanes per plan
+    using RG = Ring<kReclaim>;
+    constexpr int kBuffers = RG::kBuffers, kFullP = RG::kFullP, kFullR = RG::kFullR, kEmpty = RG::kEmpty,
+                  kOpen = RG::kOpen;
     extern __shared__ __align__(128) uint8_t sm[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int32_t N = dp.N, D = dp.D, M = dp.M, W = dp.W;
@@ -284,6 +416,8 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
     int32_t *cap = (int32_t *)(sm + L.cap);
     int32_t *load = (int32_t *)(sm + L.load);
     uint32_t *arrival = (uint32_t *)(sm + L.arr);
+    uint32_t *open = (uint32_t *)(sm + L.open);
+    uint32_t *gmask = (uint32_t *)(sm + L.gmask);  // [buffer][device group][plan]
     for (int32_t k = threadIdx.x; k < M; k += blockDim.x) weight[k] = __ldg(dp.weight + k);
     for (int32_t k = threadIdx.x; k < D; k += blockDim.x) cap[k] = __ldg(dp.cap + k);
     for (int32_t k = threadIdx.x; k < M * D; k += blockDim.x) load[k] = __ldg(dp.load + k);
@@ -293,91 +427,123 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
   for (int64_t j0 = (int64_t)blockIdx.x * kP; j0 < total; j0 += (int64_t)gridDim.x * kP) {
     const int ng = (int)(total - j0 < kP ? total - j0 : kP);
     if (threadIdx.x == 0) *gave_up = 0;
+    if (threadIdx.x < kP) open[threadIdx.x] = 0;
 
-    // Lanes at or beyond kP own no plan and touch no per-plan state.
-    const bool mine = lane < kP;
-    const int64_t p = (mine && lane < ng) ? (in_list ? (int64_t)in_list[j0 + lane] : j0 + lane) : 0;
-    const bool live = warp < 2 && mine && lane < ng && out.status[p] == 0;
-
-    if (warp >= 2) {
+    if (warp > S::kRes) {
         // ---------------- producers: lane = dispatch position ----------------
         __syncthreads();
+        const int pw = warp - 1 - S::kRes;
         const int pos = lane % kChunk, sub = lane / kChunk;
         // The plans this lane serves, fixed for the whole sweep: row pointers
         // and whether the plan is live, resolved once.
         constexpr int kStep = S::kProducers * kPlansPerIter;
         constexpr int kIters = (kP + kStep - 1) / kStep;
-        PlanPtrs rp[kIters];
+        RowPtrs rp[kIters];
         bool okq[kIters];
+        int qq[kIters];
         int64_t qplan[kIters];
 #pragma unroll
         for (int j = 0; j < kIters; ++j) {
-            const int q = (warp - 2) * kPlansPerIter + j * kStep + sub;
+            const int q = pw * kPlansPerIter + j * kStep + sub;
+            qq[j] = q < kP ? q : -1;
             okq[j] = q < kP && q < ng;
             qplan[j] = 0;
+            rp[j].place = nullptr;
+            rp[j].order = nullptr;
+            rp[j].boff = 0;
             if (okq[j]) {
                 const int64_t pq = in_list ? (int64_t)__ldg(in_list + j0 + q) : j0 + q;
                 qplan[j] = pq;
                 okq[j] = __ldg(out.status + pq) == 0;
                 rp[j].place = pl.place + pq * pl.place_stride;
                 rp[j].order = (const uint16_t *)((const uint8_t *)pl.order + pq * pl.order_stride);
-                rp[j].fuse = (const uint32_t *)((const uint8_t *)pl.fuse + pq * pl.bits_stride);
-                rp[j].prefetch = (const uint32_t *)((const uint8_t *)pl.prefetch + pq * pl.bits_stride);
-                rp[j].retain = pl.retain ? (const uint32_t *)((const uint8_t *)pl.retain + pq * pl.bits_stride)
-                                         : nullptr;
+                rp[j].boff = pq * pl.bits_stride;
             }
         }
+        // Dispatch entries are read one chunk ahead of their use.
+        int32_t h0[kIters];
+#pragma unroll
+        for (int j = 0; j < kIters; ++j) h0[j] = okq[j] && pos < N ? __ldg(rp[j].order + pos) : 0;
         for (int32_t c = 0; c < chunks; ++c) {
             const int b = c % kBuffers;
             if (c >= kBuffers) named_sync(kEmpty + b, kProdThreads + 32);  // timing released buffer b
             const bool quit = kNarrow && *gave_up;
             uint32_t *rb = ring + b * kRW * kChunk * kPitch;
             const int32_t i = c * kChunk + pos;
+            int32_t h1[kIters];
+            bool act[kIters];
 #pragma unroll
             for (int j = 0; j < kIters; ++j) {
-                const int q = (warp - 2) * kPlansPerIter + j * kStep + sub;
-                if (q >= kP) continue;
-                uint32_t rec[kRecWords] = {0, 0, 0, kSkip, 0, 0};
-                if (okq[j] && i < N && !quit) produce(dp, rp[j], i, rec);
-#pragma unroll
-                for (int w = 0; w < kRecWords; ++w) rb[(w * kChunk + pos) * kPitch + q] = rec[w];
-                if (kReclaim)  // the next use of this unit's model on its device
-                    rb[(kRecWords * kChunk + pos) * kPitch + q] =
-                        (okq[j] && i < N && !quit) ? (uint32_t)__ldg(dp.nextuse + qplan[j] * (int64_t)N + i)
-                                                   : 0xFFFFu;
+                h1[j] = okq[j] && i + kChunk < N && !quit ? __ldg(rp[j].order + i + kChunk) : 0;
+                act[j] = okq[j] && i < N && !quit;
+                if (kReclaim && qq[j] >= 0)  // the next use of this unit's model on its device
+                    rb[(kRecWords * kChunk + pos) * kPitch + qq[j]] =
+                        act[j] ? (uint32_t)__ldg(dp.nextuse + qplan[j] * (int64_t)N + i) : 0xFFFFu;
             }
-            named_arrive(kFullP + b, kProdThreads + 32);  // buffer b is full
+            uint32_t dev[kIters];
+            produce_batch<kIters, kPitch>(dp, pl, rp, act, h0, rb, pos, qq, dev);
+            // For each residency lane, the chunk's units on its devices: one
+            // ballot per device group; each half-warp holds one plan.
+#pragma unroll
+            for (int j = 0; j < kIters; ++j) {
+                const uint32_t key = dev[j] == 0xFFFFFFFFu ? (uint32_t)kG : dev[j] % kG;
+#pragma unroll
+                for (int gg = 0; gg < kG; ++gg) {
+                    const uint32_t bal = __ballot_sync(0xFFFFFFFFu, key == (uint32_t)gg);
+                    if (pos == gg && qq[j] >= 0) gmask[(b * kG + gg) * kP + qq[j]] = (bal >> (kChunk * sub)) & 0xFFFFu;
+                }
+            }
+#pragma unroll
+            for (int j = 0; j < kIters; ++j) h0[j] = h1[j];
+            named_arrive(kFullP + b, kProdThreads + kResThreads);  // buffer b is full
         }
         // Match the timing stage's releases of the last buffers.
         for (int32_t c = chunks; c < chunks + kBuffers; ++c)
             if (c >= kBuffers) named_sync(kEmpty + c % kBuffers, kProdThreads + 32);
-    } else if (warp == 1) {
-        // ---------------- residency: lane = plan (Eq. 11, Section 3.5) ----------------
-        uint32_t *used = (uint32_t *)(sm + L.used) + lane;
-        Q *queue = (Q *)(sm + L.queue) + lane;
-        uint8_t *nres = sm + L.nres + lane;
-        uint16_t *nuse = (uint16_t *)(sm + L.nuse) + lane;  // [device][model][plan]
-        uint8_t *rcnt = sm + L.rcnt + lane;                 // [model][plan]
-        if (mine) {
-            for (int32_t d = 0; d < D; ++d) { used[d * kP] = 0; queue[d * kP] = 0; nres[d * kP] = 0; }
+    } else if (warp >= 1) {
+        // ---------------- residency (Eq. 11, Section 3.5) ----------------
+        // Lane (plan, device group): kG lanes per plan, and lane g plays the
+        // plan's units on the devices d = g (mod kG) in dispatch order;
+        // under least-recently-used reclamation devices do not interact.
+        // Reclamation by next use counts a model's copies over all devices,
+        // so there one lane per plan plays every device.  The producers
+        // leave each lane's units of the chunk as a mask (gmask).
+        const int rl = (warp - 1) * 32 + lane;
+        const int qp = rl / kG, g = rl % kG;
+        const bool rmine = qp < kP;
+        const int64_t p = (rmine && qp < ng) ? (in_list ? (int64_t)in_list[j0 + qp] : j0 + qp) : 0;
+        const bool live = rmine && qp < ng && out.status[p] == 0;
+        constexpr int kRow = PcGroups<kP, kReclaim>::kLanes;
+        uint32_t *used = (uint32_t *)(sm + L.used) + rl;  // [device / kG][lane]
+        Q *queue = (Q *)(sm + L.queue) + rl;
+        uint8_t *nres = sm + L.nres + rl;
+        uint16_t *nuse = (uint16_t *)(sm + L.nuse) + qp;  // [device][model][plan]
+        uint8_t *rcnt = sm + L.rcnt + qp;                 // [model][plan]
+        if (rmine) {
+            for (int32_t t = 0; t * kG + g < D; ++t) { used[t * kRow] = 0; queue[t * kRow] = 0; nres[t * kRow] = 0; }
             if (kReclaim)
                 for (int32_t k = 0; k < M; ++k) rcnt[k * kP] = 0;
         }
         __syncthreads();
         for (int32_t c = 0; c < chunks; ++c) {
             const int b = c % kBuffers;
-            named_sync(kFullP + b, kProdThreads + 32);
-            uint32_t *rb = ring + b * kRW * kChunk * kPitch + lane;
-            const int32_t kmax = min(kChunk, N - c * kChunk);
-            for (int32_t k = 0; k < kmax && live; ++k) {
-                const uint32_t r3 = rb[(3 * kChunk + k) * kPitch];
-                if (r3 & kSkip) continue;
-                uint32_t &r1 = rb[(1 * kChunk + k) * kPitch];
+            named_sync(kFullP + b, kProdThreads + kResThreads);
+            uint32_t *rb = ring + b * kRW * kChunk * kPitch + qp;
+            uint32_t todo = live ? gmask[(b * kG + g) * kP + qp] : 0u;
+            // The ring words of the lane's next unit are read while this one plays.
+            int32_t k = todo ? __ffs((int)todo) - 1 : 0;
+            uint32_t r3 = todo ? rb[(3 * kChunk + k) * kPitch] : 0u;
+            uint32_t r1 = todo ? rb[(1 * kChunk + k) * kPitch] : 0u;
+            while (todo) {
+                todo &= todo - 1;
+                const int32_t kn = todo ? __ffs((int)todo) - 1 : k;
+                const uint32_t n3 = rb[(3 * kChunk + kn) * kPitch], n1 = rb[(1 * kChunk + kn) * kPitch];
                 const int32_t d = (int32_t)(r3 & 31u);
                 const uint32_t m = (r3 >> 5) & 15u;
-                Q q = queue[d * kP];
-                uint32_t n = nres[d * kP];
-                uint32_t u_d = used[d * kP];  // used + need <= cap + peak < 2^32
+                const int32_t t = d / kG;
+                Q q = queue[t * kRow];
+                uint32_t n = nres[t * kRow];
+                uint32_t u_d = used[t * kRow];  // used + need <= cap + peak < 2^32
                 const uint32_t wm = (uint32_t)weight[m];
                 const uint32_t capd = (uint32_t)cap[d];
                 const bool was_empty = n == 0;
@@ -443,26 +609,31 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
                     emptied = n == 0;
                     if (kReclaim) rcnt[m * kP] -= 1;
                 }
-                queue[d * kP] = q;
-                nres[d * kP] = (uint8_t)n;
-                used[d * kP] = u_d;
+                queue[t * kRow] = q;
+                nres[t * kRow] = (uint8_t)n;
+                used[t * kRow] = u_d;
                 // For timing: the load to wait for (none on a hit, Eq. 5) and
                 // the occupancy changes of section 4.3.
-                r1 = hit ? 0u : (uint32_t)load[m * D + d];
+                rb[(1 * kChunk + k) * kPitch] = hit ? 0u : (uint32_t)load[m * D + d];
                 rb[(3 * kChunk + k) * kPitch] = (r3 & ~(kPrefetch | kWasEmpty)) | (hit ? 0u : (r3 & kPrefetch)) |
                                                 (was_empty ? kWasEmpty : 0u) | (emptied ? kEmptied : 0u);
+                k = kn;
+                r3 = n3;
+                r1 = n1;
             }
-            named_arrive(kFullR + b, 64);
+            named_arrive(kFullR + b, kResThreads + 32);
         }
-        uint32_t *open = (uint32_t *)(sm + L.open);
-        if (live) {
+        if (live) {  // devices still occupied at the end
             uint32_t o = 0;
-            for (int32_t d = 0; d < D; ++d) o += nres[d * kP] != 0;
-            open[lane] = o;
+            for (int32_t t = 0; t * kG + g < D; ++t) o += nres[t * kRow] != 0;
+            if (o) atomicAdd(open + qp, o);
         }
-        named_arrive(kOpen, 64);
+        named_arrive(kOpen, kResThreads + 32);
     } else {
     // ---------------- timing: lane = plan (Eq. 2, 5, 7, 10) ----------------
+    const bool mine = lane < kP;  // lanes at or beyond kP own no plan and touch no per-plan state
+    const int64_t p = (mine && lane < ng) ? (in_list ? (int64_t)in_list[j0 + lane] : j0 + lane) : 0;
+    const bool live = mine && lane < ng && out.status[p] == 0;
     TT *slots = (TT *)(sm + L.slots) + lane;
     TT *tfree = (TT *)(sm + L.tfree) + lane;
     if (mine) {
@@ -479,44 +650,57 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
     int64_t gsum = 0;
     for (int32_t c = 0; c < chunks; ++c) {
         const int b = c % kBuffers;
-        named_sync(kFullR + b, 64);
+        named_sync(kFullR + b, kResThreads + 32);
         const uint32_t *rb = ring + b * kRW * kChunk * kPitch + lane;
         const int32_t kmax = min(kChunk, N - c * kChunk);
-        for (int32_t k = 0; k < kmax && live; ++k) {
-            const uint32_t r3 = rb[(3 * kChunk + k) * kPitch];
-            if (r3 & kSkip) continue;
-            const uint32_t run = rb[(0 * kChunk + k) * kPitch];
-            const uint32_t ld = rb[(1 * kChunk + k) * kPitch];
-            const uint32_t arr = rb[(2 * kChunk + k) * kPitch];
-            const uint32_t r4 = rb[(4 * kChunk + k) * kPitch];
-            const uint32_t r5 = rb[(5 * kChunk + k) * kPitch];
-            TT *tf_d = tfree + (r3 & 31u) * kP;
+        if (live) {
+            // The ring words of the next position are read while this one plays.
+            uint32_t w[kRecWords];
+#pragma unroll
+            for (int x = 0; x < kRecWords; ++x) w[x] = rb[(x * kChunk) * kPitch];
+            for (int32_t k = 0; k < kmax; ++k) {
+                const int32_t kn = k + 1 < kmax ? k + 1 : k;
+                uint32_t nw[kRecWords];
+#pragma unroll
+                for (int x = 0; x < kRecWords; ++x) nw[x] = rb[(x * kChunk + kn) * kPitch];
+                const uint32_t r3 = w[3];
+                if (!(r3 & kSkip)) {
+                    const uint32_t run = w[0], ld = w[1], arr = w[2], r4 = w[4], r5 = w[5];
+                    TT *tf_d = tfree + (r3 & 31u) * kP;
+                    // Release (Eq. 2, Eq. 7); an accumulator slot is reset by its reader.
+                    const uint32_t rs = r5 >> 16;
+                    const TT rel = max((TT)arr, slots[(rs & 0x7FFFu) * kP]);
+                    slots[((rs & 0x8000u) ? (rs & 0x7FFFu) : trash) * kP] = 0;
+                    // A miss loads on this device first (ld > 0 only on a miss); a
+                    // prefetched load waits only for the arrival (Eq. 5).  On a hit
+                    // the residency stage cleared the prefetch bit and ld is 0.
+                    const TT ls = max(*tf_d, (r3 & kPrefetch) ? (TT)arr : rel);
+                    const TT le = ls + ld;
+                    const TT start = max(le, rel);
+                    const TT cfin = start + run;
+                    if (kNarrow) ovf |= (le < ls) | (cfin < start);
+                    else ovf |= run == kRunCap;
+                    end = max(end, cfin);
+                    if (r3 & kWasEmpty) gsum -= (int64_t)ls;   // an empty device becomes occupied
+                    if (r3 & kEmptied) gsum += (int64_t)cfin;  // the device empties after the unit
 
-            // Release (Eq. 2, Eq. 7); an accumulator slot is reset by its reader.
-            const uint32_t rs = r5 >> 16;
-            const TT rel = max((TT)arr, slots[(rs & 0x7FFFu) * kP]);
-            slots[((rs & 0x8000u) ? (rs & 0x7FFFu) : trash) * kP] = 0;
-            // A miss loads on this device first (ld > 0 only on a miss); a
-            // prefetched load waits only for the arrival (Eq. 5).  On a hit
-            // the residency stage cleared the prefetch bit and ld is 0.
-            const TT ls = max(*tf_d, (r3 & kPrefetch) ? (TT)arr : rel);
-            const TT le = ls + ld;
-            const TT start = max(le, rel);
-            const TT cfin = start + run;
-            if (kNarrow) ovf |= (le < ls) | (cfin < start);
-            else ovf |= run == kRunCap;
-            end = max(end, cfin);
-            if (r3 & kWasEmpty) gsum -= (int64_t)ls;   // an empty device becomes occupied
-            if (r3 & kEmptied) gsum += (int64_t)cfin;  // the device empties after the unit
-
-            publish<TT, kP>(slots, r3 >> 16, cfin);  // the sink when the unit writes nothing
-            publish<TT, kP>(slots, r4 & 0xFFFFu, cfin);
-            if (((r3 >> 11) & 7u) > 2) {
-                publish<TT, kP>(slots, r4 >> 16, cfin);
-                const int4 wr = __ldg(dp.noderec + 2 * (int32_t)(r5 & 0xFFFFu) + 1);
-                for (int32_t e = 3; e < wr.y; ++e) publish<TT, kP>(slots, __ldg(dp.wl + wr.x + e), cfin);
+                    publish<TT, kP>(slots, r3 >> 16, cfin);  // the sink when the unit writes nothing
+                    publish<TT, kP>(slots, r4 & 0xFFFFu, cfin);
+                    const uint32_t nwl = (r3 >> 11) & 7u;
+                    if (nwl > 2) {
+                        publish<TT, kP>(slots, r4 >> 16, cfin);
+                        if (nwl == 4) {
+                            publish<TT, kP>(slots, r5 & 0xFFFFu, cfin);
+                        } else if (nwl > 4) {  // five or more codes: the list from global memory
+                            const int4 wr = __ldg(dp.noderec + 2 * (int32_t)(r5 & 0xFFFFu) + 1);
+                            for (int32_t e = 3; e < wr.y; ++e) publish<TT, kP>(slots, __ldg(dp.wl + wr.x + e), cfin);
+                        }
+                    }
+                    *tf_d = cfin;
+                }
+#pragma unroll
+                for (int x = 0; x < kRecWords; ++x) w[x] = nw[x];
             }
-            *tf_d = cfin;
         }
         // Once every plan of the CTA has left 32 bits, the producers stop
         // loading (they see the flag at their next wait on this buffer).
@@ -524,16 +708,16 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
         named_arrive(kEmpty + b, kProdThreads + 32);  // buffer b may be refilled
     }
     if (kNarrow) ovf |= end == (TT)kRunCap;
-    named_sync(kOpen, 64);  // the residency stage's final device counts
+    named_sync(kOpen, kResThreads + 32);  // the residency stage's final device counts
     if (live && ovf) {  // handed to the next path
         const int32_t kk = atomicAdd(ovf_count, 1);
         ovf_list[kk] = (int32_t)p;
     } else if (live) {
-        const int64_t open = ((const uint32_t *)(sm + L.open))[lane];
+        const int64_t nopen = open[lane];
         for (int32_t w = 0; w < W; ++w) slots[w * kP] -= arrival[w];  // session completion latency
         const int32_t rank = (int32_t)((95 * (int64_t)W + 99) / 100 - 1);
         out.makespan_us[p] = (int64_t)end - dp.first_arrival;
-        out.gpu_us[p] = gsum + open * (int64_t)end;
+        out.gpu_us[p] = gsum + nopen * (int64_t)end;
         out.p95_us[p] = (int64_t)select_strided<TT, kP>(slots, W, rank);
     }
     }
@@ -550,12 +734,13 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
 // pooled nearest-rank p95 over samples x sessions.
 // ---------------------------------------------------------------------------
 constexpr int kSamples = 64;                  // timing lanes (two warps)
+constexpr int kSBuffers = 3;                  // record ring buffers
 constexpr int kSChunk = 32;                   // positions per chunk (one producer warp)
 constexpr int kSRec = kRecWords + 1;          // + head node
 constexpr int kSWarps = kSamples / 32 + 2;    // timing warps, residency warp, producer warp
 constexpr int kSTiming = kSamples;            // threads of the timing stage
 // Named barriers of this kernel (ids reuse those of the deterministic one).
-constexpr int kSFullP = 1, kSFullR = kSFullP + kBuffers, kSEmpty = kSFullR + kBuffers, kSOpen = kSEmpty + kBuffers,
+constexpr int kSFullP = 1, kSFullR = kSFullP + kSBuffers, kSEmpty = kSFullR + kSBuffers, kSOpen = kSEmpty + kSBuffers,
               kSRed = kSOpen + 1;
 
 struct StochLayout {
@@ -570,7 +755,7 @@ __host__ __device__ inline StochLayout stoch_layout(int32_t D, int32_t M, int32_
     l.cap = o; o += round16(4u * D);
     l.load = o; o += round16(4u * M * D);
     l.arr = o; o += round16(4u * W);
-    l.ring = o; o += 4u * kBuffers * kSRec * kSChunk;
+    l.ring = o; o += 4u * kSBuffers * kSRec * kSChunk;
     l.slots = o; o += 4u * (uint32_t)NS * kSamples;
     l.tfree = o; o += 4u * D * kSamples;
     l.used = o; o += round16(4u * D);
@@ -622,8 +807,8 @@ stoch_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list,
         r.prefetch = (const uint32_t *)((const uint8_t *)pl.prefetch + p * pl.bits_stride);
         r.retain = pl.retain ? (const uint32_t *)((const uint8_t *)pl.retain + p * pl.bits_stride) : nullptr;
         for (int32_t c = 0; c < chunks; ++c) {
-            const int b = c % kBuffers;
-            if (c >= kBuffers) named_sync(kSEmpty + b, kSTiming + 32);
+            const int b = c % kSBuffers;
+            if (c >= kSBuffers) named_sync(kSEmpty + b, kSTiming + 32);
             uint32_t *rb = ring + b * kSRec * kSChunk;
             const int32_t i = c * kSChunk + lane;
             uint32_t rec[kRecWords] = {0, 0, 0, kSkip, 0, 0};
@@ -634,8 +819,8 @@ stoch_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list,
             rb[kRecWords * kSChunk + lane] = (uint32_t)head;
             named_arrive(kSFullP + b, 64);
         }
-        for (int32_t c = chunks; c < chunks + kBuffers; ++c)
-            if (c >= kBuffers) named_sync(kSEmpty + c % kBuffers, kSTiming + 32);
+        for (int32_t c = chunks; c < chunks + kSBuffers; ++c)
+            if (c >= kSBuffers) named_sync(kSEmpty + c % kSBuffers, kSTiming + 32);
         return;
     }
 
@@ -650,7 +835,7 @@ stoch_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list,
         const bool dev = lane < D;
         const uint32_t capd = dev ? (uint32_t)cap[lane] : 0u;
         for (int32_t c = 0; c < chunks; ++c) {
-            const int b = c % kBuffers;
+            const int b = c % kSBuffers;
             named_sync(kSFullP + b, 64);
             uint32_t *rb = ring + b * kSRec * kSChunk;
             const int32_t kmax = min(kSChunk, N - c * kSChunk);
@@ -721,7 +906,7 @@ stoch_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list,
     uint32_t end = 0, ovf = 0;
     int64_t gsum = 0;
     for (int32_t c = 0; c < chunks; ++c) {
-        const int b = c % kBuffers;
+        const int b = c % kSBuffers;
         named_sync(kSFullR + b, kSTiming + 32);
         const uint32_t *rb = ring + b * kSRec * kSChunk;
         const int32_t kmax = min(kSChunk, N - c * kSChunk);
@@ -1037,12 +1222,19 @@ int launch_pc_r(const wf_ctx *ctx, int kp, const wf_plans *pl, const wf_eval_out
 {
     const wf_dev_problem &dp = ctx->dp;
     const int sms = ctx->sms;
-    if (kp == 16)
+    if constexpr (sizeof(TT) == 4) {  // the u32 sweep has one shape
+        (void)kp;
         return dp.M <= 8
-                   ? launch_pc<uint32_t, TT, 16, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
-                   : launch_pc<uint64_t, TT, 16, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
-    return dp.M <= 8 ? launch_pc<uint32_t, TT, 6, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
-                     : launch_pc<uint64_t, TT, 6, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
+                   ? launch_pc<uint32_t, TT, kPlans32, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
+                   : launch_pc<uint64_t, TT, kPlans32, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
+    } else {
+        if (kp == 16)
+            return dp.M <= 8
+                       ? launch_pc<uint32_t, TT, 16, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
+                       : launch_pc<uint64_t, TT, 16, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
+        return dp.M <= 8 ? launch_pc<uint32_t, TT, 6, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
+                         : launch_pc<uint64_t, TT, 6, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
+    }
 }
 
 template <typename TT>
@@ -1070,8 +1262,8 @@ wf_sweep_cfg wf_sweep_config(const wf_dev_problem &dp)
     if (!sweep_usable(dp)) return c;
     const int32_t NS = dp.nslots + 2;
     const bool r = dp.reclaim != 0;
-    const size_t s32 = r ? pc_layout<16, uint32_t, 1>(dp.D, dp.M, dp.W, NS).total
-                         : pc_layout<16, uint32_t, 0>(dp.D, dp.M, dp.W, NS).total;
+    const size_t s32 = r ? pc_layout<kPlans32, uint32_t, 1>(dp.D, dp.M, dp.W, NS).total
+                         : pc_layout<kPlans32, uint32_t, 0>(dp.D, dp.M, dp.W, NS).total;
     if (s32 <= 227 * 1024) c.smem32 = s32;
     // The u64 sweep: 16 plans per CTA, or 6 where that keeps more plans per SM.
     const size_t s16 = r ? pc_layout<16, uint64_t, 1>(dp.D, dp.M, dp.W, NS).total
@@ -1094,7 +1286,7 @@ int wf_launch_sweep(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, con
     if (cfg.smem32 && !(wide_first && cfg.smem64)) {
         // u32 times for every plan; the plans that leave 32 bits go on to the
         // u64 sweep, and from there (or straight) to the int64 path.
-        rc = launch_pc_q<uint32_t>(ctx, 16, pl, out, cfg.smem32, nullptr, nullptr, list1, counts, st);
+        rc = launch_pc_q<uint32_t>(ctx, kPlans32, pl, out, cfg.smem32, nullptr, nullptr, list1, counts, st);
         if (rc) return rc;
         if (!cfg.smem64) { *rest_list = list1; *rest_count = counts; return WF_OK; }
         rc = launch_pc_q<uint64_t>(ctx, cfg.plans64, pl, out, cfg.smem64, list1, counts, list2, counts + 1, st);

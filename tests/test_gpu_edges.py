@@ -136,3 +136,39 @@ def test_two_contexts_on_two_streams():
         want = oracle.eval_plans(prob, host, threads=8)
         for a, b in zip(res.numpy(), want):
             assert np.array_equal(a, b)
+
+
+def fanout_window(F, sessions=3, D=3, M=4, seed=0):
+    """Per session a source A, F helpers B_i and F joins C_i with
+    predecessors {A, B_i}: every C_i waits on its own accumulator slot, so
+    A's write list holds F codes (F = 4 travels in the unit record; F >= 5
+    is read by the timing stage from global memory, F > 7 beyond the
+    record's 3-bit count)."""
+    rng = np.random.default_rng(seed)
+    preds, session = [], []
+    for w in range(sessions):
+        a = len(preds)
+        preds.append([])
+        preds += [[] for _ in range(F)]
+        preds += [[a, a + 1 + i] for i in range(F)]
+        session += [w] * (2 * F + 1)
+    N = len(preds)
+    off = np.zeros(N + 1, np.int32)
+    off[1:] = np.cumsum([len(x) for x in preds])
+    idx = np.array([y for x in preds for y in x], np.int32)
+    weight = rng.integers(2, 5, M).astype(np.int32)
+    return wfgen.Problem(N=N, D=D, M=M, W=sessions, pred_off=off, pred_idx=idx,
+                         model=rng.integers(0, M, N).astype(np.uint8), session=np.array(session, np.int32),
+                         arrival_us=rng.integers(0, 500, sessions).astype(np.int64),
+                         lat_us=rng.integers(10, 400, N * D).astype(np.int32),
+                         peak_mib=rng.integers(5, 9, N * D).astype(np.int32), weight_mib=weight,
+                         load_us=rng.integers(1, 60, M * D).astype(np.int32), cap_mib=np.full(D, 12, np.int32))
+
+
+@pytest.mark.parametrize("F", [3, 4, 5, 7, 9])
+def test_long_write_lists(F):
+    """Units that publish their finish to F slots (the sweep's record paths
+    for three, four, five to seven and more than seven codes)."""
+    prob = fanout_window(F, seed=F)
+    plans = wfgen.make_plans(prob, 300, F)
+    assert_same(gpu_eval(prob, plans), oracle_eval(prob, plans))
