@@ -101,6 +101,14 @@ struct Ring {
 };
 constexpr int kRecWords = 6;
 
+// The ring holds a record as word pairs (8-byte shared-memory accesses):
+// (w0, w2) for timing, (w1, w3) read and rewritten by residency, (w4, w5)
+// for timing, and under reclamation by next use (the unit's next use, 0).
+template <int kReclaim>
+struct RecPairs {
+    static constexpr int kPairs = 3 + kReclaim;
+};
+
 template <int kP>
 struct PcShape {
     static constexpr int kProducers = kP >= 32 ? 8 : kP >= 16 ? 4 : kP >= 6 ? 3 : 2;
@@ -109,10 +117,11 @@ struct PcShape {
     // Four 16-plan CTAs share an SM (shared memory allows it at 2,000
     // activations), which bounds the registers per thread.
     static constexpr int kMinBlocks = kP >= 32 ? 2 : kP >= 16 ? 4 : 1;
-    // Words per (word, position) row of the ring.  A producer store covers 16
-    // positions x 2 plans; a pitch of 2 (mod 4) puts those 32 words in 32
-    // distinct banks, and the consumers' plan-major loads are contiguous.
-    static constexpr int kPitch = ((kP + 1) | 3) - 1;
+    // Elements (8-byte word pairs) per (pair, position) row of the ring.  A
+    // producer store covers 16 positions x 2 plans in two halves of 16
+    // lanes; an odd pitch puts each half's 16 pairs on 32 distinct banks, and
+    // the consumers' plan-major loads are contiguous.
+    static constexpr int kPitch = kP | 1;
     static_assert(kChunk == 16 && kP >= 1 && kP <= 32, "ring pitch assumes 16 positions per chunk");
 };
 
@@ -166,7 +175,7 @@ __host__ __device__ inline PcLayout pc_layout(int32_t D, int32_t M, int32_t W, i
     l.cap = o; o += round16(4u * D);
     l.load = o; o += round16(4u * M * D);
     l.arr = o; o += round16(4u * W);
-    l.ring = o; o += round16(4u * Ring<kReclaim>::kBuffers * (kRecWords + kReclaim) * kChunk * PcShape<kP>::kPitch);
+    l.ring = o; o += round16(8u * Ring<kReclaim>::kBuffers * RecPairs<kReclaim>::kPairs * kChunk * PcShape<kP>::kPitch);
     l.slots = o; o += round16(t * (uint32_t)NS * kP);
     l.tfree = o; o += round16(t * D * kP);
     const uint32_t rs = (uint32_t)(PcGroups<kP, kReclaim>::rows(D) * PcGroups<kP, kReclaim>::kLanes);
@@ -299,7 +308,7 @@ __device__ __forceinline__ const uint32_t *bits_row(const uint32_t *base, int64_
 // skip record).
 template <int kI, int kPitch>
 __device__ __forceinline__ void produce_batch(const wf_dev_problem &dp, const wf_plans &pl, const RowPtrs *rp,
-                                              const bool *act, const int32_t *hh, uint32_t *rb, int pos,
+                                              const bool *act, const int32_t *hh, uint2 *rb, int pos,
                                               const int *qq, uint32_t *dev)
 {
     const int32_t D = dp.D;
@@ -329,12 +338,13 @@ __device__ __forceinline__ void produce_batch(const wf_dev_problem &dp, const wf
     for (int j = 0; j < kI; ++j) {
         dev[j] = 0xFFFFFFFFu;
         if (qq[j] < 0) continue;  // a lane beyond the CTA's plans
-        uint32_t *dst = rb + pos * kPitch + qq[j];
+        uint2 *dst = rb + pos * kPitch + qq[j];
         const int32_t h = hh[j];
         const uint32_t s0 = hr[j].x >> 16;
         if (!act[j] || (((fw[j] >> (h & 31)) & 1u) && pprev[j] == d[j])) {  // no unit, or inside its head's
-#pragma unroll
-            for (int w = 0; w < kRecWords; ++w) dst[w * kChunk * kPitch] = w == 3 ? kSkip : 0u;
+            dst[0] = make_uint2(0u, 0u);
+            dst[1 * kChunk * kPitch] = make_uint2(0u, kSkip);
+            dst[2 * kChunk * kPitch] = make_uint2(0u, 0u);
             continue;
         }
         uint32_t run = (uint32_t)lk0[j].x + (uint32_t)dp.grant, ovf = 0;  // both < 2^31: no wrap
@@ -361,15 +371,57 @@ __device__ __forceinline__ void produce_batch(const wf_dev_problem &dp, const wf
         const uint32_t nwl = (ty >> 20) & 7u;
         const uint32_t pf = (pw[j] >> (h & 31)) & 1u;
         const uint32_t reclaim = ((rwt >> (tail & 31)) & 1u) ^ 1u;
-        dst[0 * kChunk * kPitch] = ovf ? kRunCap : run;
-        dst[1 * kChunk * kPitch] = (uint32_t)kv;
-        dst[2 * kChunk * kPitch] = hr[j].z;
-        dst[3 * kChunk * kPitch] =
-            d[j] | (((hr[j].y >> 16) & 15u) << 5) | (pf << 9) | (reclaim << 10) | (nwl << 11) | (tw << 16);
+        dst[0] = make_uint2(ovf ? kRunCap : run, hr[j].z);
+        dst[1 * kChunk * kPitch] = make_uint2(
+            (uint32_t)kv, d[j] | (((hr[j].y >> 16) & 15u) << 5) | (pf << 9) | (reclaim << 10) | (nwl << 11) | (tw << 16));
+        dst[2 * kChunk * kPitch] = make_uint2((tw >> 16) | (c2t << 16),
+                                              (nwl == 4 ? c2t >> 16 : (uint32_t)tail) | (hr[j].y << 16));
         dev[j] = d[j];
-        dst[4 * kChunk * kPitch] = (tw >> 16) | (c2t << 16);
-        dst[5 * kChunk * kPitch] = (nwl == 4 ? c2t >> 16 : (uint32_t)tail) | (hr[j].y << 16);
     }
+}
+
+// One unit on its device under least-recently-used reclamation (Eq. 11,
+// Section 3.5): q / n / u_d are the device's queue, resident count and
+// resident weights.  The unit's own model leaves the queue first; the
+// victims are then exactly the queue's first entries (least recently used
+// first), and the unit's model goes back in as the most recently used.
+// Returns the record's rewritten (w1, w3): the load the unit waits for (none
+// on a hit, Eq. 5) and the occupancy changes of section 4.3.
+template <typename Q>
+__device__ __forceinline__ uint2 settle_lru(Q &q, uint32_t &n, uint32_t &u_d, uint32_t capd, uint32_t r1,
+                                            uint32_t r3, const int32_t *weight, const int32_t *load, int32_t D,
+                                            int *err)
+{
+    const int32_t d = (int32_t)(r3 & 31u);
+    const uint32_t m = (r3 >> 5) & 15u;
+    const uint32_t wm = (uint32_t)weight[m];
+    const bool was_empty = n == 0;
+    const int32_t kq = Lru<Q>::find(q, n, m);
+    const bool hit = kq < (int32_t)n;
+    q = hit ? Lru<Q>::remove(q, hit ? kq : 0) : q;  // (an index below the queue length)
+    n -= hit ? 1u : 0u;
+    const uint32_t need = hit ? r1 : wm + r1;  // used + need <= cap + peak < 2^32
+    uint32_t e = 0;
+    while (u_d + need > capd && e < n) {
+        u_d -= (uint32_t)weight[(uint32_t)(q >> (4 * e)) & 15u];
+        ++e;
+    }
+    if (u_d + need > capd) atomicExch(err, 2);  // unreachable for a valid plan
+    q = e < (uint32_t)Lru<Q>::kSlots ? (q >> (4 * e)) : (Q)0;
+    n -= e;
+    q |= (Q)m << (4 * n);
+    n += 1;
+    u_d += hit ? 0u : wm;
+    uint32_t emptied = 0;
+    if ((r3 >> 10) & 1u) {  // retain bit 0: reclaim at the end of the unit
+        q &= ~((Q)0xF << (4 * (n - 1)));
+        n -= 1;
+        u_d -= wm;
+        emptied = n == 0;
+    }
+    return make_uint2(hit ? 0u : (uint32_t)load[m * D + d],
+                      (r3 & ~(kPrefetch | kWasEmpty)) | (hit ? 0u : (r3 & kPrefetch)) |
+                          (was_empty ? kWasEmpty : 0u) | (emptied ? kEmptied : 0u));
 }
 
 // A finish time into a slot: an accumulator keeps the latest of its
@@ -392,7 +444,7 @@ __global__ void __launch_bounds__(32 * PcShape<kP>::kWarps, PcShape<kP>::kMinBlo
 pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_list, const int32_t *in_count,
           int32_t *ovf_list, int32_t *ovf_count)
 {
-    constexpr int kRW = kRecWords + kReclaim;  // words per record in the ring
+    constexpr int kRW = RecPairs<kReclaim>::kPairs;  // word pairs per record in the ring
     using S = PcShape<kP>;
     constexpr int kPitch = S::kPitch;
     constexpr int kProdThreads = 32 * S::kProducers;
@@ -408,7 +460,7 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
     const PcLayout L = pc_layout<kP, TT, kReclaim>(D, M, W, dp.nslots + 2);
     const int64_t total = in_list ? (int64_t)*in_count : pl.P;
     if ((int64_t)blockIdx.x * kP >= total) return;  // the whole CTA: no plan
-    uint32_t *ring = (uint32_t *)(sm + L.ring);
+    uint2 *ring = (uint2 *)(sm + L.ring);
     const int32_t chunks = (N + kChunk - 1) / kChunk;
     volatile uint32_t *gave_up = (volatile uint32_t *)(sm + L.flag);
 
@@ -464,11 +516,13 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
         int32_t h0[kIters];
 #pragma unroll
         for (int j = 0; j < kIters; ++j) h0[j] = okq[j] && pos < N ? __ldg(rp[j].order + pos) : 0;
+        // The timing stage's give-up flag, read a chunk before it is used so
+        // that no load of this chunk waits for it.
+        bool quit = false;
         for (int32_t c = 0; c < chunks; ++c) {
             const int b = c % kBuffers;
             if (c >= kBuffers) named_sync(kEmpty + b, kProdThreads + 32);  // timing released buffer b
-            const bool quit = kNarrow && *gave_up;
-            uint32_t *rb = ring + b * kRW * kChunk * kPitch;
+            uint2 *rb = ring + b * kRW * kChunk * kPitch;
             const int32_t i = c * kChunk + pos;
             int32_t h1[kIters];
             bool act[kIters];
@@ -477,8 +531,8 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
                 h1[j] = okq[j] && i + kChunk < N && !quit ? __ldg(rp[j].order + i + kChunk) : 0;
                 act[j] = okq[j] && i < N && !quit;
                 if (kReclaim && qq[j] >= 0)  // the next use of this unit's model on its device
-                    rb[(kRecWords * kChunk + pos) * kPitch + qq[j]] =
-                        act[j] ? (uint32_t)__ldg(dp.nextuse + qplan[j] * (int64_t)N + i) : 0xFFFFu;
+                    rb[(3 * kChunk + pos) * kPitch + qq[j]] =
+                        make_uint2(act[j] ? (uint32_t)__ldg(dp.nextuse + qplan[j] * (int64_t)N + i) : 0xFFFFu, 0u);
             }
             uint32_t dev[kIters];
             produce_batch<kIters, kPitch>(dp, pl, rp, act, h0, rb, pos, qq, dev);
@@ -495,6 +549,7 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
             }
 #pragma unroll
             for (int j = 0; j < kIters; ++j) h0[j] = h1[j];
+            quit = kNarrow && *gave_up;
             named_arrive(kFullP + b, kProdThreads + kResThreads);  // buffer b is full
         }
         // Match the timing stage's releases of the last buffers.
@@ -528,38 +583,45 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
         for (int32_t c = 0; c < chunks; ++c) {
             const int b = c % kBuffers;
             named_sync(kFullP + b, kProdThreads + kResThreads);
-            uint32_t *rb = ring + b * kRW * kChunk * kPitch + qp;
+            uint2 *rb = ring + b * kRW * kChunk * kPitch + qp;
             uint32_t todo = live ? gmask[(b * kG + g) * kP + qp] : 0u;
-            // The ring words of the lane's next unit are read while this one plays.
+            // The ring words of the lane's next unit are read while this one
+            // plays (pair 1: w1 | w3).
             int32_t k = todo ? __ffs((int)todo) - 1 : 0;
-            uint32_t r3 = todo ? rb[(3 * kChunk + k) * kPitch] : 0u;
-            uint32_t r1 = todo ? rb[(1 * kChunk + k) * kPitch] : 0u;
+            uint2 v = todo ? rb[(1 * kChunk + k) * kPitch] : make_uint2(0u, 0u);
             while (todo) {
                 todo &= todo - 1;
                 const int32_t kn = todo ? __ffs((int)todo) - 1 : k;
-                const uint32_t n3 = rb[(3 * kChunk + kn) * kPitch], n1 = rb[(1 * kChunk + kn) * kPitch];
+                const uint2 nv = rb[(1 * kChunk + kn) * kPitch];
+                const uint32_t r1 = v.x, r3 = v.y;
                 const int32_t d = (int32_t)(r3 & 31u);
-                const uint32_t m = (r3 >> 5) & 15u;
-                const int32_t t = d / kG;
-                Q q = queue[t * kRow];
-                uint32_t n = nres[t * kRow];
-                uint32_t u_d = used[t * kRow];  // used + need <= cap + peak < 2^32
-                const uint32_t wm = (uint32_t)weight[m];
-                const uint32_t capd = (uint32_t)cap[d];
-                const bool was_empty = n == 0;
-                const int32_t kq = Lru<Q>::find(q, n, m);
-                const bool hit = kq < (int32_t)n;
-                // Take the unit's own model out of the queue; the reclamation
-                // victims are then exactly its first e entries (least recently
-                // used first), and the unit's model goes back in at the end.
-                q = hit ? Lru<Q>::remove(q, hit ? kq : 0) : q;  // (an index below the queue length)
-                n -= hit ? 1u : 0u;
-                const uint32_t need = hit ? r1 : wm + r1;
-                if (kReclaim) {
-                    // Victims one at a time: a copy also resident elsewhere,
-                    // then the largest (next use - position) / reload cost
-                    // (no next use or a free reload: infinite), then the
-                    // least recently used (the earlier queue entry).
+                if (!kReclaim) {
+                    const int32_t t = d / kG;
+                    Q q = queue[t * kRow];
+                    uint32_t n = nres[t * kRow];
+                    uint32_t u_d = used[t * kRow];
+                    const uint2 w = settle_lru<Q>(q, n, u_d, (uint32_t)cap[d], r1, r3, weight, load, D, dp.err);
+                    queue[t * kRow] = q;
+                    nres[t * kRow] = (uint8_t)n;
+                    used[t * kRow] = u_d;
+                    rb[(1 * kChunk + k) * kPitch] = w;
+                } else {
+                    // Reclamation by next use: victims one at a time, a copy
+                    // also resident elsewhere first, then the largest (next
+                    // use - position) / reload cost (no next use or a free
+                    // reload: infinite), then the least recently used.
+                    const uint32_t m = (r3 >> 5) & 15u;
+                    Q q = queue[d * kRow];
+                    uint32_t n = nres[d * kRow];
+                    uint32_t u_d = used[d * kRow];  // used + need <= cap + peak < 2^32
+                    const uint32_t wm = (uint32_t)weight[m];
+                    const uint32_t capd = (uint32_t)cap[d];
+                    const bool was_empty = n == 0;
+                    const int32_t kq = Lru<Q>::find(q, n, m);
+                    const bool hit = kq < (int32_t)n;
+                    q = hit ? Lru<Q>::remove(q, hit ? kq : 0) : q;  // (an index below the queue length)
+                    n -= hit ? 1u : 0u;
+                    const uint32_t need = hit ? r1 : wm + r1;
                     const int64_t here = c * kChunk + k;
                     while (u_d + need > capd && n > 0) {
                         int32_t best = 0;
@@ -587,39 +649,28 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
                     }
                     if (u_d + need > capd) atomicExch(dp.err, 2);  // unreachable for a valid plan
                     if (!hit) rcnt[m * kP] += 1;
-                    nuse[(d * M + m) * kP] = (uint16_t)rb[(kRecWords * kChunk + k) * kPitch];
-                } else {
-                    uint32_t e = 0;
-                    while (u_d + need > capd && e < n) {
-                        u_d -= (uint32_t)weight[(uint32_t)(q >> (4 * e)) & 15u];
-                        ++e;
+                    nuse[(d * M + m) * kP] = (uint16_t)rb[(3 * kChunk + k) * kPitch].x;
+                    q |= (Q)m << (4 * n);  // the unit's model is now the most recently used
+                    n += 1;
+                    u_d += hit ? 0u : wm;
+                    uint32_t emptied = 0;
+                    if ((r3 >> 10) & 1u) {  // retain bit 0: reclaim at the end of the unit
+                        q &= ~((Q)0xF << (4 * (n - 1)));
+                        n -= 1;
+                        u_d -= wm;
+                        emptied = n == 0;
+                        rcnt[m * kP] -= 1;
                     }
-                    if (u_d + need > capd) atomicExch(dp.err, 2);  // unreachable for a valid plan
-                    q = e < (uint32_t)Lru<Q>::kSlots ? (q >> (4 * e)) : (Q)0;
-                    n -= e;
+                    queue[d * kRow] = q;
+                    nres[d * kRow] = (uint8_t)n;
+                    used[d * kRow] = u_d;
+                    rb[(1 * kChunk + k) * kPitch] =
+                        make_uint2(hit ? 0u : (uint32_t)load[m * D + d],
+                                   (r3 & ~(kPrefetch | kWasEmpty)) | (hit ? 0u : (r3 & kPrefetch)) |
+                                       (was_empty ? kWasEmpty : 0u) | (emptied ? kEmptied : 0u));
                 }
-                q |= (Q)m << (4 * n);  // the unit's model is now the most recently used
-                n += 1;
-                u_d += hit ? 0u : wm;
-                uint32_t emptied = 0;
-                if ((r3 >> 10) & 1u) {  // retain bit 0: reclaim at the end of the unit
-                    q &= ~((Q)0xF << (4 * (n - 1)));
-                    n -= 1;
-                    u_d -= wm;
-                    emptied = n == 0;
-                    if (kReclaim) rcnt[m * kP] -= 1;
-                }
-                queue[t * kRow] = q;
-                nres[t * kRow] = (uint8_t)n;
-                used[t * kRow] = u_d;
-                // For timing: the load to wait for (none on a hit, Eq. 5) and
-                // the occupancy changes of section 4.3.
-                rb[(1 * kChunk + k) * kPitch] = hit ? 0u : (uint32_t)load[m * D + d];
-                rb[(3 * kChunk + k) * kPitch] = (r3 & ~(kPrefetch | kWasEmpty)) | (hit ? 0u : (r3 & kPrefetch)) |
-                                                (was_empty ? kWasEmpty : 0u) | (emptied ? kEmptied : 0u);
                 k = kn;
-                r3 = n3;
-                r1 = n1;
+                v = nv;
             }
             named_arrive(kFullR + b, kResThreads + 32);
         }
@@ -651,21 +702,21 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
     for (int32_t c = 0; c < chunks; ++c) {
         const int b = c % kBuffers;
         named_sync(kFullR + b, kResThreads + 32);
-        const uint32_t *rb = ring + b * kRW * kChunk * kPitch + lane;
+        const uint2 *rb = ring + b * kRW * kChunk * kPitch + lane;
         const int32_t kmax = min(kChunk, N - c * kChunk);
         if (live) {
             // The ring words of the next position are read while this one plays.
-            uint32_t w[kRecWords];
+            uint2 w[3];
 #pragma unroll
-            for (int x = 0; x < kRecWords; ++x) w[x] = rb[(x * kChunk) * kPitch];
+            for (int x = 0; x < 3; ++x) w[x] = rb[(x * kChunk) * kPitch];
             for (int32_t k = 0; k < kmax; ++k) {
                 const int32_t kn = k + 1 < kmax ? k + 1 : k;
-                uint32_t nw[kRecWords];
+                uint2 nw[3];
 #pragma unroll
-                for (int x = 0; x < kRecWords; ++x) nw[x] = rb[(x * kChunk + kn) * kPitch];
-                const uint32_t r3 = w[3];
+                for (int x = 0; x < 3; ++x) nw[x] = rb[(x * kChunk + kn) * kPitch];
+                const uint32_t r3 = w[1].y;
                 if (!(r3 & kSkip)) {
-                    const uint32_t run = w[0], ld = w[1], arr = w[2], r4 = w[4], r5 = w[5];
+                    const uint32_t run = w[0].x, ld = w[1].x, arr = w[0].y, r4 = w[2].x, r5 = w[2].y;
                     TT *tf_d = tfree + (r3 & 31u) * kP;
                     // Release (Eq. 2, Eq. 7); an accumulator slot is reset by its reader.
                     const uint32_t rs = r5 >> 16;
@@ -699,11 +750,11 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
                     *tf_d = cfin;
                 }
 #pragma unroll
-                for (int x = 0; x < kRecWords; ++x) w[x] = nw[x];
+                for (int x = 0; x < 3; ++x) w[x] = nw[x];
             }
         }
         // Once every plan of the CTA has left 32 bits, the producers stop
-        // loading (they see the flag at their next wait on this buffer).
+        // loading (they see the flag a chunk or two later).
         if (kNarrow && __all_sync(0xFFFFFFFFu, !live || ovf) && lane == 0) *gave_up = 1;
         named_arrive(kEmpty + b, kProdThreads + 32);  // buffer b may be refilled
     }
