@@ -1,5 +1,5 @@
 // Plan construction: the paper's per-tick scheduler (Algorithm 1) read as a
-// list scheduler over the whole window, one plan per thread.
+// list scheduler over the whole window, one plan per warp.
 //
 //   RankReady            a node is ready once every graph predecessor is
 //                        dispatched; the ready node with the smallest
@@ -17,8 +17,8 @@
 // Each unit is played forward with the evaluation rules (admission and LRU
 // reclamation, Eq. 11; loads, Eq. 5; starts and finishes, Eq. 2, 7, 10), so
 // the constructor's timeline is the one wf_eval_plans reports for its plan.
-// State per thread lives in global scratch: finish times (a ready node's
-// release until it runs), a binary heap of (rank << 16 | node) keys, the
+// State per plan lives in global scratch: finish times (a ready node's
+// release until it runs), the unordered ready keys (rank << 16 | node), the
 // pending predecessor counts, and per device the free time, resident weights
 // and last-use stamps.
 #include <algorithm>
@@ -27,8 +27,9 @@
 
 namespace {
 
-constexpr int kThreads = 32;     // one warp per CTA, so the plans spread over every SM
-constexpr int kPlansPerSm = 128;  // plans built at once per SM (the scratch is sized for them)
+constexpr int kWarps = 4;          // warps per CTA, a plan per warp
+constexpr int kCtasPerSm = 10;     // resident CTAs per SM (48 registers per thread)
+constexpr int kSlotsPerSm = kWarps * kCtasPerSm;  // plans built at once per SM (the scratch is sized for them)
 
 __device__ __forceinline__ uint64_t mix64(uint64_t x)  // SplitMix64 output function
 {
@@ -38,157 +39,220 @@ __device__ __forceinline__ uint64_t mix64(uint64_t x)  // SplitMix64 output func
     return x ^ (x >> 31);
 }
 
-struct Scratch {
-    int64_t *c;        // [N] finish (release while ready)
-    uint64_t *heap;    // [N]
-    int32_t *pending;  // [N]
-    int64_t *t_free;   // [D]
-    int64_t *used;     // [D]
-    int64_t *stamp;    // [D][M] last-use sequence number, 0 = not resident
+// x mod d for d >= 2, exact for every 64-bit x, from the 128-bit reciprocal
+// M = floor((2^128 - 1) / d) + 1 (Lemire, Kaser and Kurz, "Faster remainder
+// by direct computation", 2019): the remainder is the top 64 bits of
+// (M x mod 2^128) d.  A handful of multiplies instead of a 64-bit division.
+struct Mod64 {
+    uint64_t mh, ml, d;
 };
 
-__host__ __device__ inline size_t scratch_bytes(int32_t N, int32_t D, int32_t M)
+__device__ __forceinline__ uint64_t mod64(uint64_t x, const Mod64 &m)
 {
-    const size_t b = 8 * (size_t)N + 8 * (size_t)N + 4 * (size_t)N + 16 * (size_t)D + 8 * (size_t)D * M;
-    return (b + 255) & ~(size_t)255;
+    const uint64_t l0 = m.ml * x;
+    const uint64_t l1 = __umul64hi(m.ml, x) + m.mh * x;
+    const uint64_t a1 = __umul64hi(l0, m.d);
+    const uint64_t s = a1 + l1 * m.d;
+    return __umul64hi(l1, m.d) + (s < a1 ? 1u : 0u);
 }
 
-__device__ __forceinline__ void heap_push(uint64_t *h, int32_t &n, uint64_t key)
+// Per-plan state in global scratch.  A node's release is accumulated as its
+// predecessors' units finish (every predecessor of a node released this way
+// is the last member of its unit), so no finish time is read back.
+struct Scratch {
+    uint64_t *key;     // [N] ready keys (rank << 16 | node), unordered
+    int64_t *rel;      // [N] the release of the ready node beside it
+    int64_t *relmax;   // [N] session arrival, raised to each finished predecessor's finish
+    int32_t *pending;  // [N] predecessors not yet finished
+};
+
+__host__ __device__ inline size_t scratch_bytes(int32_t N)
 {
-    int32_t i = n++;
-    while (i > 0) {
-        const int32_t parent = (i - 1) >> 1;
-        const uint64_t pk = h[parent];
-        if (pk <= key) break;
-        h[i] = pk;
-        i = parent;
+    return ((8 + 8 + 8 + 4) * (size_t)N + 255) & ~(size_t)255;
+}
+
+// Per-warp device state in shared memory: free time and resident weight per
+// device, last-use stamp per (device, model) (0 = not resident; stamps count
+// units, below 2^16).
+__host__ __device__ inline size_t warp_smem(int32_t D, int32_t M)
+{
+    return ((16 * (size_t)D + 2 * (size_t)D * M) + 15) & ~(size_t)15;
+}
+
+// Warp-wide minimum of a 64-bit key (two 32-bit warp reductions: high
+// halves, then low halves among the lanes holding the smallest high half);
+// returns the lowest lane holding it, and every lane gets the minimum.
+__device__ __forceinline__ int warp_argmin64(uint64_t &key)
+{
+    const uint32_t hi = __reduce_min_sync(0xFFFFFFFFu, (uint32_t)(key >> 32));
+    const uint32_t lo = __reduce_min_sync(0xFFFFFFFFu, (uint32_t)(key >> 32) == hi ? (uint32_t)key : 0xFFFFFFFFu);
+    const uint64_t k = ((uint64_t)hi << 32) | lo;
+    const int src = __ffs((int)__ballot_sync(0xFFFFFFFFu, key == k)) - 1;
+    key = k;
+    return src;
+}
+
+// Appends (key, rel) of the lanes with take set to the ready arrays at n.
+__device__ __forceinline__ void append(const Scratch &s, int32_t &n, bool take, uint64_t key, int64_t rel,
+                                       int lane)
+{
+    const uint32_t bal = __ballot_sync(0xFFFFFFFFu, take);
+    if (take) {
+        const int32_t i = n + __popc(bal & ((1u << lane) - 1u));
+        s.key[i] = key;
+        s.rel[i] = rel;
     }
-    h[i] = key;
+    n += __popc(bal);
 }
 
-__device__ __forceinline__ uint64_t heap_pop(uint64_t *h, int32_t &n)
+// A warp per plan.  The ready set is an unordered array; each step takes its
+// smallest key (a warp minimum over the array, the node a heap would give,
+// keys being unique), scores every device in its own lane, picks
+// reclamation victims as a warp minimum over the device's stamps, and
+// releases the unit's successors in parallel lanes.  Lane 0 writes the
+// plan's rows and the device state; __syncwarp orders those writes before
+// the other lanes read them.
+__global__ void __launch_bounds__(32 * kWarps, kCtasPerSm)
+construct_kernel(wf_dev_problem dp, wf_plans out, uint64_t seed, int64_t jitter, Mod64 jm, uint8_t *scratch,
+                 int64_t slots)
 {
-    const uint64_t top = h[0];
-    const uint64_t last = h[--n];
-    int32_t i = 0;
-    for (;;) {
-        int32_t child = 2 * i + 1;
-        if (child >= n) break;
-        uint64_t ck = h[child];
-        if (child + 1 < n) {
-            const uint64_t rk = h[child + 1];
-            if (rk < ck) { ck = rk; ++child; }
-        }
-        if (last <= ck) break;
-        h[i] = ck;
-        i = child;
-    }
-    if (n > 0) h[i] = last;
-    return top;
-}
-
-__global__ void __launch_bounds__(kThreads)
-construct_kernel(wf_dev_problem dp, wf_plans out, uint64_t seed, int64_t jitter, uint8_t *scratch, int64_t threads)
-{
-    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (t >= threads) return;
+    extern __shared__ __align__(16) uint8_t csm[];
+    const int lane = threadIdx.x & 31;
+    const int64_t w = (int64_t)blockIdx.x * kWarps + (threadIdx.x >> 5);
+    if (w >= slots) return;
     const int32_t N = dp.N, D = dp.D, M = dp.M;
     const int32_t words = (N + 31) / 32;
-    uint8_t *base = scratch + (size_t)t * scratch_bytes(N, D, M);
+    uint8_t *base = scratch + (size_t)w * scratch_bytes(N);
     Scratch s;
-    s.c = (int64_t *)base;
-    s.heap = (uint64_t *)(s.c + N);
-    s.t_free = (int64_t *)(s.heap + N);
-    s.used = s.t_free + D;
-    s.stamp = s.used + D;
-    s.pending = (int32_t *)(s.stamp + (size_t)D * M);
-    const uint64_t jmod = (uint64_t)jitter + 1;
-
-    for (int64_t p = t; p < out.P; p += threads) {
+    s.key = (uint64_t *)base;
+    s.rel = (int64_t *)(s.key + N);
+    s.relmax = s.rel + N;
+    s.pending = (int32_t *)(s.relmax + N);
+    uint8_t *wsm = csm + (size_t)(threadIdx.x >> 5) * warp_smem(D, M);
+    int64_t *t_free = (int64_t *)wsm;
+    int64_t *used_d = t_free + D;
+    uint16_t *stamp = (uint16_t *)(used_d + D);
+    // Jitter draws are taken mod (jitter + 1) >= 2 when jitter > 0.
+    for (int64_t p = w; p < out.P; p += slots) {
         const uint64_t g = (uint64_t)(out.plan_base + p);
         const uint64_t hp = mix64(seed ^ g);
         uint8_t *place = (uint8_t *)out.place + p * out.place_stride;
         uint16_t *order = (uint16_t *)((uint8_t *)out.order + p * out.order_stride);
         uint32_t *fuse = (uint32_t *)((uint8_t *)out.fuse + p * out.bits_stride);
         uint32_t *prefetch = (uint32_t *)((uint8_t *)out.prefetch + p * out.bits_stride);
-        for (int32_t k = 0; k < words; ++k) { fuse[k] = 0; prefetch[k] = 0; }
+        for (int32_t k = lane; k < words; k += 32) { fuse[k] = 0; prefetch[k] = 0; }
         if (out.retain) {
             uint32_t *retain = (uint32_t *)((uint8_t *)out.retain + p * out.bits_stride);
-            for (int32_t k = 0; k < words; ++k)
+            for (int32_t k = lane; k < words; k += 32)
                 retain[k] = (k + 1 < words || (N & 31) == 0) ? 0xFFFFFFFFu : ((1u << (N & 31)) - 1u);
         }
-        for (int32_t d = 0; d < D; ++d) { s.t_free[d] = 0; s.used[d] = 0; }
-        for (int32_t k = 0; k < D * M; ++k) s.stamp[k] = 0;
-        int32_t nheap = 0;
-        for (int32_t v = 0; v < N; ++v) {
-            const int32_t np = __ldg(dp.pred_off + v + 1) - __ldg(dp.pred_off + v);
-            s.pending[v] = np;
-            if (np == 0) {
-                const int64_t rel = __ldg(dp.arrival + __ldg(dp.session + v));
-                s.c[v] = rel;
-                const uint64_t j = jitter > 0 ? mix64(hp ^ (uint64_t)v) % jmod : 0;
-                heap_push(s.heap, nheap, (((uint64_t)rel + j) << 16) | (uint64_t)v);
+        for (int32_t d = lane; d < D; d += 32) { t_free[d] = 0; used_d[d] = 0; }
+        for (int32_t k = lane; k < D * M; k += 32) stamp[k] = 0;
+        int32_t nready = 0;
+        for (int32_t v0 = 0; v0 < N; v0 += 32) {
+            const int32_t v = v0 + lane;
+            bool take = false;
+            uint64_t key = 0;
+            int64_t arr = 0;
+            if (v < N) {
+                const int32_t np = __ldg(dp.pred_off + v + 1) - __ldg(dp.pred_off + v);
+                arr = __ldg(dp.arrival + __ldg(dp.session + v));
+                s.pending[v] = np;
+                s.relmax[v] = arr;
+                if (np == 0) {
+                    const uint64_t j = jitter > 0 ? mod64(mix64(hp ^ (uint64_t)v), jm) : 0;
+                    key = (((uint64_t)arr + j) << 16) | (uint64_t)v;
+                    take = true;
+                }
             }
+            append(s, nready, take, key, arr, lane);
         }
+        __syncwarp();
         int32_t pos = 0;
-        int64_t seq = 0;
-        while (nheap > 0) {
-            const int32_t u = (int32_t)(heap_pop(s.heap, nheap) & 0xFFFFu);
-            const int64_t rel = s.c[u];
+        uint32_t seq = 0;
+        while (nready > 0) {
+            // RankReady: the smallest key, with its release.
+            uint64_t best = ~0ull;
+            int32_t at = 0;
+            for (int32_t i = lane; i < nready; i += 32) {
+                const uint64_t k = s.key[i];
+                if (k < best) { best = k; at = i; }
+            }
+            const int src = warp_argmin64(best);  // keys are unique
+            at = __shfl_sync(0xFFFFFFFFu, at, src);
+            const int64_t rel = s.rel[at];
+            const int32_t u = (int32_t)(best & 0xFFFFu);
+            const uint64_t last_k = s.key[nready - 1];
+            const int64_t last_r = s.rel[nready - 1];
+            __syncwarp();
+            if (lane == 0) { s.key[at] = last_k; s.rel[at] = last_r; }
+            --nready;
             const int32_t m = __ldg(dp.model + u);
             const int64_t arr = __ldg(dp.arrival + __ldg(dp.session + u));
-            const uint64_t hu = mix64(hp ^ (uint64_t)u);
             const uint32_t fit_u = __ldg(dp.fitmask + u);
 
-            // BestFeasibleBinding.
-            int32_t d = -1;
-            int64_t best = 0;
-            for (int32_t dd = 0; dd < D; ++dd) {
-                if (!((fit_u >> dd) & 1u)) continue;
-                const int64_t tf = s.t_free[dd];
+            // BestFeasibleBinding: device lane by lane, then the smallest
+            // (score, device).
+            uint64_t score = ~0ull;
+            int64_t tf_l = 0;
+            if (lane < D && ((fit_u >> lane) & 1u)) {
+                tf_l = t_free[lane];
                 int64_t start;
-                if (s.stamp[dd * M + m] != 0) {
-                    start = max(tf, rel);
+                if (stamp[lane * M + m] != 0) {
+                    start = max(tf_l, rel);
                 } else {
-                    const int64_t ls = tf < rel ? max(tf, arr) : max(tf, rel);
-                    start = max(ls + (int64_t)__ldg(dp.load + m * D + dd), rel);
+                    const int64_t ls = tf_l < rel ? max(tf_l, arr) : max(tf_l, rel);
+                    start = max(ls + (int64_t)__ldg(dp.load + m * D + lane), rel);
                 }
-                const int64_t fin = start + dp.grant + (int64_t)__ldg(&dp.lk[u * D + dd].x);
-                const int64_t score = fin + (jitter > 0 ? (int64_t)(mix64(hu ^ (uint64_t)(dd + 1)) % jmod) : 0);
-                if (d < 0 || score < best) { d = dd; best = score; }
+                const int64_t fin = start + dp.grant + (int64_t)__ldg(&dp.lk[u * D + lane].x);
+                const uint64_t hu = mix64(hp ^ (uint64_t)u);
+                score = (uint64_t)(fin + (jitter > 0 ? (int64_t)mod64(mix64(hu ^ (uint64_t)(lane + 1)), jm) : 0));
             }
-            if (d < 0) { atomicExch(dp.err, 4); return; }  // unreachable: every node fits somewhere
+            const int32_t d = warp_argmin64(score);  // ties: the lower device
+            if (score == ~0ull) {  // unreachable: every node fits somewhere
+                if (lane == 0) atomicExch(dp.err, 4);
+                return;
+            }
+            const int64_t tf = __shfl_sync(0xFFFFFFFFu, tf_l, d);
+            uint16_t *st = stamp + d * M;
+            const bool hit = st[m] != 0;
 
             // The unit: u and its fusible chain while the members fit on d.
-            const bool hit = s.stamp[d * M + m] != 0;
-            const int64_t tf = s.t_free[d];
             const bool pf = !hit && tf < rel;
             int64_t kv = __ldg(&dp.lk[u * D + d].y);
-            place[u] = (uint8_t)d;
-            order[pos++] = (uint16_t)u;
+            if (lane == 0) { place[u] = (uint8_t)d; order[pos] = (uint16_t)u; }
+            ++pos;
             int32_t tail = u;
             for (int32_t x = __ldg(dp.fnext + u); x >= 0 && ((__ldg(dp.fitmask + x) >> d) & 1u);
                  x = __ldg(dp.fnext + x)) {
-                place[x] = (uint8_t)d;
-                order[pos++] = (uint16_t)x;
-                fuse[x >> 5] |= 1u << (x & 31);
+                if (lane == 0) {
+                    place[x] = (uint8_t)d;
+                    order[pos] = (uint16_t)x;
+                    fuse[x >> 5] |= 1u << (x & 31);
+                }
+                ++pos;
                 kv = max(kv, (int64_t)__ldg(&dp.lk[x * D + d].y));
                 tail = x;
             }
-            if (pf) prefetch[u >> 5] |= 1u << (u & 31);
+            if (pf && lane == 0) prefetch[u >> 5] |= 1u << (u & 31);
 
             // Play it forward: admission with LRU reclamation (Eq. 11), load, run.
-            int64_t *st = s.stamp + d * M;
             const int64_t wm = __ldg(dp.weight + m);
             const int64_t need = hit ? kv : wm + kv;
             const int64_t capd = __ldg(dp.cap + d);
-            while (s.used[d] + need > capd) {
-                int32_t victim = -1;
-                for (int32_t k = 0; k < M; ++k)
-                    if (k != m && st[k] != 0 && (victim < 0 || st[k] < st[victim])) victim = k;
-                if (victim < 0) { atomicExch(dp.err, 4); return; }  // unreachable: the unit fits on d
-                s.used[d] -= __ldg(dp.weight + victim);
-                st[victim] = 0;
+            int64_t used = used_d[d];
+            while (used + need > capd) {
+                const uint32_t sk = (lane < M && lane != m && st[lane] != 0) ? st[lane] : 0xFFFFFFFFu;
+                const uint32_t smin = __reduce_min_sync(0xFFFFFFFFu, sk);
+                if (smin == 0xFFFFFFFFu) {  // unreachable: the unit fits on d
+                    if (lane == 0) atomicExch(dp.err, 4);
+                    return;
+                }
+                const int32_t victim = __ffs((int)__ballot_sync(0xFFFFFFFFu, sk == smin)) - 1;
+                used -= __ldg(dp.weight + victim);
+                __syncwarp();
+                if (lane == 0) st[victim] = 0;
+                __syncwarp();
             }
             int64_t start;
             if (hit) {
@@ -196,28 +260,45 @@ construct_kernel(wf_dev_problem dp, wf_plans out, uint64_t seed, int64_t jitter,
             } else {
                 const int64_t ls = pf ? max(tf, arr) : max(tf, rel);
                 start = max(ls + (int64_t)__ldg(dp.load + m * D + d), rel);
-                s.used[d] += wm;
+                used += wm;
             }
             int64_t fin = start + dp.grant;
             for (int32_t x = u;; x = __ldg(dp.fnext + x)) {
                 fin += __ldg(&dp.lk[x * D + d].x);
-                s.c[x] = fin;
                 if (x == tail) break;
             }
-            s.t_free[d] = fin;
-            st[m] = ++seq;
-
-            // Successors of the unit's last member.
-            for (int32_t e = __ldg(dp.succ_off + tail); e < __ldg(dp.succ_off + tail + 1); ++e) {
-                const int32_t y = __ldg(dp.succ_idx + e);
-                if (--s.pending[y] > 0) continue;
-                int64_t r = __ldg(dp.arrival + __ldg(dp.session + y));
-                for (int32_t f = __ldg(dp.pred_off + y); f < __ldg(dp.pred_off + y + 1); ++f)
-                    r = max(r, s.c[__ldg(dp.pred_idx + f)]);
-                s.c[y] = r;
-                const uint64_t j = jitter > 0 ? mix64(hp ^ (uint64_t)y) % jmod : 0;
-                heap_push(s.heap, nheap, (((uint64_t)r + j) << 16) | (uint64_t)y);
+            ++seq;
+            __syncwarp();
+            if (lane == 0) {
+                used_d[d] = used;
+                t_free[d] = fin;
+                st[m] = (uint16_t)seq;
             }
+            __syncwarp();
+
+            // Successors of the unit's last member, one per lane: each takes
+            // this finish into its release; the last predecessor makes it ready.
+            const int32_t e0 = __ldg(dp.succ_off + tail), e1 = __ldg(dp.succ_off + tail + 1);
+            for (int32_t eb = e0; eb < e1; eb += 32) {
+                const int32_t e = eb + lane;
+                bool take = false;
+                uint64_t key = 0;
+                int64_t r = 0;
+                if (e < e1) {
+                    const int32_t y = __ldg(dp.succ_idx + e);
+                    const int32_t left = s.pending[y] - 1;
+                    r = max(s.relmax[y], fin);
+                    s.pending[y] = left;
+                    s.relmax[y] = r;
+                    if (left == 0) {
+                        const uint64_t j = jitter > 0 ? mod64(mix64(hp ^ (uint64_t)y), jm) : 0;
+                        key = (((uint64_t)r + j) << 16) | (uint64_t)y;
+                        take = true;
+                    }
+                }
+                append(s, nready, take, key, r, lane);
+            }
+            __syncwarp();
         }
     }
 }
@@ -237,15 +318,22 @@ extern "C" int wf_construct_plans(wf_ctx *c, const wf_plans *out, uint64_t seed,
     if (rc) return rc;
     const wf_dev_problem &dp = c->dp;
     if (!c->construct_scratch) {
-        // First call: per-thread state for up to kPlansPerSm plans per SM at once.
-        c->construct_threads = std::min<int64_t>(c->max_P, (int64_t)c->sms * kPlansPerSm);
-        rc = wf_cuda_check(cudaMalloc(&c->construct_scratch, scratch_bytes(dp.N, dp.D, dp.M) * c->construct_threads),
+        // First call: per-plan state for up to kSlotsPerSm plans per SM at once.
+        c->construct_threads = std::min<int64_t>(c->max_P, (int64_t)c->sms * kSlotsPerSm);
+        rc = wf_cuda_check(cudaMalloc(&c->construct_scratch, scratch_bytes(dp.N) * c->construct_threads),
                            "cudaMalloc(constructor scratch)");
         if (rc) { c->construct_scratch = nullptr; return rc; }
     }
-    const int64_t threads = std::min<int64_t>(out->P, c->construct_threads);
-    const unsigned blocks = (unsigned)((threads + kThreads - 1) / kThreads);
-    construct_kernel<<<blocks, kThreads, 0, (cudaStream_t)stream>>>(dp, *out, seed, jitter_us,
-                                                                    (uint8_t *)c->construct_scratch, threads);
+    const int64_t slots = std::min<int64_t>(out->P, c->construct_threads);
+    const unsigned blocks = (unsigned)((slots + kWarps - 1) / kWarps);
+    const size_t smem = kWarps * warp_smem(dp.D, dp.M);
+    Mod64 jm = {0, 0, (uint64_t)jitter_us + 1};
+    if (jitter_us > 0) {
+        const unsigned __int128 r = ~(unsigned __int128)0 / jm.d + 1;
+        jm.mh = (uint64_t)(r >> 64);
+        jm.ml = (uint64_t)r;
+    }
+    construct_kernel<<<blocks, 32 * kWarps, smem, (cudaStream_t)stream>>>(dp, *out, seed, jitter_us, jm,
+                                                                          (uint8_t *)c->construct_scratch, slots);
     return wf_cuda_check(cudaGetLastError(), "construct launch");
 }

@@ -91,8 +91,8 @@ struct wf_ctx {
     bool wide_pending;
     int64_t wide_P;
     void *search_scratch;       // local search: the union's results [max_P], top-k ids, slot pairs
-    void *construct_scratch;    // plan constructor: per-thread state, allocated by its first call
-    int64_t construct_threads;
+    void *construct_scratch;    // plan constructor: per-plan state of the plans built at once, allocated by its first call
+    int64_t construct_threads;  // plans built at once (a warp each)
     int32_t *h_ovf;             // pinned host copy of ovf_count[0]
     cudaEvent_t sweep_done;     // recorded on the caller's stream after the sweeps
     cudaEvent_t ovf_event;      // recorded on side after the read-back

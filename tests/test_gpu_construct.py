@@ -50,6 +50,17 @@ def test_random_windows(case):
         assert bits.all() and not np.unpackbits(got[4].view(np.uint8), bitorder="little", axis=1)[:, N:].any()
 
 
+@pytest.mark.parametrize("jitter", [2, 3, (1 << 40) + 12345, (1 << 46) - 1])
+def test_jitter_remainders(jitter):
+    """Jitter draws mod (jitter + 1) over the whole 64-bit range of the hash:
+    the kernel's reciprocal-multiply remainder against the oracle's %."""
+    rng = np.random.default_rng(77)
+    prob = random_problem(rng, n_sessions=5, D=4, M=4)
+    got, res = build(prob, 64, seed=9, jitter=jitter, plan_base=5)
+    want, ends = oracle.construct(prob, 64, seed=9, jitter=jitter, plan_base=5)
+    check(prob, got, res, want, ends)
+
+
 @pytest.mark.parametrize("name,P", [("tiny", 300), ("mix", 200), ("burst", 64), ("large", 8)])
 def test_named_workloads(name, P):
     prob = wfgen.config(name).problem
