@@ -2,12 +2,16 @@
 // gpu, plan index), ascending.
 //
 //  1. select: one CTA finds T, the k-th smallest of the 64-bit keys
-//     (status != 0) << 63 | makespan, by radix selection (8 bits a pass);
+//     (status != 0) << 63 | makespan, by radix selection (8 bits a pass,
+//     the digit found by a warp scan of the histogram);
 //  2. compact: every plan whose 64-bit key is at most T becomes a candidate
 //     (all ties with T included, so the full key decides among them);
 //  3. final: one CTA sorts the candidates by the full key in shared memory
 //     (bitonic network) and writes the first k; more candidates than one
 //     tile (massive ties) are folded tile by tile into the running best k.
+//
+// Up to kOneCta plans, one CTA does all three with the keys staged in shared
+// memory (one launch).
 #include <algorithm>
 
 #include "wf_internal.cuh"
@@ -64,6 +68,81 @@ __device__ __forceinline__ TopkScratch scratch_of(void *base)
 
 constexpr int64_t kSelectShared = 20480;  // keys staged in shared memory up to this many plans
 
+// Warp-wide minimum / maximum of 64-bit values (two 32-bit reductions each).
+__device__ __forceinline__ uint64_t warp_min64(uint64_t v)
+{
+    const uint32_t hi = __reduce_min_sync(0xFFFFFFFFu, (uint32_t)(v >> 32));
+    const uint32_t lo = __reduce_min_sync(0xFFFFFFFFu, (uint32_t)(v >> 32) == hi ? (uint32_t)v : 0xFFFFFFFFu);
+    return ((uint64_t)hi << 32) | lo;
+}
+
+__device__ __forceinline__ uint64_t warp_max64(uint64_t v)
+{
+    const uint32_t hi = __reduce_max_sync(0xFFFFFFFFu, (uint32_t)(v >> 32));
+    const uint32_t lo = __reduce_max_sync(0xFFFFFFFFu, (uint32_t)(v >> 32) == hi ? (uint32_t)v : 0u);
+    return ((uint64_t)hi << 32) | lo;
+}
+
+// The radix passes can start at the highest byte in which the keys differ:
+// the bytes above it are the same in every key (those of the smallest).
+// From this thread's smallest and largest keys, the block's range gives
+// prefix and the first pass's shift (-8: all keys are equal, no pass).
+__device__ void first_pass(uint64_t mn, uint64_t mx, unsigned long long *wmin, unsigned long long *wmax,
+                           unsigned long long &prefix, int &first)
+{
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    mn = warp_min64(mn);
+    mx = warp_max64(mx);
+    if (lane == 0) { wmin[warp] = mn; wmax[warp] = mx; }
+    __syncthreads();
+    if (warp == 0) {
+        const int nw = (int)(blockDim.x >> 5);
+        mn = warp_min64(lane < nw ? wmin[lane] : ~0ull);
+        mx = warp_max64(lane < nw ? wmax[lane] : 0ull);
+        if (lane == 0) {
+            const uint64_t diff = mn ^ mx;
+            if (diff == 0) {
+                prefix = mn;
+                first = -8;
+            } else {
+                const int shift = ((63 - __clzll((long long)diff)) / 8) * 8;
+                prefix = shift == 56 ? 0ull : (mn & (~0ull << (shift + 8)));
+                first = shift;
+            }
+        }
+    }
+    __syncthreads();
+}
+
+// The digit of the k-th smallest key in this radix pass: warp 0 scans the
+// 256-bucket histogram (8 buckets a lane), finds the bucket holding rank,
+// and narrows prefix and rank to it.
+__device__ __forceinline__ void pick_digit(const unsigned int *hist, int shift, unsigned long long &prefix,
+                                           long long &rank)
+{
+    const int lane = threadIdx.x & 31;
+    unsigned int h[8], sum = 0;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) { h[j] = hist[8 * lane + j]; sum += h[j]; }
+    unsigned int inc = sum;  // inclusive prefix over lanes
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const unsigned int v = __shfl_up_sync(0xFFFFFFFFu, inc, o);
+        if (lane >= o) inc += v;
+    }
+    const long long r = rank;
+    const unsigned int over = __ballot_sync(0xFFFFFFFFu, (long long)inc > r);
+    const int src = __ffs((int)over) - 1;  // the lane whose buckets hold rank (rank < count)
+    if (lane == src) {
+        long long left = r - (long long)(inc - sum);
+        int b = 0;
+        while ((long long)h[b] <= left) { left -= h[b]; ++b; }
+        rank = left;
+        prefix |= (unsigned long long)(8 * lane + b) << shift;
+    }
+}
+
+
 template <bool kStaged>
 __global__ void __launch_bounds__(kThreads)
 select_kernel(wf_eval_out res, int64_t P, int32_t k, void *scr)
@@ -73,11 +152,18 @@ select_kernel(wf_eval_out res, int64_t P, int32_t k, void *scr)
     __shared__ unsigned long long prefix;
     __shared__ long long rank;
     const TopkScratch s = scratch_of(scr);
-    if (threadIdx.x == 0) { prefix = 0; rank = k - 1; *s.count = 0; }
-    if (kStaged)
-        for (int64_t p = threadIdx.x; p < P; p += blockDim.x) keys[p] = key64(res, p);
-    __syncthreads();
-    for (int shift = 56; shift >= 0; shift -= 8) {
+    __shared__ unsigned long long wmin[32], wmax[32];
+    __shared__ int shift0;
+    if (threadIdx.x == 0) { rank = k - 1; *s.count = 0; }
+    uint64_t mn = ~0ull, mx = 0;
+    for (int64_t p = threadIdx.x; p < P; p += blockDim.x) {
+        const uint64_t v = key64(res, p);
+        if (kStaged) keys[p] = v;
+        mn = min(mn, v);
+        mx = max(mx, v);
+    }
+    first_pass(mn, mx, wmin, wmax, prefix, shift0);
+    for (int shift = shift0; shift >= 0; shift -= 8) {
         for (int b = threadIdx.x; b < 256; b += blockDim.x) hist[b] = 0;
         __syncthreads();
         const unsigned long long hi = shift == 56 ? 0ull : (~0ull << (shift + 8));
@@ -87,13 +173,7 @@ select_kernel(wf_eval_out res, int64_t P, int32_t k, void *scr)
             if ((v & hi) == pre) atomicAdd(&hist[(v >> shift) & 255u], 1u);
         }
         __syncthreads();
-        if (threadIdx.x == 0) {
-            long long r = rank;
-            int b = 0;
-            while ((long long)hist[b] <= r) { r -= hist[b]; ++b; }
-            rank = r;
-            prefix |= (unsigned long long)b << shift;
-        }
+        if (threadIdx.x < 32) pick_digit(hist, shift, prefix, rank);
         __syncthreads();
     }
     if (threadIdx.x == 0) *s.T = prefix;
@@ -166,6 +246,84 @@ final_kernel(int32_t k, void *scr, int32_t *ids, int64_t *keys)
     }
 }
 
+constexpr int64_t kOneCta = 16384;  // plans handled by the single-CTA top-k
+
+__global__ void __launch_bounds__(kThreads)
+topk_one_kernel(wf_eval_out res, int64_t P, int32_t k, void *scr, int32_t *ids, int64_t *keys)
+{
+    extern __shared__ __align__(16) uint8_t tsm[];
+    Cand *t = (Cand *)tsm;                                               // kTile
+    unsigned long long *kk = (unsigned long long *)(tsm + kTile * sizeof(Cand));  // [P]
+    __shared__ unsigned int hist[256];
+    __shared__ unsigned long long prefix;
+    __shared__ long long rank;
+    __shared__ unsigned int ncand;
+    const TopkScratch s = scratch_of(scr);
+    __shared__ unsigned long long wmin[32], wmax[32];
+    __shared__ int shift0;
+    if (threadIdx.x == 0) { rank = k - 1; ncand = 0; }
+    uint64_t mn = ~0ull, mx = 0;
+    for (int64_t p = threadIdx.x; p < P; p += blockDim.x) {
+        const uint64_t v = key64(res, p);
+        kk[p] = v;
+        mn = min(mn, v);
+        mx = max(mx, v);
+    }
+    // 1. select T, the k-th smallest 64-bit key, 8 bits a pass from the
+    // highest byte in which the keys differ.
+    first_pass(mn, mx, wmin, wmax, prefix, shift0);
+    for (int shift = shift0; shift >= 0; shift -= 8) {
+        for (int b = threadIdx.x; b < 256; b += blockDim.x) hist[b] = 0;
+        __syncthreads();
+        const unsigned long long hi = shift == 56 ? 0ull : (~0ull << (shift + 8));
+        const unsigned long long pre = prefix;
+        for (int64_t p = threadIdx.x; p < P; p += blockDim.x) {
+            const uint64_t v = kk[p];
+            if ((v & hi) == pre) atomicAdd(&hist[(v >> shift) & 255u], 1u);
+        }
+        __syncthreads();
+        if (threadIdx.x < 32) pick_digit(hist, shift, prefix, rank);
+        __syncthreads();
+    }
+    const unsigned long long T = prefix;
+    // 2. every plan whose 64-bit key is at most T is a candidate.
+    for (int64_t p = threadIdx.x; p < P; p += blockDim.x) {
+        if (kk[p] > T) continue;
+        Cand c;
+        c.mk = res.makespan_us[p];
+        c.p95 = res.p95_us[p];
+        c.gpu = res.gpu_us[p];
+        c.id = (int32_t)p;
+        c.bad = res.status[p] != 0 ? 1u : 0u;
+        s.cand[atomicAdd(&ncand, 1u)] = c;
+    }
+    __syncthreads();
+    // 3. sort, as final_kernel.
+    const int64_t n = ncand;
+    int len = 64;
+    while (len < n && len < kTile) len <<= 1;
+    int64_t next = 0;
+    bool first = true;
+    while (first || next < n) {
+        const int base = first ? 0 : k;
+        for (int u = threadIdx.x; u < len - base; u += blockDim.x) {
+            const int64_t c = next + u;
+            t[base + u] = c < n ? s.cand[c] : padding();
+        }
+        next += len - base;
+        first = false;
+        bitonic_sort(t, len);
+    }
+    for (int u = threadIdx.x; u < k; u += blockDim.x) {
+        ids[u] = t[u].id;
+        if (keys) {
+            keys[3 * u] = t[u].mk;
+            keys[3 * u + 1] = t[u].p95;
+            keys[3 * u + 2] = t[u].gpu;
+        }
+    }
+}
+
 }  // namespace
 
 size_t wf_topk_scratch_bytes(int64_t max_P)
@@ -177,6 +335,14 @@ int wf_launch_topk(wf_ctx *ctx, const wf_eval_out *res, int64_t P, int32_t k, in
                    int64_t *keys, cudaStream_t st)
 {
     const size_t smem = kTile * sizeof(Cand);
+    if (P <= kOneCta) {
+        const size_t one = smem + 8 * (size_t)P;
+        int rc = wf_cuda_check(cudaFuncSetAttribute(topk_one_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                    (int)one), "topk smem attribute");
+        if (rc) return rc;
+        topk_one_kernel<<<1, kThreads, one, st>>>(*res, P, k, ctx->topk_scratch, ids, keys);
+        return wf_cuda_check(cudaGetLastError(), "topk launch");
+    }
     int rc = wf_cuda_check(cudaFuncSetAttribute(final_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                 (int)smem), "topk smem attribute");
     if (rc) return rc;
