@@ -126,7 +126,8 @@ typedef struct {
  *     retain may be NULL (every model retained after its units).
  *   Strides are in bytes and multiples of 16; place_stride >= N,
  *   order_stride >= 2N, bits_stride >= 4*ceil(N/32).  Base pointers must be
- *   16-byte aligned.  plan_base is the global index of row 0 (it seeds the
+ *   16-byte aligned, and each array spans P whole rows of its stride (the
+ *   kernels read rows in 16-byte pieces, up to the row's padding).  plan_base is the global index of row 0 (it seeds the
  *   latency samples, so shards of one batch reproduce the whole batch).
  */
 typedef struct {

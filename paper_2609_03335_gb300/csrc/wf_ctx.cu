@@ -267,16 +267,16 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
     size_t o_lk = img.add(lk.data(), sizeof(int2) * lk.size());
     // Status tables: the devices each activation fits on (Eq. 8), padded to a
     // multiple of four entries, and every edge packed as pred | succ << 16.
-    std::vector<uint32_t> fitmask(((size_t)N + 3) & ~(size_t)3, 0u);
+    std::vector<uint32_t> fitmask(((size_t)N + 15) & ~(size_t)15, 0u);  // read 16 at a time
     for (int32_t n = 0; n < N; ++n)
         for (int32_t d = 0; d < D; ++d)
             if (adm[(int64_t)n * D + d] <= pb->cap_mib[d]) fitmask[n] |= 1u << d;
     size_t o_fit = img.add(fitmask.data(), sizeof(uint32_t) * fitmask.size());
-    std::vector<uint32_t> edges(E);
+    std::vector<uint32_t> edges(((size_t)E + 3) & ~(size_t)3, 0u);  // read 4 at a time
     for (int32_t v = 0; v < N; ++v)
         for (int32_t e = pb->pred_off[v]; e < pb->pred_off[v + 1]; ++e)
             edges[e] = (uint32_t)pb->pred_idx[e] | ((uint32_t)v << 16);
-    size_t o_edges = img.add(edges.data(), sizeof(uint32_t) * E);
+    size_t o_edges = img.add(edges.data(), sizeof(uint32_t) * edges.size());
     // Successor lists (the transpose of pred CSR) for the plan constructor,
     // and a bound on any time a plan of the window can reach.
     std::vector<int32_t> succ_off(N + 1, 0), succ_idx(E > 0 ? E : 1);

@@ -1137,41 +1137,57 @@ status_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out)
         const uint8_t *place = pl.place + p * pl.place_stride;
         const uint16_t *order = (const uint16_t *)((const uint8_t *)pl.order + p * pl.order_stride);
         uint32_t st = 0;
-        // Rows start 16-byte aligned and hold at least N entries; a word read
-        // past N stays inside the row's padding to 4 bytes only when used
-        // below N, so lanes mask the entries at or beyond N.
-        for (int32_t n4 = 4 * lane; n4 < N; n4 += 128) {
-            const uint32_t pw = __ldg((const uint32_t *)(place + n4));
-            const uint4 fm = __ldg((const uint4 *)(dp.fitmask + n4));
-            const uint32_t f[4] = {fm.x, fm.y, fm.z, fm.w};
+        // Rows start 16-byte aligned and their strides are multiples of 16
+        // bytes, so 16-byte reads at multiples of 16 bytes below N stay in
+        // the row; lanes mask the entries at or beyond N.  The fit masks are
+        // padded to 16 entries.
+        for (int32_t n16 = 16 * lane; n16 < N; n16 += 512) {
+            const uint4 pw = __ldg((const uint4 *)(place + n16));
+            const uint32_t pws[4] = {pw.x, pw.y, pw.z, pw.w};
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const uint32_t d = (pw >> (8 * j)) & 255u;
-                if (n4 + j < N) st |= d >= (uint32_t)D ? WF_ST_DEVICE : (((f[j] >> d) & 1u) ? 0u : WF_ST_CAPACITY);
+            for (int q = 0; q < 4; ++q) {
+                const uint4 fm = __ldg((const uint4 *)(dp.fitmask + n16 + 4 * q));
+                const uint32_t f[4] = {fm.x, fm.y, fm.z, fm.w};
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const uint32_t d = (pws[q] >> (8 * j)) & 255u;
+                    if (n16 + 4 * q + j < N)
+                        st |= d >= (uint32_t)D ? WF_ST_DEVICE : (((f[j] >> d) & 1u) ? 0u : WF_ST_CAPACITY);
+                }
             }
         }
-        for (int32_t i = 2 * lane; i < N; i += 64) {
-            const uint32_t ow = __ldg((const uint32_t *)(order + i));
-            const uint32_t h0 = ow & 0xFFFFu, h1 = ow >> 16;
-            if (h0 < (uint32_t)N) pos[h0] = (uint16_t)i;
-            else st |= WF_ST_PERMUTATION;
-            if (i + 1 < N) {
-                if (h1 < (uint32_t)N) pos[h1] = (uint16_t)(i + 1);
-                else st |= WF_ST_PERMUTATION;
+        // The inverse permutation, 8 dispatch entries a lane at a time, then
+        // read back: a repeated node leaves some entry unmatched.
+        for (int32_t i8 = 8 * lane; i8 < N; i8 += 256) {
+            const uint4 ow = __ldg((const uint4 *)(order + i8));
+            const uint32_t w[4] = {ow.x, ow.y, ow.z, ow.w};
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const uint32_t h = (w[j >> 1] >> (16 * (j & 1))) & 0xFFFFu;
+                if (i8 + j < N) {
+                    if (h < (uint32_t)N) pos[h] = (uint16_t)(i8 + j);
+                    else st |= WF_ST_PERMUTATION;
+                }
             }
         }
         __syncwarp();
-        for (int32_t i = 2 * lane; i < N; i += 64) {
-            const uint32_t ow = __ldg((const uint32_t *)(order + i));
-            const uint32_t h0 = ow & 0xFFFFu, h1 = ow >> 16;
-            if (h0 < (uint32_t)N && pos[h0] != (uint16_t)i) st |= WF_ST_PERMUTATION;
-            if (i + 1 < N && h1 < (uint32_t)N && pos[h1] != (uint16_t)(i + 1)) st |= WF_ST_PERMUTATION;
+        for (int32_t i8 = 8 * lane; i8 < N; i8 += 256) {
+            const uint4 ow = __ldg((const uint4 *)(order + i8));
+            const uint32_t w[4] = {ow.x, ow.y, ow.z, ow.w};
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const uint32_t h = (w[j >> 1] >> (16 * (j & 1))) & 0xFFFFu;
+                if (i8 + j < N && h < (uint32_t)N && pos[h] != (uint16_t)(i8 + j)) st |= WF_ST_PERMUTATION;
+            }
         }
         st = __reduce_or_sync(0xFFFFFFFFu, st);
         if (!(st & WF_ST_PERMUTATION)) {
-            for (int32_t e = lane; e < E; e += 32) {
-                const uint32_t uv = __ldg(dp.edges + e);
-                if (pos[uv & 0xFFFFu] > pos[uv >> 16]) st |= WF_ST_TOPOLOGY;
+            for (int32_t e4 = 4 * lane; e4 < E; e4 += 128) {  // edges padded to 4
+                const uint4 uv = __ldg((const uint4 *)(dp.edges + e4));
+                const uint32_t w[4] = {uv.x, uv.y, uv.z, uv.w};
+#pragma unroll
+                for (int j = 0; j < 4; ++j)
+                    if (e4 + j < E && pos[w[j] & 0xFFFFu] > pos[w[j] >> 16]) st |= WF_ST_TOPOLOGY;
             }
             st = __reduce_or_sync(0xFFFFFFFFu, st);
         }
