@@ -1299,8 +1299,12 @@ int launch_pc_r(const wf_ctx *ctx, int kp, const wf_plans *pl, const wf_eval_out
             return dp.M <= 8
                        ? launch_pc<uint32_t, TT, 16, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
                        : launch_pc<uint64_t, TT, 16, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
-        return dp.M <= 8 ? launch_pc<uint32_t, TT, 6, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
-                         : launch_pc<uint64_t, TT, 6, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
+        if (kp == 6)
+            return dp.M <= 8
+                       ? launch_pc<uint32_t, TT, 6, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
+                       : launch_pc<uint64_t, TT, 6, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
+        return dp.M <= 8 ? launch_pc<uint32_t, TT, 3, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
+                         : launch_pc<uint64_t, TT, 3, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
     }
 }
 
@@ -1332,14 +1336,18 @@ wf_sweep_cfg wf_sweep_config(const wf_dev_problem &dp)
     const size_t s32 = r ? pc_layout<kPlans32, uint32_t, 1>(dp.D, dp.M, dp.W, NS).total
                          : pc_layout<kPlans32, uint32_t, 0>(dp.D, dp.M, dp.W, NS).total;
     if (s32 <= 227 * 1024) c.smem32 = s32;
-    // The u64 sweep: 16 plans per CTA, or 6 where that keeps more plans per SM.
+    // The u64 sweep: 16, 6 or 3 plans per CTA, whichever keeps the most plans
+    // per SM (ties: the smaller CTAs, more of them to hide latency).
     const size_t s16 = r ? pc_layout<16, uint64_t, 1>(dp.D, dp.M, dp.W, NS).total
                          : pc_layout<16, uint64_t, 0>(dp.D, dp.M, dp.W, NS).total;
     const size_t s6 = r ? pc_layout<6, uint64_t, 1>(dp.D, dp.M, dp.W, NS).total
                         : pc_layout<6, uint64_t, 0>(dp.D, dp.M, dp.W, NS).total;
-    const int a = plans_per_sm(s16, 16), b = plans_per_sm(s6, 6);
-    if (a > 0 && a >= b) { c.smem64 = s16; c.plans64 = 16; }
-    else if (b > 0) { c.smem64 = s6; c.plans64 = 6; }
+    const size_t s3 = r ? pc_layout<3, uint64_t, 1>(dp.D, dp.M, dp.W, NS).total
+                        : pc_layout<3, uint64_t, 0>(dp.D, dp.M, dp.W, NS).total;
+    const int a = plans_per_sm(s16, 16), b = plans_per_sm(s6, 6), e = plans_per_sm(s3, 3);
+    if (e > 0 && e >= a && e >= b) { c.smem64 = s3; c.plans64 = 3; }
+    else if (b > 0 && b >= a) { c.smem64 = s6; c.plans64 = 6; }
+    else if (a > 0) { c.smem64 = s16; c.plans64 = 16; }
     return c;
 }
 
