@@ -115,6 +115,25 @@ def test_random_windows_with_invalid_plans_retain_and_grant(seed):
     assert np.array_equal(got["rel"], rel) and np.array_equal(got["comp"], comp)
 
 
+@pytest.mark.parametrize("seed", range(10))
+def test_random_device_and_model_counts(seed):
+    """Device counts 1-32 and model counts 1-16 (so residency lanes own one to
+    eight devices, queues of 32 or 64 bits), with retain bits, grant and
+    admission margin, and both reclamation policies."""
+    rng = np.random.default_rng(5200 + seed)
+    D, M = int(rng.integers(1, 33)), int(rng.integers(1, 17))
+    prob = random_problem(rng, n_sessions=int(rng.integers(2, 10)), sizes=(4, 12), D=D, M=M)
+    prob = prob.with_(grant_us=int(rng.integers(0, 300)), margin_mib=int(rng.integers(0, 3)),
+                      reclaim=int(seed % 3 == 2))
+    if not prob.fits().any(axis=1).all():  # every activation must fit somewhere
+        prob = prob.with_(margin_mib=0)
+    P = int(rng.integers(50, 600))
+    plans = wfgen.make_plans(prob, P, seed, p_fuse=float(rng.uniform(0, 1)),
+                             p_prefetch=float(rng.uniform(0, 1)),
+                             p_retain=float(rng.uniform(0.3, 1)) if seed % 2 else None)
+    assert_same(gpu_eval(prob, plans, k=min(P, 8)), oracle_eval(prob, plans))
+
+
 @pytest.mark.parametrize("seed", range(3))
 def test_random_stochastic_windows(seed):
     rng = np.random.default_rng(4100 + seed)
