@@ -622,24 +622,27 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
                     q = hit ? Lru<Q>::remove(q, hit ? kq : 0) : q;  // (an index below the queue length)
                     n -= hit ? 1u : 0u;
                     const uint32_t need = hit ? r1 : wm + r1;
-                    const int64_t here = c * kChunk + k;
+                    const int32_t here = c * kChunk + k;
                     while (u_d + need > capd && n > 0) {
+                        // The class (redundant << 1 | infinite) ranks first; within
+                        // a finite class the larger distance per unit of cost
+                        // (32-bit factors, exact 64-bit products); ties keep the
+                        // earlier queue entry.
                         int32_t best = 0;
-                        uint32_t bred = 0, binf = 0;
-                        int64_t bdist = 0, bcost = 0;
+                        uint32_t bcls = 0;
+                        int32_t bdist = 0, bcost = 0;
                         for (int32_t e = 0; e < (int32_t)n; ++e) {
                             const uint32_t kk = (uint32_t)(q >> (4 * e)) & 15u;
                             const uint32_t red = rcnt[kk * kP] > 1;
                             const uint32_t nu = nuse[(d * M + kk) * kP];
-                            const int64_t cost = load[kk * D + d];
+                            const int32_t cost = load[kk * D + d];
                             const uint32_t inf = nu == 0xFFFFu || cost == 0;
-                            const int64_t dist = (int64_t)nu - here;
-                            bool better;
-                            if (e == 0) better = true;
-                            else if (red != bred) better = red > bred;
-                            else if (inf != binf) better = inf > binf;
-                            else better = !inf && dist * bcost > bdist * cost;
-                            if (better) { best = e; bred = red; binf = inf; bdist = dist; bcost = cost; }
+                            const uint32_t cls = (red << 1) | inf;
+                            const int32_t dist = (int32_t)nu - here;
+                            if (e == 0 || cls > bcls ||
+                                (cls == bcls && !inf && (int64_t)dist * bcost > (int64_t)bdist * cost)) {
+                                best = e; bcls = cls; bdist = dist; bcost = cost;
+                            }
                         }
                         const uint32_t victim = (uint32_t)(q >> (4 * best)) & 15u;
                         u_d -= (uint32_t)weight[victim];
