@@ -45,8 +45,9 @@ def algorithmic_bytes_per_plan(N: int) -> int:
 
 
 def topk_launches(P: int, k: int) -> int:
-    """Kernel launches of one wf_topk call: select, compact, final."""
-    return 3
+    """Kernel launches of one wf_topk call: one CTA does select, compact and
+    sort up to 16,384 plans; beyond, three kernels."""
+    return 1 if P <= 16384 else 3
 
 
 def kernel_source_hash() -> str:
