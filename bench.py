@@ -46,7 +46,8 @@ def algorithmic_bytes_per_plan(N: int) -> int:
 
 def topk_launches(P: int, k: int) -> int:
     """Kernel launches of one wf_topk call: one CTA does select, compact and
-    sort up to 16,384 plans; beyond, three kernels."""
+    sort up to 16,384 plans; beyond, three kernels (tile bounds, compaction,
+    final select and sort; the two scratch words are reset by memsets)."""
     return 1 if P <= 16384 else 3
 
 

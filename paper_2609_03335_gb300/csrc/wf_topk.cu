@@ -1,9 +1,8 @@
 // Top-k of evaluated plans (row a12) by the key (status != 0, makespan, p95,
 // gpu, plan index), ascending.
 //
-//  1. select: one CTA finds T, the k-th smallest of the 64-bit keys
-//     (status != 0) << 63 | makespan, by radix selection (8 bits a pass,
-//     the digit found by a warp scan of the histogram);
+//  1. threshold: T, a 64-bit key (status != 0) << 63 | makespan that at
+//     least k plans' keys do not exceed;
 //  2. compact: every plan whose 64-bit key is at most T becomes a candidate
 //     (all ties with T included, so the full key decides among them);
 //  3. final: one CTA sorts the candidates by the full key in shared memory
@@ -11,7 +10,12 @@
 //     tile (massive ties) are folded tile by tile into the running best k.
 //
 // Up to kOneCta plans, one CTA does all three with the keys staged in shared
-// memory (one launch).
+// memory (one launch): T is the exact k-th smallest key, found by radix
+// selection (8 bits a pass, the digit found by a warp scan of the
+// histogram), so usually about k candidates reach the sort.  Beyond, T is
+// first the smallest of the tiles' own k-th keys (kth_kernel, one CTA a
+// tile); the final CTA then runs the same exact selection over those
+// candidates before sorting.
 #include <algorithm>
 
 #include "wf_internal.cuh"
@@ -65,8 +69,6 @@ __device__ __forceinline__ TopkScratch scratch_of(void *base)
     s.cand = (Cand *)((uint8_t *)base + 64);
     return s;
 }
-
-constexpr int64_t kSelectShared = 20480;  // keys staged in shared memory up to this many plans
 
 // Warp-wide minimum / maximum of 64-bit values (two 32-bit reductions each).
 __device__ __forceinline__ uint64_t warp_min64(uint64_t v)
@@ -143,42 +145,6 @@ __device__ __forceinline__ void pick_digit(const unsigned int *hist, int shift, 
 }
 
 
-template <bool kStaged>
-__global__ void __launch_bounds__(kThreads)
-select_kernel(wf_eval_out res, int64_t P, int32_t k, void *scr)
-{
-    extern __shared__ unsigned long long keys[];
-    __shared__ unsigned int hist[256];
-    __shared__ unsigned long long prefix;
-    __shared__ long long rank;
-    const TopkScratch s = scratch_of(scr);
-    __shared__ unsigned long long wmin[32], wmax[32];
-    __shared__ int shift0;
-    if (threadIdx.x == 0) { rank = k - 1; *s.count = 0; }
-    uint64_t mn = ~0ull, mx = 0;
-    for (int64_t p = threadIdx.x; p < P; p += blockDim.x) {
-        const uint64_t v = key64(res, p);
-        if (kStaged) keys[p] = v;
-        mn = min(mn, v);
-        mx = max(mx, v);
-    }
-    first_pass(mn, mx, wmin, wmax, prefix, shift0);
-    for (int shift = shift0; shift >= 0; shift -= 8) {
-        for (int b = threadIdx.x; b < 256; b += blockDim.x) hist[b] = 0;
-        __syncthreads();
-        const unsigned long long hi = shift == 56 ? 0ull : (~0ull << (shift + 8));
-        const unsigned long long pre = prefix;
-        for (int64_t p = threadIdx.x; p < P; p += blockDim.x) {
-            const uint64_t v = kStaged ? keys[p] : key64(res, p);
-            if ((v & hi) == pre) atomicAdd(&hist[(v >> shift) & 255u], 1u);
-        }
-        __syncthreads();
-        if (threadIdx.x < 32) pick_digit(hist, shift, prefix, rank);
-        __syncthreads();
-    }
-    if (threadIdx.x == 0) *s.T = prefix;
-}
-
 __global__ void compact_kernel(wf_eval_out res, int64_t P, void *scr)
 {
     const TopkScratch s = scratch_of(scr);
@@ -193,6 +159,61 @@ __global__ void compact_kernel(wf_eval_out res, int64_t P, void *scr)
         c.bad = res.status[p] != 0 ? 1u : 0u;
         s.cand[atomicAdd(s.count, 1u)] = c;
     }
+}
+
+// The k-th smallest of kk[0, n) (shared memory, k <= n), by radix selection
+// from the highest byte in which the keys differ.  Every thread of the CTA
+// calls it with the smallest and largest of the keys it wrote.
+__device__ unsigned long long radix_kth(const unsigned long long *kk, int64_t n, int32_t k, uint64_t mn,
+                                        uint64_t mx)
+{
+    __shared__ unsigned int hist[256];
+    __shared__ unsigned long long prefix;
+    __shared__ long long rank;
+    __shared__ unsigned long long wmin[32], wmax[32];
+    __shared__ int shift0;
+    if (threadIdx.x == 0) rank = k - 1;
+    first_pass(mn, mx, wmin, wmax, prefix, shift0);
+    for (int shift = shift0; shift >= 0; shift -= 8) {
+        for (int b = threadIdx.x; b < 256; b += blockDim.x) hist[b] = 0;
+        __syncthreads();
+        const unsigned long long hi = shift == 56 ? 0ull : (~0ull << (shift + 8));
+        const unsigned long long pre = prefix;
+        for (int64_t i = threadIdx.x; i < n; i += blockDim.x) {
+            const uint64_t v = kk[i];
+            if ((v & hi) == pre) atomicAdd(&hist[(v >> shift) & 255u], 1u);
+        }
+        __syncthreads();
+        if (threadIdx.x < 32) pick_digit(hist, shift, prefix, rank);
+        __syncthreads();
+    }
+    return prefix;
+}
+
+// Beyond kOneCta plans: each CTA finds the k-th smallest 64-bit key of a
+// tile of kKth plans and lowers T to it.  Every tile's k-th key bounds the
+// batch's k-th from above, so the keys at most T (the smallest bound) hold
+// the k best, ties included; compact and final take it from there.  T starts
+// at all ones and the candidate count at 0 (host memsets).
+constexpr int kKth = 4096;
+
+__global__ void __launch_bounds__(kThreads)
+kth_kernel(wf_eval_out res, int64_t P, int32_t k, void *scr)
+{
+    __shared__ unsigned long long v[kKth];
+    const TopkScratch s = scratch_of(scr);
+    const int64_t base = (int64_t)blockIdx.x * kKth;
+    const int n = P - base < kKth ? (int)(P - base) : kKth;
+    if (n < k) return;  // a short last tile bounds nothing
+    uint64_t mn = ~0ull, mx = 0;
+    for (int u = threadIdx.x; u < n; u += blockDim.x) {
+        const uint64_t x = key64(res, base + u);
+        v[u] = x;
+        mn = min(mn, x);
+        mx = max(mx, x);
+    }
+    const unsigned long long T = radix_kth(v, n, k, mn, mx);
+    if (threadIdx.x == 0) atomicMin(s.T, T);
 }
 
 // Sorts t[0, len) ascending; len is a power of two, at most kTile.
@@ -213,29 +234,8 @@ __device__ void bitonic_sort(Cand *t, int len)
     __syncthreads();
 }
 
-__global__ void __launch_bounds__(kThreads)
-final_kernel(int32_t k, void *scr, int32_t *ids, int64_t *keys)
+__device__ void write_first(const Cand *t, int32_t k, int32_t *ids, int64_t *keys)
 {
-    extern __shared__ Cand t[];
-    const TopkScratch s = scratch_of(scr);
-    const int64_t n = *s.count;
-    // One network of the smallest power-of-two size that holds every candidate
-    // when they fit a tile; otherwise the running best k occupy t[0, k) and
-    // each round fills the rest of a full tile with new candidates.
-    int len = 64;
-    while (len < n && len < kTile) len <<= 1;
-    int64_t next = 0;
-    bool first = true;
-    while (first || next < n) {
-        const int base = first ? 0 : k;
-        for (int u = threadIdx.x; u < len - base; u += blockDim.x) {
-            const int64_t c = next + u;
-            t[base + u] = c < n ? s.cand[c] : padding();
-        }
-        next += len - base;
-        first = false;
-        bitonic_sort(t, len);
-    }
     for (int u = threadIdx.x; u < k; u += blockDim.x) {
         ids[u] = t[u].id;
         if (keys) {
@@ -246,60 +246,36 @@ final_kernel(int32_t k, void *scr, int32_t *ids, int64_t *keys)
     }
 }
 
-constexpr int64_t kOneCta = 16384;  // plans handled by the single-CTA top-k
-
-__global__ void __launch_bounds__(kThreads)
-topk_one_kernel(wf_eval_out res, int64_t P, int32_t k, void *scr, int32_t *ids, int64_t *keys)
-{
-    extern __shared__ __align__(16) uint8_t tsm[];
-    Cand *t = (Cand *)tsm;                                               // kTile
-    unsigned long long *kk = (unsigned long long *)(tsm + kTile * sizeof(Cand));  // [P]
-    __shared__ unsigned int hist[256];
-    __shared__ unsigned long long prefix;
-    __shared__ long long rank;
-    __shared__ unsigned int ncand;
-    const TopkScratch s = scratch_of(scr);
-    __shared__ unsigned long long wmin[32], wmax[32];
-    __shared__ int shift0;
-    if (threadIdx.x == 0) { rank = k - 1; ncand = 0; }
-    uint64_t mn = ~0ull, mx = 0;
-    for (int64_t p = threadIdx.x; p < P; p += blockDim.x) {
-        const uint64_t v = key64(res, p);
-        kk[p] = v;
-        mn = min(mn, v);
-        mx = max(mx, v);
-    }
-    // 1. select T, the k-th smallest 64-bit key, 8 bits a pass from the
-    // highest byte in which the keys differ.
-    first_pass(mn, mx, wmin, wmax, prefix, shift0);
-    for (int shift = shift0; shift >= 0; shift -= 8) {
-        for (int b = threadIdx.x; b < 256; b += blockDim.x) hist[b] = 0;
-        __syncthreads();
-        const unsigned long long hi = shift == 56 ? 0ull : (~0ull << (shift + 8));
-        const unsigned long long pre = prefix;
-        for (int64_t p = threadIdx.x; p < P; p += blockDim.x) {
-            const uint64_t v = kk[p];
-            if ((v & hi) == pre) atomicAdd(&hist[(v >> shift) & 255u], 1u);
-        }
-        __syncthreads();
-        if (threadIdx.x < 32) pick_digit(hist, shift, prefix, rank);
-        __syncthreads();
-    }
-    const unsigned long long T = prefix;
-    // 2. every plan whose 64-bit key is at most T is a candidate.
-    for (int64_t p = threadIdx.x; p < P; p += blockDim.x) {
-        if (kk[p] > T) continue;
+// Items to rank: the plans of an evaluated batch, or the candidates
+// compacted into scratch.
+struct PlanSrc {
+    wf_eval_out res;
+    __device__ uint64_t key(int64_t i) const { return key64(res, i); }
+    __device__ Cand get(int64_t i) const
+    {
         Cand c;
-        c.mk = res.makespan_us[p];
-        c.p95 = res.p95_us[p];
-        c.gpu = res.gpu_us[p];
-        c.id = (int32_t)p;
-        c.bad = res.status[p] != 0 ? 1u : 0u;
-        s.cand[atomicAdd(&ncand, 1u)] = c;
+        c.mk = res.makespan_us[i];
+        c.p95 = res.p95_us[i];
+        c.gpu = res.gpu_us[i];
+        c.id = (int32_t)i;
+        c.bad = res.status[i] != 0 ? 1u : 0u;
+        return c;
     }
-    __syncthreads();
-    // 3. sort, as final_kernel.
-    const int64_t n = ncand;
+};
+
+struct CandSrc {
+    const Cand *cand;
+    __device__ uint64_t key(int64_t i) const { return ((uint64_t)cand[i].bad << 63) | (uint64_t)cand[i].mk; }
+    __device__ Cand get(int64_t i) const { return cand[i]; }
+};
+
+// Sorts the items of src[0, n) that qualify (all when kk is null, else those
+// with kk[i] <= T) by the full key, a tile at a time: the running best k stay
+// in t[0, k) and each round fills the rest of the tile; writes the first k.
+template <class Src>
+__device__ void fold_sort(const Src &src, int64_t n, int32_t k, const unsigned long long *kk,
+                          unsigned long long T, Cand *t, int32_t *ids, int64_t *keys)
+{
     int len = 64;
     while (len < n && len < kTile) len <<= 1;
     int64_t next = 0;
@@ -308,20 +284,72 @@ topk_one_kernel(wf_eval_out res, int64_t P, int32_t k, void *scr, int32_t *ids, 
         const int base = first ? 0 : k;
         for (int u = threadIdx.x; u < len - base; u += blockDim.x) {
             const int64_t c = next + u;
-            t[base + u] = c < n ? s.cand[c] : padding();
+            t[base + u] = c < n && (!kk || kk[c] <= T) ? src.get(c) : padding();
         }
         next += len - base;
         first = false;
         bitonic_sort(t, len);
     }
-    for (int u = threadIdx.x; u < k; u += blockDim.x) {
-        ids[u] = t[u].id;
-        if (keys) {
-            keys[3 * u] = t[u].mk;
-            keys[3 * u + 1] = t[u].p95;
-            keys[3 * u + 2] = t[u].gpu;
-        }
+    write_first(t, k, ids, keys);
+}
+
+// The k best of src[0, n) (k <= n <= kOneCta): the 64-bit keys staged in kk,
+// T the exact k-th smallest of them, the items with keys at most T gathered
+// into t and sorted there by the full key.
+template <class Src>
+__device__ void select_and_sort(const Src &src, int64_t n, int32_t k, unsigned long long *kk, Cand *t,
+                                int32_t *ids, int64_t *keys)
+{
+    __shared__ unsigned int m;
+    if (threadIdx.x == 0) m = 0;
+    uint64_t mn = ~0ull, mx = 0;
+    for (int64_t i = threadIdx.x; i < n; i += blockDim.x) {
+        const uint64_t v = src.key(i);
+        kk[i] = v;
+        mn = min(mn, v);
+        mx = max(mx, v);
     }
+    const unsigned long long T = radix_kth(kk, n, k, mn, mx);
+    for (int64_t i = threadIdx.x; i < n; i += blockDim.x) {
+        if (kk[i] > T) continue;
+        const unsigned int slot = atomicAdd(&m, 1u);
+        if (slot < (unsigned)kTile) t[slot] = src.get(i);
+    }
+    __syncthreads();
+    const unsigned int cnt = m;
+    if (cnt > (unsigned)kTile) {  // massive ties with T
+        fold_sort(src, n, k, kk, T, t, ids, keys);
+        return;
+    }
+    int len = 64;
+    while (len < (int)cnt) len <<= 1;
+    for (int u = (int)cnt + threadIdx.x; u < len; u += blockDim.x) t[u] = padding();
+    bitonic_sort(t, len);
+    write_first(t, k, ids, keys);
+}
+
+constexpr int64_t kOneCta = 16384;  // keys staged in shared memory by one CTA
+
+__global__ void __launch_bounds__(kThreads)
+final_kernel(int32_t k, void *scr, int32_t *ids, int64_t *keys)
+{
+    extern __shared__ __align__(16) uint8_t tsm[];
+    Cand *t = (Cand *)tsm;
+    unsigned long long *kk = (unsigned long long *)(tsm + kTile * sizeof(Cand));  // [kOneCta]
+    const TopkScratch s = scratch_of(scr);
+    const int64_t n = *s.count;
+    const CandSrc src{s.cand};
+    if (n <= kOneCta) select_and_sort(src, n, k, kk, t, ids, keys);
+    else fold_sort(src, n, k, nullptr, 0ull, t, ids, keys);
+}
+
+__global__ void __launch_bounds__(kThreads)
+topk_one_kernel(wf_eval_out res, int64_t P, int32_t k, int32_t *ids, int64_t *keys)
+{
+    extern __shared__ __align__(16) uint8_t tsm[];
+    Cand *t = (Cand *)tsm;
+    unsigned long long *kk = (unsigned long long *)(tsm + kTile * sizeof(Cand));  // [P]
+    select_and_sort(PlanSrc{res}, P, k, kk, t, ids, keys);
 }
 
 }  // namespace
@@ -334,27 +362,22 @@ size_t wf_topk_scratch_bytes(int64_t max_P)
 int wf_launch_topk(wf_ctx *ctx, const wf_eval_out *res, int64_t P, int32_t k, int32_t *ids,
                    int64_t *keys, cudaStream_t st)
 {
-    const size_t smem = kTile * sizeof(Cand);
+    const size_t smem = kTile * sizeof(Cand) + 8 * (size_t)std::min<int64_t>(P, kOneCta);
     if (P <= kOneCta) {
-        const size_t one = smem + 8 * (size_t)P;
         int rc = wf_cuda_check(cudaFuncSetAttribute(topk_one_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                    (int)one), "topk smem attribute");
+                                                    (int)smem), "topk smem attribute");
         if (rc) return rc;
-        topk_one_kernel<<<1, kThreads, one, st>>>(*res, P, k, ctx->topk_scratch, ids, keys);
+        topk_one_kernel<<<1, kThreads, smem, st>>>(*res, P, k, ids, keys);
         return wf_cuda_check(cudaGetLastError(), "topk launch");
     }
     int rc = wf_cuda_check(cudaFuncSetAttribute(final_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                 (int)smem), "topk smem attribute");
     if (rc) return rc;
-    if (P <= kSelectShared) {
-        const size_t ks = 8 * (size_t)P;
-        rc = wf_cuda_check(cudaFuncSetAttribute(select_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                (int)ks), "topk select smem attribute");
-        if (rc) return rc;
-        select_kernel<true><<<1, kThreads, ks, st>>>(*res, P, k, ctx->topk_scratch);
-    } else {
-        select_kernel<false><<<1, kThreads, 0, st>>>(*res, P, k, ctx->topk_scratch);
-    }
+    // T = all ones, candidate count = 0 (scratch words 0 and 1).
+    rc = wf_cuda_check(cudaMemsetAsync(ctx->topk_scratch, 0xFF, 8, st), "topk reset");
+    if (!rc) rc = wf_cuda_check(cudaMemsetAsync((uint8_t *)ctx->topk_scratch + 8, 0, 4, st), "topk reset");
+    if (rc) return rc;
+    kth_kernel<<<(unsigned)((P + kKth - 1) / kKth), kThreads, 0, st>>>(*res, P, k, ctx->topk_scratch);
     const int64_t blocks = std::min<int64_t>((P + 255) / 256, (int64_t)ctx->sms * 8);
     compact_kernel<<<(unsigned)blocks, 256, 0, st>>>(*res, P, ctx->topk_scratch);
     final_kernel<<<1, kThreads, smem, st>>>(k, ctx->topk_scratch, ids, keys);

@@ -1,0 +1,71 @@
+"""Top-k on synthetic result arrays, at batch sizes past the single-CTA
+path: ties within and across tiles, invalid plans, a short last tile, and
+k up to its limit.  The keys are written straight into the result arrays, so
+only the top-k kernels run."""
+import numpy as np
+import pytest
+
+import oracle
+import wfgen
+from gpu_util import lib
+
+pytestmark = pytest.mark.gpu
+
+
+def run_topk(mk, p95, gpu, st, k):
+    import torch
+    wf = lib()
+    P = len(mk)
+    ctx = wf.Ctx(wfgen.config("tiny").problem, max_P=P)
+    res = wf.Results(P)
+    res.makespan.copy_(torch.from_numpy(mk))
+    res.p95.copy_(torch.from_numpy(p95))
+    res.gpu.copy_(torch.from_numpy(gpu))
+    res.status.copy_(torch.from_numpy(st.view(np.int32)))
+    ids = torch.empty(k, dtype=torch.int32, device="cuda")
+    keys = torch.empty((k, 3), dtype=torch.int64, device="cuda")
+    wf.wf_topk(ctx, res, P, k, ids, keys)
+    torch.cuda.synchronize()
+    return ids.cpu().numpy(), keys.cpu().numpy()
+
+
+@pytest.mark.parametrize("P,spread,bad", [
+    (16385, 10**9, 0.0),      # one plan past the single-CTA path
+    (40000, 50, 0.1),         # heavy ties: more candidates than a sorting tile
+    (65536 + 17, 10**6, 0.5),  # a 17-plan last tile, half the plans invalid
+    (200000, 3000, 0.02),
+])
+@pytest.mark.parametrize("k", [1, 32, 1024])
+def test_large_batches(P, spread, bad, k):
+    rng = np.random.default_rng(P + k)
+    mk = rng.integers(1000, 1000 + spread, P).astype(np.int64)
+    p95 = rng.integers(0, 20, P).astype(np.int64)
+    gpu = rng.integers(0, 5, P).astype(np.int64)
+    st = np.where(rng.random(P) < bad, rng.integers(1, 16, P), 0).astype(np.uint32)
+    ids, keys = run_topk(mk, p95, gpu, st, k)
+    want_ids, want_keys = oracle.topk(mk, p95, gpu, st, k)
+    assert np.array_equal(ids, want_ids) and np.array_equal(keys, want_keys)
+
+
+def test_best_plans_in_one_tile():
+    """All of the k best plans sit in one tile: the other tiles' k-th keys
+    are all worse, so the threshold comes from that tile alone."""
+    P, k = 50000, 64
+    rng = np.random.default_rng(3)
+    mk = rng.integers(10**6, 2 * 10**6, P).astype(np.int64)
+    mk[4096:4096 + 200] = rng.integers(0, 1000, 200)
+    zeros = np.zeros(P, np.int64)
+    st = np.zeros(P, np.uint32)
+    ids, keys = run_topk(mk, zeros, zeros, st, k)
+    want_ids, want_keys = oracle.topk(mk, zeros, zeros, st, k)
+    assert np.array_equal(ids, want_ids) and np.array_equal(keys, want_keys)
+
+
+def test_all_plans_invalid_and_tied():
+    P, k = 30000, 1024
+    mk = np.full(P, 7, np.int64)
+    zeros = np.zeros(P, np.int64)
+    st = np.ones(P, np.uint32)
+    ids, keys = run_topk(mk, zeros, zeros, st, k)
+    want_ids, want_keys = oracle.topk(mk, zeros, zeros, st, k)
+    assert np.array_equal(ids, want_ids) and np.array_equal(keys, want_keys)
