@@ -205,7 +205,7 @@ def local_search_timing(wf, ctx, dp, prob, P, stream, flush, peak_gbs, k=32, rou
     """Local search around the batch's first k plans: P - k children per
     round (mutate -> evaluate -> merge; the context holds P plans).  The
     mutation kernel alone is timed too; it writes the child rows and reads
-    the k parent rows (from L2)."""
+    the k parent rows (once from DRAM, then from L2)."""
     import torch
     N = prob.N
     P = P - k
@@ -230,11 +230,14 @@ def local_search_timing(wf, ctx, dp, prob, P, stream, flush, peak_gbs, k=32, rou
     torch.cuda.synchronize()
     mut_ms = float(np.median([a.elapsed_time(b) for a, b in mut]))
     ls_ms = e[2].elapsed_time(e[3])
+    # Compulsory DRAM bytes: every child row written once, the k parent rows
+    # read once (the children's further reads of them hit L2).
     row = N + 2 * N + 2 * 4 * ((N + 31) // 32)
-    gbs = 2 * row * P / (mut_ms * 1e-3) / 1e9
+    bytes_per_child = row * (P + k) / P
+    gbs = bytes_per_child * P / (mut_ms * 1e-3) / 1e9
     return {"k": k, "children_per_round": P, "rounds": rounds, "n_ops": 3,
             "ms_per_round": ls_ms / rounds, "children_per_s": P * rounds / (ls_ms * 1e-3),
-            "mutate_kernel": {"ms": mut_ms, "timing": "median of 5 launches, L2 flushed before each", "bytes_per_child": 2 * row, "achieved_gbs": gbs,
+            "mutate_kernel": {"ms": mut_ms, "timing": "median of 5 launches, L2 flushed before each", "bytes_per_child": bytes_per_child, "achieved_gbs": gbs,
                               "frac": gbs / peak_gbs if peak_gbs else None, "bound": "hbm"}}
 
 

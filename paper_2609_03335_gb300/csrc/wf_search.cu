@@ -4,8 +4,11 @@
 // the children are evaluated by the sweep, and the elite keeps the k best of
 // itself and its children.
 //
-//   mutate_kernel   a CTA per child: copy the parent's rows in 16-byte
-//                   pieces, then apply the child's changes (one thread)
+//   mutate_kernel   a CTA per child: the parent's rows copied to the child
+//                   in 16-byte pieces, then the child's changes applied by
+//                   one thread; for short rows mutate_staged_kernel, a warp
+//                   per child, stages the rows in shared memory with bulk
+//                   copies and decodes the changes on all lanes
 //   union_kernel    elite and child results side by side for the top-k key
 //   pairs_kernel    one CTA: which elite slots leave, which children enter
 //   replace_kernel  a CTA per entering child: its rows and results into the
@@ -17,6 +20,8 @@
 namespace {
 
 constexpr int kCopyThreads = 128;
+constexpr int kMutWarps = 8;                // children a staged mutate CTA works on at once, a warp each
+constexpr int64_t kStagedMax = 96 * 1024;  // shared memory of a staged mutate CTA, at most
 constexpr int kMaxK = 1024;
 
 __device__ __forceinline__ uint64_t mix64(uint64_t x)  // SplitMix64 output function
@@ -29,12 +34,26 @@ __device__ __forceinline__ uint64_t mix64(uint64_t x)  // SplitMix64 output func
 
 __host__ __device__ inline int64_t pad16(int64_t bytes) { return (bytes + 15) & ~(int64_t)15; }
 
-// bytes (a multiple of 16) from src to dst, both 16-byte aligned, by the CTA.
-__device__ __forceinline__ void copy_row(void *dst, const void *src, int64_t bytes)
+// bytes (a multiple of 16) from src to dst, both 16-byte aligned, by `lanes`
+// threads (this one is `lane`), four pieces a thread in flight (kWide) or one.
+// src is global memory that no thread writes during the kernel (read through
+// the non-coherent path).
+template <bool kWide = true>
+__device__ __forceinline__ void copy_row(void *dst, const void *src, int64_t bytes, int lane, int lanes)
 {
     const uint4 *s = (const uint4 *)src;
     uint4 *d = (uint4 *)dst;
-    for (int64_t i = threadIdx.x; i < bytes / 16; i += blockDim.x) d[i] = __ldg(s + i);
+    const int64_t n = bytes / 16;
+    int64_t i = lane;
+    for (; kWide && i + 3 * lanes < n; i += 4 * lanes) {
+        const uint4 a = __ldg(s + i), b = __ldg(s + i + lanes), c = __ldg(s + i + 2 * lanes),
+                    e = __ldg(s + i + 3 * lanes);
+        d[i] = a;
+        d[i + lanes] = b;
+        d[i + 2 * lanes] = c;
+        d[i + 3 * lanes] = e;
+    }
+    for (; i < n; i += lanes) d[i] = __ldg(s + i);
 }
 
 struct Row {
@@ -56,15 +75,15 @@ __device__ __forceinline__ Row row_of(const wf_plans &pl, int64_t p)
 
 // Every row of plan b of `from` into plan a of `to` (padding to 16 bytes included).
 __device__ __forceinline__ void copy_plan(const wf_dev_problem &dp, const wf_plans &to, int64_t a,
-                                          const wf_plans &from, int64_t b)
+                                          const wf_plans &from, int64_t b, int lane, int lanes)
 {
     const int64_t N = dp.N, wbytes = pad16(4 * ((N + 31) / 32));
     const Row d = row_of(to, a), s = row_of(from, b);
-    copy_row(d.place, s.place, pad16(N));
-    copy_row(d.order, s.order, pad16(2 * N));
-    copy_row(d.fuse, s.fuse, wbytes);
-    copy_row(d.prefetch, s.prefetch, wbytes);
-    if (d.retain && s.retain) copy_row(d.retain, s.retain, wbytes);
+    copy_row(d.place, s.place, pad16(N), lane, lanes);
+    copy_row(d.order, s.order, pad16(2 * N), lane, lanes);
+    copy_row(d.fuse, s.fuse, wbytes, lane, lanes);
+    copy_row(d.prefetch, s.prefetch, wbytes, lane, lanes);
+    if (d.retain && s.retain) copy_row(d.retain, s.retain, wbytes, lane, lanes);
 }
 
 __device__ bool is_pred(const wf_dev_problem &dp, int32_t u, int32_t v)
@@ -77,47 +96,215 @@ __device__ bool is_pred(const wf_dev_problem &dp, int32_t u, int32_t v)
 // Child c copies parent c mod n_par; change s is decoded from
 // h = mix(mix(mix(seed ^ round) ^ c) ^ s): h mod 4 picks a move to a fitting
 // device (Eq. 8), a fuse flip (Eq. 3), a prefetch flip (Eq. 5) or an adjacent
-// swap that never crosses a graph edge (Eq. 10).
+// swap that never crosses a graph edge (Eq. 10).  The changes apply in turn.
+struct Change {
+    uint32_t kind;  // 0 none, 1 move node a to device b, 2 fuse flip of a, 3 prefetch flip of a,
+                    // 4 swap of positions a and a + 1 (when legal at that point)
+    int32_t a, b;
+};
+
+// hc = mix(mix(seed ^ round) ^ c), shared by the child's changes.
+__device__ __forceinline__ Change decode_change(const wf_dev_problem &dp, uint64_t hc, int32_t s)
+{
+    const int32_t N = dp.N;
+    const uint64_t h = mix64(hc ^ (uint64_t)s);
+    const uint32_t x = (uint32_t)(h >> 8), y = (uint32_t)(h >> 40);
+    const uint32_t op = (uint32_t)h & 3u;
+    Change g{0u, 0, 0};
+    if (op == 3u) {
+        if (N >= 2) g = Change{4u, (int32_t)(x % (uint32_t)(N - 1)), 0};
+        return g;
+    }
+    const int32_t n = (int32_t)(x % (uint32_t)N);
+    if (op == 0u) {
+        uint32_t fit = __ldg(dp.fitmask + n);
+        const int32_t f = __popc(fit);
+        if (f == 0) return g;
+        for (int32_t k = (int32_t)(y % (uint32_t)f); k > 0; --k) fit &= fit - 1;  // drop the lowest k
+        return Change{1u, n, __ffs((int)fit) - 1};
+    }
+    return Change{op == 1u ? 2u : 3u, n, 0};
+}
+
+__device__ __forceinline__ void apply_change(const wf_dev_problem &dp, const Row &r, const Change &g)
+{
+    const int32_t N = dp.N, a = g.a;
+    if (g.kind == 4u) {
+        const int32_t u = r.order[a], v = r.order[a + 1];
+        if (v < N && !(u < N && is_pred(dp, u, v))) {
+            r.order[a] = (uint16_t)v;
+            r.order[a + 1] = (uint16_t)u;
+        }
+    } else if (g.kind == 1u) {
+        r.place[a] = (uint8_t)g.b;
+    } else if (g.kind == 2u) {
+        r.fuse[a >> 5] ^= 1u << (a & 31);
+    } else if (g.kind == 3u) {
+        r.prefetch[a >> 5] ^= 1u << (a & 31);
+    }
+}
+
+__device__ __forceinline__ uint64_t child_hash(uint64_t seed, int64_t round, int64_t c)
+{
+    return mix64(mix64(seed ^ (uint64_t)round) ^ (uint64_t)c);
+}
+
+// Long rows: a CTA per child, the changes applied to the child's rows in
+// global memory.
 __global__ void __launch_bounds__(kCopyThreads)
 mutate_kernel(wf_dev_problem dp, wf_plans par, int64_t n_par, wf_plans ch, uint64_t seed, int64_t round,
               int32_t n_ops)
 {
-    const int32_t N = dp.N;
     for (int64_t c = blockIdx.x; c < ch.P; c += gridDim.x) {
-        copy_plan(dp, ch, c, par, c % n_par);
+        copy_plan(dp, ch, c, par, c % n_par, (int)threadIdx.x, (int)blockDim.x);
         __syncthreads();
         if (threadIdx.x == 0) {
             const Row r = row_of(ch, c);
-            for (int32_t s = 0; s < n_ops; ++s) {
-                const uint64_t h = mix64(mix64(mix64(seed ^ (uint64_t)round) ^ (uint64_t)c) ^ (uint64_t)s);
-                const uint32_t x = (uint32_t)(h >> 8), y = (uint32_t)(h >> 40);
-                const uint32_t op = (uint32_t)h & 3u;
-                if (op == 3u) {
-                    if (N < 2) continue;
-                    const int32_t i = (int32_t)(x % (uint32_t)(N - 1));
-                    const int32_t u = r.order[i], v = r.order[i + 1];
-                    if (v < N && !(u < N && is_pred(dp, u, v))) {
-                        r.order[i] = (uint16_t)v;
-                        r.order[i + 1] = (uint16_t)u;
-                    }
-                    continue;
-                }
-                const int32_t n = (int32_t)(x % (uint32_t)N);
-                if (op == 0u) {
-                    uint32_t fit = __ldg(dp.fitmask + n);
-                    const int32_t f = __popc(fit);
-                    if (f == 0) continue;
-                    for (int32_t k = (int32_t)(y % (uint32_t)f); k > 0; --k) fit &= fit - 1;  // drop the lowest k
-                    r.place[n] = (uint8_t)(__ffs((int)fit) - 1);
-                } else if (op == 1u) {
-                    r.fuse[n >> 5] ^= 1u << (n & 31);
-                } else {
-                    r.prefetch[n >> 5] ^= 1u << (n & 31);
-                }
-            }
+            const uint64_t hc = child_hash(seed, round, c);
+            for (int32_t s = 0; s < n_ops; ++s) apply_change(dp, r, decode_change(dp, hc, s));
         }
         __syncthreads();
     }
+}
+
+// Shared-memory address of a generic pointer into this CTA's shared memory.
+__device__ __forceinline__ uint32_t smem_addr(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void mbar_init(uint64_t *bar)
+{
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_addr(bar)) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+// Arms bar for one phase that completes when `bytes` have landed.
+__device__ __forceinline__ void mbar_expect(uint64_t *bar, uint32_t bytes)
+{
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
+                 : "memory");
+}
+
+// Waits, a bounded number of polls, for bar's phase of the given parity.
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity)
+{
+    for (uint32_t it = 0; it < (1u << 20); ++it) {
+        uint32_t done;
+        asm volatile("{\n\t.reg .pred p;\n\t"
+                     "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+                     "selp.u32 %0, 1, 0, p;\n\t}"
+                     : "=r"(done)
+                     : "r"(smem_addr(bar)), "r"(parity)
+                     : "memory");
+        if (done) return true;
+    }
+    return false;
+}
+
+// 1-D bulk copy (TMA) of `bytes` (a multiple of 16, both ends 16-byte
+// aligned) from global memory into this CTA's shared memory, counted on bar.
+__device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar)
+{
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     smem_addr(dst)),
+                 "l"(src), "r"(bytes), "r"(smem_addr(bar))
+                 : "memory");
+}
+
+// 1-D bulk copy from shared memory to global memory, in the thread's open
+// bulk group.
+__device__ __forceinline__ void bulk_store(void *dst, const void *src, uint32_t bytes)
+{
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst), "r"(smem_addr(src)),
+                 "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// The thread's bulk stores have read their shared-memory sources.
+__device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+// The thread's bulk stores are complete.
+__device__ __forceinline__ void bulk_wait() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+// Orders this thread's shared-memory accesses before later bulk copies.
+__device__ __forceinline__ void fence_async_shared() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+// Bytes of one warp's staged rows: place, order, fuse, prefetch and, when
+// both batches carry one, retain, each padded to 16 bytes.
+__host__ __device__ inline int64_t staged_row_bytes(int64_t N, bool retain)
+{
+    return pad16(N) + pad16(2 * N) + (retain ? 3 : 2) * pad16(4 * ((N + 31) / 32));
+}
+
+// Short rows: a warp per child.  Lane 0 stages the parent's rows in the
+// warp's slice of shared memory with bulk copies while the lanes decode the
+// child's changes (lane t the t-th of each group of 32); lane 0 then applies
+// them on chip, in turn, and writes the rows to the child with bulk copies.
+// The slice is reloaded only after those stores have read it.  A bulk load
+// that has not landed after the bounded wait sets error word 3, and the warp
+// stops after a second bounded wait.
+__global__ void __launch_bounds__(32 * kMutWarps, 4)
+mutate_staged_kernel(wf_dev_problem dp, wf_plans par, int64_t n_par, wf_plans ch, uint64_t seed, int64_t round,
+                     int32_t n_ops)
+{
+    extern __shared__ __align__(16) uint8_t msm[];
+    __shared__ uint64_t bars[kMutWarps];
+    const int64_t N = dp.N, pl = pad16(N), ol = pad16(2 * N), wb = pad16(4 * ((N + 31) / 32));
+    const bool ret = par.retain != nullptr && ch.retain != nullptr;
+    const int lane = (int)(threadIdx.x & 31), warp = (int)(threadIdx.x >> 5);
+    uint8_t *base = msm + warp * staged_row_bytes(N, ret);
+    uint64_t *bar = &bars[warp];
+    Row sm;
+    sm.place = base;
+    sm.order = (uint16_t *)(base + pl);
+    sm.fuse = (uint32_t *)(base + pl + ol);
+    sm.prefetch = (uint32_t *)(base + pl + ol + wb);
+    sm.retain = ret ? (uint32_t *)(base + pl + ol + 2 * wb) : nullptr;
+    const uint32_t bytes = (uint32_t)staged_row_bytes(N, ret);
+    if (lane == 0) mbar_init(bar);
+    __syncwarp();
+    uint32_t parity = 0;
+    for (int64_t c = (int64_t)blockIdx.x * kMutWarps + warp; c < ch.P; c += (int64_t)gridDim.x * kMutWarps) {
+        const Row s = row_of(par, c % n_par), d = row_of(ch, c);
+        if (lane == 0) {
+            bulk_wait_read();  // the previous child's stores are done with the slice
+            fence_async_shared();
+            mbar_expect(bar, bytes);
+            bulk_load(sm.place, s.place, (uint32_t)pl, bar);
+            bulk_load(sm.order, s.order, (uint32_t)ol, bar);
+            bulk_load(sm.fuse, s.fuse, (uint32_t)wb, bar);
+            bulk_load(sm.prefetch, s.prefetch, (uint32_t)wb, bar);
+            if (ret) bulk_load(sm.retain, s.retain, (uint32_t)wb, bar);
+        }
+        const uint64_t hc = child_hash(seed, round, c);
+        Change g = lane < n_ops ? decode_change(dp, hc, lane) : Change{0u, 0, 0};
+        bool landed = true;
+        if (lane == 0) {
+            landed = mbar_wait(bar, parity);
+            if (!landed) {
+                atomicExch(dp.err, 3);
+                mbar_wait(bar, parity);
+            }
+        }
+        parity ^= 1u;
+        if (!__shfl_sync(0xFFFFFFFFu, landed, 0)) break;
+        for (int32_t g0 = 0; g0 < n_ops; g0 += 32) {
+            if (g0 > 0) g = g0 + lane < n_ops ? decode_change(dp, hc, g0 + lane) : Change{0u, 0, 0};
+            const int cnt = min(32, n_ops - g0);
+            for (int t = 0; t < cnt; ++t) {
+                const Change e{__shfl_sync(0xFFFFFFFFu, g.kind, t), __shfl_sync(0xFFFFFFFFu, g.a, t),
+                               __shfl_sync(0xFFFFFFFFu, g.b, t)};
+                if (lane == 0) apply_change(dp, sm, e);
+            }
+        }
+        if (lane == 0) {
+            fence_async_shared();  // lane 0's changes are seen by the bulk stores
+            bulk_store(d.place, sm.place, (uint32_t)pl);
+            bulk_store(d.order, sm.order, (uint32_t)ol);
+            bulk_store(d.fuse, sm.fuse, (uint32_t)wb);
+            bulk_store(d.prefetch, sm.prefetch, (uint32_t)wb);
+            if (ret) bulk_store(d.retain, sm.retain, (uint32_t)wb);
+            bulk_commit();
+        }
+    }
+    if (lane == 0) bulk_wait();
 }
 
 // Elite results (index < k) and child results (index k + c) side by side.
@@ -181,7 +368,7 @@ replace_kernel(wf_dev_problem dp, wf_plans elite, wf_eval_out elite_res, wf_plan
     const int32_t j = blockIdx.x;
     if (j >= *npairs) return;
     const int2 pr = pairs[j];
-    copy_plan(dp, elite, pr.x, ch, pr.y);
+    copy_plan(dp, elite, pr.x, ch, pr.y, (int)threadIdx.x, (int)blockDim.x);
     if (threadIdx.x == 0) {
         elite_res.makespan_us[pr.x] = ch_res.makespan_us[pr.y];
         elite_res.p95_us[pr.x] = ch_res.p95_us[pr.y];
@@ -216,8 +403,24 @@ SearchScratch scratch_of(const wf_ctx *c)
 int launch_mutate(wf_ctx *c, const wf_plans *par, const wf_plans *ch, uint64_t seed, int64_t round, int32_t n_ops,
                   cudaStream_t st)
 {
-    const int64_t blocks = std::min<int64_t>(ch->P, (int64_t)c->sms * 64);
-    mutate_kernel<<<(unsigned)blocks, kCopyThreads, 0, st>>>(c->dp, *par, par->P, *ch, seed, round, n_ops);
+    const int64_t staged = kMutWarps * staged_row_bytes(c->dp.N, par->retain && ch->retain);
+    if (staged <= kStagedMax) {
+        // One wave of resident CTAs, each warp striding over the children.
+        int rc = wf_cuda_check(cudaFuncSetAttribute(mutate_staged_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                    (int)staged), "mutate smem attribute");
+        int per_sm = 0;
+        if (!rc) rc = wf_cuda_check(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, mutate_staged_kernel,
+                                                                                    32 * kMutWarps, (size_t)staged),
+                                    "mutate occupancy");
+        if (rc) return rc;
+        const int64_t blocks = std::min<int64_t>((ch->P + kMutWarps - 1) / kMutWarps,
+                                                 (int64_t)c->sms * std::max(per_sm, 1));
+        mutate_staged_kernel<<<(unsigned)blocks, 32 * kMutWarps, (size_t)staged, st>>>(c->dp, *par, par->P, *ch,
+                                                                                       seed, round, n_ops);
+    } else {
+        const int64_t blocks = std::min<int64_t>(ch->P, (int64_t)c->sms * 64);
+        mutate_kernel<<<(unsigned)blocks, kCopyThreads, 0, st>>>(c->dp, *par, par->P, *ch, seed, round, n_ops);
+    }
     return wf_cuda_check(cudaGetLastError(), "mutate launch");
 }
 
