@@ -321,6 +321,16 @@ int wf_ctx_set_reclaim(wf_ctx *ctx, int32_t policy);
  */
 int wf_ctx_status(wf_ctx *ctx, void *stream);
 
+/*
+ * Diagnostic: launches, on `stream`, one device-side bounded wait that
+ * nothing completes (an mbarrier armed for bytes that no copy delivers, the
+ * wait the bulk-copy kernels use).  It gives up after about a second and
+ * records the expiry, so the next wf_ctx_status returns WF_ETIMEOUT; the
+ * context stays usable.  Returns WF_EINVAL for a NULL context, WF_ECUDA when
+ * the launch fails.
+ */
+int wf_ctx_check_wait_expiry(wf_ctx *ctx, void *stream);
+
 /* Release every device and host allocation of the context (NULL is a no-op). */
 void wf_ctx_destroy(wf_ctx *ctx);
 

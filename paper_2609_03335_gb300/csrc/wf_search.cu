@@ -183,16 +183,18 @@ __device__ __forceinline__ void mbar_expect(uint64_t *bar, uint32_t bytes)
                  : "memory");
 }
 
-// Waits, a bounded number of polls, for bar's phase of the given parity.
+// Waits for bar's phase of the given parity: at most 2^20 polls, each
+// suspending the thread for up to about a microsecond, so about a second in
+// all before it gives up.
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity)
 {
     for (uint32_t it = 0; it < (1u << 20); ++it) {
         uint32_t done;
         asm volatile("{\n\t.reg .pred p;\n\t"
-                     "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+                     "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
                      "selp.u32 %0, 1, 0, p;\n\t}"
                      : "=r"(done)
-                     : "r"(smem_addr(bar)), "r"(parity)
+                     : "r"(smem_addr(bar)), "r"(parity), "r"(1000u)
                      : "memory");
         if (done) return true;
     }
@@ -305,6 +307,16 @@ mutate_staged_kernel(wf_dev_problem dp, wf_plans par, int64_t n_par, wf_plans ch
         }
     }
     if (lane == 0) bulk_wait();
+}
+
+// The bounded wait's expiry path: an mbarrier armed for 16 bytes that no copy
+// delivers, so the wait gives up and sets error word 3.
+__global__ void wait_expiry_kernel(int *err)
+{
+    __shared__ uint64_t bar;
+    mbar_init(&bar);
+    mbar_expect(&bar, 16);
+    if (!mbar_wait(&bar, 0)) atomicExch(err, 3);
 }
 
 // Elite results (index < k) and child results (index k + c) side by side.
@@ -456,6 +468,15 @@ int check_pair(const wf_ctx *c, const wf_plans *a, const wf_plans *b)
 size_t wf_search_scratch_bytes(int64_t max_P)
 {
     return (size_t)((28 * max_P + 255) & ~(int64_t)255) + 16 * kMaxK + 256;
+}
+
+extern "C" int wf_ctx_check_wait_expiry(wf_ctx *c, void *stream)
+{
+    if (!c) return wf_set_error(WF_EINVAL, "NULL context");
+    int rc = wf_select_device(c);
+    if (rc) return rc;
+    wait_expiry_kernel<<<1, 1, 0, (cudaStream_t)stream>>>(c->dp.err);
+    return wf_cuda_check(cudaGetLastError(), "wait expiry launch");
 }
 
 extern "C" int wf_mutate_plans(wf_ctx *c, const wf_plans *parents, const wf_plans *children, uint64_t seed,

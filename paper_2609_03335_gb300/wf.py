@@ -24,7 +24,7 @@ INT64_MAX = np.iinfo(np.int64).max
 EXPORTS = ("wf_problem_check", "wf_ctx_create", "wf_forecast_readiness", "wf_eval_plans",
            "wf_topk", "wf_ctx_status", "wf_ctx_destroy", "wf_strerror", "wf_last_error",
            "wf_eval_plans_static", "wf_mutate_plans", "wf_merge_elite", "wf_local_search",
-           "wf_construct_plans", "wf_ctx_set_reclaim")
+           "wf_construct_plans", "wf_ctx_set_reclaim", "wf_ctx_check_wait_expiry")
 
 
 class WfError(RuntimeError):
@@ -84,6 +84,7 @@ def load_library():
         "wf_construct_plans": ([p, p, ctypes.c_uint64, i64, p], ctypes.c_int),
         "wf_ctx_set_reclaim": ([p, i32], ctypes.c_int),
         "wf_ctx_status": ([p, p], ctypes.c_int),
+        "wf_ctx_check_wait_expiry": ([p, p], ctypes.c_int),
         "wf_ctx_destroy": ([p], None),
         "wf_strerror": ([ctypes.c_int], ctypes.c_char_p),
         "wf_last_error": ([], ctypes.c_char_p),
@@ -208,6 +209,10 @@ def wf_ctx_destroy(ctx: Ctx):
 
 def wf_ctx_status(ctx: Ctx, stream=None):
     _check(load_library().wf_ctx_status(ctx.ptr, _stream_handle(stream)), "wf_ctx_status")
+
+
+def wf_ctx_check_wait_expiry(ctx: Ctx, stream=None):
+    _check(load_library().wf_ctx_check_wait_expiry(ctx.ptr, _stream_handle(stream)), "wf_ctx_check_wait_expiry")
 
 
 def wf_forecast_readiness(ctx: Ctx, rel, comp, stream=None):

@@ -172,3 +172,29 @@ def test_long_write_lists(F):
     prob = fanout_window(F, seed=F)
     plans = wfgen.make_plans(prob, 300, F)
     assert_same(gpu_eval(prob, plans), oracle_eval(prob, plans))
+
+
+def test_bounded_wait_expiry_is_reported():
+    """A device-side wait that nothing completes gives up on its own (in
+    about a second), the host reads WF_ETIMEOUT from wf_ctx_status, and the
+    context evaluates correctly afterwards."""
+    import time
+    import torch
+    wf = lib()
+    w = wfgen.config("tiny")
+    ctx = wf.Ctx(w.problem, max_P=64)
+    t0 = time.perf_counter()
+    wf.wf_ctx_check_wait_expiry(ctx)
+    with pytest.raises(wf.WfError) as e:
+        wf.wf_ctx_status(ctx)
+    assert e.value.code == wf.WF_ETIMEOUT
+    assert time.perf_counter() - t0 < 30
+    wf.wf_ctx_status(ctx)  # cleared
+    host = wfgen.make_plans(w.problem, 64, 3)
+    plans = wf.DevicePlans.from_host(host, "cuda")
+    res = wf.Results(64)
+    wf.wf_eval_plans(ctx, plans, res)
+    torch.cuda.synchronize()
+    wf.wf_ctx_status(ctx)
+    for a, b in zip(res.numpy(), oracle.eval_plans(w.problem, host)):
+        assert np.array_equal(a, b)
