@@ -631,7 +631,11 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
                         int32_t best = 0;
                         uint32_t bcls = 0;
                         int32_t bdist = 0, bcost = 0;
-                        for (int32_t e = 0; e < (int32_t)n; ++e) {
+                        // (Unrolled over the queue's capacity, so the entries'
+                        // loads are not chained through the loop counter.)
+#pragma unroll
+                        for (int32_t e = 0; e < Lru<Q>::kSlots; ++e) {
+                            if (e >= (int32_t)n) break;
                             const uint32_t kk = (uint32_t)(q >> (4 * e)) & 15u;
                             const uint32_t red = rcnt[kk * kP] > 1;
                             const uint32_t nu = nuse[(d * M + kk) * kP];
