@@ -272,6 +272,10 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
         for (int32_t d = 0; d < D; ++d)
             if (adm[(int64_t)n * D + d] <= pb->cap_mib[d]) fitmask[n] |= 1u << d;
     size_t o_fit = img.add(fitmask.data(), sizeof(uint32_t) * fitmask.size());
+    // The same masks a byte each when every device index fits a byte's bits.
+    std::vector<uint8_t> fit8(fitmask.size(), 0u);
+    for (size_t n = 0; n < fitmask.size(); ++n) fit8[n] = (uint8_t)(fitmask[n] & 0xFFu);
+    size_t o_fit8 = img.add(fit8.data(), fit8.size());
     std::vector<uint32_t> edges(((size_t)E + 3) & ~(size_t)3, 0u);  // read 4 at a time
     for (int32_t v = 0; v < N; ++v)
         for (int32_t e = pb->pred_off[v]; e < pb->pred_off[v + 1]; ++e)
@@ -363,6 +367,7 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
     dp.hrec = (const uint4 *)(base + o_hrec);
     dp.wc23 = (const uint32_t *)(base + o_wc23);
     dp.fitmask = (const uint32_t *)(base + o_fit);
+    dp.fit8 = (const uint8_t *)(base + o_fit8);
     dp.edges = (const uint32_t *)(base + o_edges);
     dp.succ_off = (const int32_t *)(base + o_soff);
     dp.succ_idx = (const int32_t *)(base + o_sidx);

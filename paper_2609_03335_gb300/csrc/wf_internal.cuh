@@ -48,6 +48,7 @@ struct wf_dev_problem {
     const uint4 *hrec;          // [N] {links, release slot | model << 16 | writes << 20, arrival, codes 0 | 1 << 16}
     const uint32_t *wc23;       // [N] third | fourth << 16 write code of each node's write list (the sink slot when shorter)
     const uint32_t *fitmask;    // [N rounded up to 16] bit d: peak[n][d] <= cap[d]
+    const uint8_t *fit8;        // [N rounded up to 16] the low byte of fitmask (all of it when D <= 8)
     const uint32_t *edges;      // [E rounded up to 4] predecessor | successor << 16
     const int32_t *succ_off;    // [N+1] successor lists (CSR)
     const int32_t *succ_idx;    // [E]

@@ -1133,6 +1133,9 @@ __host__ __device__ inline uint32_t status_warp_bytes(int32_t N)
     return round16(2u * (uint32_t)N);
 }
 
+// kByte: every device index is below 8, so one byte per node holds its fit
+// mask (fit8): a quarter of the table reads of the 32-bit masks.
+template <bool kByte>
 __global__ void __launch_bounds__(128)
 status_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out)
 {
@@ -1151,15 +1154,29 @@ status_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out)
         for (int32_t n16 = 16 * lane; n16 < N; n16 += 512) {
             const uint4 pw = __ldg((const uint4 *)(place + n16));
             const uint32_t pws[4] = {pw.x, pw.y, pw.z, pw.w};
+            if (kByte) {
+                const uint4 fb = __ldg((const uint4 *)(dp.fit8 + n16));
+                const uint32_t fbs[4] = {fb.x, fb.y, fb.z, fb.w};
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const uint4 fm = __ldg((const uint4 *)(dp.fitmask + n16 + 4 * q));
-                const uint32_t f[4] = {fm.x, fm.y, fm.z, fm.w};
+                for (int q = 0; q < 4; ++q) {
 #pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    const uint32_t d = (pws[q] >> (8 * j)) & 255u;
-                    if (n16 + 4 * q + j < N)
-                        st |= d >= (uint32_t)D ? WF_ST_DEVICE : (((f[j] >> d) & 1u) ? 0u : WF_ST_CAPACITY);
+                    for (int j = 0; j < 4; ++j) {
+                        const uint32_t d = (pws[q] >> (8 * j)) & 255u, f = (fbs[q] >> (8 * j)) & 255u;
+                        if (n16 + 4 * q + j < N)
+                            st |= d >= (uint32_t)D ? WF_ST_DEVICE : (((f >> (d & 7u)) & 1u) ? 0u : WF_ST_CAPACITY);
+                    }
+                }
+            } else {
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const uint4 fm = __ldg((const uint4 *)(dp.fitmask + n16 + 4 * q));
+                    const uint32_t f[4] = {fm.x, fm.y, fm.z, fm.w};
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        const uint32_t d = (pws[q] >> (8 * j)) & 255u;
+                        if (n16 + 4 * q + j < N)
+                            st |= d >= (uint32_t)D ? WF_ST_DEVICE : (((f[j] >> d) & 1u) ? 0u : WF_ST_CAPACITY);
+                    }
                 }
             }
         }
@@ -1206,18 +1223,25 @@ status_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out)
     }
 }
 
-int launch_status(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, cudaStream_t st)
+template <bool kByte>
+int launch_status_as(const wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, cudaStream_t st)
 {
     const wf_dev_problem &dp = ctx->dp;
     const size_t wbytes = status_warp_bytes(dp.N);
     const int swarps = (int)std::max<size_t>(1, std::min<size_t>(4, (227 * 1024) / wbytes));
     const size_t ssmem = wbytes * swarps;
-    int rc = wf_cuda_check(cudaFuncSetAttribute(status_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                (int)ssmem), "status smem attribute");
+    int rc = wf_cuda_check(cudaFuncSetAttribute(status_kernel<kByte>,
+                                                cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ssmem),
+                           "status smem attribute");
     if (rc) return rc;
     const int64_t sblocks = std::min<int64_t>((pl->P + swarps - 1) / swarps, (int64_t)ctx->sms * 16);
-    status_kernel<<<(unsigned)sblocks, 32 * swarps, ssmem, st>>>(dp, *pl, *out);
+    status_kernel<kByte><<<(unsigned)sblocks, 32 * swarps, ssmem, st>>>(dp, *pl, *out);
     return WF_OK;
+}
+
+int launch_status(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, cudaStream_t st)
+{
+    return ctx->dp.D <= 8 ? launch_status_as<true>(ctx, pl, out, st) : launch_status_as<false>(ctx, pl, out, st);
 }
 
 }  // namespace
