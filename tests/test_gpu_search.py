@@ -119,3 +119,23 @@ def test_local_search_matches_oracle(name, k, C, rounds, n_ops, S):
     best0 = min(zip(met0[3].tolist(), met0[0].tolist()))
     best1 = min(zip(met[3].tolist(), met[0].tolist()))
     assert best1 <= best0
+
+
+@pytest.mark.parametrize("N", [3600, 3700, 5000])
+@pytest.mark.parametrize("retain", [False, True])
+def test_mutate_long_rows(N, retain):
+    """Rows on both sides of the staged kernel's limit (eight warps' row sets
+    in 96 KB of shared memory; the retain row counts): 3,600 activations are
+    staged with and without retain rows, 3,700 only without, 5,000 never."""
+    import torch
+    from test_gpu_edges import chains_window
+    wf = lib()
+    prob = chains_window([N // 4] * 4, D=3, M=3, seed=N)
+    par = wfgen.make_plans(prob, 7, N, p_retain=0.5 if retain else None)
+    C = 300
+    ctx = wf.Ctx(prob, max_P=C)
+    dpar = wf.DevicePlans.from_host(par, "cuda")
+    dch = wf.DevicePlans.empty(C, prob.N, retain)
+    wf.wf_mutate_plans(ctx, dpar, dch, seed=99, round_=2, n_ops=5)
+    torch.cuda.synchronize()
+    assert_rows(dch, oracle.mutate(prob, par, C, 99, 2, 5), prob.N)
