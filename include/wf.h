@@ -19,7 +19,9 @@
  *   wf_local_search         rounds of mutate -> evaluate -> merge
  *   wf_construct_plans      plans built by a list scheduler (Algorithm 1)
  *   wf_ctx_set_reclaim      reclamation order: LRU or by next use
- *   wf_ctx_destroy, wf_strerror
+ *   wf_ctx_status           device-side failures of earlier calls
+ *   wf_ctx_check_wait_expiry  the bounded device wait's expiry path (tests)
+ *   wf_ctx_destroy, wf_strerror, wf_last_error
  *
  * Conventions.
  *   - Times are int64 microseconds, memory int32 MiB; every output is an
