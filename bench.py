@@ -44,6 +44,31 @@ def algorithmic_bytes_per_plan(N: int) -> int:
     return N + 2 * N + 2 * ((N + 7) // 8) + 28
 
 
+def host_cpu() -> dict:
+    """The host the oracle runs on: logical cores and the CPU model as lscpu
+    (or /proc/cpuinfo) names it."""
+    model = None
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.split(":")[0].strip() == "Model name":
+                model = line.split(":", 1)[1].strip()
+                break
+    except (OSError, subprocess.SubprocessError):
+        pass
+    if model is None:
+        try:
+            with open("/proc/cpuinfo") as f:
+                for line in f:
+                    if line.lower().startswith("model name"):
+                        model = line.split(":", 1)[1].strip()
+                        break
+        except OSError:
+            pass
+    import platform
+    return {"nproc": os.cpu_count(), "cpu_model": model or platform.machine()}
+
+
 def topk_launches(P: int, k: int) -> int:
     """Kernel launches of one wf_topk call: one CTA does select, compact and
     sort up to 16,384 plans; beyond, three kernels (tile bounds, compaction,
@@ -195,7 +220,8 @@ def run_reference(args, rank, world):
         "config": {"workload": f"{WORKLOAD}: {w.description}; oracle step = first {sample} plans of the batch",
                    "P": sample, "N": w.problem.N},
         "cpu_baseline": {"value": value, "unit": "plans/s", "cores": 1, "kind": "oracle",
-                         "sample": f"first {sample} plans of the {WORKLOAD} batch per step, one thread"},
+                         "sample": f"first {sample} plans of the {WORKLOAD} batch per step, one thread",
+                         **host_cpu()},
         "e2e": {"value": value, "unit": "plans/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -459,7 +485,7 @@ def run_gpu(args, rank, world, local):
         dt = time.perf_counter() - t0
         cpu = {"value": sample / dt, "unit": "plans/s", "cores": 1, "kind": "oracle",
                "sample": f"{'all' if sample == P else 'the first'} {sample} plans of the {WORKLOAD} batch, "
-                         f"one thread, {dt:.2f} s"}
+                         f"one thread, {dt:.2f} s", **host_cpu()}
 
     if rank == 0:
         line = {
