@@ -70,6 +70,7 @@ def _setup(lib):
     lib.orc_status.argtypes = [p, p, p, p]
     lib.orc_eval_plan.argtypes = [p, p, p, p, p, p, p, i64, p, p, p]
     lib.orc_eval_batch.argtypes = [p, p, p, i64, p, i64, p, p, p, i64, i64, i64, i64, p, p, p, p]
+    lib.orc_eval_phi_batch.argtypes = [p, p, p, i64, p, i64, p, p, p, i64, i64, i64, p, p]
     lib.orc_splitmix64.argtypes = [ctypes.c_uint64]
     lib.orc_splitmix64.restype = ctypes.c_uint64
     lib.orc_multiplier.argtypes = [p, ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint64]
@@ -78,7 +79,7 @@ def _setup(lib):
                                ctypes.c_uint64, i64, ctypes.c_int32]
     lib.orc_construct.argtypes = [p, p, ctypes.c_uint64, ctypes.c_uint64, i64, p, p, p, p, p]
     for f in ("orc_fusible_next", "orc_forecast", "orc_status", "orc_eval_plan", "orc_eval_batch", "orc_mutate",
-              "orc_construct"):
+              "orc_construct", "orc_eval_phi_batch"):
         getattr(lib, f).restype = ctypes.c_int
     return lib
 
@@ -235,6 +236,52 @@ def eval_plans(prob, plans, lo: int = 0, hi: int | None = None, threads: int = 1
         with ThreadPoolExecutor(threads) as ex:
             list(ex.map(run, [(a, min(n, a + step)) for a in range(0, n, step)]))
     return mk, p95, gpu, st
+
+
+def eval_phi(prob, plans, lo: int = 0, hi: int | None = None, threads: int = 1):
+    """The window terms of Eq. 12's ranking key for plans [lo, hi) of a
+    deterministic batch: (timely prefetches P_N, lifecycle overhead H_life in
+    us), INT64_MAX for invalid plans.  See orc_eval_phi_batch."""
+    op = OracleProblem(prob)
+    hi = plans.P if hi is None else hi
+    n = hi - lo
+    timely = np.zeros(n, np.int64)
+    life = np.zeros(n, np.int64)
+    place = np.ascontiguousarray(plans.place[lo:hi])
+    order = np.ascontiguousarray(plans.order[lo:hi])
+    fuse = np.ascontiguousarray(plans.fuse[lo:hi])
+    pref = np.ascontiguousarray(plans.prefetch[lo:hi])
+    ret = None if plans.retain is None else np.ascontiguousarray(plans.retain[lo:hi])
+
+    def run(rng):
+        a, b = rng
+        rc = op.lib.orc_eval_phi_batch(ctypes.byref(op.c), op.fnext.ctypes.data,
+                                       place.ctypes.data, place.shape[1], order.ctypes.data,
+                                       order.shape[1] * 2, fuse.ctypes.data, pref.ctypes.data,
+                                       None if ret is None else ret.ctypes.data, fuse.shape[1] * 4,
+                                       a, b, timely.ctypes.data, life.ctypes.data)
+        if rc != 0:
+            raise RuntimeError(f"oracle phi failed ({rc})")
+
+    if threads <= 1 or n < 2:
+        run((0, n))
+    else:
+        step = max(1, (n + threads * 4 - 1) // (threads * 4))
+        with ThreadPoolExecutor(threads) as ex:
+            list(ex.map(run, [(a, min(n, a + step)) for a in range(0, n, step)]))
+    return timely, life
+
+
+def topk_phi(makespan, timely, life, status, k: int, plan_base: int = 0):
+    """The k best plans by Eq. 12's window key (invalid last, latest
+    completion, most timely prefetches, least lifecycle overhead, plan id).
+    Returns (ids int32 [k], keys int64 [k][3] = makespan, timely, life)."""
+    P = len(makespan)
+    key = sorted(range(P), key=lambda p: (int(status[p]) != 0, int(makespan[p]), -int(timely[p]),
+                                          int(life[p]), p))
+    ids = np.array(key[:k], np.int32)
+    keys = np.stack([np.asarray(makespan)[ids], np.asarray(timely)[ids], np.asarray(life)[ids]], axis=1)
+    return ids + plan_base, keys.astype(np.int64)
 
 
 def topk(makespan, p95, gpu, status, k: int, plan_base: int = 0):

@@ -274,7 +274,7 @@ static int simulate(const orc_problem *pb, const int32_t *fnext,
                     const uint8_t *place, const uint16_t *order,
                     const uint32_t *fuse, const uint32_t *prefetch, const uint32_t *retain,
                     const int64_t *L, int64_t *c, int64_t *comp_w,
-                    int64_t *makespan, int64_t *gpu_total, orc_trace *tr)
+                    int64_t *makespan, int64_t *gpu_total, orc_trace *tr, int64_t *phi)
 {
     const int32_t N = pb->N, D = pb->D, M = pb->M, W = pb->W;
     int64_t *t_free = (int64_t *)malloc(sizeof(int64_t) * (size_t)D);
@@ -284,11 +284,14 @@ static int simulate(const orc_problem *pb, const int32_t *fnext,
     int32_t *nres = (int32_t *)malloc(sizeof(int32_t) * (size_t)D);
     int64_t *stamp = (int64_t *)malloc(sizeof(int64_t) * (size_t)D * (size_t)M);
     uint8_t *done = (uint8_t *)malloc((size_t)N);
+    uint8_t *loaded = (uint8_t *)calloc((size_t)D * (size_t)M, 1);  /* model m was ever resident on d */
+    int64_t timely = 0, life = 0;
     int32_t *chain = (int32_t *)malloc(sizeof(int32_t) * (size_t)N);
     uint8_t *is_head = (uint8_t *)malloc((size_t)N);
     int32_t *fprev = (int32_t *)malloc(sizeof(int32_t) * (size_t)N);
     int rc = 0;
-    if (!t_free || !occ_since || !gpu || !used || !nres || !stamp || !done || !chain || !is_head || !fprev) {
+    if (!t_free || !occ_since || !gpu || !used || !nres || !stamp || !done || !chain || !is_head || !fprev ||
+        !loaded) {
         rc = -1;
         goto out;
     }
@@ -370,7 +373,16 @@ static int simulate(const orc_problem *pb, const int32_t *fnext,
             used[d] += pb->weight[m];
             nres[d] += 1;
             start = imax64(le, rel);
+            /* Eq. 12's lifecycle terms: a prefetched load that started before
+             * the release and ended by it is timely; a load of a model this
+             * device held before is a reload caused by reclamation. */
+            if (bit_of(prefetch, h) && ls < rel && le <= rel) ++timely;
+            if (loaded[(int64_t)d * M + m]) life += pb->load[(int64_t)m * D + d];
+            loaded[(int64_t)d * M + m] = 1;
         }
+        /* The ready-work loading delay: how far the load pushes the start
+         * beyond the later of the release and the device's free time. */
+        life += start - imax64(t_free[d], rel);
         start += pb->grant;  /* one grant per unit, however long the chain */
 
         /* Execute the chain back to back (Eq. 4 run time = sum of members). */
@@ -436,9 +448,10 @@ static int simulate(const orc_problem *pb, const int32_t *fnext,
         comp_w[w] = imax64(comp_w[w], c[n] - pb->arrival[w]);
     }
     if (tr) for (int32_t n = 0; n < N; ++n) tr->finish[n] = c[n];
+    if (phi) { phi[0] = timely; phi[1] = life; }
 out:
     free(t_free); free(occ_since); free(gpu); free(used); free(nres); free(stamp); free(done); free(chain);
-    free(is_head); free(fprev);
+    free(is_head); free(fprev); free(loaded);
     return rc;
 }
 
@@ -506,7 +519,7 @@ int orc_eval_plan(const orc_problem *pb, const int32_t *fnext,
             }
         int64_t mk, g;
         rc = simulate(pb, fnext, place, order, fuse, prefetch, retain, L, c,
-                      &pool[(int64_t)s * W], &mk, &g, pb->S > 0 ? NULL : tr);
+                      &pool[(int64_t)s * W], &mk, &g, pb->S > 0 ? NULL : tr, NULL);
         if (rc) goto out;
         sum_mk += mk;
         sum_gpu += g;
@@ -542,6 +555,54 @@ int orc_eval_batch(const orc_problem *pb, const int32_t *fnext,
         makespan[p] = o[0]; p95[p] = o[1]; gpu[p] = o[2];
     }
     return 0;
+}
+
+/*
+ * The window terms of the ranking key of Eq. 12 for plans [lo, hi) of a
+ * deterministic batch (S = 0).  Over a whole window every unit is admitted,
+ * so the coverage counts A_k are equal for all valid plans and the key
+ * reduces to (latest completion, -P_N, H_life):
+ *   timely[p]  P_N, the units whose model load ran under their prefetch bit,
+ *              started before the unit's release and ended by it;
+ *   life[p]    H_life, the sum over units of the delay the load adds to the
+ *              start, max(load end, release) - max(device free, release)
+ *              (zero on a hit), plus the load time of every load of a model
+ *              its device had held before (a reload after reclamation).
+ * Invalid plans get INT64_MAX for both.  Returns -3 when S > 0.
+ */
+int orc_eval_phi_batch(const orc_problem *pb, const int32_t *fnext,
+                       const uint8_t *place, int64_t place_stride,
+                       const uint16_t *order, int64_t order_stride,
+                       const uint32_t *fuse, const uint32_t *prefetch, const uint32_t *retain,
+                       int64_t bits_stride, int64_t lo, int64_t hi, int64_t *timely, int64_t *life)
+{
+    if (pb->S > 0) return -3;
+    const int32_t N = pb->N, D = pb->D, W = pb->W;
+    int64_t *L = (int64_t *)malloc(sizeof(int64_t) * (size_t)N * (size_t)D);
+    int64_t *c = (int64_t *)malloc(sizeof(int64_t) * (size_t)N);
+    int64_t *comp = (int64_t *)malloc(sizeof(int64_t) * (size_t)W);
+    int rc = 0;
+    if (!L || !c || !comp) { rc = -1; goto out; }
+    for (int64_t k = 0; k < (int64_t)N * D; ++k) L[k] = pb->lat[k];
+    for (int64_t p = lo; p < hi; ++p) {
+        const uint8_t *pl = place + p * place_stride;
+        const uint16_t *od = (const uint16_t *)((const uint8_t *)order + p * order_stride);
+        const uint32_t *fu = (const uint32_t *)((const uint8_t *)fuse + p * bits_stride);
+        const uint32_t *pf = (const uint32_t *)((const uint8_t *)prefetch + p * bits_stride);
+        const uint32_t *rt = retain ? (const uint32_t *)((const uint8_t *)retain + p * bits_stride) : NULL;
+        uint32_t st;
+        rc = orc_status(pb, pl, od, &st);
+        if (rc) goto out;
+        if (st != 0) { timely[p] = life[p] = ORC_INF; continue; }
+        int64_t mk, g, phi[2];
+        rc = simulate(pb, fnext, pl, od, fu, pf, rt, L, c, comp, &mk, &g, NULL, phi);
+        if (rc) goto out;
+        timely[p] = phi[0];
+        life[p] = phi[1];
+    }
+out:
+    free(L); free(c); free(comp);
+    return rc;
 }
 
 /*

@@ -33,6 +33,9 @@ def test_golden_case(name, idx):
         assert int((tr["load_start"] >= 0).sum()) == exp["loads"]
     if "units" in exp:
         assert len(tr["unit_head"]) == exp["units"]
+    if "timely" in exp:  # the window terms of Eq. 12's ranking key
+        timely, life = oracle.eval_phi(prob, plans)
+        assert (int(timely[0]), int(life[0])) == (exp["timely"], exp["life"])
     if "evicted" in exp:
         got = {str(h): [m for m in range(32) if (int(tr["evicted"][h]) >> m) & 1]
                for h in tr["unit_head"] if tr["evicted"][h]}

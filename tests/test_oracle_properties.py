@@ -347,3 +347,29 @@ def test_grant_and_load_costs_never_speed_up(seed):
     b = oracle.eval_plans(prob.with_(grant_us=5), plans)
     c = oracle.eval_plans(prob.with_(load_us=prob.load_us * 2), plans)
     assert (b[0] >= a[0]).all() and (c[0] >= a[0]).all()
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_phi_terms_closed_form_without_reclamation(seed):
+    """Eq. 12's window terms with room for every model and no prefetch bits:
+    each model loads once per device, at its first use there, and each load
+    delays its unit by exactly the load time, so H_life is the sum of C[m,d]
+    over the (device, model) pairs a plan uses, and P_N is 0.  Setting every
+    prefetch bit can only make loads timely, never more than there are units."""
+    rng = np.random.default_rng(7100 + seed)
+    prob = random_problem(rng, n_sessions=int(rng.integers(1, 5)), D=int(rng.integers(1, 5)),
+                          M=int(rng.integers(1, 6)), tight=False)
+    prob = prob.with_(cap_mib=np.full(prob.D, 10**8, np.int32))
+    plans = wfgen.make_plans(prob, 40, seed, p_prefetch=0.0)
+    mk, p95, gpu, st = oracle.eval_plans(prob, plans)
+    timely, life = oracle.eval_phi(prob, plans)
+    load = np.asarray(prob.load_us).reshape(prob.M, prob.D)
+    model = np.asarray(prob.model)
+    for p in range(plans.P):
+        assert st[p] == 0
+        pairs = {(int(plans.place[p, n]), int(model[n])) for n in range(prob.N)}
+        assert timely[p] == 0
+        assert life[p] == sum(int(load[m, d]) for d, m in pairs)
+    allpf = wfgen.make_plans(prob, 40, seed, p_prefetch=1.0)
+    timely2, life2 = oracle.eval_phi(prob, allpf)
+    assert (timely2 <= prob.N).all() and (life2 <= life).all()
