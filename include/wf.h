@@ -19,6 +19,8 @@
  *   wf_local_search         rounds of mutate -> evaluate -> merge
  *   wf_construct_plans      plans built by a list scheduler (Algorithm 1)
  *   wf_ctx_set_reclaim      reclamation order: LRU or by next use
+ *   wf_eval_plans_phi       wf_eval_plans plus the window terms of Eq. 12
+ *   wf_topk_phi             the k best plans by Eq. 12's window key
  *   wf_ctx_status           device-side failures of earlier calls
  *   wf_ctx_check_wait_expiry  the bounded device wait's expiry path (tests)
  *   wf_ctx_destroy, wf_strerror, wf_last_error
@@ -316,6 +318,37 @@ int wf_construct_plans(wf_ctx *ctx, const wf_plans *out, uint64_t seed, int64_t 
  * context.  wf_eval_plans_static always uses WF_RECLAIM_LRU.
  */
 int wf_ctx_set_reclaim(wf_ctx *ctx, int32_t policy);
+
+/*
+ * wf_eval_plans, plus the window terms of the ranking key of Eq. 12.  That
+ * key ranks a tick's partial plan by (-A_1, ..., -A_K, C_F, -P_N, H_life);
+ * over a whole window every unit is admitted, so the coverage counts A_k are
+ * equal for all valid plans and it reduces to (C_F, -P_N, H_life), C_F the
+ * latest completion (the makespan's order).  Per plan:
+ *   timely_dev[p]  P_N: the units whose model load ran under their prefetch
+ *                  bit (Eq. 5), started before the unit's release and ended
+ *                  by it;
+ *   life_dev[p]    H_life (us): over the units, the delay the load adds to
+ *                  the start, max(load end, release) - max(device free,
+ *                  release) (0 on a hit), plus the load time of every load of
+ *                  a model its device held before (a reload after reclamation,
+ *                  Eq. 11 or a retain bit of 0).
+ * Both are INT64_MAX for an invalid plan.  DEVICE int64 [P] each.  Needs
+ * S = 0 (WF_EINVAL otherwise); either reclamation order.  The context carries
+ * the two pointers during the call, so calls on one context are not
+ * thread-safe.  Otherwise as wf_eval_plans.
+ */
+int wf_eval_plans_phi(wf_ctx *ctx, const wf_plans *plans, const wf_eval_out *out, int64_t *timely_dev,
+                      int64_t *life_dev, void *stream);
+
+/*
+ * The k best plans by Eq. 12's window key (status != 0, makespan, -timely,
+ * life, plan index), ascending, from wf_eval_plans_phi's outputs.  keys_dev:
+ * DEVICE int64 [k][3] (makespan, timely, life) or NULL.  Otherwise as
+ * wf_topk.
+ */
+int wf_topk_phi(wf_ctx *ctx, const wf_eval_out *out, const int64_t *timely_dev, const int64_t *life_dev, int64_t P,
+                int32_t k, int32_t *ids_dev, int64_t *keys_dev, void *stream);
 
 /*
  * Synchronize `stream` and report device-side failures of earlier calls on

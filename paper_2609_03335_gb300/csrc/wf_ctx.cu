@@ -492,6 +492,37 @@ extern "C" int wf_topk(wf_ctx *c, const wf_eval_out *res, int64_t P, int32_t k, 
     return wf_launch_topk(c, res, P, k, ids, keys, (cudaStream_t)stream);
 }
 
+extern "C" int wf_eval_plans_phi(wf_ctx *c, const wf_plans *pl, const wf_eval_out *out, int64_t *timely,
+                                 int64_t *life, void *stream)
+{
+    REQUIRE(c && pl && out && timely && life, "NULL argument");
+    REQUIRE(c->dp.S == 0, "the window terms of Eq. 12 need deterministic latencies (S = 0)");
+    int rc = wf_check_plans(c, pl, "plans");
+    if (!rc) rc = wf_check_out(out, "results");
+    if (!rc) rc = select_device(c);
+    if (rc) return rc;
+    // The kernels take the outputs from the problem they are launched with;
+    // the context carries them for this call only.
+    c->dp.phi_timely = timely;
+    c->dp.phi_life = life;
+    rc = wf_launch_eval(c, pl, out, (cudaStream_t)stream);
+    c->dp.phi_timely = nullptr;
+    c->dp.phi_life = nullptr;
+    return rc;
+}
+
+extern "C" int wf_topk_phi(wf_ctx *c, const wf_eval_out *res, const int64_t *timely, const int64_t *life,
+                           int64_t P, int32_t k, int32_t *ids, int64_t *keys, void *stream)
+{
+    REQUIRE(c && res && timely && life && ids, "NULL argument");
+    REQUIRE(res->makespan_us && res->status, "NULL result array");
+    REQUIRE(P >= 1 && P <= c->max_P, "P outside 1..max_P");
+    REQUIRE(k >= 1 && k <= 1024 && k <= P, "k=%d outside 1..min(P, 1024)", k);
+    int rc = select_device(c);
+    if (rc) return rc;
+    return wf_launch_topk(c, res, P, k, ids, keys, (cudaStream_t)stream, timely, life, -1);
+}
+
 extern "C" int wf_ctx_set_reclaim(wf_ctx *c, int32_t policy)
 {
     REQUIRE(c, "NULL context");

@@ -52,6 +52,7 @@ struct Row {
     int32_t *used;    // [D] resident weights
     int32_t *nres;    // [D] resident model count
     int32_t *stamp;   // [D][M] last dispatch position + 1 using the model, 0 = not resident
+    int32_t *loaded;  // [D] bit m: model m was ever resident on the device (Eq. 12 window terms)
 };
 
 __device__ __forceinline__ size_t up8(size_t x) { return (x + 7) & ~(size_t)7; }
@@ -67,7 +68,8 @@ __device__ __forceinline__ Row row_at(const wf_dev_problem &dp, uint8_t *base)
     r.comp = (int64_t *)(base + o); o += 8 * (size_t)dp.W;
     r.used = (int32_t *)(base + o); o += up8(4 * (size_t)dp.D);
     r.nres = (int32_t *)(base + o); o += up8(4 * (size_t)dp.D);
-    r.stamp = (int32_t *)(base + o);
+    r.stamp = (int32_t *)(base + o); o += up8(4 * (size_t)dp.D * dp.M);
+    r.loaded = (int32_t *)(base + o);
     return r;
 }
 
@@ -122,14 +124,20 @@ __device__ __forceinline__ int64_t run_time(const wf_dev_problem &dp, int32_t n,
 }
 
 // One play of a valid plan.  Returns makespan and GPU time; per-session
-// completion latencies are left in row.comp.
+// completion latencies are left in row.comp.  With phi, also the window
+// terms of Eq. 12: phi[0] the timely prefetches (a prefetched load that
+// starts before the unit's release and ends by it), phi[1] the lifecycle
+// overhead (the delay each load adds to its unit's start, plus the load time
+// of every reload of a model the device held before).
 template <bool kStoch>
 __device__ void play(const wf_dev_problem &dp, const PlanRows &pr, Row &row, uint64_t key,
-                     int64_t *makespan, int64_t *gpu_total)
+                     int64_t *makespan, int64_t *gpu_total, int64_t *phi = nullptr)
 {
     const int32_t N = dp.N, D = dp.D, M = dp.M, W = dp.W;
+    int64_t timely = 0, life = 0;
     for (int32_t d = 0; d < D; ++d) {
         row.tfree[d] = 0; row.occ[d] = kNone; row.gpu[d] = 0; row.used[d] = 0; row.nres[d] = 0;
+        row.loaded[d] = 0;
     }
     for (int32_t k = 0; k < D * M; ++k) row.stamp[k] = 0;
     for (int32_t w = 0; w < W; ++w) row.comp[w] = kNone;
@@ -178,12 +186,20 @@ __device__ void play(const wf_dev_problem &dp, const PlanRows &pr, Row &row, uin
         if (hit) {
             start = max(tf, rel);
         } else {
-            const int64_t ls = max(tf, bit_at(pr.prefetch, h) ? arr : rel);
+            const bool pf = bit_at(pr.prefetch, h);
+            const int64_t ls = max(tf, pf ? arr : rel);
             if (row.occ[d] == kNone) row.occ[d] = ls;
             row.used[d] += wm;
             row.nres[d] += 1;
-            start = max(ls + dp.load[m * D + d], rel);
+            const int64_t le = ls + dp.load[m * D + d];
+            start = max(le, rel);
+            if (phi) {
+                timely += pf && ls < rel && le <= rel;
+                if ((row.loaded[d] >> m) & 1) life += dp.load[m * D + d];
+                row.loaded[d] |= 1 << m;
+            }
         }
+        if (phi) life += start - max(tf, rel);
         const int64_t c = start + dp.grant + run;
         row.ctail[tail] = c;
         row.tfree[d] = c;
@@ -208,6 +224,7 @@ __device__ void play(const wf_dev_problem &dp, const PlanRows &pr, Row &row, uin
     for (int32_t w = 0; w < W; ++w) row.comp[w] -= dp.arrival[w];
     *makespan = end - dp.first_arrival;
     *gpu_total = g;
+    if (phi) { phi[0] = timely; phi[1] = life; }
 }
 
 // r-th smallest (0-based) of v[0..n), reordering v (Hoare quickselect).
@@ -244,13 +261,15 @@ eval_det_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, uint8_t *scratc
         out.status[p] = st;
         if (st) {
             out.makespan_us[p] = out.p95_us[p] = out.gpu_us[p] = WF_INF64;
+            if (dp.phi_life) dp.phi_timely[p] = dp.phi_life[p] = WF_INF64;
             continue;
         }
-        int64_t mk, g;
-        play<false>(dp, pr, row, 0, &mk, &g);
+        int64_t mk, g, phi[2];
+        play<false>(dp, pr, row, 0, &mk, &g, dp.phi_life ? phi : nullptr);
         out.makespan_us[p] = mk;
         out.gpu_us[p] = g;
         out.p95_us[p] = select_rank(row.comp, dp.W, p95_rank(dp.W));
+        if (dp.phi_life) { dp.phi_timely[p] = phi[0]; dp.phi_life[p] = phi[1]; }
     }
 }
 
@@ -270,13 +289,15 @@ eval_list_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, uint8_t *scrat
         out.status[p] = st;
         if (st) {
             out.makespan_us[p] = out.p95_us[p] = out.gpu_us[p] = WF_INF64;
+            if (dp.phi_life) dp.phi_timely[p] = dp.phi_life[p] = WF_INF64;
             continue;
         }
-        int64_t mk, g;
-        play<false>(dp, pr, row, 0, &mk, &g);
+        int64_t mk, g, phi[2];
+        play<false>(dp, pr, row, 0, &mk, &g, dp.phi_life ? phi : nullptr);
         out.makespan_us[p] = mk;
         out.gpu_us[p] = g;
         out.p95_us[p] = select_rank(row.comp, dp.W, p95_rank(dp.W));
+        if (dp.phi_life) { dp.phi_timely[p] = phi[0]; dp.phi_life[p] = phi[1]; }
     }
 }
 
@@ -363,7 +384,8 @@ eval_stoch_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, uint8_t *scra
 size_t wf_eval_row_bytes(const wf_dev_problem &dp)
 {
     size_t b = ((8 * (size_t)dp.N + 7) & ~(size_t)7) + 8 * 3 * (size_t)dp.D + 8 * (size_t)dp.W +
-               2 * ((4 * (size_t)dp.D + 7) & ~(size_t)7) + 4 * (size_t)dp.D * dp.M;
+               2 * ((4 * (size_t)dp.D + 7) & ~(size_t)7) + ((4 * (size_t)dp.D * dp.M + 7) & ~(size_t)7) +
+               4 * (size_t)dp.D;
     return (b + 127) & ~(size_t)127;
 }
 

@@ -59,6 +59,10 @@ struct wf_dev_problem {
     int32_t reclaim;
     uint16_t *nextuse;
     int64_t max_chain_run;      // the longest fusible chain's run time on its slowest devices, plus the grant
+    // Outputs of the window terms of Eq. 12 ([P] each, wf_eval_plans_phi);
+    // null outside such a call.
+    int64_t *phi_timely;
+    int64_t *phi_life;
     int64_t max_arrival;
 };
 
@@ -116,8 +120,12 @@ int wf_select_device(const wf_ctx *c);
 // Launchers (one per translation unit).
 int wf_launch_forecast(wf_ctx *ctx, int64_t *rel, int64_t *comp, cudaStream_t st);
 int wf_launch_eval(wf_ctx *ctx, const wf_plans *plans, const wf_eval_out *out, cudaStream_t st);
+// The k best plans by (invalid, makespan, term2, term3, index); term2 and
+// term3 default to p95 and GPU time, and sign2 = -1 ranks term2 largest
+// first (the timely prefetches of Eq. 12).
 int wf_launch_topk(wf_ctx *ctx, const wf_eval_out *res, int64_t P, int32_t k, int32_t *ids,
-                   int64_t *keys, cudaStream_t st);
+                   int64_t *keys, cudaStream_t st, const int64_t *term2 = nullptr, const int64_t *term3 = nullptr,
+                   int64_t sign2 = 1);
 size_t wf_eval_row_bytes(const wf_dev_problem &dp);
 size_t wf_eval_scratch_bytes(const wf_dev_problem &dp, int64_t max_P, int64_t *units);
 size_t wf_topk_scratch_bytes(int64_t max_P);

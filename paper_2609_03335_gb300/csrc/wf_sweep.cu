@@ -158,14 +158,17 @@ struct PcGroups {
 };
 
 struct PcLayout {
-    uint32_t weight, cap, load, arr, ring, slots, tfree, used, queue, nres, open, flag, nuse, rcnt, gmask, total;
+    uint32_t weight, cap, load, arr, ring, slots, tfree, used, queue, nres, open, flag, nuse, rcnt, gmask, everl,
+        total;
 };
 
 // Shared memory of a CTA of kP plans with TT times and NS slots per plan;
 // with reclamation by next use (kReclaim) the ring carries a seventh record
 // word and each plan keeps per (device, model) the next use of the resident
-// copy and per model the number of devices holding it.
-template <int kP, typename TT, int kReclaim = 0>
+// copy and per model the number of devices holding it; with the window terms
+// of Eq. 12 (kPhi) each residency lane keeps per device the models it ever
+// held.
+template <int kP, typename TT, int kReclaim = 0, bool kPhi = false>
 __host__ __device__ inline PcLayout pc_layout(int32_t D, int32_t M, int32_t W, int32_t NS)
 {
     constexpr uint32_t t = sizeof(TT);
@@ -187,6 +190,7 @@ __host__ __device__ inline PcLayout pc_layout(int32_t D, int32_t M, int32_t W, i
     l.nuse = o; o += kReclaim ? round16(2u * D * M * kP) : 0u;
     l.rcnt = o; o += kReclaim ? round16((uint32_t)M * kP) : 0u;
     l.gmask = o; o += round16(4u * Ring<kReclaim>::kBuffers * PcGroups<kP, kReclaim>::kG * kP);
+    l.everl = o; o += kPhi ? round16(2u * rs) : 0u;
     l.total = o;
     return l;
 }
@@ -390,7 +394,7 @@ __device__ __forceinline__ void produce_batch(const wf_dev_problem &dp, const wf
 template <typename Q>
 __device__ __forceinline__ uint2 settle_lru(Q &q, uint32_t &n, uint32_t &u_d, uint32_t capd, uint32_t r1,
                                             uint32_t r3, const int32_t *weight, const int32_t *load, int32_t D,
-                                            int *err)
+                                            int *err, bool &missed)
 {
     const int32_t d = (int32_t)(r3 & 31u);
     const uint32_t m = (r3 >> 5) & 15u;
@@ -398,6 +402,7 @@ __device__ __forceinline__ uint2 settle_lru(Q &q, uint32_t &n, uint32_t &u_d, ui
     const bool was_empty = n == 0;
     const int32_t kq = Lru<Q>::find(q, n, m);
     const bool hit = kq < (int32_t)n;
+    missed = !hit;
     q = hit ? Lru<Q>::remove(q, hit ? kq : 0) : q;  // (an index below the queue length)
     n -= hit ? 1u : 0u;
     const uint32_t need = hit ? r1 : wm + r1;  // used + need <= cap + peak < 2^32
@@ -439,7 +444,7 @@ __device__ __forceinline__ void publish(TT *slots, uint32_t code, TT c)
 // ovf_list; once every plan of a CTA has, its stages run on without loads.
 // TT = uint64_t: only a unit whose summed run time reaches 2^32 - 1 sends its
 // plan to ovf_list.
-template <typename Q, typename TT, int kP, int kReclaim>
+template <typename Q, typename TT, int kP, int kReclaim, bool kPhi>
 __global__ void __launch_bounds__(32 * PcShape<kP>::kWarps, PcShape<kP>::kMinBlocks)
 pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_list, const int32_t *in_count,
           int32_t *ovf_list, int32_t *ovf_count)
@@ -457,7 +462,7 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
     extern __shared__ __align__(128) uint8_t sm[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int32_t N = dp.N, D = dp.D, M = dp.M, W = dp.W;
-    const PcLayout L = pc_layout<kP, TT, kReclaim>(D, M, W, dp.nslots + 2);
+    const PcLayout L = pc_layout<kP, TT, kReclaim, kPhi>(D, M, W, dp.nslots + 2);
     const int64_t total = in_list ? (int64_t)*in_count : pl.P;
     if ((int64_t)blockIdx.x * kP >= total) return;  // the whole CTA: no plan
     uint2 *ring = (uint2 *)(sm + L.ring);
@@ -574,8 +579,12 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
         uint8_t *nres = sm + L.nres + rl;
         uint16_t *nuse = (uint16_t *)(sm + L.nuse) + qp;  // [device][model][plan]
         uint8_t *rcnt = sm + L.rcnt + qp;                 // [model][plan]
+        uint16_t *everl = (uint16_t *)(sm + L.everl) + rl;  // [device / kG][lane], bit m: m was held (kPhi)
         if (rmine) {
-            for (int32_t t = 0; t * kG + g < D; ++t) { used[t * kRow] = 0; queue[t * kRow] = 0; nres[t * kRow] = 0; }
+            for (int32_t t = 0; t * kG + g < D; ++t) {
+                used[t * kRow] = 0; queue[t * kRow] = 0; nres[t * kRow] = 0;
+                if (kPhi) everl[t * kRow] = 0;
+            }
             if (kReclaim)
                 for (int32_t k = 0; k < M; ++k) rcnt[k * kP] = 0;
         }
@@ -600,7 +609,13 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
                     Q q = queue[t * kRow];
                     uint32_t n = nres[t * kRow];
                     uint32_t u_d = used[t * kRow];
-                    const uint2 w = settle_lru<Q>(q, n, u_d, (uint32_t)cap[d], r1, r3, weight, load, D, dp.err);
+                    bool missed;
+                    uint2 w = settle_lru<Q>(q, n, u_d, (uint32_t)cap[d], r1, r3, weight, load, D, dp.err, missed);
+                    if (kPhi && missed) {  // a reload of a model this device held before: bit 31 of the load word
+                        const uint32_t m = (r3 >> 5) & 15u, e = everl[t * kRow];
+                        w.x |= ((e >> m) & 1u) << 31;
+                        everl[t * kRow] = (uint16_t)(e | (1u << m));
+                    }
                     queue[t * kRow] = q;
                     nres[t * kRow] = (uint8_t)n;
                     used[t * kRow] = u_d;
@@ -671,8 +686,14 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
                     queue[d * kRow] = q;
                     nres[d * kRow] = (uint8_t)n;
                     used[d * kRow] = u_d;
+                    uint32_t reload = 0;
+                    if (kPhi && !hit) {
+                        const uint32_t e = everl[d * kRow];
+                        reload = ((e >> m) & 1u) << 31;
+                        everl[d * kRow] = (uint16_t)(e | (1u << m));
+                    }
                     rb[(1 * kChunk + k) * kPitch] =
-                        make_uint2(hit ? 0u : (uint32_t)load[m * D + d],
+                        make_uint2(hit ? 0u : ((uint32_t)load[m * D + d] | reload),
                                    (r3 & ~(kPrefetch | kWasEmpty)) | (hit ? 0u : (r3 & kPrefetch)) |
                                        (was_empty ? kWasEmpty : 0u) | (emptied ? kEmptied : 0u));
                 }
@@ -706,6 +727,8 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
     TT end = 0;
     uint32_t ovf = 0;
     int64_t gsum = 0;
+    uint32_t ph_timely = 0;  // Eq. 12 window terms (kPhi)
+    uint64_t ph_life = 0;
     for (int32_t c = 0; c < chunks; ++c) {
         const int b = c % kBuffers;
         named_sync(kFullR + b, kResThreads + 32);
@@ -723,7 +746,8 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
                 for (int x = 0; x < 3; ++x) nw[x] = rb[(x * kChunk + kn) * kPitch];
                 const uint32_t r3 = w[1].y;
                 if (!(r3 & kSkip)) {
-                    const uint32_t run = w[0].x, ld = w[1].x, arr = w[0].y, r4 = w[2].x, r5 = w[2].y;
+                    const uint32_t run = w[0].x, arr = w[0].y, r4 = w[2].x, r5 = w[2].y;
+                    const uint32_t ld = kPhi ? w[1].x & 0x7FFFFFFFu : w[1].x;  // bit 31: a reload (kPhi)
                     TT *tf_d = tfree + (r3 & 31u) * kP;
                     // Release (Eq. 2, Eq. 7); an accumulator slot is reset by its reader.
                     const uint32_t rs = r5 >> 16;
@@ -732,9 +756,18 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
                     // A miss loads on this device first (ld > 0 only on a miss); a
                     // prefetched load waits only for the arrival (Eq. 5).  On a hit
                     // the residency stage cleared the prefetch bit and ld is 0.
-                    const TT ls = max(*tf_d, (r3 & kPrefetch) ? (TT)arr : rel);
+                    const TT tf = *tf_d;
+                    const TT ls = max(tf, (r3 & kPrefetch) ? (TT)arr : rel);
                     const TT le = ls + ld;
                     const TT start = max(le, rel);
+                    if (kPhi) {
+                        // A prefetched load (the bit survives residency only on a
+                        // miss) that starts before the release and ends by it is
+                        // timely; every unit adds the delay its load puts on its
+                        // start, and a reload its load time.
+                        ph_timely += (r3 & kPrefetch) && ls < rel && le <= rel;
+                        ph_life += (uint64_t)(start - max(tf, rel)) + (w[1].x >> 31 ? (uint64_t)ld : 0ull);
+                    }
                     const TT cfin = start + run;
                     if (kNarrow) ovf |= (le < ls) | (cfin < start);
                     else ovf |= run == kRunCap;
@@ -777,6 +810,10 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
         out.makespan_us[p] = (int64_t)end - dp.first_arrival;
         out.gpu_us[p] = gsum + nopen * (int64_t)end;
         out.p95_us[p] = (int64_t)select_strided<TT, kP>(slots, W, rank);
+        if (kPhi) {
+            dp.phi_timely[p] = ph_timely;
+            dp.phi_life[p] = (int64_t)ph_life;
+        }
     }
     }
     __syncthreads();  // the group's shared state is free for the next group
@@ -1218,6 +1255,7 @@ status_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out)
         if (lane == 0) {
             out.status[p] = st;
             if (st) out.makespan_us[p] = out.p95_us[p] = out.gpu_us[p] = WF_INF64;
+            if (st && dp.phi_life) dp.phi_timely[p] = dp.phi_life[p] = WF_INF64;
         }
         __syncwarp();  // pos[] is reused by the warp's next plan
     }
@@ -1294,11 +1332,11 @@ int plans_per_sm(size_t smem, int kp)
     return smem <= 227 * 1024 ? kp * (int)((228 * 1024) / (smem + 1024)) : 0;
 }
 
-template <typename Q, typename TT, int kP, int kR>
+template <typename Q, typename TT, int kP, int kR, bool kF>
 int launch_pc(const wf_dev_problem &dp, int sms, const wf_plans *pl, const wf_eval_out *out, size_t smem,
               const int32_t *in_list, const int32_t *in_count, int32_t *list, int32_t *count, cudaStream_t st)
 {
-    int rc = wf_cuda_check(cudaFuncSetAttribute(pc_kernel<Q, TT, kP, kR>,
+    int rc = wf_cuda_check(cudaFuncSetAttribute(pc_kernel<Q, TT, kP, kR, kF>,
                                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
                            "sweep smem attribute");
     if (rc) return rc;
@@ -1309,12 +1347,12 @@ int launch_pc(const wf_dev_problem &dp, int sms, const wf_plans *pl, const wf_ev
         const int64_t per_sm = std::max<int64_t>(1, std::min<int64_t>(8, (228 * 1024) / (int64_t)(smem + 1024)));
         blocks = std::min<int64_t>(blocks, per_sm * sms);
     }
-    pc_kernel<Q, TT, kP, kR><<<(unsigned)blocks, 32 * PcShape<kP>::kWarps, smem, st>>>(dp, *pl, *out, in_list, in_count, list,
+    pc_kernel<Q, TT, kP, kR, kF><<<(unsigned)blocks, 32 * PcShape<kP>::kWarps, smem, st>>>(dp, *pl, *out, in_list, in_count, list,
                                                                           count);
     return wf_cuda_check(cudaGetLastError(), "sweep launch");
 }
 
-template <typename TT, int kR>
+template <typename TT, int kR, bool kF>
 int launch_pc_r(const wf_ctx *ctx, int kp, const wf_plans *pl, const wf_eval_out *out, size_t smem,
                 const int32_t *in_list, const int32_t *in_count, int32_t *list, int32_t *count, cudaStream_t st)
 {
@@ -1323,19 +1361,19 @@ int launch_pc_r(const wf_ctx *ctx, int kp, const wf_plans *pl, const wf_eval_out
     if constexpr (sizeof(TT) == 4) {  // the u32 sweep has one shape
         (void)kp;
         return dp.M <= 8
-                   ? launch_pc<uint32_t, TT, kPlans32, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
-                   : launch_pc<uint64_t, TT, kPlans32, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
+                   ? launch_pc<uint32_t, TT, kPlans32, kR, kF>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
+                   : launch_pc<uint64_t, TT, kPlans32, kR, kF>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
     } else {
         if (kp == 16)
             return dp.M <= 8
-                       ? launch_pc<uint32_t, TT, 16, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
-                       : launch_pc<uint64_t, TT, 16, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
+                       ? launch_pc<uint32_t, TT, 16, kR, kF>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
+                       : launch_pc<uint64_t, TT, 16, kR, kF>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
         if (kp == 6)
             return dp.M <= 8
-                       ? launch_pc<uint32_t, TT, 6, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
-                       : launch_pc<uint64_t, TT, 6, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
-        return dp.M <= 8 ? launch_pc<uint32_t, TT, 3, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
-                         : launch_pc<uint64_t, TT, 3, kR>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
+                       ? launch_pc<uint32_t, TT, 6, kR, kF>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
+                       : launch_pc<uint64_t, TT, 6, kR, kF>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
+        return dp.M <= 8 ? launch_pc<uint32_t, TT, 3, kR, kF>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
+                         : launch_pc<uint64_t, TT, 3, kR, kF>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
     }
 }
 
@@ -1343,8 +1381,11 @@ template <typename TT>
 int launch_pc_q(const wf_ctx *ctx, int kp, const wf_plans *pl, const wf_eval_out *out, size_t smem,
                 const int32_t *in_list, const int32_t *in_count, int32_t *list, int32_t *count, cudaStream_t st)
 {
-    return ctx->dp.reclaim ? launch_pc_r<TT, 1>(ctx, kp, pl, out, smem, in_list, in_count, list, count, st)
-                           : launch_pc_r<TT, 0>(ctx, kp, pl, out, smem, in_list, in_count, list, count, st);
+    if (ctx->dp.phi_life)
+        return ctx->dp.reclaim ? launch_pc_r<TT, 1, true>(ctx, kp, pl, out, smem, in_list, in_count, list, count, st)
+                               : launch_pc_r<TT, 0, true>(ctx, kp, pl, out, smem, in_list, in_count, list, count, st);
+    return ctx->dp.reclaim ? launch_pc_r<TT, 1, false>(ctx, kp, pl, out, smem, in_list, in_count, list, count, st)
+                           : launch_pc_r<TT, 0, false>(ctx, kp, pl, out, smem, in_list, in_count, list, count, st);
 }
 
 }  // namespace
@@ -1358,23 +1399,30 @@ int wf_launch_nextuse(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, c
     return wf_cuda_check(cudaGetLastError(), "next-use launch");
 }
 
+// Shared memory of a sweep CTA for this problem, its reclamation order and
+// whether the window terms of Eq. 12 are wanted.
+template <int kP, typename TT>
+size_t layout_bytes(const wf_dev_problem &dp)
+{
+    const int32_t NS = dp.nslots + 2;
+    if (dp.phi_life)
+        return dp.reclaim ? pc_layout<kP, TT, 1, true>(dp.D, dp.M, dp.W, NS).total
+                          : pc_layout<kP, TT, 0, true>(dp.D, dp.M, dp.W, NS).total;
+    return dp.reclaim ? pc_layout<kP, TT, 1, false>(dp.D, dp.M, dp.W, NS).total
+                      : pc_layout<kP, TT, 0, false>(dp.D, dp.M, dp.W, NS).total;
+}
+
 wf_sweep_cfg wf_sweep_config(const wf_dev_problem &dp)
 {
     wf_sweep_cfg c = {0, 0, 0};
     if (!sweep_usable(dp)) return c;
-    const int32_t NS = dp.nslots + 2;
-    const bool r = dp.reclaim != 0;
-    const size_t s32 = r ? pc_layout<kPlans32, uint32_t, 1>(dp.D, dp.M, dp.W, NS).total
-                         : pc_layout<kPlans32, uint32_t, 0>(dp.D, dp.M, dp.W, NS).total;
+    const size_t s32 = layout_bytes<kPlans32, uint32_t>(dp);
     if (s32 <= 227 * 1024) c.smem32 = s32;
     // The u64 sweep: 16, 6 or 3 plans per CTA, whichever keeps the most plans
     // per SM (ties: the smaller CTAs, more of them to hide latency).
-    const size_t s16 = r ? pc_layout<16, uint64_t, 1>(dp.D, dp.M, dp.W, NS).total
-                         : pc_layout<16, uint64_t, 0>(dp.D, dp.M, dp.W, NS).total;
-    const size_t s6 = r ? pc_layout<6, uint64_t, 1>(dp.D, dp.M, dp.W, NS).total
-                        : pc_layout<6, uint64_t, 0>(dp.D, dp.M, dp.W, NS).total;
-    const size_t s3 = r ? pc_layout<3, uint64_t, 1>(dp.D, dp.M, dp.W, NS).total
-                        : pc_layout<3, uint64_t, 0>(dp.D, dp.M, dp.W, NS).total;
+    const size_t s16 = layout_bytes<16, uint64_t>(dp);
+    const size_t s6 = layout_bytes<6, uint64_t>(dp);
+    const size_t s3 = layout_bytes<3, uint64_t>(dp);
     const int a = plans_per_sm(s16, 16), b = plans_per_sm(s6, 6), e = plans_per_sm(s3, 3);
     if (e > 0 && e >= a && e >= b) { c.smem64 = s3; c.plans64 = 3; }
     else if (b > 0 && b >= a) { c.smem64 = s6; c.plans64 = 6; }

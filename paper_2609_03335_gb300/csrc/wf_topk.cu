@@ -145,19 +145,31 @@ __device__ __forceinline__ void pick_digit(const unsigned int *hist, int shift, 
 }
 
 
-__global__ void compact_kernel(wf_eval_out res, int64_t P, void *scr)
+// The second and third terms of the key: p95 and GPU time, or (Eq. 12's
+// window terms) minus the timely prefetches and the lifecycle overhead.
+struct Terms {
+    const int64_t *a, *b;
+    int64_t sa;  // +1, or -1 for a term ranked largest first
+};
+
+__device__ __forceinline__ Cand cand_of(const wf_eval_out &res, const Terms &tm, int64_t p)
+{
+    Cand c;
+    c.mk = res.makespan_us[p];
+    c.p95 = tm.sa * tm.a[p];
+    c.gpu = tm.b[p];
+    c.id = (int32_t)p;
+    c.bad = res.status[p] != 0 ? 1u : 0u;
+    return c;
+}
+
+__global__ void compact_kernel(wf_eval_out res, Terms tm, int64_t P, void *scr)
 {
     const TopkScratch s = scratch_of(scr);
     const unsigned long long T = *s.T;
     for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < P; p += (int64_t)gridDim.x * blockDim.x) {
         if (key64(res, p) > T) continue;
-        Cand c;
-        c.mk = res.makespan_us[p];
-        c.p95 = res.p95_us[p];
-        c.gpu = res.gpu_us[p];
-        c.id = (int32_t)p;
-        c.bad = res.status[p] != 0 ? 1u : 0u;
-        s.cand[atomicAdd(s.count, 1u)] = c;
+        s.cand[atomicAdd(s.count, 1u)] = cand_of(res, tm, p);
     }
 }
 
@@ -234,13 +246,13 @@ __device__ void bitonic_sort(Cand *t, int len)
     __syncthreads();
 }
 
-__device__ void write_first(const Cand *t, int32_t k, int32_t *ids, int64_t *keys)
+__device__ void write_first(const Cand *t, int32_t k, int32_t *ids, int64_t *keys, int64_t sa)
 {
     for (int u = threadIdx.x; u < k; u += blockDim.x) {
         ids[u] = t[u].id;
         if (keys) {
             keys[3 * u] = t[u].mk;
-            keys[3 * u + 1] = t[u].p95;
+            keys[3 * u + 1] = sa * t[u].p95;
             keys[3 * u + 2] = t[u].gpu;
         }
     }
@@ -250,17 +262,9 @@ __device__ void write_first(const Cand *t, int32_t k, int32_t *ids, int64_t *key
 // compacted into scratch.
 struct PlanSrc {
     wf_eval_out res;
+    Terms tm;
     __device__ uint64_t key(int64_t i) const { return key64(res, i); }
-    __device__ Cand get(int64_t i) const
-    {
-        Cand c;
-        c.mk = res.makespan_us[i];
-        c.p95 = res.p95_us[i];
-        c.gpu = res.gpu_us[i];
-        c.id = (int32_t)i;
-        c.bad = res.status[i] != 0 ? 1u : 0u;
-        return c;
-    }
+    __device__ Cand get(int64_t i) const { return cand_of(res, tm, i); }
 };
 
 struct CandSrc {
@@ -274,7 +278,7 @@ struct CandSrc {
 // in t[0, k) and each round fills the rest of the tile; writes the first k.
 template <class Src>
 __device__ void fold_sort(const Src &src, int64_t n, int32_t k, const unsigned long long *kk,
-                          unsigned long long T, Cand *t, int32_t *ids, int64_t *keys)
+                          unsigned long long T, Cand *t, int32_t *ids, int64_t *keys, int64_t sa)
 {
     int len = 64;
     while (len < n && len < kTile) len <<= 1;
@@ -290,7 +294,7 @@ __device__ void fold_sort(const Src &src, int64_t n, int32_t k, const unsigned l
         first = false;
         bitonic_sort(t, len);
     }
-    write_first(t, k, ids, keys);
+    write_first(t, k, ids, keys, sa);
 }
 
 // The k best of src[0, n) (k <= n <= kOneCta): the 64-bit keys staged in kk,
@@ -298,7 +302,7 @@ __device__ void fold_sort(const Src &src, int64_t n, int32_t k, const unsigned l
 // into t and sorted there by the full key.
 template <class Src>
 __device__ void select_and_sort(const Src &src, int64_t n, int32_t k, unsigned long long *kk, Cand *t,
-                                int32_t *ids, int64_t *keys)
+                                int32_t *ids, int64_t *keys, int64_t sa)
 {
     __shared__ unsigned int m;
     if (threadIdx.x == 0) m = 0;
@@ -318,20 +322,20 @@ __device__ void select_and_sort(const Src &src, int64_t n, int32_t k, unsigned l
     __syncthreads();
     const unsigned int cnt = m;
     if (cnt > (unsigned)kTile) {  // massive ties with T
-        fold_sort(src, n, k, kk, T, t, ids, keys);
+        fold_sort(src, n, k, kk, T, t, ids, keys, sa);
         return;
     }
     int len = 64;
     while (len < (int)cnt) len <<= 1;
     for (int u = (int)cnt + threadIdx.x; u < len; u += blockDim.x) t[u] = padding();
     bitonic_sort(t, len);
-    write_first(t, k, ids, keys);
+    write_first(t, k, ids, keys, sa);
 }
 
 constexpr int64_t kOneCta = 16384;  // keys staged in shared memory by one CTA
 
 __global__ void __launch_bounds__(kThreads)
-final_kernel(int32_t k, void *scr, int32_t *ids, int64_t *keys)
+final_kernel(int32_t k, void *scr, int32_t *ids, int64_t *keys, int64_t sa)
 {
     extern __shared__ __align__(16) uint8_t tsm[];
     Cand *t = (Cand *)tsm;
@@ -339,17 +343,17 @@ final_kernel(int32_t k, void *scr, int32_t *ids, int64_t *keys)
     const TopkScratch s = scratch_of(scr);
     const int64_t n = *s.count;
     const CandSrc src{s.cand};
-    if (n <= kOneCta) select_and_sort(src, n, k, kk, t, ids, keys);
-    else fold_sort(src, n, k, nullptr, 0ull, t, ids, keys);
+    if (n <= kOneCta) select_and_sort(src, n, k, kk, t, ids, keys, sa);
+    else fold_sort(src, n, k, nullptr, 0ull, t, ids, keys, sa);
 }
 
 __global__ void __launch_bounds__(kThreads)
-topk_one_kernel(wf_eval_out res, int64_t P, int32_t k, int32_t *ids, int64_t *keys)
+topk_one_kernel(wf_eval_out res, Terms tm, int64_t P, int32_t k, int32_t *ids, int64_t *keys)
 {
     extern __shared__ __align__(16) uint8_t tsm[];
     Cand *t = (Cand *)tsm;
     unsigned long long *kk = (unsigned long long *)(tsm + kTile * sizeof(Cand));  // [P]
-    select_and_sort(PlanSrc{res}, P, k, kk, t, ids, keys);
+    select_and_sort(PlanSrc{res, tm}, P, k, kk, t, ids, keys, tm.sa);
 }
 
 }  // namespace
@@ -360,14 +364,15 @@ size_t wf_topk_scratch_bytes(int64_t max_P)
 }
 
 int wf_launch_topk(wf_ctx *ctx, const wf_eval_out *res, int64_t P, int32_t k, int32_t *ids,
-                   int64_t *keys, cudaStream_t st)
+                   int64_t *keys, cudaStream_t st, const int64_t *term2, const int64_t *term3, int64_t sign2)
 {
+    const Terms tm{term2 ? term2 : res->p95_us, term3 ? term3 : res->gpu_us, term2 ? sign2 : 1};
     const size_t smem = kTile * sizeof(Cand) + 8 * (size_t)std::min<int64_t>(P, kOneCta);
     if (P <= kOneCta) {
         int rc = wf_cuda_check(cudaFuncSetAttribute(topk_one_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                     (int)smem), "topk smem attribute");
         if (rc) return rc;
-        topk_one_kernel<<<1, kThreads, smem, st>>>(*res, P, k, ids, keys);
+        topk_one_kernel<<<1, kThreads, smem, st>>>(*res, tm, P, k, ids, keys);
         return wf_cuda_check(cudaGetLastError(), "topk launch");
     }
     int rc = wf_cuda_check(cudaFuncSetAttribute(final_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -379,7 +384,7 @@ int wf_launch_topk(wf_ctx *ctx, const wf_eval_out *res, int64_t P, int32_t k, in
     if (rc) return rc;
     kth_kernel<<<(unsigned)((P + kKth - 1) / kKth), kThreads, 0, st>>>(*res, P, k, ctx->topk_scratch);
     const int64_t blocks = std::min<int64_t>((P + 255) / 256, (int64_t)ctx->sms * 8);
-    compact_kernel<<<(unsigned)blocks, 256, 0, st>>>(*res, P, ctx->topk_scratch);
-    final_kernel<<<1, kThreads, smem, st>>>(k, ctx->topk_scratch, ids, keys);
+    compact_kernel<<<(unsigned)blocks, 256, 0, st>>>(*res, tm, P, ctx->topk_scratch);
+    final_kernel<<<1, kThreads, smem, st>>>(k, ctx->topk_scratch, ids, keys, tm.sa);
     return wf_cuda_check(cudaGetLastError(), "topk launch");
 }

@@ -24,7 +24,8 @@ INT64_MAX = np.iinfo(np.int64).max
 EXPORTS = ("wf_problem_check", "wf_ctx_create", "wf_forecast_readiness", "wf_eval_plans",
            "wf_topk", "wf_ctx_status", "wf_ctx_destroy", "wf_strerror", "wf_last_error",
            "wf_eval_plans_static", "wf_mutate_plans", "wf_merge_elite", "wf_local_search",
-           "wf_construct_plans", "wf_ctx_set_reclaim", "wf_ctx_check_wait_expiry")
+           "wf_construct_plans", "wf_ctx_set_reclaim", "wf_ctx_check_wait_expiry", "wf_eval_plans_phi",
+           "wf_topk_phi")
 
 
 class WfError(RuntimeError):
@@ -78,6 +79,8 @@ def load_library():
         "wf_forecast_readiness": ([p, p, p, p], ctypes.c_int),
         "wf_eval_plans": ([p, p, p, p], ctypes.c_int),
         "wf_topk": ([p, p, i64, i32, p, p, p], ctypes.c_int),
+        "wf_eval_plans_phi": ([p, p, p, p, p, p], ctypes.c_int),
+        "wf_topk_phi": ([p, p, p, p, i64, i32, p, p, p], ctypes.c_int),
         "wf_mutate_plans": ([p, p, p, ctypes.c_uint64, i64, i32, p], ctypes.c_int),
         "wf_merge_elite": ([p, p, p, p, p, p], ctypes.c_int),
         "wf_local_search": ([p, p, p, p, p, ctypes.c_uint64, i64, i32, i32, p], ctypes.c_int),
@@ -308,6 +311,22 @@ def wf_topk(ctx: Ctx, res: Results, P: int, k: int, ids, keys=None, stream=None)
     _check(load_library().wf_topk(ctx.ptr, ctypes.byref(oc), int(P), int(k), ids.data_ptr(),
                                   None if keys is None else keys.data_ptr(), _stream_handle(stream)),
            "wf_topk")
+
+
+def wf_eval_plans_phi(ctx: Ctx, plans: DevicePlans, out: Results, timely, life, stream=None):
+    """wf_eval_plans plus Eq. 12's window terms; timely, life: device int64 [P]."""
+    pl = plans.c(None, 0)
+    oc = out.c(0)
+    _check(load_library().wf_eval_plans_phi(ctx.ptr, ctypes.byref(pl), ctypes.byref(oc), timely.data_ptr(),
+                                            life.data_ptr(), _stream_handle(stream)), "wf_eval_plans_phi")
+
+
+def wf_topk_phi(ctx: Ctx, res: Results, timely, life, P: int, k: int, ids, keys=None, stream=None):
+    """The k best by Eq. 12's window key; keys: device int64 [k, 3] (makespan, timely, life) or None."""
+    oc = res.c()
+    _check(load_library().wf_topk_phi(ctx.ptr, ctypes.byref(oc), timely.data_ptr(), life.data_ptr(), int(P),
+                                      int(k), ids.data_ptr(), None if keys is None else keys.data_ptr(),
+                                      _stream_handle(stream)), "wf_topk_phi")
 
 
 def wf_mutate_plans(ctx: Ctx, parents: DevicePlans, children: DevicePlans, seed: int, round_: int,
