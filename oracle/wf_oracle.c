@@ -28,7 +28,10 @@
  *   - makespan = last finish - first arrival, p95 = nearest-rank 95th
  *     percentile of per-session completion latency (Section 4.2), GPU time =
  *     time each device holds at least one model: loading, generating or idle
- *     resident (Section 4.3).
+ *     resident (Section 4.3);
+ *   - beside them, the window terms of the ranking key of Eq. 12: timely
+ *     prefetches and the lifecycle overhead (ready-work loading delay plus
+ *     reloads after reclamation), see orc_eval_phi_batch.
  *
  * Every time is an int64 microsecond count and every memory an int32 MiB
  * count, so results are exact.  Points the paper leaves open are read as
