@@ -337,6 +337,35 @@ def reclaim_timing(wf, ctx, dp, res_lru, P, stream, flush):
             "mean_gpu_us": {"lru": mean(lru[1]), "next_use": mean(res.gpu)}}
 
 
+def phi_timing(wf, ctx, dp, P, k, stream, flush):
+    """The batch through wf_eval_plans_phi (Eq. 12's window terms beside the
+    metrics) and its top-k by that key: eval time (median of 3, L2 flushed
+    before each) and the best plan's (makespan, timely prefetches, lifecycle
+    overhead)."""
+    import torch
+    res = wf.Results(P, dp.place.device)
+    timely = torch.empty(P, dtype=torch.int64, device=dp.place.device)
+    life = torch.empty_like(timely)
+    ids = torch.empty(k, dtype=torch.int32, device=dp.place.device)
+    keys = torch.empty((k, 3), dtype=torch.int64, device=dp.place.device)
+    ts = []
+    with torch.cuda.stream(stream):
+        wf.wf_eval_plans_phi(ctx, dp, res, timely, life, stream)
+        for _ in range(3):
+            e = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+            flush.zero_()
+            e[0].record(stream)
+            wf.wf_eval_plans_phi(ctx, dp, res, timely, life, stream)
+            e[1].record(stream)
+            ts.append(e)
+        wf.wf_topk_phi(ctx, res, timely, life, P, k, ids, keys, stream)
+    torch.cuda.synchronize()
+    ms = float(np.median([a.elapsed_time(b) for a, b in ts]))
+    best = keys[0].tolist()
+    return {"eval_ms": ms, "plans_per_s": P / (ms * 1e-3),
+            "best": {"makespan_us": best[0], "timely_prefetches": best[1], "life_us": best[2]}}
+
+
 def run_gpu(args, rank, world, local):
     import torch
 
@@ -456,6 +485,7 @@ def run_gpu(args, rank, world, local):
     barrier(world)
     # before the search rewrites rows 0..31; the policy needs deterministic latencies
     nextuse = reclaim_timing(wf, ctx, dp, res, P, stream, flush) if prob.S == 0 else None
+    phi = phi_timing(wf, ctx, dp, P, k, stream, flush) if prob.S == 0 else None
     search = local_search_timing(wf, ctx, dp, prob, P, stream, flush, peak_gbs=read_peaks().get("hbm_gbs"))
     built = construct_timing(wf, ctx, prob, P, k, stream, flush, random_best=int(keys[0, 0].item()))
     clk = clocks.stop()
@@ -515,6 +545,7 @@ def run_gpu(args, rank, world, local):
             "local_search": search,
             "construct": built,
             "reclaim_next_use": nextuse,
+            "eq12_window_terms": phi,
         }
         print(json.dumps(line), flush=True)
     ctx.close()
