@@ -6,7 +6,9 @@
 //
 // Mapping: one thread plays one (plan, sample).  Its mutable state (chain-tail
 // finish times, per-device and per-session state) lives in a scratch row of
-// the context; plans beyond the number of rows are taken in rounds.
+// the context; plans beyond the number of rows are taken in rounds.  For
+// wf_eval_plans_phi a deterministic play also returns the window terms of
+// Eq. 12's ranking key (timely prefetches, lifecycle overhead).
 #include <algorithm>
 #include <mutex>
 

@@ -20,6 +20,11 @@
 //
 // Times are u32; a plan whose times reach 2^32 us is listed for the exact
 // int64 path in wf_eval.cu.
+//
+// A compile-time variant (kPhi) also returns the window terms of Eq. 12's
+// ranking key: residency marks a reload (a model its device held before) in
+// bit 31 of the record's load word, and timing counts the timely prefetches
+// and sums each unit's load delay plus its reload time.
 #include <algorithm>
 
 #include "wf_internal.cuh"
