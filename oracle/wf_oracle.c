@@ -43,7 +43,9 @@
  * Parity pins: every function here is pinned by the CPU test suite
  * (hand-worked windows, closed forms, textbook-routine reductions,
  * invariants replayed from the trace, brute force).  The stochastic
- * multiplier draw is pinned by the published SplitMix64 vector and by the
+ * multiplier draw is pinned by the published SplitMix64 vector, by three
+ * multipliers worked by hand from that vector and the table formulas (each
+ * nested hash input chosen to be a published generator state), and by the
  * sample statistics of the multipliers.
  */
 #include <stdint.h>

@@ -43,6 +43,9 @@ MUTANTS = {
     "z_truncates": ("if (prod % 262144 != 0 && prod < 0) zq -= 1;", ""),
     "multiplier_no_rounding": ("(base * mult + 32768) >> 16", "(base * mult) >> 16"),
     "angle_from_low_bits": ("(h >> 32) & (uint64_t)(pb->bm_cn - 1)", "h & (uint64_t)(pb->bm_cn - 1)"),
+    "hash_nests_sample_first": ("orc_splitmix64(orc_splitmix64(orc_splitmix64(pb->seed ^ plan) ^ sample) ^ node)",
+                                "orc_splitmix64(orc_splitmix64(orc_splitmix64(pb->seed ^ sample) ^ plan) ^ node)"),
+    "radius_from_bits_12": ("(int64_t)(h & (uint64_t)(pb->bm_rn - 1))", "(int64_t)((h >> 12) & (uint64_t)(pb->bm_rn - 1))"),
     "mean_rounds_up": ("out3[0] = sum_mk / S;", "out3[0] = (sum_mk + S - 1) / S;"),
     "device_free_at_head_end": ("t_free[d] = c[last];", "t_free[d] = c[h];"),
     "hash_ignores_plan": ("orc_splitmix64(pb->seed ^ plan)", "orc_splitmix64(pb->seed)"),

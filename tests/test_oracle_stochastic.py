@@ -30,6 +30,35 @@ def test_splitmix64_published_vector():
         assert oracle.splitmix64((state + k * GAMMA) % (1 << 64)) == int(want)
 
 
+def test_multiplier_hand_derived():
+    """The multiplier of three (seed, plan, sample, node) tuples worked by hand
+    in tests/golden/multiplier_hand_derived.json: each nested mix input is a
+    Rosetta state, so every hash value is a published SplitMix64 output; the
+    table entries, the floored product and the multiplier follow from the
+    table formulas.  A wrong nesting order, wrong index bits, a truncating
+    zq or a wrong table entry changes the result."""
+    with open(os.path.join(GOLDEN, "multiplier_hand_derived.json")) as f:
+        fx = json.load(f)
+    with open(os.path.join(GOLDEN, "splitmix64_rosetta.json")) as f:
+        out = [int(x) for x in json.load(f)["outputs"]]
+    state = {int(k): int(v) for k, v in fx["states"].items()}
+    for k, v in state.items():
+        assert v == (1234567 + k * GAMMA) % (1 << 64)
+    r, c, e = wfgen.box_muller_tables()
+    rng = np.random.default_rng(0)
+    for case in fx["cases"]:
+        seed, plan, sample, node = (int(case[x]) for x in ("seed", "plan", "sample", "node"))
+        a, b, cc = case["a"], case["b"], case["c"]
+        # the chosen inputs land each nested step on a published state
+        assert seed ^ plan == state[a]
+        assert out[a] ^ sample == state[b]
+        assert out[b] ^ node == state[cc]
+        steps = list(case["steps"].values())
+        assert int(steps[2]) == out[cc]
+        prob = _stoch_problem(rng, S=1, tables=(r, c, e)).with_(seed=seed)
+        assert oracle.multiplier(prob, plan, sample, node) == case["multiplier"]
+
+
 def _stoch_problem(rng, S, tables=None, **kw):
     prob = random_problem(rng, **kw)
     r, c, e = tables or wfgen.box_muller_tables()
