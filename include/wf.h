@@ -14,6 +14,7 @@
  *   wf_eval_plans           play every plan forward (Eq. 2-11) -> metrics
  *   wf_topk                 the k best plans by the ranking key
  *   wf_eval_plans_static    wf_eval_plans without a context or any allocation
+ *   wf_static_status        device-side outcome of the last wf_eval_plans_static
  *   wf_mutate_plans         children of plans with a few point changes each
  *   wf_merge_elite          keep the k best of an elite and its children
  *   wf_local_search         rounds of mutate -> evaluate -> merge
@@ -68,8 +69,10 @@ enum {
     WF_ST_DEVICE = 1u,      /* some place[n] >= D */
     WF_ST_CAPACITY = 2u,    /* some peak[n][place[n]] > cap[place[n]] (Eq. 8) */
     WF_ST_PERMUTATION = 4u, /* order is not a permutation of 0..N-1 */
-    WF_ST_TOPOLOGY = 8u     /* an edge u -> v with v dispatched before u (Eq. 9-10);
+    WF_ST_TOPOLOGY = 8u,    /* an edge u -> v with v dispatched before u (Eq. 9-10);
                                examined only when WF_ST_PERMUTATION is clear */
+    WF_ST_TABLES = 16u      /* wf_eval_plans_static only: the problem tables failed its
+                               device check, so no plan of the batch was evaluated */
 };
 
 typedef struct wf_ctx wf_ctx;
@@ -208,26 +211,45 @@ int wf_topk(wf_ctx *ctx, const wf_eval_out *res, int64_t P, int32_t k,
  * the cache -- or whose device memory belongs to an allocator that must not
  * be bypassed.
  *
- * Same results as wf_eval_plans for a deterministic problem (S must be 0),
- * without a context and without allocating anything: every table of *prob is
- * a DEVICE pointer here (same layouts as above; the caller guarantees the
- * problem passes wf_problem_check, which this call cannot repeat without
- * copying it back), plans and outputs are DEVICE pointers as for
- * wf_eval_plans.  Scratch is a 32 MiB file-scope device array that every GPU
- * loading this library holds until the process exits.  A call needs 256 B,
- * plus three tables of 4*N bytes each rounded up to 256 B, plus one state row
- * per plan of about 8*(N + W + 3*D) + 4*D*(M + 2) bytes (rounded up to
- * 128 B); a batch that does not fit returns WF_EINVAL naming the largest
- * batch that does (about 1,900 plans of a 2,000-activation window) -- split
- * larger batches by plan_base.  The first call on a device looks the array's
- * address up (cudaGetSymbolAddress) with that device current; make that first
- * call before any stream capture.  All calls share the array and each call
- * re-initialises what it relies on; calls that overlap on the GPU (other
- * streams, other threads) race on it and must be serialised by the caller.
- * Asynchronous on `stream`; returns WF_OK, WF_EINVAL or WF_ECUDA.
+ * Same results as wf_eval_plans with least-recently-used reclamation (the
+ * default of a context) for a deterministic problem (S must be 0), without a
+ * context and without allocating anything: every table of *prob is a DEVICE
+ * pointer here (same layouts as above), plans and outputs are DEVICE
+ * pointers as for wf_eval_plans.  Before anything is indexed by them, a
+ * device check confirms model < M, 0 <= session < W, pred_off starting at 0
+ * and non-decreasing, 0 <= pred_idx < N without self-loops, non-negative run
+ * times, loads and arrivals, weights and capacities >= 1 and peak >= weight;
+ * when it fails, every plan of the batch gets status WF_ST_TABLES and
+ * INT64_MAX metrics, and wf_static_status reports it.  (Acyclicity,
+ * duplicate or cross-session edges and "every activation fits somewhere" are
+ * not checked: the caller guarantees them, as wf_problem_check does for a
+ * context; pred_off[N] must be the length of pred_idx.)
+ * Scratch is a 32 MiB file-scope device array that every GPU loading this
+ * library holds until the process exits.  A call needs 256 B, plus three
+ * tables of 4*N bytes each rounded up to 256 B, plus one state row per plan
+ * of 8*(N + W + 3*D) + 4*D*(M + 3) bytes rounded up to 128 B; a batch that
+ * does not fit returns WF_EINVAL naming the largest batch that does (about
+ * 1,900 plans of a 2,000-activation window) -- split larger batches by
+ * plan_base.  Each call made outside stream capture looks the array's
+ * address up (cudaGetSymbolAddress) with the current device; a call under
+ * capture reuses the address of the last call outside capture on that
+ * device, so make one call before capturing, and again after a device
+ * reset.  All calls share the array and each call re-initialises what it
+ * relies on; calls that overlap on the GPU (other streams, other threads)
+ * race on it and must be serialised by the caller.  Asynchronous on
+ * `stream`; returns WF_OK, WF_EINVAL or WF_ECUDA.
  */
 int wf_eval_plans_static(const wf_problem *prob, const wf_plans *plans, const wf_eval_out *out,
                          void *stream);
+
+/*
+ * The paper has no counterpart to this call either: the device-side outcome
+ * of the last wf_eval_plans_static call on the current device.  Synchronizes
+ * `stream`, reads the static array's error word (no allocation) and clears
+ * it: WF_OK, WF_EINVAL when the problem tables failed the device check, or
+ * WF_ECUDA when an evaluation hit a state no valid plan reaches.
+ */
+int wf_static_status(void *stream);
 
 /*
  * Local search around the best plans.  The paper's scheduler re-ranks its

@@ -525,6 +525,11 @@ __host__ __device__ __forceinline__ StaticLayout static_layout(int32_t N, int64_
     return l;
 }
 
+// Error word of the static array (header offset 8): 0, or kStaticBadTables
+// when the problem tables failed the device check (bits 8.. name the first
+// check that failed), or the evaluation's own error codes.
+constexpr int kStaticBadTables = 4;
+
 // Everything the derived tables start from: zero successor counts, no links,
 // the first arrival at +infinity, a clear error word.
 __global__ void static_init_kernel(uint8_t *s, int32_t N, StaticLayout l)
@@ -541,8 +546,41 @@ __global__ void static_init_kernel(uint8_t *s, int32_t N, StaticLayout l)
     }
 }
 
+// The device check of the caller's tables (one thread per node, model,
+// device, session and (model, device) pair), before any of them indexes
+// another table.  A failure sets the error word; the kernels after it then
+// index nothing.
+__global__ void static_check_kernel(uint8_t *s, wf_dev_problem dp)
+{
+    const int32_t v = blockIdx.x * blockDim.x + threadIdx.x;
+    const int32_t N = dp.N, D = dp.D, M = dp.M, W = dp.W;
+    int bad = 0;
+    if (v < N) {
+        const int32_t a = dp.pred_off[v], b = dp.pred_off[v + 1];
+        if ((v == 0 && a != 0) || b < a) bad = 1;
+        else
+            for (int32_t e = a; e < b; ++e) {
+                const int32_t u = dp.pred_idx[e];
+                if (u < 0 || u >= N || u == v) { bad = 2; break; }
+            }
+        const uint32_t m = dp.model[v];
+        const int32_t w = dp.session[v];
+        if (m >= (uint32_t)M) bad = 3;
+        else if (w < 0 || w >= W) bad = 4;
+        else
+            for (int32_t d = 0; d < D; ++d)
+                if (dp.lat[(int64_t)v * D + d] < 0 || dp.peak[(int64_t)v * D + d] < dp.weight[m]) { bad = 5; break; }
+    }
+    if (v < M && dp.weight[v] < 1) bad = 6;
+    if (v < D && dp.cap[v] < 1) bad = 7;
+    if (v < M * D && dp.load[v] < 0) bad = 8;
+    if (v < W && dp.arrival[v] < 0) bad = 9;
+    if (bad) atomicCAS((int *)(s + 8), 0, kStaticBadTables | (bad << 8));
+}
+
 __global__ void static_count_kernel(uint8_t *s, wf_dev_problem dp, StaticLayout l)
 {
+    if (*(volatile int *)(s + 8)) return;  // the tables failed the check
     const int32_t v = blockIdx.x * blockDim.x + threadIdx.x;
     if (v < dp.W) atomicMin((long long *)s, (long long)dp.arrival[v]);
     if (v >= dp.N) return;
@@ -553,6 +591,7 @@ __global__ void static_count_kernel(uint8_t *s, wf_dev_problem dp, StaticLayout 
 // Eq. 3: (u, v) fusible iff succ(u) = {v}, pred(v) = {u}, same model.
 __global__ void static_link_kernel(uint8_t *s, wf_dev_problem dp, StaticLayout l)
 {
+    if (*(volatile int *)(s + 8)) return;  // the tables failed the check
     const int32_t v = blockIdx.x * blockDim.x + threadIdx.x;
     if (v >= dp.N || dp.pred_off[v + 1] - dp.pred_off[v] != 1) return;
     const int32_t u = dp.pred_idx[dp.pred_off[v]];
@@ -570,6 +609,11 @@ eval_static_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, uint8_t *s, 
 {
     const int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (p >= pl.P) return;
+    if ((*(volatile int *)(s + 8) & 0xFF) == kStaticBadTables) {  // nothing is evaluated
+        out.status[p] = WF_ST_TABLES;
+        out.makespan_us[p] = out.p95_us[p] = out.gpu_us[p] = WF_INF64;
+        return;
+    }
     wf_dev_problem d = dp;
     d.first_arrival = *(const int64_t *)s;
     Row row = row_at(d, s + l.rows + (size_t)p * row_bytes);
@@ -587,7 +631,8 @@ eval_static_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, uint8_t *s, 
     out.p95_us[p] = select_rank(row.comp, d.W, p95_rank(d.W));
 }
 
-// Device address of the static array, looked up once per device.
+// Device address of the static array per device, from the last lookup
+// outside stream capture.
 uint8_t *g_static_addr[64];
 bool g_static_ready[64];
 std::mutex g_static_mu;
@@ -646,15 +691,24 @@ extern "C" int wf_eval_plans_static(const wf_problem *pb, const wf_plans *pl, co
     int rc = wf_cuda_check(cudaGetDevice(&dev), "cudaGetDevice");
     if (rc) return rc;
     if (dev < 0 || dev >= 64) return wf_set_error(WF_EINVAL, "device ordinal %d >= 64", dev);
+    cudaStream_t st = (cudaStream_t)stream;
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    rc = wf_cuda_check(cudaStreamIsCapturing(st, &cs), "stream capture status");
+    if (rc) return rc;
     uint8_t *s = nullptr;
     {
+        // Outside capture the address is looked up with the current device
+        // (valid in the current context, also after a device reset); under
+        // capture the last such lookup on this device is reused.
         std::lock_guard<std::mutex> lock(g_static_mu);
-        if (!g_static_ready[dev]) {
+        if (cs == cudaStreamCaptureStatusNone) {
             void *p = nullptr;
             rc = wf_cuda_check(cudaGetSymbolAddress(&p, g_static_scratch), "cudaGetSymbolAddress");
             if (rc) return rc;
             g_static_addr[dev] = (uint8_t *)p;
             g_static_ready[dev] = true;
+        } else if (!g_static_ready[dev]) {
+            return wf_set_error(WF_EINVAL, "the first wf_eval_plans_static call on a device must not be captured");
         }
         s = g_static_addr[dev];
     }
@@ -662,13 +716,38 @@ extern "C" int wf_eval_plans_static(const wf_problem *pb, const wf_plans *pl, co
     dp.fprev = (const int32_t *)(s + l.fprev);
     dp.err = (int *)(s + 8);
 
-    cudaStream_t st = (cudaStream_t)stream;
     const int32_t span = std::max(N, W);
     const unsigned grid = (unsigned)((span + 255) / 256);
+    const int32_t cspan = std::max(span, M * D);
     static_init_kernel<<<(unsigned)((N + 255) / 256), 256, 0, st>>>(s, N, l);
+    static_check_kernel<<<(unsigned)((cspan + 255) / 256), 256, 0, st>>>(s, dp);
     static_count_kernel<<<grid, 256, 0, st>>>(s, dp, l);
     static_link_kernel<<<(unsigned)((N + 255) / 256), 256, 0, st>>>(s, dp, l);
     eval_static_kernel<<<(unsigned)((pl->P + kEvalThreads - 1) / kEvalThreads), kEvalThreads, 0, st>>>(
         dp, *pl, *out, s, l, row);
     return wf_cuda_check(cudaGetLastError(), "static evaluation launch");
+}
+
+extern "C" int wf_static_status(void *stream)
+{
+    int rc = wf_cuda_check(cudaStreamSynchronize((cudaStream_t)stream), "cudaStreamSynchronize");
+    if (rc) return rc;
+    int err = 0;
+    rc = wf_cuda_check(cudaMemcpyFromSymbol(&err, g_static_scratch, sizeof(int), 8), "read the static error word");
+    if (rc) return rc;
+    if (!err) return WF_OK;
+    const int zero = 0;
+    rc = wf_cuda_check(cudaMemcpyToSymbol(g_static_scratch, &zero, sizeof(int), 8), "clear the static error word");
+    if (rc) return rc;
+    if ((err & 0xFF) == kStaticBadTables) {
+        static const char *what[] = {"", "pred_off does not start at 0 or decreases",
+                                     "a pred_idx entry is out of range or a self-loop", "a model id is >= M",
+                                     "a session id is out of range", "a run time is negative or a peak below its weight",
+                                     "a weight is below 1", "a capacity is below 1", "a load time is negative",
+                                     "an arrival is negative"};
+        const int k = err >> 8;
+        return wf_set_error(WF_EINVAL, "the problem tables failed the device check: %s",
+                            k >= 1 && k <= 9 ? what[k] : "unknown");
+    }
+    return wf_set_error(WF_ECUDA, "device error word %d in the static evaluation", err);
 }

@@ -17,7 +17,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libwf.so")
 
 WF_OK, WF_EINVAL, WF_ENOMEM, WF_ECUDA, WF_ETIMEOUT = 0, 1, 2, 3, 4
-ST_DEVICE, ST_CAPACITY, ST_PERMUTATION, ST_TOPOLOGY = 1, 2, 4, 8
+ST_DEVICE, ST_CAPACITY, ST_PERMUTATION, ST_TOPOLOGY, ST_TABLES = 1, 2, 4, 8, 16
 INT64_MAX = np.iinfo(np.int64).max
 
 # Every entry point declared in include/wf.h.
@@ -25,7 +25,7 @@ EXPORTS = ("wf_problem_check", "wf_ctx_create", "wf_forecast_readiness", "wf_eva
            "wf_topk", "wf_ctx_status", "wf_ctx_destroy", "wf_strerror", "wf_last_error",
            "wf_eval_plans_static", "wf_mutate_plans", "wf_merge_elite", "wf_local_search",
            "wf_construct_plans", "wf_ctx_set_reclaim", "wf_ctx_check_wait_expiry", "wf_eval_plans_phi",
-           "wf_topk_phi")
+           "wf_topk_phi", "wf_static_status")
 
 
 class WfError(RuntimeError):
@@ -92,6 +92,7 @@ def load_library():
         "wf_strerror": ([ctypes.c_int], ctypes.c_char_p),
         "wf_last_error": ([], ctypes.c_char_p),
         "wf_eval_plans_static": ([p, p, p, p], ctypes.c_int),
+        "wf_static_status": ([p], ctypes.c_int),
     }
     for name, (args, res) in sig.items():
         f = getattr(lib, name)
@@ -398,3 +399,9 @@ def wf_eval_plans_static(prob: DeviceProblem, plans: DevicePlans, out: Results, 
     oc = out.c()
     _check(load_library().wf_eval_plans_static(ctypes.byref(prob.c), ctypes.byref(pl), ctypes.byref(oc),
                                                _stream_handle(stream)), "wf_eval_plans_static")
+
+
+def wf_static_status(stream=None):
+    """Synchronize the stream and report (then clear) the device-side outcome
+    of the last wf_eval_plans_static call on the current device."""
+    _check(load_library().wf_static_status(_stream_handle(stream)), "wf_static_status")
