@@ -366,6 +366,123 @@ def phi_timing(wf, ctx, dp, P, k, stream, flush):
             "best": {"makespan_us": best[0], "timely_prefetches": best[1], "life_us": best[2]}}
 
 
+# Fixed oracle samples of the other windows (plans), each a few seconds of
+# one host thread at most.
+OTHER_WORKLOADS = {"tiny": 1024, "mix": 1024, "stochastic": 16, "large": 128}
+
+
+def workload_entry(name, wf, dev, steps=5, warmup=3, with_cpu=True):
+    """One forecast / eval / top-k step of another named window at its full
+    size, timed like the headline (CUDA events, L2 flushed before each step),
+    with the oracle on a fixed sample of the same batch and the clocks seen.
+    Stochastic windows report simulations (plans x samples) per second."""
+    import torch
+
+    import wfgen
+    w = wfgen.config(name)
+    prob, P, k = w.problem, w.P, w.k
+    plans = wfgen.make_plans(prob, P, w.plan_seed)
+    ctx = wf.Ctx(prob, max_P=P, device=dev.index)
+    dp = wf.DevicePlans.from_host(plans, dev)
+    res = wf.Results(P, dev)
+    rel = torch.empty(prob.N, dtype=torch.int64, device=dev)
+    comp = torch.empty_like(rel)
+    ids = torch.empty(k, dtype=torch.int32, device=dev)
+    keys = torch.empty((k, 3), dtype=torch.int64, device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
+    stream = torch.cuda.Stream(device=dev)
+    with torch.cuda.stream(stream):
+        for _ in range(warmup):
+            flush.zero_()
+            wf.wf_forecast_readiness(ctx, rel, comp, stream)
+            wf.wf_eval_plans(ctx, dp, res, stream)
+            wf.wf_topk(ctx, res, P, k, ids, keys, stream)
+    wf.wf_ctx_status(ctx, stream)
+    clocks = ClockSampler(dev.index)
+    clocks.start()
+    time.sleep(0.2)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(steps)]
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        for e in ev:
+            flush.zero_()
+            e[0].record(stream)
+            wf.wf_forecast_readiness(ctx, rel, comp, stream)
+            e[1].record(stream)
+            wf.wf_eval_plans(ctx, dp, res, stream)
+            e[2].record(stream)
+            wf.wf_topk(ctx, res, P, k, ids, keys, stream)
+            e[3].record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    wf.wf_ctx_status(ctx, stream)
+    step_ms = float(np.median([e[0].elapsed_time(e[3]) for e in ev]))
+    eval_ms = float(np.median([e[1].elapsed_time(e[2]) for e in ev]))
+    peak = read_peaks().get("hbm_gbs")
+    bpp = algorithmic_bytes_per_plan(prob.N)
+    entry = {"description": w.description, "P": P, "N": prob.N, "D": prob.D, "k": k,
+             "step_ms": step_ms, "eval_ms": eval_ms, "plans_per_s": P / (step_ms * 1e-3),
+             "roofline": {"bound": "alu" if prob.S else "hbm",
+                          "achieved_gbs": bpp * P / (eval_ms * 1e-3) / 1e9, "peak_gbs": peak,
+                          "frac_of_hbm": bpp * P / (eval_ms * 1e-3) / 1e9 / peak if peak else None,
+                          "algorithmic_bytes_per_plan": bpp},
+             "clocks": clk, "timing": f"median of {steps} steps after {warmup}, L2 flushed before each"}
+    if prob.S:
+        entry["samples"] = prob.S
+        entry["sims_per_s"] = P * prob.S / (step_ms * 1e-3)
+    if with_cpu:
+        import oracle
+        oracle.build()
+        n = min(P, OTHER_WORKLOADS[name])
+        t0 = time.perf_counter()
+        oracle.eval_plans(prob, plans, 0, n)
+        dt = time.perf_counter() - t0
+        entry["cpu_baseline"] = {"value": n / dt, "unit": "plans/s", "cores": 1, "kind": "oracle",
+                                 "sample": f"the first {n} plans of the {name} batch, one thread, {dt:.2f} s"}
+        if prob.S:
+            entry["cpu_baseline"]["sims_per_s"] = n * prob.S / dt
+    ctx.close()
+    del dp, res, plans
+    torch.cuda.empty_cache()
+    return entry
+
+
+def static_timing(wf, prob, plans, dev, flush, reps=5):
+    """wf_eval_plans_static (no context, no allocation) on the largest batch
+    of this window its static scratch holds: median of reps calls, L2 flushed
+    before each."""
+    import re
+
+    import torch
+    dprob = wf.DeviceProblem(prob, dev)
+    fit = plans.P
+    try:
+        wf.wf_eval_plans_static(dprob, wf.DevicePlans.from_host(plans, dev), wf.Results(plans.P, dev))
+        wf.wf_static_status()
+    except wf.WfError as e:
+        m = re.search(r"at most (\d+) plans", str(e))
+        if not m:
+            raise
+        fit = int(m.group(1))
+    sub = plans.slice(0, fit)
+    dp = wf.DevicePlans.from_host(sub, dev)
+    out = wf.Results(fit, dev)
+    ts = []
+    for _ in range(reps):
+        flush.zero_()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        wf.wf_eval_plans_static(dprob, dp, out)
+        b.record()
+        torch.cuda.synchronize()
+        ts.append(a.elapsed_time(b))
+    wf.wf_static_status()
+    ms = float(np.median(ts))
+    return {"plans": fit, "ms": ms, "plans_per_s": fit / (ms * 1e-3),
+            "timing": f"median of {reps} calls, L2 flushed before each",
+            "note": "the largest batch of this window the 32 MiB static scratch holds; a thread per plan"}
+
+
 def run_gpu(args, rank, world, local):
     import torch
 
@@ -489,6 +606,7 @@ def run_gpu(args, rank, world, local):
     search = local_search_timing(wf, ctx, dp, prob, P, stream, flush, peak_gbs=read_peaks().get("hbm_gbs"))
     built = construct_timing(wf, ctx, prob, P, k, stream, flush, random_best=int(keys[0, 0].item()))
     clk = clocks.stop()
+    static = static_timing(wf, prob, plans, dev, flush) if prob.S == 0 and world == 1 else None
     e2e_ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, world)
     # the host reads the top-k it copied back
     assert int(ids_h.numpy().min()) >= 0
@@ -546,7 +664,15 @@ def run_gpu(args, rank, world, local):
             "construct": built,
             "reclaim_next_use": nextuse,
             "eq12_window_terms": phi,
+            "static_entry": static,
         }
+        if world == 1 and not args.no_workloads and WORKLOAD == "burst":
+            # the other named windows, each at its full size (context, plans
+            # and L2 flush of their own)
+            del dp, res
+            torch.cuda.empty_cache()
+            line["workloads"] = {n: workload_entry(n, wf, dev, with_cpu=not args.no_cpu_baseline)
+                                 for n in OTHER_WORKLOADS}
         print(json.dumps(line), flush=True)
     ctx.close()
 
@@ -558,6 +684,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=("gpu", "reference"), default="gpu")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-workloads", action="store_true", help="skip the other named windows")
     ap.add_argument("--workload", default="burst", choices=("tiny", "mix", "burst", "stochastic", "large"),
                     help="the synthetic window (burst is the headline configuration)")
     ap.add_argument("--plans", type=int, default=0, help="plans per GPU (default: the workload's)")

@@ -24,6 +24,7 @@
  *   wf_topk_phi             the k best plans by Eq. 12's window key
  *   wf_ctx_status           device-side failures of earlier calls
  *   wf_ctx_check_wait_expiry  the bounded device wait's expiry path (tests)
+ *   wf_ctx_set_eval_path    every plan on the exact int64 path (tests, cross-checks)
  *   wf_ctx_destroy, wf_strerror, wf_last_error
  *
  * Conventions.
@@ -56,6 +57,12 @@ enum {
     WF_ENOMEM = 2,    /* device or host allocation failed */
     WF_ECUDA = 3,     /* a CUDA launch or runtime error (see wf_strerror) */
     WF_ETIMEOUT = 4   /* a bounded device-side wait expired; results are invalid */
+};
+
+/* Evaluation path (wf_ctx_set_eval_path). */
+enum {
+    WF_PATH_AUTO = 0,   /* the shared-memory sweeps, the exact int64 path for what they hand on (the default) */
+    WF_PATH_INT64 = 1   /* every plan on the exact int64 path (a thread per plan, state in global memory) */
 };
 
 /* Reclamation order (wf_ctx_set_reclaim). */
@@ -381,12 +388,22 @@ int wf_ctx_status(wf_ctx *ctx, void *stream);
 /*
  * Diagnostic: launches, on `stream`, one device-side bounded wait that
  * nothing completes (an mbarrier armed for bytes that no copy delivers, the
- * wait the bulk-copy kernels use).  It gives up after about a second and
+ * wait the bulk-copy kernels use).  It gives up after 2^20 polls of about
+ * 4 us each (about 4 s on a GB300) and
  * records the expiry, so the next wf_ctx_status returns WF_ETIMEOUT; the
  * context stays usable.  Returns WF_EINVAL for a NULL context, WF_ECUDA when
  * the launch fails.
  */
 int wf_ctx_check_wait_expiry(wf_ctx *ctx, void *stream);
+
+/*
+ * Which kernels later evaluation calls on this context use: WF_PATH_AUTO
+ * (default) or WF_PATH_INT64, every plan on the exact int64 path.  Both give
+ * the same results; the int64 path is slower and serves tests and
+ * cross-checks of the sweeps.  Not thread-safe with calls in flight on the
+ * context.  Returns WF_EINVAL for a NULL context or another value.
+ */
+int wf_ctx_set_eval_path(wf_ctx *ctx, int32_t path);
 
 /* Release every device and host allocation of the context (NULL is a no-op). */
 void wf_ctx_destroy(wf_ctx *ctx);

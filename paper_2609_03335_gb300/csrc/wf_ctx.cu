@@ -319,8 +319,7 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
     if (!c) return wf_set_error(WF_ENOMEM, "host allocation of the context");
     c->device = device;
     c->max_P = max_P;
-    const char *path = getenv("WF_EVAL_PATH");
-    c->force_int64 = path && strcmp(path, "int64") == 0;
+    c->force_int64 = false;
     c->tables_bytes = img.bytes.size();
     rc = wf_cuda_check(cudaMalloc(&c->tables, c->tables_bytes), "cudaMalloc(tables)");
     if (!rc) rc = wf_cuda_check(cudaMemcpy(c->tables, img.bytes.data(), c->tables_bytes,
@@ -565,5 +564,14 @@ extern "C" int wf_ctx_status(wf_ctx *c, void *stream)
         cudaMemcpy(c->err, &zero, sizeof(int), cudaMemcpyHostToDevice);
         return wf_set_error(WF_ETIMEOUT, "device error word %d", err);
     }
+    return WF_OK;
+}
+
+extern "C" int wf_ctx_set_eval_path(wf_ctx *c, int32_t path)
+{
+    REQUIRE(c, "NULL context");
+    REQUIRE(path == WF_PATH_AUTO || path == WF_PATH_INT64, "eval path %d is neither WF_PATH_AUTO nor WF_PATH_INT64",
+            path);
+    c->force_int64 = path == WF_PATH_INT64;
     return WF_OK;
 }

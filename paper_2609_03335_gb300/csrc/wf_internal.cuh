@@ -85,7 +85,7 @@ struct wf_ctx {
     size_t topk_scratch_bytes;
     int *err;
     int sms;                    // streaming multiprocessors of the device
-    bool force_int64;           // WF_EVAL_PATH=int64: always take the int64 path (tests)
+    bool force_int64;           // wf_ctx_set_eval_path(WF_PATH_INT64): every plan on the int64 path
     int32_t *ovf_count;         // [2]: plans the u32 sweep hands on, plans left for the int64 path
     int32_t *ovf_list;          // [max_P] the u32 sweep's hand-offs (and the stochastic sweep's)
     int32_t *ovf_list2;         // [max_P] plans for the int64 path

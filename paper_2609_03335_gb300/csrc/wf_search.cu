@@ -183,9 +183,9 @@ __device__ __forceinline__ void mbar_expect(uint64_t *bar, uint32_t bytes)
                  : "memory");
 }
 
-// Waits for bar's phase of the given parity: at most 2^20 polls, each
-// suspending the thread for up to about a microsecond, so about a second in
-// all before it gives up.
+// Waits for bar's phase of the given parity: at most 2^20 polls, each with a
+// suspend-time hint of 1 us; one poll takes about 4 us on a GB300, so the
+// wait gives up after about 4 s.
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity)
 {
     for (uint32_t it = 0; it < (1u << 20); ++it) {
@@ -240,8 +240,11 @@ __host__ __device__ inline int64_t staged_row_bytes(int64_t N, bool retain)
 // child's changes (lane t the t-th of each group of 32); lane 0 then applies
 // them on chip, in turn, and writes the rows to the child with bulk copies.
 // The slice is reloaded only after those stores have read it.  A bulk load
-// that has not landed after the bounded wait sets error word 3, and the warp
-// stops after a second bounded wait.
+// that has not landed after the bounded wait sets error word 3; the warp then
+// waits once more, with the same bound, for the copies it issued (an issued
+// bulk copy cannot be withdrawn, and an unbounded wait could hang the GPU),
+// stops taking children, and drains its own bulk stores before the CTA
+// exits.
 __global__ void __launch_bounds__(32 * kMutWarps, 4)
 mutate_staged_kernel(wf_dev_problem dp, wf_plans par, int64_t n_par, wf_plans ch, uint64_t seed, int64_t round,
                      int32_t n_ops)

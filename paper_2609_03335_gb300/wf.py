@@ -25,7 +25,7 @@ EXPORTS = ("wf_problem_check", "wf_ctx_create", "wf_forecast_readiness", "wf_eva
            "wf_topk", "wf_ctx_status", "wf_ctx_destroy", "wf_strerror", "wf_last_error",
            "wf_eval_plans_static", "wf_mutate_plans", "wf_merge_elite", "wf_local_search",
            "wf_construct_plans", "wf_ctx_set_reclaim", "wf_ctx_check_wait_expiry", "wf_eval_plans_phi",
-           "wf_topk_phi", "wf_static_status")
+           "wf_topk_phi", "wf_static_status", "wf_ctx_set_eval_path")
 
 
 class WfError(RuntimeError):
@@ -93,6 +93,7 @@ def load_library():
         "wf_last_error": ([], ctypes.c_char_p),
         "wf_eval_plans_static": ([p, p, p, p], ctypes.c_int),
         "wf_static_status": ([p], ctypes.c_int),
+        "wf_ctx_set_eval_path": ([p, i32], ctypes.c_int),
     }
     for name, (args, res) in sig.items():
         f = getattr(lib, name)
@@ -213,6 +214,14 @@ def wf_ctx_destroy(ctx: Ctx):
 
 def wf_ctx_status(ctx: Ctx, stream=None):
     _check(load_library().wf_ctx_status(ctx.ptr, _stream_handle(stream)), "wf_ctx_status")
+
+
+PATH_AUTO, PATH_INT64 = 0, 1
+
+
+def wf_ctx_set_eval_path(ctx: Ctx, path: int):
+    """PATH_AUTO (the sweeps) or PATH_INT64 (every plan on the exact int64 path)."""
+    _check(load_library().wf_ctx_set_eval_path(ctx.ptr, int(path)), "wf_ctx_set_eval_path")
 
 
 def wf_ctx_check_wait_expiry(ctx: Ctx, stream=None):

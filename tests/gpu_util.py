@@ -15,13 +15,16 @@ def lib():
     return wf
 
 
-def gpu_eval(prob, plans, k=None, ctx=None, forecast=False):
-    """Evaluate on cuda:0 through the C ABI; returns a dict of numpy arrays."""
+def gpu_eval(prob, plans, k=None, ctx=None, forecast=False, int64_path=False):
+    """Evaluate on cuda:0 through the C ABI; returns a dict of numpy arrays.
+    int64_path: every plan on the exact int64 path (wf_ctx_set_eval_path)."""
     import torch
     wf = lib()
     dev = torch.device("cuda", 0)
     own = ctx is None
     ctx = ctx or wf.Ctx(prob, max_P=plans.P, device=0)
+    if int64_path:
+        wf.wf_ctx_set_eval_path(ctx, wf.PATH_INT64)
     dp = wf.DevicePlans.from_host(plans, dev)
     res = wf.Results(plans.P, dev)
     wf.wf_eval_plans(ctx, dp, res)

@@ -176,7 +176,7 @@ def test_long_write_lists(F):
 
 def test_bounded_wait_expiry_is_reported():
     """A device-side wait that nothing completes gives up on its own (in
-    about a second), the host reads WF_ETIMEOUT from wf_ctx_status, and the
+    about 4 s), the host reads WF_ETIMEOUT from wf_ctx_status, and the
     context evaluates correctly afterwards."""
     import time
     import torch

@@ -165,13 +165,12 @@ def test_stochastic_sample_counts(S):
     assert np.array_equal(got["ids"], ids) and np.array_equal(got["keys"], keys)
 
 
-def test_stochastic_int64_path_matches_oracle(monkeypatch):
+def test_stochastic_int64_path_matches_oracle():
     """The per-sample int64 path on its own, forced for every plan."""
-    monkeypatch.setenv("WF_EVAL_PATH", "int64")
     w = wfgen.config("stochastic")
     plans = wfgen.make_plans(w.problem, 512, 91, p_retain=0.5)
     inject_invalid(plans, w.problem, np.random.default_rng(2))
-    got = gpu_eval(w.problem, plans, k=8)
+    got = gpu_eval(w.problem, plans, k=8, int64_path=True)
     assert_same(got, oracle_eval(w.problem, plans))
 
 
@@ -267,14 +266,13 @@ def test_long_chain_window():
 
 
 @pytest.mark.parametrize("name", ["mix", "burst"])
-def test_int64_path_matches_oracle(name, monkeypatch):
+def test_int64_path_matches_oracle(name):
     """The exact int64 path (taken for plans whose times overflow the
     shared-memory sweep's u32 slots) on its own, forced for every plan."""
-    monkeypatch.setenv("WF_EVAL_PATH", "int64")
     w = wfgen.config(name)
     plans = wfgen.make_plans(w.problem, 2048, 77, p_retain=0.5)
     inject_invalid(plans, w.problem, np.random.default_rng(1))
-    got = gpu_eval(w.problem, plans, k=8)
+    got = gpu_eval(w.problem, plans, k=8, int64_path=True)
     assert_same(got, oracle_eval(w.problem, plans))
 
 

@@ -12,12 +12,14 @@ from test_gpu_parity import inject_invalid
 pytestmark = pytest.mark.gpu
 
 
-def gpu_phi(prob, plans, k, reclaim=0):
+def gpu_phi(prob, plans, k, reclaim=0, int64_path=False):
     import torch
     wf = lib()
     ctx = wf.Ctx(prob, max_P=plans.P)
     if reclaim:
         wf.wf_ctx_set_reclaim(ctx, 1)
+    if int64_path:
+        wf.wf_ctx_set_eval_path(ctx, wf.PATH_INT64)
     dp = wf.DevicePlans.from_host(plans, "cuda")
     res = wf.Results(plans.P)
     timely = torch.empty(plans.P, dtype=torch.int64, device="cuda")
@@ -35,8 +37,8 @@ def gpu_phi(prob, plans, k, reclaim=0):
     return out
 
 
-def check(prob, plans, k, reclaim=0):
-    got = gpu_phi(prob, plans, k, reclaim)
+def check(prob, plans, k, reclaim=0, int64_path=False):
+    got = gpu_phi(prob, plans, k, reclaim, int64_path)
     p = prob.with_(reclaim=reclaim)
     mk, p95, gpu, st = oracle.eval_plans(p, plans, threads=THREADS)
     timely, life = oracle.eval_phi(p, plans, threads=THREADS)
@@ -72,12 +74,11 @@ def test_random_windows(seed, reclaim):
     check(prob, plans, k=int(rng.integers(1, min(P, 64) + 1)), reclaim=reclaim)
 
 
-def test_int64_path(monkeypatch):
-    monkeypatch.setenv("WF_EVAL_PATH", "int64")
+def test_int64_path():
     w = wfgen.config("mix")
     plans = wfgen.make_plans(w.problem, 1024, 5, p_retain=0.5)
     inject_invalid(plans, w.problem, np.random.default_rng(2))
-    check(w.problem, plans, k=16)
+    check(w.problem, plans, k=16, int64_path=True)
 
 
 def test_times_beyond_u32():
