@@ -53,13 +53,13 @@ class _Problem(ctypes.Structure):
                 ("grant", ctypes.c_int32), ("S", ctypes.c_int32), ("seed", ctypes.c_uint64),
                 ("bm_r", ctypes.c_void_p), ("bm_c", ctypes.c_void_p), ("bm_e", ctypes.c_void_p),
                 ("bm_rn", ctypes.c_int32), ("bm_cn", ctypes.c_int32), ("bm_en", ctypes.c_int32),
-                ("reclaim", ctypes.c_int32)]
+                ("reclaim", ctypes.c_int32), ("batch", ctypes.c_int32)]
 
 
 class _Trace(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in (
         "unit_head", "n_units", "head_of", "start", "finish", "rel", "load_start", "load_end",
-        "kv_adm", "used_after", "evicted", "reclaimed", "occ_start", "occ_end", "occ_dev", "n_occ")]
+        "kv_adm", "used_after", "evicted", "reclaimed", "occ_start", "occ_end", "occ_dev", "n_occ", "adm")]
 
 
 def _setup(lib):
@@ -127,7 +127,8 @@ class OracleProblem:
                           int(prob.grant_us), self.S, int(prob.seed) & ((1 << 64) - 1),
                           ar["bm_r"].ctypes.data, ar["bm_c"].ctypes.data, ar["bm_e"].ctypes.data,
                           int(np.asarray(prob.bm_r).size), int(np.asarray(prob.bm_c).size),
-                          int(np.asarray(prob.bm_e).size), int(getattr(prob, "reclaim", 0)))
+                          int(np.asarray(prob.bm_e).size), int(getattr(prob, "reclaim", 0)),
+                          int(getattr(prob, "batch", 0)))
         self.fnext = np.empty(self.N, np.int32)
         if self.lib.orc_fusible_next(ctypes.byref(self.c), self.fnext.ctypes.data) != 0:
             raise MemoryError("oracle allocation failed")
@@ -182,7 +183,8 @@ def eval_plan(prob, plans, p: int, trace: bool = False, op: OracleProblem | None
                    kv_adm=np.zeros(N, np.int32), used_after=np.zeros(N, np.int32),
                    evicted=np.zeros(N, np.uint32), reclaimed=np.zeros(N, np.uint8),
                    occ_start=np.zeros(N + D, np.int64), occ_end=np.zeros(N + D, np.int64),
-                   occ_dev=np.zeros(N + D, np.int32), n_occ=np.zeros(1, np.int32))
+                   occ_dev=np.zeros(N + D, np.int32), n_occ=np.zeros(1, np.int32),
+                   adm=np.full(N, -1, np.int64))
         tr = _Trace(*[tra[f].ctypes.data for f, _ in _Trace._fields_])
     rc = op.lib.orc_eval_plan(ctypes.byref(op.c), op.fnext.ctypes.data, pl.ctypes.data, od.ctypes.data,
                               fu.ctypes.data, pf.ctypes.data, None if rt is None else rt.ctypes.data,

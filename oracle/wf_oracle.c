@@ -31,7 +31,10 @@
  *     resident (Section 4.3);
  *   - beside them, the window terms of the ranking key of Eq. 12: timely
  *     prefetches and the lifecycle overhead (ready-work loading delay plus
- *     reloads after reclamation), see orc_eval_phi_batch.
+ *     reloads after reclamation), see orc_eval_phi_batch;
+ *   - with a replica batch limit B_q (Section 3.5, batch >= 1), units of a
+ *     device's current replica run up to B_q at once and Eq. 11 sums the KV
+ *     needs of every running unit, see simulate_batched.
  *
  * Every time is an int64 microsecond count and every memory an int32 MiB
  * count, so results are exact.  Points the paper leaves open are read as
@@ -73,6 +76,7 @@ typedef struct {
     const int32_t *bm_r, *bm_c, *bm_e;
     int32_t bm_rn, bm_cn, bm_en;
     int32_t reclaim;           /* 0: least recently used first; 1: by next use (see next_use_victim) */
+    int32_t batch;             /* replica batch limit B_q (simulate_batched); 0: one unit at a time per device */
 } orc_problem;
 
 /* Optional record of one deterministic run, for the invariant checker. */
@@ -93,6 +97,7 @@ typedef struct {
     int64_t *occ_end;
     int32_t *occ_dev;
     int32_t *n_occ;       /* [1] */
+    int64_t *adm;         /* [N] per head: admission time (the load start on a miss); NULL: not kept */
 } orc_trace;
 
 static int64_t imax64(int64_t a, int64_t b) { return a > b ? a : b; }
@@ -460,6 +465,224 @@ out:
     return rc;
 }
 
+/*
+ * The same play with the replica batch limit B_q of Section 3.5 (B = batch
+ * >= 1).  Eq. 11 sums the request memory of every unit active at a
+ * transition boundary, and concurrent units of one replica respect its batch
+ * limit.  A replica is a model resident on a device; a device runs units of
+ * one replica at a time, up to B of them at once:
+ *   - units are admitted in the plan's dispatch order;
+ *   - a unit of the device's current replica joins it: it takes the slot
+ *     (of B) that frees earliest, no earlier than its release and than the
+ *     previous admission on the device, and is admitted once resident
+ *     weights + the KV needs of the units still running + its own KV fit the
+ *     capacity (least-recently-used idle models are reclaimed first; if that
+ *     is not enough, it waits for the next running unit to end);
+ *   - a unit of another model waits until the device has drained (every
+ *     running unit ended) and then hits or loads exactly as in simulate,
+ *     with the device free at the drain time; it becomes the current
+ *     replica, and its other slots free when the model is ready;
+ *   - a unit's KV is held from its admission (the load start on a miss) to
+ *     its end.
+ * With admissions in dispatch order, memory use over a unit's interval peaks
+ * at its admission, so one check there covers Eq. 11 for it.  With B = 1 the
+ * play equals simulate's.  Retain rows are modelled for B = 1 only; the
+ * window terms of Eq. 12 and reclamation by next use are not modelled here.
+ */
+static int simulate_batched(const orc_problem *pb, const int32_t *fnext,
+                            const uint8_t *place, const uint16_t *order,
+                            const uint32_t *fuse, const uint32_t *prefetch, const uint32_t *retain,
+                            const int64_t *L, int64_t *c, int64_t *comp_w,
+                            int64_t *makespan, int64_t *gpu_total, orc_trace *tr)
+{
+    const int32_t N = pb->N, D = pb->D, M = pb->M, W = pb->W, B = pb->batch;
+    if (B < 1 || (B > 1 && retain) || pb->reclaim) return -3;
+    int64_t *slot_end = (int64_t *)malloc(sizeof(int64_t) * (size_t)D * (size_t)B);
+    int64_t *slot_kv = (int64_t *)malloc(sizeof(int64_t) * (size_t)D * (size_t)B);
+    int64_t *last_adm = (int64_t *)malloc(sizeof(int64_t) * (size_t)D);
+    int32_t *cur = (int32_t *)malloc(sizeof(int32_t) * (size_t)D);
+    int64_t *occ_since = (int64_t *)malloc(sizeof(int64_t) * (size_t)D);
+    int64_t *gpu = (int64_t *)malloc(sizeof(int64_t) * (size_t)D);
+    int64_t *used = (int64_t *)malloc(sizeof(int64_t) * (size_t)D);
+    int32_t *nres = (int32_t *)malloc(sizeof(int32_t) * (size_t)D);
+    int64_t *stamp = (int64_t *)malloc(sizeof(int64_t) * (size_t)D * (size_t)M);
+    uint8_t *done = (uint8_t *)malloc((size_t)N);
+    int32_t *chain = (int32_t *)malloc(sizeof(int32_t) * (size_t)N);
+    int rc = 0;
+    if (!slot_end || !slot_kv || !last_adm || !cur || !occ_since || !gpu || !used || !nres || !stamp || !done ||
+        !chain) {
+        rc = -1;
+        goto out;
+    }
+    for (int32_t d = 0; d < D; ++d) {
+        for (int32_t j = 0; j < B; ++j) { slot_end[(int64_t)d * B + j] = 0; slot_kv[(int64_t)d * B + j] = 0; }
+        last_adm[d] = 0; cur[d] = -1; occ_since[d] = ORC_NONE; gpu[d] = 0; used[d] = 0; nres[d] = 0;
+        for (int32_t m = 0; m < M; ++m) stamp[(int64_t)d * M + m] = 0;  /* 0 = not resident */
+    }
+    memset(done, 0, (size_t)N);
+    int64_t seq = 0;
+    if (tr) { *tr->n_units = 0; *tr->n_occ = 0; }
+
+    for (int32_t i = 0; i < N; ++i) {
+        const int32_t h = order[i];
+        if (done[h]) continue;  /* already ran inside an earlier chain */
+        int32_t len = 0;
+        chain[len++] = h;
+        for (;;) {
+            int32_t s = fnext[chain[len - 1]];
+            if (s < 0 || !bit_of(fuse, s) || place[s] != place[h]) break;
+            chain[len++] = s;
+        }
+        const int32_t last = chain[len - 1];
+        const int32_t d = place[h];
+        const int32_t m = pb->model[h];
+        const int32_t w = pb->session[h];
+        int64_t *st = &stamp[(int64_t)d * M];
+        int64_t *se = &slot_end[(int64_t)d * B];
+        int64_t *sk = &slot_kv[(int64_t)d * B];
+        int64_t rel = pb->arrival[w];
+        for (int32_t e = pb->pred_off[h]; e < pb->pred_off[h + 1]; ++e)
+            rel = imax64(rel, c[pb->pred_idx[e]]);
+        int64_t kv_adm = 0;
+        for (int32_t j = 0; j < len; ++j)
+            kv_adm = imax64(kv_adm, (int64_t)pb->peak[(int64_t)chain[j] * D + d] - pb->weight[m]);
+
+        int64_t adm, start, ls = -1, le = -1;
+        int32_t slot = 0;
+        uint32_t evicted = 0;
+        if (m == cur[d]) {
+            /* Join the current replica: the earliest-free slot (lowest index
+             * on ties), in dispatch order, once memory allows (Eq. 11). */
+            for (int32_t j = 1; j < B; ++j)
+                if (se[j] < se[slot]) slot = j;
+            adm = imax64(imax64(rel, se[slot]), last_adm[d]);
+            for (;;) {
+                int64_t running = 0;
+                for (int32_t j = 0; j < B; ++j)
+                    if (se[j] > adm) running += sk[j];
+                while (used[d] + running + kv_adm > pb->cap[d]) {
+                    int32_t victim = -1;
+                    for (int32_t k = 0; k < M; ++k)
+                        if (k != m && st[k] != 0 && (victim < 0 || st[k] < st[victim])) victim = k;
+                    if (victim < 0) break;
+                    used[d] -= pb->weight[victim];
+                    st[victim] = 0;
+                    nres[d] -= 1;
+                    evicted |= 1u << victim;
+                }
+                if (used[d] + running + kv_adm <= pb->cap[d]) break;
+                /* not even without idle models: wait for the next running unit to end */
+                int64_t next = ORC_INF;
+                for (int32_t j = 0; j < B; ++j)
+                    if (se[j] > adm) next = imin64(next, se[j]);
+                if (next == ORC_INF) { rc = -2; goto out; }  /* unreachable for a valid plan */
+                adm = next;
+            }
+            start = adm;
+        } else {
+            /* Another model: the device drains, then the unit hits or loads as
+             * in simulate with the device free at the drain time. */
+            int64_t drain = 0;
+            for (int32_t j = 0; j < B; ++j) drain = imax64(drain, se[j]);
+            const int hit = st[m] != 0;
+            const int64_t need = hit ? kv_adm : pb->weight[m] + kv_adm;
+            while (used[d] + need > pb->cap[d]) {
+                int32_t victim = -1;
+                for (int32_t k = 0; k < M; ++k)
+                    if (k != m && st[k] != 0 && (victim < 0 || st[k] < st[victim])) victim = k;
+                if (victim < 0) { rc = -2; goto out; }
+                used[d] -= pb->weight[victim];
+                st[victim] = 0;
+                nres[d] -= 1;
+                evicted |= 1u << victim;
+            }
+            int64_t ready;
+            if (hit) {
+                adm = start = imax64(drain, rel);
+                ready = drain;
+            } else {
+                ls = bit_of(prefetch, h) ? imax64(drain, pb->arrival[w]) : imax64(drain, rel);
+                if (occ_since[d] == ORC_NONE) occ_since[d] = ls;
+                le = ls + pb->load[(int64_t)m * D + d];
+                used[d] += pb->weight[m];
+                nres[d] += 1;
+                adm = ls;
+                start = imax64(le, rel);
+                ready = le;
+            }
+            for (int32_t j = 0; j < B; ++j) { se[j] = ready; sk[j] = 0; }
+            cur[d] = m;
+        }
+        start += pb->grant;
+        int64_t t = start;
+        for (int32_t j = 0; j < len; ++j) {
+            int32_t n = chain[j];
+            if (tr) { tr->start[n] = t; tr->head_of[n] = h; tr->rel[n] = (j == 0) ? rel : -1; }
+            t += L[(int64_t)n * D + d];
+            c[n] = t;
+            done[n] = 1;
+        }
+        se[slot] = c[last];
+        sk[slot] = kv_adm;
+        last_adm[d] = adm;
+        st[m] = ++seq;
+        if (tr) {
+            tr->unit_head[(*tr->n_units)++] = h;
+            tr->load_start[h] = ls;
+            tr->load_end[h] = le;
+            tr->kv_adm[h] = (int32_t)kv_adm;
+            tr->used_after[h] = (int32_t)used[d];
+            tr->evicted[h] = evicted;
+            tr->reclaimed[h] = 0;
+            if (tr->adm) tr->adm[h] = adm;
+        }
+        /* Retain bit 0 (B = 1 only): the model leaves when the unit ends, and
+         * the device has no current replica. */
+        if (retain && !bit_of(retain, last)) {
+            used[d] -= pb->weight[m];
+            st[m] = 0;
+            nres[d] -= 1;
+            cur[d] = -1;
+            if (tr) tr->reclaimed[h] = 1;
+            if (nres[d] == 0) {
+                gpu[d] += c[last] - occ_since[d];
+                if (tr) {
+                    int32_t k = (*tr->n_occ)++;
+                    tr->occ_start[k] = occ_since[d]; tr->occ_end[k] = c[last]; tr->occ_dev[k] = d;
+                }
+                occ_since[d] = ORC_NONE;
+            }
+        }
+    }
+
+    int64_t end = 0, first = ORC_INF;
+    for (int32_t n = 0; n < N; ++n) end = imax64(end, c[n]);
+    for (int32_t w = 0; w < W; ++w) first = imin64(first, pb->arrival[w]);
+    *makespan = end - first;
+    int64_t g = 0;
+    for (int32_t d = 0; d < D; ++d) {
+        if (occ_since[d] != ORC_NONE) {
+            gpu[d] += end - occ_since[d];
+            if (tr) {
+                int32_t k = (*tr->n_occ)++;
+                tr->occ_start[k] = occ_since[d]; tr->occ_end[k] = end; tr->occ_dev[k] = d;
+            }
+        }
+        g += gpu[d];
+    }
+    *gpu_total = g;
+    for (int32_t w = 0; w < W; ++w) comp_w[w] = ORC_NONE;
+    for (int32_t n = 0; n < N; ++n) {
+        int32_t w = pb->session[n];
+        comp_w[w] = imax64(comp_w[w], c[n] - pb->arrival[w]);
+    }
+    if (tr) for (int32_t n = 0; n < N; ++n) tr->finish[n] = c[n];
+out:
+    free(slot_end); free(slot_kv); free(last_adm); free(cur); free(occ_since); free(gpu); free(used); free(nres);
+    free(stamp); free(done); free(chain);
+    return rc;
+}
+
 /* SplitMix64 (Steele, Lea and Flood, OOPSLA 2014): advance by the golden
  * gamma, then the variant-13 finaliser.  mix(x) is one output for state x. */
 uint64_t orc_splitmix64(uint64_t x)
@@ -523,8 +746,11 @@ int orc_eval_plan(const orc_problem *pb, const int32_t *fnext,
                 }
             }
         int64_t mk, g;
-        rc = simulate(pb, fnext, place, order, fuse, prefetch, retain, L, c,
-                      &pool[(int64_t)s * W], &mk, &g, pb->S > 0 ? NULL : tr, NULL);
+        rc = pb->batch > 0
+                 ? simulate_batched(pb, fnext, place, order, fuse, prefetch, retain, L, c, &pool[(int64_t)s * W],
+                                    &mk, &g, pb->S > 0 ? NULL : tr)
+                 : simulate(pb, fnext, place, order, fuse, prefetch, retain, L, c,
+                            &pool[(int64_t)s * W], &mk, &g, pb->S > 0 ? NULL : tr, NULL);
         if (rc) goto out;
         sum_mk += mk;
         sum_gpu += g;
@@ -581,7 +807,7 @@ int orc_eval_phi_batch(const orc_problem *pb, const int32_t *fnext,
                        const uint32_t *fuse, const uint32_t *prefetch, const uint32_t *retain,
                        int64_t bits_stride, int64_t lo, int64_t hi, int64_t *timely, int64_t *life)
 {
-    if (pb->S > 0) return -3;
+    if (pb->S > 0 || pb->batch > 0) return -3;  /* deterministic, one unit at a time per device */
     const int32_t N = pb->N, D = pb->D, W = pb->W;
     int64_t *L = (int64_t *)malloc(sizeof(int64_t) * (size_t)N * (size_t)D);
     int64_t *c = (int64_t *)malloc(sizeof(int64_t) * (size_t)N);

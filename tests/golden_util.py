@@ -27,11 +27,17 @@ def problem_of(fx, case=None):
     lat = np.array([n["lat"] for n in nodes], np.int32)
     peak = np.array([n["peak"] for n in nodes], np.int32)
     grant = pb["grant"]
+    cap = pb["cap"]
+    batch = pb.get("batch", 0)
     if case is not None:
         if "patch_peak" in case:
             peak = np.array(case["patch_peak"], np.int32)
         if "patch_grant" in case:
             grant = case["patch_grant"]
+        if "patch_cap" in case:
+            cap = case["patch_cap"]
+        if "patch_batch" in case:
+            batch = case["patch_batch"]
     return wfgen.Problem(
         N=N, D=D, M=pb["M"], W=pb["W"], pred_off=off,
         pred_idx=np.array([u for n in nodes for u in n["preds"]], np.int32),
@@ -41,7 +47,7 @@ def problem_of(fx, case=None):
         lat_us=lat.reshape(-1), peak_mib=peak.reshape(-1),
         weight_mib=np.array(pb["weight"], np.int32),
         load_us=np.array(pb["load"], np.int32).reshape(-1),
-        cap_mib=np.array(pb["cap"], np.int32), grant_us=grant, name=fx["name"])
+        cap_mib=np.array(cap, np.int32), grant_us=grant, name=fx["name"], batch=batch)
 
 
 def set_bits(row, nodes):

@@ -46,6 +46,13 @@ MUTANTS = {
     "hash_nests_sample_first": ("orc_splitmix64(orc_splitmix64(orc_splitmix64(pb->seed ^ plan) ^ sample) ^ node)",
                                 "orc_splitmix64(orc_splitmix64(orc_splitmix64(pb->seed ^ sample) ^ plan) ^ node)"),
     "radius_from_bits_12": ("(int64_t)(h & (uint64_t)(pb->bm_rn - 1))", "(int64_t)((h >> 12) & (uint64_t)(pb->bm_rn - 1))"),
+    "batch_admits_out_of_order": ("adm = imax64(imax64(rel, se[slot]), last_adm[d]);", "adm = imax64(rel, se[slot]);"),
+    "batch_ignores_running_kv": ("if (se[j] > adm) running += sk[j];", "if (0) running += sk[j];"),
+    "batch_latest_slot": ("if (se[j] < se[slot]) slot = j;", "if (se[j] > se[slot]) slot = j;"),
+    "batch_switch_without_drain": ("for (int32_t j = 0; j < B; ++j) drain = imax64(drain, se[j]);",
+                                   "for (int32_t j = 0; j < B; ++j) drain = imin64(drain, se[j]);"),
+    "batch_other_slots_free_before_load": ("for (int32_t j = 0; j < B; ++j) { se[j] = ready; sk[j] = 0; }",
+                                           "for (int32_t j = 0; j < B; ++j) { se[j] = drain; sk[j] = 0; }"),
     "mean_rounds_up": ("out3[0] = sum_mk / S;", "out3[0] = (sum_mk + S - 1) / S;"),
     "device_free_at_head_end": ("t_free[d] = c[last];", "t_free[d] = c[h];"),
     "hash_ignores_plan": ("orc_splitmix64(pb->seed ^ plan)", "orc_splitmix64(pb->seed)"),
@@ -69,16 +76,24 @@ MUTANTS = {
 
 PIN_FILES = ["tests/test_oracle_golden.py", "tests/test_oracle_properties.py",
              "tests/test_oracle_stochastic.py", "tests/test_oracle_search.py", "tests/test_oracle_construct.py",
-             "tests/test_oracle_reclaim.py"]
+             "tests/test_oracle_reclaim.py", "tests/test_oracle_batch.py"]
 
 
 def _run_mutant(name, tmp):
+    """A site that simulate_batched repeats (the same step of the play) is
+    mutated at its first occurrence, which lies in simulate; the batched copy
+    is pinned against simulate by the B_q = 1 test.  Every other site is
+    unique."""
     old, new = MUTANTS[name]
     src = open(SRC).read()
-    assert src.count(old) == 1, f"mutation site for {name} not unique / not found"
+    n = src.count(old)
+    assert n >= 1, f"mutation site for {name} not found"
+    if n > 1:
+        assert src.index(old) < src.index("static int simulate_batched("), f"site for {name} not in simulate"
+        assert n == 1 + src[src.index("static int simulate_batched("):].count(old), f"site for {name} not unique"
     path = os.path.join(tmp, f"{name}.c")
     with open(path, "w") as f:
-        f.write(src.replace(old, new))
+        f.write(src.replace(old, new, 1))
     lib = os.path.join(tmp, f"lib{name}.so")
     subprocess.check_call(["gcc", "-O1", "-std=c11", "-fPIC", "-shared", "-o", lib, path])
     env = dict(os.environ, WF_ORACLE_LIB=lib)

@@ -101,6 +101,7 @@ class Problem:
     name: str = ""
     reclaim: int = 0          # reclamation order: 0 least recently used, 1 by next use
     margin_mib: int = 0       # admission margin: capacity checks use peak + margin
+    batch: int = 0            # replica batch limit B_q (0: one unit at a time per device)
 
     @property
     def E(self) -> int:
