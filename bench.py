@@ -447,6 +447,34 @@ def workload_entry(name, wf, dev, steps=5, warmup=3, with_cpu=True):
     return entry
 
 
+def batch_timing(wf, prob, dp, P, dev, flush, limits=(1, 2, 4), reps=3):
+    """The batch under the replica batch limit B_q (wf_ctx_set_batch, the
+    int64 path): eval time (median of reps, L2 flushed before each) and the
+    mean makespan and GPU time of the valid plans per limit."""
+    import torch
+    ctx = wf.Ctx(prob, max_P=P, device=dev.index)
+    res = wf.Results(P, dev)
+    out = {}
+    for B in limits:
+        wf.wf_ctx_set_batch(ctx, B)
+        ts = []
+        for _ in range(reps):
+            flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            wf.wf_eval_plans(ctx, dp, res)
+            b.record()
+            torch.cuda.synchronize()
+            ts.append(a.elapsed_time(b))
+        wf.wf_ctx_status(ctx)
+        mk, _, gpu, st = res.numpy()
+        ok = st == 0
+        out[str(B)] = {"eval_ms": float(np.median(ts)), "plans_per_s": P / (float(np.median(ts)) * 1e-3),
+                       "mean_makespan_us": float(mk[ok].mean()), "mean_gpu_us": float(gpu[ok].mean())}
+    ctx.close()
+    return out
+
+
 def static_timing(wf, prob, plans, dev, flush, reps=5):
     """wf_eval_plans_static (no context, no allocation) on the largest batch
     of this window its static scratch holds: median of reps calls, L2 flushed
@@ -607,6 +635,7 @@ def run_gpu(args, rank, world, local):
     built = construct_timing(wf, ctx, prob, P, k, stream, flush, random_best=int(keys[0, 0].item()))
     clk = clocks.stop()
     static = static_timing(wf, prob, plans, dev, flush) if prob.S == 0 and world == 1 else None
+    batched = batch_timing(wf, prob, dp, P, dev, flush) if prob.S == 0 and world == 1 else None
     e2e_ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, world)
     # the host reads the top-k it copied back
     assert int(ids_h.numpy().min()) >= 0
@@ -665,6 +694,7 @@ def run_gpu(args, rank, world, local):
             "reclaim_next_use": nextuse,
             "eq12_window_terms": phi,
             "static_entry": static,
+            "replica_batch": batched,
         }
         if world == 1 and not args.no_workloads and WORKLOAD == "burst":
             # the other named windows, each at its full size (context, plans

@@ -25,6 +25,7 @@
  *   wf_ctx_status           device-side failures of earlier calls
  *   wf_ctx_check_wait_expiry  the bounded device wait's expiry path (tests)
  *   wf_ctx_set_eval_path    every plan on the exact int64 path (tests, cross-checks)
+ *   wf_ctx_set_batch        replica batch limit B_q (Eq. 11, Section 3.5)
  *   wf_ctx_destroy, wf_strerror, wf_last_error
  *
  * Conventions.
@@ -404,6 +405,27 @@ int wf_ctx_check_wait_expiry(wf_ctx *ctx, void *stream);
  * context.  Returns WF_EINVAL for a NULL context or another value.
  */
 int wf_ctx_set_eval_path(wf_ctx *ctx, int32_t path);
+
+/*
+ * Replica batch limit B_q (Eq. 11 and the batch limit stated with it,
+ * Section 3.5) for later evaluation calls on this context; 0 (the default)
+ * keeps one unit at a time per device.  With B_q >= 1 a device runs units of
+ * one replica (a model resident on it) at a time, up to B_q of them at once:
+ * units are admitted in dispatch order; a unit of the device's current
+ * replica takes the slot that frees earliest, no earlier than its release
+ * and the device's latest admission, once resident weights + the KV needs
+ * of the units still running + its own KV fit the capacity (idle models are
+ * reclaimed least recently used first; if that is not enough the unit waits
+ * for the next running unit to end); a unit of another model waits for the
+ * device to drain, then hits or loads as without the limit.  B_q = 1 gives
+ * the same results as 0.  Deterministic problems with least-recently-used
+ * reclamation only; evaluation calls then take the exact int64 path (a
+ * thread per plan) and reject retain rows when B_q > 1 and the window terms
+ * of Eq. 12 (WF_EINVAL).  The first increase may reallocate the evaluation
+ * scratch; not thread-safe with calls in flight on the context.  Returns
+ * WF_EINVAL for a value outside 0..64 or such a problem.
+ */
+int wf_ctx_set_batch(wf_ctx *ctx, int32_t batch);
 
 /* Release every device and host allocation of the context (NULL is a no-op). */
 void wf_ctx_destroy(wf_ctx *ctx);

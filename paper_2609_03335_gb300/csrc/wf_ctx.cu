@@ -531,6 +531,7 @@ extern "C" int wf_ctx_set_reclaim(wf_ctx *c, int32_t policy)
         return WF_OK;
     }
     REQUIRE(c->dp.S == 0, "reclamation by next use needs deterministic latencies (S = 0)");
+    REQUIRE(c->dp.batch == 0, "reclamation by next use is not modelled with a replica batch limit");
     REQUIRE(c->dp.max_chain_run < (int64_t)UINT32_MAX,
             "a fusible chain may run %lld us, beyond the shared-memory sweep", (long long)c->dp.max_chain_run);
     wf_dev_problem probe = c->dp;
@@ -573,5 +574,36 @@ extern "C" int wf_ctx_set_eval_path(wf_ctx *c, int32_t path)
     REQUIRE(path == WF_PATH_AUTO || path == WF_PATH_INT64, "eval path %d is neither WF_PATH_AUTO nor WF_PATH_INT64",
             path);
     c->force_int64 = path == WF_PATH_INT64;
+    return WF_OK;
+}
+
+extern "C" int wf_ctx_set_batch(wf_ctx *c, int32_t batch)
+{
+    REQUIRE(c, "NULL context");
+    REQUIRE(batch >= 0 && batch <= 64, "replica batch limit %d outside 0..64", batch);
+    if (batch > 0) {
+        REQUIRE(c->dp.S == 0, "the replica batch limit needs deterministic latencies (S = 0)");
+        REQUIRE(c->dp.reclaim == 0, "the replica batch limit is modelled with least-recently-used reclamation");
+    }
+    wf_dev_problem probe = c->dp;
+    probe.batch = batch;
+    const size_t row = wf_eval_row_bytes(probe);
+    if (row > c->eval_row_bytes) {  // a longer state row: the evaluation scratch is rebuilt
+        int rc = select_device(c);
+        if (rc) return rc;
+        int64_t threads = 0;
+        const size_t bytes = wf_eval_scratch_bytes(probe, c->max_P, &threads);
+        void *fresh = nullptr;
+        rc = wf_cuda_check(cudaMalloc(&fresh, bytes), "cudaMalloc(eval scratch)");
+        if (rc) return rc;
+        rc = wf_cuda_check(cudaDeviceSynchronize(), "cudaDeviceSynchronize");
+        if (rc) { cudaFree(fresh); return rc; }
+        cudaFree(c->eval_scratch);
+        c->eval_scratch = fresh;
+        c->eval_scratch_bytes = bytes;
+        c->eval_threads = threads;
+        c->eval_row_bytes = row;
+    }
+    c->dp.batch = batch;
     return WF_OK;
 }

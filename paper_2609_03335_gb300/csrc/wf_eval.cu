@@ -55,6 +55,11 @@ struct Row {
     int32_t *nres;    // [D] resident model count
     int32_t *stamp;   // [D][M] last dispatch position + 1 using the model, 0 = not resident
     int32_t *loaded;  // [D] bit m: model m was ever resident on the device (Eq. 12 window terms)
+    // With a replica batch limit B = dp.batch (only then laid out):
+    int64_t *slot_end;  // [D][B] when each slot of the device's current replica frees
+    int64_t *slot_kv;   // [D][B] KV need of the unit in each slot
+    int64_t *last_adm;  // [D] the device's latest admission
+    int32_t *cur;       // [D] model of the device's current replica, -1 for none
 };
 
 __device__ __forceinline__ size_t up8(size_t x) { return (x + 7) & ~(size_t)7; }
@@ -71,7 +76,16 @@ __device__ __forceinline__ Row row_at(const wf_dev_problem &dp, uint8_t *base)
     r.used = (int32_t *)(base + o); o += up8(4 * (size_t)dp.D);
     r.nres = (int32_t *)(base + o); o += up8(4 * (size_t)dp.D);
     r.stamp = (int32_t *)(base + o); o += up8(4 * (size_t)dp.D * dp.M);
-    r.loaded = (int32_t *)(base + o);
+    r.loaded = (int32_t *)(base + o); o += up8(4 * (size_t)dp.D);
+    if (dp.batch > 0) {
+        r.slot_end = (int64_t *)(base + o); o += 8 * (size_t)dp.D * dp.batch;
+        r.slot_kv = (int64_t *)(base + o); o += 8 * (size_t)dp.D * dp.batch;
+        r.last_adm = (int64_t *)(base + o); o += 8 * (size_t)dp.D;
+        r.cur = (int32_t *)(base + o);
+    } else {
+        r.slot_end = r.slot_kv = r.last_adm = nullptr;
+        r.cur = nullptr;
+    }
     return r;
 }
 
@@ -229,6 +243,141 @@ __device__ void play(const wf_dev_problem &dp, const PlanRows &pr, Row &row, uin
     if (phi) { phi[0] = timely; phi[1] = life; }
 }
 
+// One play with the replica batch limit B_q (Eq. 11 over every active unit,
+// Section 3.5): a device runs units of one replica (a resident model) at a
+// time, up to B = dp.batch of them at once.  Units are admitted in dispatch
+// order.  A unit of the device's current replica takes the slot that frees
+// earliest, no earlier than its release and the device's latest admission,
+// once resident weights + the KV of the units still running + its own KV
+// fit (idle least-recently-used models are reclaimed first; if that is not
+// enough the unit waits for the next running unit to end).  A unit of
+// another model waits for the device to drain and then hits or loads as in
+// play<false>; its other slots free when the model is ready.  B = 1 gives
+// play<false>'s results.  Deterministic times; retain rows only with B = 1.
+__device__ void play_batched(const wf_dev_problem &dp, const PlanRows &pr, Row &row, int64_t *makespan,
+                             int64_t *gpu_total)
+{
+    const int32_t N = dp.N, D = dp.D, M = dp.M, W = dp.W, B = dp.batch;
+    for (int32_t d = 0; d < D; ++d) {
+        row.occ[d] = kNone; row.gpu[d] = 0; row.used[d] = 0; row.nres[d] = 0;
+        row.last_adm[d] = 0; row.cur[d] = -1;
+        for (int32_t j = 0; j < B; ++j) { row.slot_end[d * B + j] = 0; row.slot_kv[d * B + j] = 0; }
+    }
+    for (int32_t k = 0; k < D * M; ++k) row.stamp[k] = 0;
+    for (int32_t w = 0; w < W; ++w) row.comp[w] = kNone;
+    int64_t end = 0;
+
+    for (int32_t i = 0; i < N; ++i) {
+        const int32_t h = pr.order[i];
+        const int32_t d = pr.place[h];
+        const int32_t fp = dp.fprev[h];
+        if (fp >= 0 && bit_at(pr.fuse, h) && pr.place[fp] == d) continue;  // inside its head's unit
+        const int32_t m = dp.model[h];
+        const int32_t w = dp.session[h];
+        const int64_t arr = dp.arrival[w];
+        int64_t rel = arr;
+        for (int32_t e = dp.pred_off[h]; e < dp.pred_off[h + 1]; ++e)
+            rel = max(rel, row.ctail[dp.pred_idx[e]]);
+        const int32_t wm = dp.weight[m];
+        int32_t tail = h;
+        int64_t kv = dp.peak[(int64_t)h * D + d] - wm;
+        int64_t run = dp.lat[(int64_t)h * D + d];
+        for (int32_t s = dp.fnext[h]; s >= 0 && bit_at(pr.fuse, s) && pr.place[s] == d; s = dp.fnext[s]) {
+            kv = max(kv, (int64_t)dp.peak[(int64_t)s * D + d] - wm);
+            run += dp.lat[(int64_t)s * D + d];
+            tail = s;
+        }
+        int32_t *st = row.stamp + d * M;
+        int64_t *se = row.slot_end + d * B, *sk = row.slot_kv + d * B;
+        const int64_t cap = dp.cap[d];
+        int64_t adm, start;
+        int32_t slot = 0;
+        if (m == row.cur[d]) {
+            // Join the current replica (Eq. 11 with the running units' KV).
+            for (int32_t j = 1; j < B; ++j)
+                if (se[j] < se[slot]) slot = j;
+            adm = max(max(rel, se[slot]), row.last_adm[d]);
+            for (;;) {
+                int64_t running = 0;
+                for (int32_t j = 0; j < B; ++j) running += se[j] > adm ? sk[j] : 0;
+                while (row.used[d] + running + kv > cap) {  // idle models, least recently used first
+                    int32_t victim = -1, vs = INT32_MAX;
+                    for (int32_t k = 0; k < M; ++k)
+                        if (k != m && st[k] != 0 && st[k] < vs) { vs = st[k]; victim = k; }
+                    if (victim < 0) break;
+                    row.used[d] -= dp.weight[victim];
+                    row.nres[d] -= 1;
+                    st[victim] = 0;
+                }
+                if (row.used[d] + running + kv <= cap) break;
+                int64_t next = kNone;  // the next running unit to end
+                for (int32_t j = 0; j < B; ++j)
+                    if (se[j] > adm && (next == kNone || se[j] < next)) next = se[j];
+                if (next == kNone) { atomicExch(dp.err, 2); break; }  // unreachable for a valid plan
+                adm = next;
+            }
+            start = adm;
+        } else {
+            // Another model: the device drains, then the unit hits or loads.
+            int64_t drain = 0;
+            for (int32_t j = 0; j < B; ++j) drain = max(drain, se[j]);
+            const bool hit = st[m] != 0;
+            const int64_t need = hit ? kv : wm + kv;
+            while (row.used[d] + need > cap) {
+                int32_t victim = -1, vs = INT32_MAX;
+                for (int32_t k = 0; k < M; ++k)
+                    if (k != m && st[k] != 0 && st[k] < vs) { vs = st[k]; victim = k; }
+                if (victim < 0) { atomicExch(dp.err, 2); break; }  // unreachable for a valid plan
+                row.used[d] -= dp.weight[victim];
+                row.nres[d] -= 1;
+                st[victim] = 0;
+            }
+            int64_t ready;
+            if (hit) {
+                adm = start = max(drain, rel);
+                ready = drain;
+            } else {
+                const int64_t ls = max(drain, bit_at(pr.prefetch, h) ? arr : rel);
+                if (row.occ[d] == kNone) row.occ[d] = ls;
+                row.used[d] += wm;
+                row.nres[d] += 1;
+                const int64_t le = ls + dp.load[m * D + d];
+                adm = ls;
+                start = max(le, rel);
+                ready = le;
+            }
+            for (int32_t j = 0; j < B; ++j) { se[j] = ready; sk[j] = 0; }
+            row.cur[d] = m;
+        }
+        const int64_t c = start + dp.grant + run;
+        row.ctail[tail] = c;
+        se[slot] = c;
+        sk[slot] = kv;
+        row.last_adm[d] = adm;
+        st[m] = i + 1;
+        end = max(end, c);
+        row.comp[w] = max(row.comp[w], c);
+        if (pr.retain && !bit_at(pr.retain, tail)) {  // B = 1 only
+            row.used[d] -= wm;
+            row.nres[d] -= 1;
+            st[m] = 0;
+            row.cur[d] = -1;
+            if (row.nres[d] == 0) {
+                row.gpu[d] += c - row.occ[d];
+                row.occ[d] = kNone;
+            }
+        }
+    }
+    int64_t g = 0;
+    for (int32_t d = 0; d < D; ++d) {
+        if (row.occ[d] != kNone) row.gpu[d] += end - row.occ[d];
+        g += row.gpu[d];
+    }
+    for (int32_t w = 0; w < W; ++w) row.comp[w] -= dp.arrival[w];
+    *makespan = end - dp.first_arrival;
+    *gpu_total = g;
+}
+
 // r-th smallest (0-based) of v[0..n), reordering v (Hoare quickselect).
 __device__ int64_t select_rank(int64_t *v, int32_t n, int32_t r)
 {
@@ -267,7 +416,8 @@ eval_det_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, uint8_t *scratc
             continue;
         }
         int64_t mk, g, phi[2];
-        play<false>(dp, pr, row, 0, &mk, &g, dp.phi_life ? phi : nullptr);
+        if (dp.batch > 0) play_batched(dp, pr, row, &mk, &g);
+        else play<false>(dp, pr, row, 0, &mk, &g, dp.phi_life ? phi : nullptr);
         out.makespan_us[p] = mk;
         out.gpu_us[p] = g;
         out.p95_us[p] = select_rank(row.comp, dp.W, p95_rank(dp.W));
@@ -295,7 +445,8 @@ eval_list_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, uint8_t *scrat
             continue;
         }
         int64_t mk, g, phi[2];
-        play<false>(dp, pr, row, 0, &mk, &g, dp.phi_life ? phi : nullptr);
+        if (dp.batch > 0) play_batched(dp, pr, row, &mk, &g);
+        else play<false>(dp, pr, row, 0, &mk, &g, dp.phi_life ? phi : nullptr);
         out.makespan_us[p] = mk;
         out.gpu_us[p] = g;
         out.p95_us[p] = select_rank(row.comp, dp.W, p95_rank(dp.W));
@@ -388,6 +539,7 @@ size_t wf_eval_row_bytes(const wf_dev_problem &dp)
     size_t b = ((8 * (size_t)dp.N + 7) & ~(size_t)7) + 8 * 3 * (size_t)dp.D + 8 * (size_t)dp.W +
                2 * ((4 * (size_t)dp.D + 7) & ~(size_t)7) + ((4 * (size_t)dp.D * dp.M + 7) & ~(size_t)7) +
                4 * (size_t)dp.D;
+    if (dp.batch > 0) b += 4 + 16 * (size_t)dp.D * dp.batch + 12 * (size_t)dp.D;  // (4: padding after loaded)
     return (b + 127) & ~(size_t)127;
 }
 
@@ -411,9 +563,14 @@ int wf_launch_eval(wf_ctx *ctx, const wf_plans *plans, const wf_eval_out *out, c
     const wf_dev_problem &dp = ctx->dp;
     uint8_t *scratch = (uint8_t *)ctx->eval_scratch;
     const int64_t units = std::min<int64_t>(ctx->eval_threads, plans->P);
+    if (dp.batch > 1 && plans->retain)
+        return wf_set_error(WF_EINVAL, "retain rows are modelled with a replica batch limit of 1 only");
+    if (dp.batch > 0 && dp.phi_life)
+        return wf_set_error(WF_EINVAL, "the window terms of Eq. 12 are not modelled with a replica batch limit");
     if (dp.S == 0) {
         const int64_t blocks = (units + kEvalThreads - 1) / kEvalThreads;
-        const wf_sweep_cfg cfg = ctx->force_int64 ? wf_sweep_cfg{0, 0, 0} : wf_sweep_config(dp);
+        // The replica batch limit is played by the int64 path only.
+        const wf_sweep_cfg cfg = ctx->force_int64 || dp.batch > 0 ? wf_sweep_cfg{0, 0, 0} : wf_sweep_config(dp);
         if (dp.reclaim && !cfg.smem64)
             return wf_set_error(WF_EINVAL, "reclamation by next use runs only in the shared-memory sweep");
         if (cfg.smem32 || cfg.smem64) {

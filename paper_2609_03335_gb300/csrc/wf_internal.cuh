@@ -58,6 +58,10 @@ struct wf_dev_problem {
     // positions (0xFFFF = none), filled per call.
     int32_t reclaim;
     uint16_t *nextuse;
+    // Replica batch limit B_q (wf_ctx_set_batch): 0 = one unit at a time per
+    // device (the sweeps); >= 1 = up to B_q units of a device's current
+    // replica at once, played by the int64 path.
+    int32_t batch;
     int64_t max_chain_run;      // the longest fusible chain's run time on its slowest devices, plus the grant
     // Outputs of the window terms of Eq. 12 ([P] each, wf_eval_plans_phi);
     // null outside such a call.

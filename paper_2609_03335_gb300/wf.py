@@ -25,7 +25,8 @@ EXPORTS = ("wf_problem_check", "wf_ctx_create", "wf_forecast_readiness", "wf_eva
            "wf_topk", "wf_ctx_status", "wf_ctx_destroy", "wf_strerror", "wf_last_error",
            "wf_eval_plans_static", "wf_mutate_plans", "wf_merge_elite", "wf_local_search",
            "wf_construct_plans", "wf_ctx_set_reclaim", "wf_ctx_check_wait_expiry", "wf_eval_plans_phi",
-           "wf_topk_phi", "wf_static_status", "wf_ctx_set_eval_path")
+           "wf_topk_phi", "wf_static_status", "wf_ctx_set_eval_path",
+           "wf_ctx_set_batch")
 
 
 class WfError(RuntimeError):
@@ -94,6 +95,7 @@ def load_library():
         "wf_eval_plans_static": ([p, p, p, p], ctypes.c_int),
         "wf_static_status": ([p], ctypes.c_int),
         "wf_ctx_set_eval_path": ([p, i32], ctypes.c_int),
+        "wf_ctx_set_batch": ([p, i32], ctypes.c_int),
     }
     for name, (args, res) in sig.items():
         f = getattr(lib, name)
@@ -180,6 +182,9 @@ class Ctx:
         reclaim = int(getattr(prob, "reclaim", 0))
         if reclaim:
             wf_ctx_set_reclaim(self, reclaim)
+        batch = int(getattr(prob, "batch", 0))
+        if batch:
+            wf_ctx_set_batch(self, batch)
 
     @property
     def N(self):
@@ -222,6 +227,11 @@ PATH_AUTO, PATH_INT64 = 0, 1
 def wf_ctx_set_eval_path(ctx: Ctx, path: int):
     """PATH_AUTO (the sweeps) or PATH_INT64 (every plan on the exact int64 path)."""
     _check(load_library().wf_ctx_set_eval_path(ctx.ptr, int(path)), "wf_ctx_set_eval_path")
+
+
+def wf_ctx_set_batch(ctx: Ctx, batch: int):
+    """Replica batch limit B_q for later evaluations (0: one unit at a time per device)."""
+    _check(load_library().wf_ctx_set_batch(ctx.ptr, int(batch)), "wf_ctx_set_batch")
 
 
 def wf_ctx_check_wait_expiry(ctx: Ctx, stream=None):
