@@ -534,13 +534,13 @@ extern "C" int wf_ctx_set_reclaim(wf_ctx *c, int32_t policy)
     REQUIRE(c->dp.batch == 0, "reclamation by next use is not modelled with a replica batch limit");
     REQUIRE(c->dp.max_chain_run < (int64_t)UINT32_MAX,
             "a fusible chain may run %lld us, beyond the shared-memory sweep", (long long)c->dp.max_chain_run);
+    int rc = select_device(c);
+    if (rc) return rc;
     wf_dev_problem probe = c->dp;
     probe.reclaim = 1;
     const wf_sweep_cfg cfg = wf_sweep_config(probe);
     REQUIRE(cfg.smem64, "reclamation by next use needs the 64-bit shared-memory sweep, "
                         "which this window does not fit");
-    int rc = select_device(c);
-    if (rc) return rc;
     if (!c->dp.nextuse) {
         rc = wf_cuda_check(cudaMalloc(&c->dp.nextuse, sizeof(uint16_t) * (size_t)c->max_P * (size_t)c->dp.N),
                            "cudaMalloc(next-use table)");

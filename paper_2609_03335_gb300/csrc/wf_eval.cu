@@ -570,7 +570,7 @@ int wf_launch_eval(wf_ctx *ctx, const wf_plans *plans, const wf_eval_out *out, c
     if (dp.S == 0) {
         const int64_t blocks = (units + kEvalThreads - 1) / kEvalThreads;
         // The replica batch limit is played by the int64 path only.
-        const wf_sweep_cfg cfg = ctx->force_int64 || dp.batch > 0 ? wf_sweep_cfg{0, 0, 0} : wf_sweep_config(dp);
+        const wf_sweep_cfg cfg = ctx->force_int64 || dp.batch > 0 ? wf_sweep_cfg{} : wf_sweep_config(dp);
         if (dp.reclaim && !cfg.smem64)
             return wf_set_error(WF_EINVAL, "reclamation by next use runs only in the shared-memory sweep");
         if (cfg.smem32 || cfg.smem64) {

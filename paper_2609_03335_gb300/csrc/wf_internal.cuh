@@ -135,11 +135,14 @@ size_t wf_eval_scratch_bytes(const wf_dev_problem &dp, int64_t max_P, int64_t *u
 size_t wf_topk_scratch_bytes(int64_t max_P);
 size_t wf_search_scratch_bytes(int64_t max_P);
 // The shared-memory sweeps that apply to a problem: u32 times with 16 plans
-// per CTA, and u64 times with plans64 plans per CTA (0 bytes = not usable).
+// per CTA, and u64 times with plans64 plans per CTA (0 bytes = not usable);
+// res32 / res64 are the CTAs of each resident on one SM.
 struct wf_sweep_cfg {
     size_t smem32;
     size_t smem64;
     int plans64;
+    int res32;
+    int res64;
 };
 wf_sweep_cfg wf_sweep_config(const wf_dev_problem &dp);
 int wf_launch_nextuse(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, cudaStream_t st);

@@ -26,6 +26,9 @@
 // bit 31 of the record's load word, and timing counts the timely prefetches
 // and sums each unit's load delay plus its reload time.
 #include <algorithm>
+#include <mutex>
+#include <utility>
+#include <vector>
 
 #include "wf_internal.cuh"
 
@@ -162,9 +165,45 @@ struct PcGroups {
     __host__ __device__ static int32_t rows(int32_t D) { return (D + kG - 1) / kG; }
 };
 
+// Storage of the finish-time slots, [slot][plan]: TT words, or (Split40, for
+// u64 times whose every value stays below 2^40 us) a 32-bit low word per
+// slot and an 8-bit high byte in an array of its own: 5 bytes instead of 8,
+// so more plans fit an SM.
+struct Split40 {};
+
+template <typename ST>
+struct SlotBytes {
+    static constexpr uint32_t kLo = sizeof(ST), kHi = 0;
+};
+template <>
+struct SlotBytes<Split40> {
+    static constexpr uint32_t kLo = 4, kHi = 1;
+};
+
+template <typename TT, typename ST, int kS>
+struct SlotArr {  // plain words
+    TT *v;
+    __device__ __forceinline__ TT get(uint32_t i) const { return v[i * kS]; }
+    __device__ __forceinline__ void set(uint32_t i, TT x) const { v[i * kS] = x; }
+};
+template <int kS>
+struct SlotArr<uint64_t, Split40, kS> {
+    uint32_t *lo;
+    uint8_t *hi;
+    __device__ __forceinline__ uint64_t get(uint32_t i) const
+    {
+        return ((uint64_t)hi[i * kS] << 32) | lo[i * kS];
+    }
+    __device__ __forceinline__ void set(uint32_t i, uint64_t x) const
+    {
+        lo[i * kS] = (uint32_t)x;
+        hi[i * kS] = (uint8_t)(x >> 32);
+    }
+};
+
 struct PcLayout {
-    uint32_t weight, cap, load, arr, ring, slots, tfree, used, queue, nres, open, flag, nuse, rcnt, gmask, everl,
-        total;
+    uint32_t weight, cap, load, arr, ring, slots, slots_hi, tfree, used, queue, nres, open, flag, nuse, rcnt, gmask,
+        everl, total;
 };
 
 // Shared memory of a CTA of kP plans with TT times and NS slots per plan;
@@ -173,7 +212,7 @@ struct PcLayout {
 // copy and per model the number of devices holding it; with the window terms
 // of Eq. 12 (kPhi) each residency lane keeps per device the models it ever
 // held.
-template <int kP, typename TT, int kReclaim = 0, bool kPhi = false>
+template <int kP, typename TT, int kReclaim = 0, bool kPhi = false, typename ST = TT>
 __host__ __device__ inline PcLayout pc_layout(int32_t D, int32_t M, int32_t W, int32_t NS)
 {
     constexpr uint32_t t = sizeof(TT);
@@ -184,7 +223,8 @@ __host__ __device__ inline PcLayout pc_layout(int32_t D, int32_t M, int32_t W, i
     l.load = o; o += round16(4u * M * D);
     l.arr = o; o += round16(4u * W);
     l.ring = o; o += round16(8u * Ring<kReclaim>::kBuffers * RecPairs<kReclaim>::kPairs * kChunk * PcShape<kP>::kPitch);
-    l.slots = o; o += round16(t * (uint32_t)NS * kP);
+    l.slots = o; o += round16(SlotBytes<ST>::kLo * (uint32_t)NS * kP);
+    l.slots_hi = o; o += round16(SlotBytes<ST>::kHi * (uint32_t)NS * kP);
     l.tfree = o; o += round16(t * D * kP);
     const uint32_t rs = (uint32_t)(PcGroups<kP, kReclaim>::rows(D) * PcGroups<kP, kReclaim>::kLanes);
     l.used = o; o += round16(4u * rs);
@@ -229,6 +269,26 @@ __device__ TT select_strided(TT *v, int32_t n, int32_t r)
         else return v[r * kS];
     }
     return v[r * kS];
+}
+
+// The same over slots 0 .. n-1 of a slot array.
+template <typename TT, typename SA>
+__device__ TT select_slots(const SA &v, int32_t n, int32_t r)
+{
+    int32_t lo = 0, hi = n - 1;
+    while (lo < hi) {
+        const TT pivot = v.get(lo + (hi - lo) / 2);
+        int32_t i = lo, j = hi;
+        while (i <= j) {
+            while (v.get(i) < pivot) ++i;
+            while (v.get(j) > pivot) --j;
+            if (i <= j) { const TT t = v.get(i); v.set(i, v.get(j)); v.set(j, t); ++i; --j; }
+        }
+        if (r <= j) hi = j;
+        else if (r >= i) lo = i;
+        else return v.get(r);
+    }
+    return v.get(r);
 }
 
 // Two extra slots follow a plan's nslots slots: a sink that absorbs writes
@@ -436,11 +496,11 @@ __device__ __forceinline__ uint2 settle_lru(Q &q, uint32_t &n, uint32_t &u_d, ui
 
 // A finish time into a slot: an accumulator keeps the latest of its
 // writers, any other slot takes the value.
-template <typename TT, int kS>
-__device__ __forceinline__ void publish(TT *slots, uint32_t code, TT c)
+template <typename TT, typename SA>
+__device__ __forceinline__ void publish(const SA &slots, uint32_t code, TT c)
 {
-    TT &sv = slots[(code & 0x7FFFu) * kS];
-    sv = (code & 0x8000u) ? max(sv, c) : c;
+    const uint32_t i = code & 0x7FFFu;
+    slots.set(i, (code & 0x8000u) ? max(slots.get(i), c) : c);
 }
 
 // The sweep of groups of kP plans: every plan of the batch (in_list NULL, plan
@@ -449,7 +509,7 @@ __device__ __forceinline__ void publish(TT *slots, uint32_t code, TT c)
 // ovf_list; once every plan of a CTA has, its stages run on without loads.
 // TT = uint64_t: only a unit whose summed run time reaches 2^32 - 1 sends its
 // plan to ovf_list.
-template <typename Q, typename TT, int kP, int kReclaim, bool kPhi>
+template <typename Q, typename TT, int kP, int kReclaim, bool kPhi, typename ST>
 __global__ void __launch_bounds__(32 * PcShape<kP>::kWarps, PcShape<kP>::kMinBlocks)
 pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_list, const int32_t *in_count,
           int32_t *ovf_list, int32_t *ovf_count)
@@ -467,7 +527,7 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
     extern __shared__ __align__(128) uint8_t sm[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int32_t N = dp.N, D = dp.D, M = dp.M, W = dp.W;
-    const PcLayout L = pc_layout<kP, TT, kReclaim, kPhi>(D, M, W, dp.nslots + 2);
+    const PcLayout L = pc_layout<kP, TT, kReclaim, kPhi, ST>(D, M, W, dp.nslots + 2);
     const int64_t total = in_list ? (int64_t)*in_count : pl.P;
     if ((int64_t)blockIdx.x * kP >= total) return;  // the whole CTA: no plan
     uint2 *ring = (uint2 *)(sm + L.ring);
@@ -718,10 +778,16 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
     const bool mine = lane < kP;  // lanes at or beyond kP own no plan and touch no per-plan state
     const int64_t p = (mine && lane < ng) ? (in_list ? (int64_t)in_list[j0 + lane] : j0 + lane) : 0;
     const bool live = mine && lane < ng && out.status[p] == 0;
-    TT *slots = (TT *)(sm + L.slots) + lane;
+    SlotArr<TT, ST, kP> slots;
+    if constexpr (SlotBytes<ST>::kHi) {
+        slots.lo = (uint32_t *)(sm + L.slots) + lane;
+        slots.hi = sm + L.slots_hi + lane;
+    } else {
+        slots.v = (TT *)(sm + L.slots) + lane;
+    }
     TT *tfree = (TT *)(sm + L.tfree) + lane;
     if (mine) {
-        for (int32_t k = 0; k < dp.nslots + 2; ++k) slots[k * kP] = 0;
+        for (int32_t k = 0; k < dp.nslots + 2; ++k) slots.set(k, 0);
         for (int32_t d = 0; d < D; ++d) tfree[d * kP] = 0;
     }
     __syncthreads();
@@ -756,8 +822,8 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
                     TT *tf_d = tfree + (r3 & 31u) * kP;
                     // Release (Eq. 2, Eq. 7); an accumulator slot is reset by its reader.
                     const uint32_t rs = r5 >> 16;
-                    const TT rel = max((TT)arr, slots[(rs & 0x7FFFu) * kP]);
-                    slots[((rs & 0x8000u) ? (rs & 0x7FFFu) : trash) * kP] = 0;
+                    const TT rel = max((TT)arr, slots.get(rs & 0x7FFFu));
+                    slots.set((rs & 0x8000u) ? (rs & 0x7FFFu) : trash, 0);
                     // A miss loads on this device first (ld > 0 only on a miss); a
                     // prefetched load waits only for the arrival (Eq. 5).  On a hit
                     // the residency stage cleared the prefetch bit and ld is 0.
@@ -780,16 +846,16 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
                     if (r3 & kWasEmpty) gsum -= (int64_t)ls;   // an empty device becomes occupied
                     if (r3 & kEmptied) gsum += (int64_t)cfin;  // the device empties after the unit
 
-                    publish<TT, kP>(slots, r3 >> 16, cfin);  // the sink when the unit writes nothing
-                    publish<TT, kP>(slots, r4 & 0xFFFFu, cfin);
+                    publish<TT>(slots, r3 >> 16, cfin);  // the sink when the unit writes nothing
+                    publish<TT>(slots, r4 & 0xFFFFu, cfin);
                     const uint32_t nwl = (r3 >> 11) & 7u;
                     if (nwl > 2) {
-                        publish<TT, kP>(slots, r4 >> 16, cfin);
+                        publish<TT>(slots, r4 >> 16, cfin);
                         if (nwl == 4) {
-                            publish<TT, kP>(slots, r5 & 0xFFFFu, cfin);
+                            publish<TT>(slots, r5 & 0xFFFFu, cfin);
                         } else if (nwl > 4) {  // five or more codes: the list from global memory
                             const int4 wr = __ldg(dp.noderec + 2 * (int32_t)(r5 & 0xFFFFu) + 1);
-                            for (int32_t e = 3; e < wr.y; ++e) publish<TT, kP>(slots, __ldg(dp.wl + wr.x + e), cfin);
+                            for (int32_t e = 3; e < wr.y; ++e) publish<TT>(slots, __ldg(dp.wl + wr.x + e), cfin);
                         }
                     }
                     *tf_d = cfin;
@@ -810,11 +876,11 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
         ovf_list[kk] = (int32_t)p;
     } else if (live) {
         const int64_t nopen = open[lane];
-        for (int32_t w = 0; w < W; ++w) slots[w * kP] -= arrival[w];  // session completion latency
+        for (int32_t w = 0; w < W; ++w) slots.set(w, slots.get(w) - arrival[w]);  // session completion latency
         const int32_t rank = (int32_t)((95 * (int64_t)W + 99) / 100 - 1);
         out.makespan_us[p] = (int64_t)end - dp.first_arrival;
         out.gpu_us[p] = gsum + nopen * (int64_t)end;
-        out.p95_us[p] = (int64_t)select_strided<TT, kP>(slots, W, rank);
+        out.p95_us[p] = (int64_t)select_slots<TT>(slots, W, rank);
         if (kPhi) {
             dp.phi_timely[p] = ph_timely;
             dp.phi_life[p] = (int64_t)ph_life;
@@ -1185,7 +1251,11 @@ status_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out)
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, warps = blockDim.x >> 5;
     const int32_t N = dp.N, D = dp.D, E = dp.E;
     uint16_t *pos = (uint16_t *)(ssm + (size_t)warp * status_warp_bytes(N));
-    for (int64_t p = (int64_t)blockIdx.x * warps + warp; p < pl.P; p += (int64_t)gridDim.x * warps) {
+    // Plans are visited from the last to the first: the rows read last stay
+    // in L2, and they are those of the sweep's first wave of CTAs (the
+    // lowest plan indices), which then re-reads them from L2 rather than DRAM.
+    for (int64_t k = (int64_t)blockIdx.x * warps + warp; k < pl.P; k += (int64_t)gridDim.x * warps) {
+        const int64_t p = pl.P - 1 - k;
         const uint8_t *place = pl.place + p * pl.place_stride;
         const uint16_t *order = (const uint16_t *)((const uint8_t *)pl.order + p * pl.order_stride);
         uint32_t st = 0;
@@ -1331,66 +1401,100 @@ bool sweep_usable(const wf_dev_problem &dp)
            dp.N <= 65534;
 }
 
-// Plans per SM at this shared-memory size (228 KB per SM, 1 KB reserved per CTA).
-int plans_per_sm(size_t smem, int kp)
-{
-    return smem <= 227 * 1024 ? kp * (int)((228 * 1024) / (smem + 1024)) : 0;
-}
+// The 64-bit sweep keeps its slots in 40 bits when no time of the window can
+// reach 2^40 us (the context's horizon bounds every finish) and reclamation
+// is least recently used.
+bool split40(const wf_dev_problem &dp) { return dp.horizon < ((int64_t)1 << 40) && dp.reclaim == 0; }
 
-template <typename Q, typename TT, int kP, int kR, bool kF>
-int launch_pc(const wf_dev_problem &dp, int sms, const wf_plans *pl, const wf_eval_out *out, size_t smem,
-              const int32_t *in_list, const int32_t *in_count, int32_t *list, int32_t *count, cudaStream_t st)
+template <typename Q, typename TT, int kP, int kR, bool kF, typename ST = TT>
+int launch_pc(const wf_dev_problem &dp, int sms, int resident, const wf_plans *pl, const wf_eval_out *out,
+              size_t smem, const int32_t *in_list, const int32_t *in_count, int32_t *list, int32_t *count, cudaStream_t st)
 {
-    int rc = wf_cuda_check(cudaFuncSetAttribute(pc_kernel<Q, TT, kP, kR, kF>,
+    int rc = wf_cuda_check(cudaFuncSetAttribute(pc_kernel<Q, TT, kP, kR, kF, ST>,
                                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
                            "sweep smem attribute");
     if (rc) return rc;
     // Every plan: a CTA per group.  A list (of unknown length): at most as
     // many CTAs as are resident at once, each walking over groups.
     int64_t blocks = (pl->P + kP - 1) / kP;
-    if (in_list) {
-        const int64_t per_sm = std::max<int64_t>(1, std::min<int64_t>(8, (228 * 1024) / (int64_t)(smem + 1024)));
-        blocks = std::min<int64_t>(blocks, per_sm * sms);
-    }
-    pc_kernel<Q, TT, kP, kR, kF><<<(unsigned)blocks, 32 * PcShape<kP>::kWarps, smem, st>>>(dp, *pl, *out, in_list, in_count, list,
-                                                                          count);
+    if (in_list) blocks = std::min<int64_t>(blocks, (int64_t)std::max(1, resident) * sms);
+    pc_kernel<Q, TT, kP, kR, kF, ST><<<(unsigned)blocks, 32 * PcShape<kP>::kWarps, smem, st>>>(
+        dp, *pl, *out, in_list, in_count, list, count);
     return wf_cuda_check(cudaGetLastError(), "sweep launch");
 }
 
-template <typename TT, int kR, bool kF>
-int launch_pc_r(const wf_ctx *ctx, int kp, const wf_plans *pl, const wf_eval_out *out, size_t smem,
-                const int32_t *in_list, const int32_t *in_count, int32_t *list, int32_t *count, cudaStream_t st)
+template <typename T> struct Ty { using type = T; };
+template <int V> struct Iv { static constexpr int value = V; };
+
+// Calls f(Ty<Q>{}, Iv<kP>{}, Ty<ST>{}) for the sweep instantiation that this
+// problem and CTA shape take: Q the LRU word (up to 8 models pack in 32 bits),
+// kP the plans per CTA, ST the finish-slot storage.
+template <typename TT, int kR, typename F>
+int pc_visit(const wf_dev_problem &dp, int kp, F &&f)
 {
-    const wf_dev_problem &dp = ctx->dp;
-    const int sms = ctx->sms;
     if constexpr (sizeof(TT) == 4) {  // the u32 sweep has one shape
         (void)kp;
-        return dp.M <= 8
-                   ? launch_pc<uint32_t, TT, kPlans32, kR, kF>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
-                   : launch_pc<uint64_t, TT, kPlans32, kR, kF>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
+        return dp.M <= 8 ? f(Ty<uint32_t>{}, Iv<kPlans32>{}, Ty<TT>{}) : f(Ty<uint64_t>{}, Iv<kPlans32>{}, Ty<TT>{});
     } else {
-        if (kp == 16)
-            return dp.M <= 8
-                       ? launch_pc<uint32_t, TT, 16, kR, kF>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
-                       : launch_pc<uint64_t, TT, 16, kR, kF>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
-        if (kp == 6)
-            return dp.M <= 8
-                       ? launch_pc<uint32_t, TT, 6, kR, kF>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
-                       : launch_pc<uint64_t, TT, 6, kR, kF>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
-        return dp.M <= 8 ? launch_pc<uint32_t, TT, 3, kR, kF>(dp, sms, pl, out, smem, in_list, in_count, list, count, st)
-                         : launch_pc<uint64_t, TT, 3, kR, kF>(dp, sms, pl, out, smem, in_list, in_count, list, count, st);
+        auto by_q = [&](auto p, auto s) { return dp.M <= 8 ? f(Ty<uint32_t>{}, p, s) : f(Ty<uint64_t>{}, p, s); };
+        auto by_p = [&](auto s) {
+            return kp == 16 ? by_q(Iv<16>{}, s) : kp == 6 ? by_q(Iv<6>{}, s) : by_q(Iv<3>{}, s);
+        };
+        if constexpr (kR == 0)
+            if (split40(dp)) return by_p(Ty<Split40>{});
+        return by_p(Ty<TT>{});
     }
 }
 
+template <typename TT, int kR, bool kF>
+int launch_pc_r(const wf_ctx *ctx, int kp, int resident, const wf_plans *pl, const wf_eval_out *out, size_t smem,
+                const int32_t *in_list, const int32_t *in_count, int32_t *list, int32_t *count, cudaStream_t st)
+{
+    const wf_dev_problem &dp = ctx->dp;
+    return pc_visit<TT, kR>(dp, kp, [&](auto q, auto p, auto s) {
+        return launch_pc<typename decltype(q)::type, TT, decltype(p)::value, kR, kF, typename decltype(s)::type>(
+            dp, ctx->sms, resident, pl, out, smem, in_list, in_count, list, count, st);
+    });
+}
+
+// CTAs of the sweep instantiation resident on one SM at this shared-memory
+// size: registers and shared memory both count (0 = it does not fit).
+template <typename TT, int kR, bool kF>
+int resident_r(const wf_dev_problem &dp, int kp, size_t smem)
+{
+    if (smem > 227 * 1024) return 0;
+    return pc_visit<TT, kR>(dp, kp, [&](auto q, auto p, auto s) {
+        const auto k = pc_kernel<typename decltype(q)::type, TT, decltype(p)::value, kR, kF, typename decltype(s)::type>;
+        int n = 0;
+        if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess ||
+            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k, 32 * PcShape<decltype(p)::value>::kWarps, smem) !=
+                cudaSuccess) {
+            (void)cudaGetLastError();
+            return 0;
+        }
+        return n;
+    });
+}
+
 template <typename TT>
-int launch_pc_q(const wf_ctx *ctx, int kp, const wf_plans *pl, const wf_eval_out *out, size_t smem,
+int resident(const wf_dev_problem &dp, int kp, size_t smem)
+{
+    if (dp.phi_life)
+        return dp.reclaim ? resident_r<TT, 1, true>(dp, kp, smem) : resident_r<TT, 0, true>(dp, kp, smem);
+    return dp.reclaim ? resident_r<TT, 1, false>(dp, kp, smem) : resident_r<TT, 0, false>(dp, kp, smem);
+}
+
+template <typename TT>
+int launch_pc_q(const wf_ctx *ctx, int kp, int resident, const wf_plans *pl, const wf_eval_out *out, size_t smem,
                 const int32_t *in_list, const int32_t *in_count, int32_t *list, int32_t *count, cudaStream_t st)
 {
     if (ctx->dp.phi_life)
-        return ctx->dp.reclaim ? launch_pc_r<TT, 1, true>(ctx, kp, pl, out, smem, in_list, in_count, list, count, st)
-                               : launch_pc_r<TT, 0, true>(ctx, kp, pl, out, smem, in_list, in_count, list, count, st);
-    return ctx->dp.reclaim ? launch_pc_r<TT, 1, false>(ctx, kp, pl, out, smem, in_list, in_count, list, count, st)
-                           : launch_pc_r<TT, 0, false>(ctx, kp, pl, out, smem, in_list, in_count, list, count, st);
+        return ctx->dp.reclaim
+                   ? launch_pc_r<TT, 1, true>(ctx, kp, resident, pl, out, smem, in_list, in_count, list, count, st)
+                   : launch_pc_r<TT, 0, true>(ctx, kp, resident, pl, out, smem, in_list, in_count, list, count, st);
+    return ctx->dp.reclaim
+               ? launch_pc_r<TT, 1, false>(ctx, kp, resident, pl, out, smem, in_list, in_count, list, count, st)
+               : launch_pc_r<TT, 0, false>(ctx, kp, resident, pl, out, smem, in_list, in_count, list, count, st);
 }
 
 }  // namespace
@@ -1410,6 +1514,9 @@ template <int kP, typename TT>
 size_t layout_bytes(const wf_dev_problem &dp)
 {
     const int32_t NS = dp.nslots + 2;
+    if (sizeof(TT) == 8 && split40(dp))
+        return dp.phi_life ? pc_layout<kP, TT, 0, true, Split40>(dp.D, dp.M, dp.W, NS).total
+                           : pc_layout<kP, TT, 0, false, Split40>(dp.D, dp.M, dp.W, NS).total;
     if (dp.phi_life)
         return dp.reclaim ? pc_layout<kP, TT, 1, true>(dp.D, dp.M, dp.W, NS).total
                           : pc_layout<kP, TT, 0, true>(dp.D, dp.M, dp.W, NS).total;
@@ -1417,21 +1524,67 @@ size_t layout_bytes(const wf_dev_problem &dp)
                       : pc_layout<kP, TT, 0, false>(dp.D, dp.M, dp.W, NS).total;
 }
 
-wf_sweep_cfg wf_sweep_config(const wf_dev_problem &dp)
+namespace {
+
+// The shape choice depends on these fields of the problem only (and on the
+// device, whose registers and shared memory bound the resident CTAs).
+struct CfgKey {
+    int dev;
+    int32_t D, M, W, nslots;
+    bool usable, split, reclaim, phi;
+    bool operator==(const CfgKey &o) const
+    {
+        return dev == o.dev && D == o.D && M == o.M && W == o.W && nslots == o.nslots && usable == o.usable &&
+               split == o.split && reclaim == o.reclaim && phi == o.phi;
+    }
+};
+
+wf_sweep_cfg choose(const wf_dev_problem &dp)
 {
-    wf_sweep_cfg c = {0, 0, 0};
+    wf_sweep_cfg c = {};
     if (!sweep_usable(dp)) return c;
     const size_t s32 = layout_bytes<kPlans32, uint32_t>(dp);
-    if (s32 <= 227 * 1024) c.smem32 = s32;
+    c.res32 = resident<uint32_t>(dp, kPlans32, s32);
+    if (c.res32 > 0) c.smem32 = s32;
     // The u64 sweep: 16, 6 or 3 plans per CTA, whichever keeps the most plans
-    // per SM (ties: the smaller CTAs, more of them to hide latency).
-    const size_t s16 = layout_bytes<16, uint64_t>(dp);
-    const size_t s6 = layout_bytes<6, uint64_t>(dp);
-    const size_t s3 = layout_bytes<3, uint64_t>(dp);
-    const int a = plans_per_sm(s16, 16), b = plans_per_sm(s6, 6), e = plans_per_sm(s3, 3);
-    if (e > 0 && e >= a && e >= b) { c.smem64 = s3; c.plans64 = 3; }
-    else if (b > 0 && b >= a) { c.smem64 = s6; c.plans64 = 6; }
-    else if (a > 0) { c.smem64 = s16; c.plans64 = 16; }
+    // resident per SM, registers and shared memory both counted.  Ties go to
+    // the larger CTA, whose producer and residency warps serve more plans.
+    const int shapes[3] = {16, 6, 3};
+    int best = 0;
+    for (int kp : shapes) {
+        const size_t sm = kp == 16 ? layout_bytes<16, uint64_t>(dp)
+                          : kp == 6 ? layout_bytes<6, uint64_t>(dp)
+                                    : layout_bytes<3, uint64_t>(dp);
+        const int n = resident<uint64_t>(dp, kp, sm);
+        if (n > 0 && kp * n > best) {
+            best = kp * n;
+            c.smem64 = sm;
+            c.plans64 = kp;
+            c.res64 = n;
+        }
+    }
+    return c;
+}
+
+}  // namespace
+
+wf_sweep_cfg wf_sweep_config(const wf_dev_problem &dp)
+{
+    static std::mutex mu;
+    static std::vector<std::pair<CfgKey, wf_sweep_cfg>> cache;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        (void)cudaGetLastError();
+        return wf_sweep_cfg{};
+    }
+    const CfgKey key = {dev, dp.D, dp.M, dp.W, dp.nslots, sweep_usable(dp), split40(dp), dp.reclaim != 0,
+                        dp.phi_life != 0};
+    std::lock_guard<std::mutex> lock(mu);
+    for (const auto &e : cache)
+        if (e.first == key) return e.second;
+    const wf_sweep_cfg c = choose(dp);
+    if (cache.size() >= 64) cache.erase(cache.begin());
+    cache.emplace_back(key, c);
     return c;
 }
 
@@ -1445,12 +1598,12 @@ int wf_launch_sweep(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, con
     if (cfg.smem32 && !(wide_first && cfg.smem64)) {
         // u32 times for every plan; the plans that leave 32 bits go on to the
         // u64 sweep, and from there (or straight) to the int64 path.
-        rc = launch_pc_q<uint32_t>(ctx, kPlans32, pl, out, cfg.smem32, nullptr, nullptr, list1, counts, st);
+        rc = launch_pc_q<uint32_t>(ctx, kPlans32, cfg.res32, pl, out, cfg.smem32, nullptr, nullptr, list1, counts, st);
         if (rc) return rc;
         if (!cfg.smem64) { *rest_list = list1; *rest_count = counts; return WF_OK; }
-        rc = launch_pc_q<uint64_t>(ctx, cfg.plans64, pl, out, cfg.smem64, list1, counts, list2, counts + 1, st);
+        rc = launch_pc_q<uint64_t>(ctx, cfg.plans64, cfg.res64, pl, out, cfg.smem64, list1, counts, list2, counts + 1, st);
     } else {
-        rc = launch_pc_q<uint64_t>(ctx, cfg.plans64, pl, out, cfg.smem64, nullptr, nullptr, list2, counts + 1, st);
+        rc = launch_pc_q<uint64_t>(ctx, cfg.plans64, cfg.res64, pl, out, cfg.smem64, nullptr, nullptr, list2, counts + 1, st);
     }
     *rest_list = list2;
     *rest_count = counts + 1;
