@@ -1243,7 +1243,7 @@ __host__ __device__ inline uint32_t status_warp_bytes(int32_t N)
 
 // kByte: every device index is below 8, so one byte per node holds its fit
 // mask (fit8): a quarter of the table reads of the 32-bit masks.
-template <bool kByte>
+template <bool kByte, int kU>
 __global__ void __launch_bounds__(128)
 status_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out)
 {
@@ -1263,67 +1263,107 @@ status_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out)
         // bytes, so 16-byte reads at multiples of 16 bytes below N stay in
         // the row; lanes mask the entries at or beyond N.  The fit masks are
         // padded to 16 entries.
-        for (int32_t n16 = 16 * lane; n16 < N; n16 += 512) {
-            const uint4 pw = __ldg((const uint4 *)(place + n16));
-            const uint32_t pws[4] = {pw.x, pw.y, pw.z, pw.w};
-            if (kByte) {
-                const uint4 fb = __ldg((const uint4 *)(dp.fit8 + n16));
-                const uint32_t fbs[4] = {fb.x, fb.y, fb.z, fb.w};
+        // Every loop issues kU 16-byte reads per lane before it uses any: on
+        // long rows a warp keeps a plan's reads in flight rather than one
+        // round trip per 512 bytes (kU = 1 on short rows, whose loops run once).
+        for (int32_t b16 = 16 * lane; b16 < N; b16 += kU * 512) {
+            uint4 pw[kU], fb[kU], fm[kU][4];
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
+            for (int u = 0; u < kU; ++u) {
+                const int32_t n16 = b16 + 512 * u;
+                const bool in = n16 < N;
+                pw[u] = in ? __ldg((const uint4 *)(place + n16)) : make_uint4(0u, 0u, 0u, 0u);
+                if (kByte) {
+                    fb[u] = in ? __ldg((const uint4 *)(dp.fit8 + n16)) : make_uint4(0u, 0u, 0u, 0u);
+                } else {
 #pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-                        const uint32_t d = (pws[q] >> (8 * j)) & 255u, f = (fbs[q] >> (8 * j)) & 255u;
-                        if (n16 + 4 * q + j < N)
-                            st |= d >= (uint32_t)D ? WF_ST_DEVICE : (((f >> (d & 7u)) & 1u) ? 0u : WF_ST_CAPACITY);
-                    }
+                    for (int q = 0; q < 4; ++q)
+                        fm[u][q] = in ? __ldg((const uint4 *)(dp.fitmask + n16 + 4 * q)) : make_uint4(0u, 0u, 0u, 0u);
                 }
-            } else {
+            }
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const uint4 fm = __ldg((const uint4 *)(dp.fitmask + n16 + 4 * q));
-                    const uint32_t f[4] = {fm.x, fm.y, fm.z, fm.w};
+            for (int u = 0; u < kU; ++u) {
+                const int32_t n16 = b16 + 512 * u;
+                const uint32_t pws[4] = {pw[u].x, pw[u].y, pw[u].z, pw[u].w};
+                if (kByte) {
+                    const uint32_t fbs[4] = {fb[u].x, fb[u].y, fb[u].z, fb[u].w};
 #pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-                        const uint32_t d = (pws[q] >> (8 * j)) & 255u;
-                        if (n16 + 4 * q + j < N)
-                            st |= d >= (uint32_t)D ? WF_ST_DEVICE : (((f[j] >> d) & 1u) ? 0u : WF_ST_CAPACITY);
+                    for (int q = 0; q < 4; ++q) {
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) {
+                            const uint32_t d = (pws[q] >> (8 * j)) & 255u, f = (fbs[q] >> (8 * j)) & 255u;
+                            if (n16 + 4 * q + j < N)
+                                st |= d >= (uint32_t)D ? WF_ST_DEVICE
+                                                       : (((f >> (d & 7u)) & 1u) ? 0u : WF_ST_CAPACITY);
+                        }
+                    }
+                } else {
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const uint32_t f[4] = {fm[u][q].x, fm[u][q].y, fm[u][q].z, fm[u][q].w};
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) {
+                            const uint32_t d = (pws[q] >> (8 * j)) & 255u;
+                            if (n16 + 4 * q + j < N)
+                                st |= d >= (uint32_t)D ? WF_ST_DEVICE : (((f[j] >> d) & 1u) ? 0u : WF_ST_CAPACITY);
+                        }
                     }
                 }
             }
         }
         // The inverse permutation, 8 dispatch entries a lane at a time, then
         // read back: a repeated node leaves some entry unmatched.
-        for (int32_t i8 = 8 * lane; i8 < N; i8 += 256) {
-            const uint4 ow = __ldg((const uint4 *)(order + i8));
-            const uint32_t w[4] = {ow.x, ow.y, ow.z, ow.w};
+        for (int32_t b8 = 8 * lane; b8 < N; b8 += kU * 256) {
+            uint4 ow[kU];
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                const uint32_t h = (w[j >> 1] >> (16 * (j & 1))) & 0xFFFFu;
-                if (i8 + j < N) {
-                    if (h < (uint32_t)N) pos[h] = (uint16_t)(i8 + j);
-                    else st |= WF_ST_PERMUTATION;
+            for (int u = 0; u < kU; ++u)
+                ow[u] = b8 + 256 * u < N ? __ldg((const uint4 *)(order + b8 + 256 * u)) : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+            for (int u = 0; u < kU; ++u) {
+                const int32_t i8 = b8 + 256 * u;
+                const uint32_t w[4] = {ow[u].x, ow[u].y, ow[u].z, ow[u].w};
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    const uint32_t h = (w[j >> 1] >> (16 * (j & 1))) & 0xFFFFu;
+                    if (i8 + j < N) {
+                        if (h < (uint32_t)N) pos[h] = (uint16_t)(i8 + j);
+                        else st |= WF_ST_PERMUTATION;
+                    }
                 }
             }
         }
         __syncwarp();
-        for (int32_t i8 = 8 * lane; i8 < N; i8 += 256) {
-            const uint4 ow = __ldg((const uint4 *)(order + i8));
-            const uint32_t w[4] = {ow.x, ow.y, ow.z, ow.w};
+        for (int32_t b8 = 8 * lane; b8 < N; b8 += kU * 256) {
+            uint4 ow[kU];
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                const uint32_t h = (w[j >> 1] >> (16 * (j & 1))) & 0xFFFFu;
-                if (i8 + j < N && h < (uint32_t)N && pos[h] != (uint16_t)(i8 + j)) st |= WF_ST_PERMUTATION;
+            for (int u = 0; u < kU; ++u)
+                ow[u] = b8 + 256 * u < N ? __ldg((const uint4 *)(order + b8 + 256 * u)) : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+            for (int u = 0; u < kU; ++u) {
+                const int32_t i8 = b8 + 256 * u;
+                const uint32_t w[4] = {ow[u].x, ow[u].y, ow[u].z, ow[u].w};
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    const uint32_t h = (w[j >> 1] >> (16 * (j & 1))) & 0xFFFFu;
+                    if (i8 + j < N && h < (uint32_t)N && pos[h] != (uint16_t)(i8 + j)) st |= WF_ST_PERMUTATION;
+                }
             }
         }
         st = __reduce_or_sync(0xFFFFFFFFu, st);
         if (!(st & WF_ST_PERMUTATION)) {
-            for (int32_t e4 = 4 * lane; e4 < E; e4 += 128) {  // edges padded to 4
-                const uint4 uv = __ldg((const uint4 *)(dp.edges + e4));
-                const uint32_t w[4] = {uv.x, uv.y, uv.z, uv.w};
+            for (int32_t b4 = 4 * lane; b4 < E; b4 += kU * 128) {  // edges padded to 4
+                uint4 uv[kU];
 #pragma unroll
-                for (int j = 0; j < 4; ++j)
-                    if (e4 + j < E && pos[w[j] & 0xFFFFu] > pos[w[j] >> 16]) st |= WF_ST_TOPOLOGY;
+                for (int u = 0; u < kU; ++u)
+                    uv[u] = b4 + 128 * u < E ? __ldg((const uint4 *)(dp.edges + b4 + 128 * u)) : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+                for (int u = 0; u < kU; ++u) {
+                    const int32_t e4 = b4 + 128 * u;
+                    const uint32_t w[4] = {uv[u].x, uv[u].y, uv[u].z, uv[u].w};
+#pragma unroll
+                    for (int j = 0; j < 4; ++j)
+                        if (e4 + j < E && pos[w[j] & 0xFFFFu] > pos[w[j] >> 16]) st |= WF_ST_TOPOLOGY;
+                }
             }
             st = __reduce_or_sync(0xFFFFFFFFu, st);
         }
@@ -1336,25 +1376,27 @@ status_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out)
     }
 }
 
-template <bool kByte>
+template <bool kByte, int kU>
 int launch_status_as(const wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, cudaStream_t st)
 {
     const wf_dev_problem &dp = ctx->dp;
     const size_t wbytes = status_warp_bytes(dp.N);
     const int swarps = (int)std::max<size_t>(1, std::min<size_t>(4, (227 * 1024) / wbytes));
     const size_t ssmem = wbytes * swarps;
-    int rc = wf_cuda_check(cudaFuncSetAttribute(status_kernel<kByte>,
+    int rc = wf_cuda_check(cudaFuncSetAttribute(status_kernel<kByte, kU>,
                                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ssmem),
                            "status smem attribute");
     if (rc) return rc;
     const int64_t sblocks = std::min<int64_t>((pl->P + swarps - 1) / swarps, (int64_t)ctx->sms * 16);
-    status_kernel<kByte><<<(unsigned)sblocks, 32 * swarps, ssmem, st>>>(dp, *pl, *out);
+    status_kernel<kByte, kU><<<(unsigned)sblocks, 32 * swarps, ssmem, st>>>(dp, *pl, *out);
     return WF_OK;
 }
 
 int launch_status(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, cudaStream_t st)
 {
-    return ctx->dp.D <= 8 ? launch_status_as<true>(ctx, pl, out, st) : launch_status_as<false>(ctx, pl, out, st);
+    const bool byte = ctx->dp.D <= 8, wide = ctx->dp.N >= 1024;
+    if (wide) return byte ? launch_status_as<true, 4>(ctx, pl, out, st) : launch_status_as<false, 4>(ctx, pl, out, st);
+    return byte ? launch_status_as<true, 1>(ctx, pl, out, st) : launch_status_as<false, 1>(ctx, pl, out, st);
 }
 
 }  // namespace

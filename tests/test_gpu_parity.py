@@ -8,7 +8,7 @@ import pytest
 import oracle
 import wfgen
 from golden_util import fixture_names, load, plans_of, problem_of
-from gpu_util import assert_same, gpu_eval, oracle_eval
+from gpu_util import assert_same, gpu_eval, lib, oracle_eval
 from randprob import random_problem
 
 pytestmark = pytest.mark.gpu
@@ -68,16 +68,23 @@ def test_stochastic_workload_full_parity():
 
 
 def test_large_window_parity():
-    """Full size (P=131072, N=8192, D=16); the oracle checks every plan."""
+    """Full size (P=131072, N=8192, D=16); the oracle checks every plan.  Two
+    calls on one context: the first plays the 32-bit sweep and hands every
+    plan to the 64-bit one; once that count has arrived, later calls start
+    with the 64-bit sweep over the whole batch, the launch the bench times."""
     w = wfgen.config("large")
     plans = wfgen.make_plans(w.problem, w.P, w.plan_seed)
-    got = gpu_eval(w.problem, plans, k=w.k, forecast=True)
     want = oracle_eval(w.problem, plans)
-    assert_same(got, want)
     ids, keys = oracle.topk(want["makespan"], want["p95"], want["gpu"], want["status"], w.k)
-    assert np.array_equal(got["ids"], ids) and np.array_equal(got["keys"], keys)
-    rel, comp = oracle.forecast(w.problem)
-    assert np.array_equal(got["rel"], rel) and np.array_equal(got["comp"], comp)
+    ctx = lib().Ctx(w.problem, max_P=plans.P, device=0)
+    for call in range(2):
+        got = gpu_eval(w.problem, plans, k=w.k, ctx=ctx, forecast=call == 0)
+        assert_same(got, want)
+        assert np.array_equal(got["ids"], ids) and np.array_equal(got["keys"], keys)
+        if call == 0:
+            rel, comp = oracle.forecast(w.problem)
+            assert np.array_equal(got["rel"], rel) and np.array_equal(got["comp"], comp)
+    ctx.close()
 
 
 @pytest.mark.parametrize("name", fixture_names())
