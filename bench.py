@@ -299,12 +299,12 @@ def metric_of(prob):
     return f"candidate plans evaluated/sec (N={prob.N},D={prob.D}" + (f",S={prob.S})" if prob.S else ")")
 
 
-def issue_roofline(eval_ms, clk, sms):
+def issue_roofline(eval_ms, clk, sms, workload=None):
     """The integer-issue roofline of the evaluation call: its warp
     instructions (ncu, same kernel source) over its CUDA-event time, against
     4 warp instructions per clock per SM at the median SM clock sampled
     during the run."""
-    inst = read_instructions(WORKLOAD)
+    inst = read_instructions(workload or WORKLOAD)
     mhz = (clk or {}).get("sm_mhz")
     if not inst or not mhz:
         return None
@@ -427,9 +427,16 @@ def workload_entry(name, wf, dev, steps=5, warmup=3, with_cpu=True):
                           "frac_of_hbm": bpp * P / (eval_ms * 1e-3) / 1e9 / peak if peak else None,
                           "algorithmic_bytes_per_plan": bpp},
              "clocks": clk, "timing": f"median of {steps} steps after {warmup}, L2 flushed before each"}
+    traffic, _ = read_traffic(name)
+    entry["roofline"]["traffic"] = traffic
+    entry["roofline_issue"] = issue_roofline(eval_ms, clk, torch.cuda.get_device_properties(dev).multi_processor_count,
+                                             name)
     if prob.S:
         entry["samples"] = prob.S
         entry["sims_per_s"] = P * prob.S / (step_ms * 1e-3)
+        ri = entry["roofline_issue"]
+        if ri:  # the sims/s this instruction count would give at the full issue rate
+            ri["sims_per_s_ceiling"] = P * prob.S / (ri["warp_instructions"] / ri["peak"])
     if with_cpu:
         import oracle
         oracle.build()
