@@ -312,6 +312,30 @@ def test_fused_run_time_beyond_u32():
     assert_same(got, want)
 
 
+def test_horizon_beyond_2_40_uses_8_byte_slots():
+    """The 64-bit sweep keeps its finish slots in 40 bits only while the
+    context's horizon (latest arrival plus every node's worst run and load)
+    stays below 2^40 us.  About 600 nodes of near 2^31 us each push it past;
+    two calls check both launch shapes of the 8-byte-slot sweep."""
+    wf = lib()
+    rng = np.random.default_rng(53)
+    prob = random_problem(rng, n_sessions=20, sizes=(26, 34), D=4, M=3)
+    lat = ((1 << 31) - 1 - prob.lat_us.astype(np.int64) % 1000).astype(np.int32)
+    prob = prob.with_(lat_us=lat)
+    worst = (lat.reshape(prob.N, prob.D).astype(np.int64)
+             + prob.load_us.reshape(prob.M, prob.D)[prob.model].astype(np.int64)).max(axis=1)
+    horizon = int(prob.arrival_us.max()) + int((worst + prob.grant_us).sum())
+    assert horizon >= 1 << 40
+    plans = wfgen.make_plans(prob, 400, 11)
+    inject_invalid(plans, prob, rng)
+    want = oracle_eval(prob, plans)
+    assert (want["makespan"][want["status"] == 0] >= (1 << 32)).all()
+    ctx = wf.Ctx(prob, max_P=plans.P, device=0)
+    for _ in range(2):
+        assert_same(gpu_eval(prob, plans, k=8, ctx=ctx), want)
+    ctx.close()
+
+
 def test_repeated_calls_after_overflow():
     """A context whose batches leave 32 bits starts later calls with the u64
     sweep; every call gives the oracle's results."""
