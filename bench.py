@@ -77,10 +77,17 @@ def topk_launches(P: int, k: int) -> int:
 
 
 def kernel_source_hash() -> str:
+    """sha256 (first 16 hex digits) of the evaluation kernels' sources with
+    their comments, indentation and blank lines removed: an edit to a comment
+    keeps the recorded counters, any edit to code drops them.  (No string
+    literal in these files holds a comment marker.)"""
+    import re
     h = hashlib.sha256()
     for f in ("wf_eval.cu", "wf_sweep.cu", "wf_internal.cuh"):
-        with open(os.path.join(ROOT, "paper_2609_03335_gb300", "csrc", f), "rb") as fh:
-            h.update(fh.read())
+        with open(os.path.join(ROOT, "paper_2609_03335_gb300", "csrc", f), encoding="utf-8") as fh:
+            src = re.sub(r"/\*.*?\*/", "", fh.read(), flags=re.S)
+        lines = (re.sub(r"//.*$", "", ln).strip() for ln in src.splitlines())
+        h.update("\n".join(ln for ln in lines if ln).encode())
     return h.hexdigest()[:16]
 
 

@@ -18,8 +18,13 @@
 // with one producer warp, residency settled once for all samples, and 64
 // timing lanes, one per sample.
 //
-// Times are u32; a plan whose times reach 2^32 us is listed for the exact
-// int64 path in wf_eval.cu.
+// Times: the deterministic sweep first plays u32 times and lists a plan whose
+// times reach 2^32 us; a second instantiation with u64 times plays the listed
+// plans (or, once a context has seen most plans leave 32 bits, the whole
+// batch), with 16, 6 or 3 plans per CTA by occupancy and finish slots of 40
+// bits (a u32 word and a byte) while no time can reach 2^40 us.  Only a unit
+// whose summed run time saturates 32 bits goes on to the exact int64 path in
+// wf_eval.cu, as does a stochastic plan whose times leave 32 bits.
 //
 // A compile-time variant (kPhi) also returns the window terms of Eq. 12's
 // ranking key: residency marks a reload (a model its device held before) in
