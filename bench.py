@@ -7,9 +7,10 @@ One step = the whole hot path over one batch: readiness forecast, evaluation
 of every plan, top-k.  Inputs are resident in HBM before the timed region; L2
 is flushed (a 256 MiB write) between timed steps, which are timed one by one
 with CUDA events on the library's stream.  ``e2e`` repeats the step through
-the public call with the plans in pinned host memory, the host-to-device copy
-(into one of two device buffers, overlapping the previous step's evaluation)
-and the read-back of the top-k inside the timed region.
+wf_eval_topk_host, the C-ABI call that takes the plans in (page-locked) host
+memory and returns the top-k and the forecast there; its host-to-device copy
+(into one of two staging slots, overlapping the previous step's evaluation)
+and the read-back lie inside the timed region.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gpu|reference]
 
@@ -589,44 +590,24 @@ def run_gpu(args, rank, world, local):
     ms_per_step = max_over_ranks(float(np.mean(step_ms)), world)
     eval_ms_mean = float(np.mean(eval_ms))
 
-    # End to end through the public call: pinned host plans -> device -> top-k -> host.  Each
-    # step copies its plans into one of two device buffers on a copy stream while the previous
-    # step evaluates (a serving loop's double buffering); every step's copies and its top-k
-    # read-back lie inside the timed region.
-    pinned = {a: torch.from_numpy(np.ascontiguousarray(getattr(plans, a))).pin_memory()
-              for a in ("place", "order", "fuse", "prefetch")}
-    e2e_bufs = [wf.DevicePlans(torch.empty_like(pinned["place"], device=dev),
-                               torch.empty(pinned["order"].shape, dtype=torch.int16, device=dev),
-                               torch.empty(pinned["fuse"].shape, dtype=torch.int32, device=dev),
-                               torch.empty(pinned["prefetch"].shape, dtype=torch.int32, device=dev),
-                               plan_base=rank * P) for _ in range(2)]
-    h2d = sum(t.numel() * t.element_size() for t in pinned.values())
+    # End to end through the host-memory call: every step hands wf_eval_topk_host the batch's
+    # page-locked host rows; the library copies them into one of its two staging slots on its own
+    # copy stream (overlapping the previous step's evaluation, as a serving loop would run),
+    # forecasts, evaluates, selects the top-k and copies the top-k and the forecast back into
+    # page-locked host memory.  Every step's copies lie inside the timed region.
+    hplans = wf.DevicePlans.host(plans)
+    hplans.plan_base = rank * P
+    pad = lambda b: (b + 15) // 16 * 16
+    h2d = P * (pad(prob.N) + pad(2 * prob.N) + 2 * pad(4 * ((prob.N + 31) // 32)))
     ids_h = torch.empty(k, dtype=torch.int32).pin_memory()
     keys_h = torch.empty((k, 3), dtype=torch.int64).pin_memory()
-    d2h = ids_h.numel() * 4 + keys_h.numel() * 8
-    copy_stream = torch.cuda.Stream(device=dev)
-    copied = [torch.cuda.Event() for _ in range(2)]
-    used = [torch.cuda.Event() for _ in range(2)]
-    for ev in used:
-        ev.record(stream)
+    rel_h = torch.empty(prob.N, dtype=torch.int64).pin_memory()
+    comp_h = torch.empty(prob.N, dtype=torch.int64).pin_memory()
+    d2h = ids_h.numel() * 4 + keys_h.numel() * 8 + 2 * prob.N * 8
+    wf.wf_ctx_reserve_host(ctx)
 
     def e2e_step(i):
-        b = i % 2
-        buf = e2e_bufs[b]
-        copy_stream.wait_event(used[b])  # the evaluation that last read this buffer is done
-        with torch.cuda.stream(copy_stream):
-            buf.place.copy_(pinned["place"], non_blocking=True)
-            buf.order.copy_(pinned["order"].view(torch.int16), non_blocking=True)
-            buf.fuse.copy_(pinned["fuse"].view(torch.int32), non_blocking=True)
-            buf.prefetch.copy_(pinned["prefetch"].view(torch.int32), non_blocking=True)
-            copied[b].record(copy_stream)
-        stream.wait_event(copied[b])
-        wf.wf_forecast_readiness(ctx, rel, comp, stream)
-        wf.wf_eval_plans(ctx, buf, res, stream)
-        used[b].record(stream)
-        wf.wf_topk(ctx, res, P, k, ids, keys, stream)
-        ids_h.copy_(ids, non_blocking=True)
-        keys_h.copy_(keys, non_blocking=True)
+        wf.wf_eval_topk_host(ctx, hplans, k, ids_h, keys_h, None, rel_h, comp_h, stream)
 
     with torch.cuda.stream(stream):
         for i in range(args.warmup):
@@ -635,8 +616,7 @@ def run_gpu(args, rank, world, local):
     barrier(world)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with torch.cuda.stream(stream):
-        e0.record(stream)
-        copy_stream.wait_event(e0)  # the first step's copies start inside the timed region
+        e0.record(stream)  # (the stream is idle: the first step's copy starts after this)
         for i in range(args.steps):
             e2e_step(i)
         e1.record(stream)

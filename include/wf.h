@@ -13,6 +13,8 @@
  *   wf_forecast_readiness   release forecast of every activation (Eq. 2)
  *   wf_eval_plans           play every plan forward (Eq. 2-11) -> metrics
  *   wf_topk                 the k best plans by the ranking key
+ *   wf_eval_topk_host       forecast + evaluation + top-k from and to host memory
+ *   wf_ctx_reserve_host     allocate wf_eval_topk_host's staging up front
  *   wf_eval_plans_static    wf_eval_plans without a context or any allocation
  *   wf_static_status        device-side outcome of the last wf_eval_plans_static
  *   wf_mutate_plans         children of plans with a few point changes each
@@ -35,11 +37,14 @@
  *     load_us is [M][D].
  *   - Problem pointers are HOST pointers, read during wf_ctx_create only; the
  *     caller keeps ownership.  Plan and output pointers are DEVICE pointers
- *     owned by the caller; the library never frees them.
+ *     owned by the caller (HOST pointers for wf_eval_topk_host); the library
+ *     never frees them.
  *   - Calls taking a stream (a cudaStream_t passed as void*, NULL = the
  *     legacy default stream) are asynchronous on it and allocate nothing:
  *     the context owns every scratch buffer, sized at creation for up to
- *     max_P plans per call.  One context serves one stream at a time.
+ *     max_P plans per call (wf_eval_topk_host's staging, and the plan
+ *     constructor's state, at their first use).  One context serves one
+ *     stream at a time.
  *   - Return codes: WF_OK (0) or a WF_E* code below.  Problems with single
  *     plans are data (status bits), never return codes.
  */
@@ -210,6 +215,44 @@ int wf_eval_plans(wf_ctx *ctx, const wf_plans *plans, const wf_eval_out *out, vo
  */
 int wf_topk(wf_ctx *ctx, const wf_eval_out *res, int64_t P, int32_t k,
             int32_t *ids_dev, int64_t *keys_dev, void *stream);
+
+/*
+ * One step of the hot path from and to HOST memory: copy a batch of plans
+ * in, optionally forecast readiness (as wf_forecast_readiness), evaluate the
+ * batch (as wf_eval_plans) and select its k best (as wf_topk), then copy the
+ * results out.  host_plans has the layout of wf_plans, but its five arrays
+ * are HOST pointers (retain may be NULL); its strides need only be >= the
+ * row sizes and multiples of 16 bytes.  ids_host: int32 [k]; keys_host: int64
+ * [k][3] or NULL; out_host: every plan's metrics and status ([P] each, HOST
+ * pointers) or NULL; rel_host / comp_host: int64 [N] each, both or neither
+ * (neither: no forecast).  1 <= k <= min(P, 1024), P <= max_P.
+ *
+ * The context copies the plans into one of two device staging slots on a
+ * copy stream of its own, and calls alternate between the slots, so a call's
+ * copy overlaps the previous call's evaluation on `stream`; each copy first
+ * waits for the evaluation that last read its slot.  The results are in host
+ * memory once `stream` has passed the call (synchronize or record an event
+ * after it).  The host plan arrays must stay unchanged until the call's copy
+ * has run (at the latest, when `stream` has passed the call).  Host memory
+ * should be page-locked (cudaHostAlloc, or a pinned torch tensor); pageable
+ * memory works, but then its copies do not overlap the GPU's work.  Under
+ * stream capture the copies go on `stream` itself (page-locked memory
+ * only).  The device results, top-k and forecast buffers are single, so the
+ * calls on one context must all use one stream.  The staging (two slots of
+ * max_P plan rows, the results, the forecast) is allocated by the first call
+ * or by wf_ctx_reserve_host, and freed with the context.  Returns WF_OK,
+ * WF_EINVAL, WF_ENOMEM or WF_ECUDA.
+ */
+int wf_eval_topk_host(wf_ctx *ctx, const wf_plans *host_plans, int32_t k, int32_t *ids_host,
+                      int64_t *keys_host, const wf_eval_out *out_host, int64_t *rel_host,
+                      int64_t *comp_host, void *stream);
+
+/*
+ * Allocate wf_eval_topk_host's staging now (see above), so that no call of
+ * it allocates.  Returns WF_OK, WF_ENOMEM or WF_ECUDA; a second call does
+ * nothing.
+ */
+int wf_ctx_reserve_host(wf_ctx *ctx);
 
 /*
  * The paper has no counterpart to this entry point; it serves callers that

@@ -11,7 +11,7 @@ ROOT = os.path.dirname(HERE)
 LIB = os.path.join(HERE, "libwf.so")
 OBJ = os.path.join(HERE, "_build")
 SOURCES = ["wf_ctx.cu", "wf_slots.cpp", "wf_forecast.cu", "wf_eval.cu", "wf_sweep.cu", "wf_topk.cu",
-           "wf_search.cu", "wf_construct.cu"]
+           "wf_search.cu", "wf_construct.cu", "wf_host.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",
          "--expt-relaxed-constexpr", "-I", os.path.join(ROOT, "include")]

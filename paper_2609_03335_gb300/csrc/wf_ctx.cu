@@ -409,6 +409,7 @@ extern "C" void wf_ctx_destroy(wf_ctx *c)
     int prev = -1;
     cudaGetDevice(&prev);
     cudaSetDevice(c->device);
+    wf_host_release(c);
     if (c->tables) cudaFree(c->tables);
     if (c->eval_scratch) cudaFree(c->eval_scratch);
     if (c->topk_scratch) cudaFree(c->topk_scratch);

@@ -106,7 +106,11 @@ struct wf_ctx {
     cudaEvent_t sweep_done;     // recorded on the caller's stream after the sweeps
     cudaEvent_t ovf_event;      // recorded on side after the read-back
     cudaStream_t side;          // the read-back's own stream, off the caller's critical path
+    struct wf_host_stage *host; // wf_eval_topk_host's staging (wf_host.cu), made by its first use
 };
+
+// Frees wf_eval_topk_host's staging once its copies have finished (wf_host.cu).
+void wf_host_release(wf_ctx *c);
 
 // Static slot assignment (wf_slots.cpp).  Fills rslot code per node, write
 // lists (CSR) and returns the slot count, or -1 when it exceeds 32767.

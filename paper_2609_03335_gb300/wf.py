@@ -26,7 +26,7 @@ EXPORTS = ("wf_problem_check", "wf_ctx_create", "wf_forecast_readiness", "wf_eva
            "wf_eval_plans_static", "wf_mutate_plans", "wf_merge_elite", "wf_local_search",
            "wf_construct_plans", "wf_ctx_set_reclaim", "wf_ctx_check_wait_expiry", "wf_eval_plans_phi",
            "wf_topk_phi", "wf_static_status", "wf_ctx_set_eval_path",
-           "wf_ctx_set_batch")
+           "wf_ctx_set_batch", "wf_eval_topk_host", "wf_ctx_reserve_host")
 
 
 class WfError(RuntimeError):
@@ -96,6 +96,8 @@ def load_library():
         "wf_static_status": ([p], ctypes.c_int),
         "wf_ctx_set_eval_path": ([p, i32], ctypes.c_int),
         "wf_ctx_set_batch": ([p, i32], ctypes.c_int),
+        "wf_eval_topk_host": ([p, p, i32, p, p, p, p, p, p], ctypes.c_int),
+        "wf_ctx_reserve_host": ([p], ctypes.c_int),
     }
     for name, (args, res) in sig.items():
         f = getattr(lib, name)
@@ -273,6 +275,22 @@ class DevicePlans:
         return out
 
     @staticmethod
+    def host(plans, pin: bool = True):
+        """The rows of a wfgen.Plans batch as host tensors (page-locked unless
+        pin=False) for wf_eval_topk_host."""
+        import torch
+
+        def t(x):
+            if x is None:
+                return None
+            h = torch.from_numpy(np.ascontiguousarray(x))
+            return h.pin_memory() if pin else h
+        return DevicePlans(t(plans.place), t(plans.order.view(np.int16)), t(plans.fuse.view(np.int32)),
+                           t(plans.prefetch.view(np.int32)), t(None if plans.retain is None
+                                                               else plans.retain.view(np.int32)),
+                           plan_base=getattr(plans, "plan_base", 0))
+
+    @staticmethod
     def from_host(plans, device="cuda", non_blocking=False):
         import torch
 
@@ -299,14 +317,17 @@ class DevicePlans:
 
 
 class Results:
-    """Per-plan outputs on the device."""
+    """Per-plan outputs on the device (or, with device="cpu", in host memory,
+    page-locked unless pin=False, for wf_eval_topk_host)."""
 
-    def __init__(self, P: int, device="cuda"):
+    def __init__(self, P: int, device="cuda", pin: bool = True):
         import torch
-        self.makespan = torch.empty(P, dtype=torch.int64, device=device)
-        self.p95 = torch.empty(P, dtype=torch.int64, device=device)
-        self.gpu = torch.empty(P, dtype=torch.int64, device=device)
-        self.status = torch.empty(P, dtype=torch.int32, device=device)
+        mk = lambda dt: torch.empty(P, dtype=dt, device=device)
+        self.makespan, self.p95, self.gpu, self.status = (mk(torch.int64), mk(torch.int64), mk(torch.int64),
+                                                          mk(torch.int32))
+        if torch.device(device).type == "cpu" and pin:
+            self.makespan, self.p95, self.gpu, self.status = (t.pin_memory() for t in
+                                                              (self.makespan, self.p95, self.gpu, self.status))
 
     def c(self, offset: int = 0) -> wf_eval_out:
         return wf_eval_out(self.makespan.data_ptr() + 8 * offset, self.p95.data_ptr() + 8 * offset,
@@ -315,6 +336,24 @@ class Results:
     def numpy(self):
         return (self.makespan.cpu().numpy(), self.p95.cpu().numpy(), self.gpu.cpu().numpy(),
                 self.status.cpu().numpy().view(np.uint32))
+
+
+def wf_eval_topk_host(ctx: Ctx, plans: DevicePlans, k: int, ids, keys=None, out: Results | None = None,
+                      rel=None, comp=None, stream=None):
+    """One step from and to host memory: plans, ids [k] int32, keys [k, 3]
+    int64, out (Results on "cpu") and the forecast rel / comp [N] int64 are
+    HOST tensors (page-locked for overlap).  Asynchronous on `stream`: the
+    results are there once the stream has passed the call."""
+    pl = plans.c()
+    oc = None if out is None else out.c()
+    ptr = lambda t: None if t is None else t.data_ptr()
+    _check(load_library().wf_eval_topk_host(ctx.ptr, ctypes.byref(pl), int(k), ptr(ids), ptr(keys),
+                                            None if oc is None else ctypes.byref(oc), ptr(rel), ptr(comp),
+                                            _stream_handle(stream)), "wf_eval_topk_host")
+
+
+def wf_ctx_reserve_host(ctx: Ctx):
+    _check(load_library().wf_ctx_reserve_host(ctx.ptr), "wf_ctx_reserve_host")
 
 
 def wf_eval_plans(ctx: Ctx, plans: DevicePlans, out: Results, stream=None, P: int | None = None,
