@@ -77,19 +77,33 @@ def topk_launches(P: int, k: int) -> int:
     return 1 if P <= 16384 else 3
 
 
-def kernel_source_hash() -> str:
-    """sha256 (first 16 hex digits) of the evaluation kernels' sources with
-    their comments, indentation and blank lines removed: an edit to a comment
-    keeps the recorded counters, any edit to code drops them.  (No string
-    literal in these files holds a comment marker.)"""
+def kernel_code(files: dict) -> str:
+    """The evaluation kernels' code from the sources {name: text}: wf_eval.cu
+    and wf_sweep.cu whole, and of wf_internal.cuh the device problem record
+    and the #defines (the rest of that header is host-side: the context
+    record and the launchers' declarations); comments, indentation and blank
+    lines removed.  (No string literal in these files holds a comment marker.)"""
     import re
-    h = hashlib.sha256()
+    hdr = files["wf_internal.cuh"]
+    rec = re.search(r"struct wf_dev_problem \{.*?\n\};", hdr, flags=re.S)
+    parts = [files["wf_eval.cu"], files["wf_sweep.cu"], rec.group(0) if rec else hdr,
+             "\n".join(ln for ln in hdr.splitlines() if ln.startswith("#define"))]
+    out = []
+    for src in parts:
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        out += [ln for ln in (re.sub(r"//.*$", "", ln).strip() for ln in src.splitlines()) if ln]
+    return "\n".join(out)
+
+
+def kernel_source_hash() -> str:
+    """sha256 (first 16 hex digits) of kernel_code(): an edit to a comment or
+    to host-side declarations keeps the recorded counters, any edit to the
+    kernels' code drops them."""
+    files = {}
     for f in ("wf_eval.cu", "wf_sweep.cu", "wf_internal.cuh"):
         with open(os.path.join(ROOT, "paper_2609_03335_gb300", "csrc", f), encoding="utf-8") as fh:
-            src = re.sub(r"/\*.*?\*/", "", fh.read(), flags=re.S)
-        lines = (re.sub(r"//.*$", "", ln).strip() for ln in src.splitlines())
-        h.update("\n".join(ln for ln in lines if ln).encode())
-    return h.hexdigest()[:16]
+            files[f] = fh.read()
+    return hashlib.sha256(kernel_code(files).encode()).hexdigest()[:16]
 
 
 def read_peaks() -> dict:
