@@ -5,7 +5,7 @@ copy peak.
 
 One step = the whole hot path over one batch: readiness forecast, evaluation
 of every plan, top-k.  Inputs are resident in HBM before the timed region; L2
-is flushed (a 256 MiB write) between timed steps, which are timed one by one
+is flushed (a 256 MiB write, read back) between timed steps, which are timed one by one
 with CUDA events on the library's stream.  ``e2e`` repeats the step through
 wf_eval_topk_host, the C-ABI call that takes the plans in (page-locked) host
 memory and returns the top-k and the forecast there; its host-to-device copy
@@ -104,6 +104,14 @@ def kernel_source_hash() -> str:
         with open(os.path.join(ROOT, "paper_2609_03335_gb300", "csrc", f), encoding="utf-8") as fh:
             files[f] = fh.read()
     return hashlib.sha256(kernel_code(files).encode()).hexdigest()[:16]
+
+
+def flush_l2(buf):
+    """Flush L2 before a timed step: write the 256 MiB buffer (larger than
+    L2), then read it back, so the write-backs of its dirty lines happen here
+    and the step starts with a cold L2 of clean lines (none of its inputs)."""
+    buf.zero_()
+    buf.amax()
 
 
 def read_peaks() -> dict:
@@ -267,11 +275,11 @@ def local_search_timing(wf, ctx, dp, prob, P, stream, flush, peak_gbs, k=32, rou
         e = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
         mut = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(5)]
         for r, (a, b) in enumerate(mut):
-            flush.zero_()
+            flush_l2(flush)
             a.record(stream)
             wf.wf_mutate_plans(ctx, elite, kids, seed=7, round_=1 + r, n_ops=3, stream=stream)
             b.record(stream)
-        flush.zero_()
+        flush_l2(flush)
         e[2].record(stream)
         wf.wf_local_search(ctx, elite, er, kids, kr, seed=7, round0=2, rounds=rounds, n_ops=3, stream=stream)
         e[3].record(stream)
@@ -302,7 +310,7 @@ def construct_timing(wf, ctx, prob, P, k, stream, flush, random_best, jitter=200
     e = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
     with torch.cuda.stream(stream):
         wf.wf_construct_plans(ctx, out, seed=11, jitter_us=jitter, stream=stream)  # first call allocates
-        flush.zero_()
+        flush_l2(flush)
         e[0].record(stream)
         wf.wf_construct_plans(ctx, out, seed=12, jitter_us=jitter, stream=stream)
         e[1].record(stream)
@@ -346,7 +354,7 @@ def reclaim_timing(wf, ctx, dp, res_lru, P, stream, flush):
     e = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
     with torch.cuda.stream(stream):
         wf.wf_eval_plans(ctx, dp, res, stream)
-        flush.zero_()
+        flush_l2(flush)
         e[0].record(stream)
         wf.wf_eval_plans(ctx, dp, res, stream)
         e[1].record(stream)
@@ -375,7 +383,7 @@ def phi_timing(wf, ctx, dp, P, k, stream, flush):
         wf.wf_eval_plans_phi(ctx, dp, res, timely, life, stream)
         for _ in range(3):
             e = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
-            flush.zero_()
+            flush_l2(flush)
             e[0].record(stream)
             wf.wf_eval_plans_phi(ctx, dp, res, timely, life, stream)
             e[1].record(stream)
@@ -415,7 +423,7 @@ def workload_entry(name, wf, dev, steps=5, warmup=3, with_cpu=True):
     stream = torch.cuda.Stream(device=dev)
     with torch.cuda.stream(stream):
         for _ in range(warmup):
-            flush.zero_()
+            flush_l2(flush)
             wf.wf_forecast_readiness(ctx, rel, comp, stream)
             wf.wf_eval_plans(ctx, dp, res, stream)
             wf.wf_topk(ctx, res, P, k, ids, keys, stream)
@@ -427,7 +435,7 @@ def workload_entry(name, wf, dev, steps=5, warmup=3, with_cpu=True):
     torch.cuda.synchronize()
     with torch.cuda.stream(stream):
         for e in ev:
-            flush.zero_()
+            flush_l2(flush)
             e[0].record(stream)
             wf.wf_forecast_readiness(ctx, rel, comp, stream)
             e[1].record(stream)
@@ -488,7 +496,7 @@ def batch_timing(wf, prob, dp, P, dev, flush, limits=(1, 2, 4), reps=3):
         wf.wf_ctx_set_batch(ctx, B)
         ts = []
         for _ in range(reps):
-            flush.zero_()
+            flush_l2(flush)
             a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             a.record()
             wf.wf_eval_plans(ctx, dp, res)
@@ -526,7 +534,7 @@ def static_timing(wf, prob, plans, dev, flush, reps=5):
     out = wf.Results(fit, dev)
     ts = []
     for _ in range(reps):
-        flush.zero_()
+        flush_l2(flush)
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record()
         wf.wf_eval_plans_static(dprob, dp, out)
@@ -573,7 +581,7 @@ def run_gpu(args, rank, world, local):
 
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
-            flush.zero_()
+            flush_l2(flush)
             step()
     wf.wf_ctx_status(ctx, stream)
 
@@ -585,7 +593,7 @@ def run_gpu(args, rank, world, local):
     torch.cuda.synchronize()
     with torch.cuda.stream(stream):
         for s in range(args.steps):
-            flush.zero_()
+            flush_l2(flush)
             e = ev[s]
             e[0].record(stream)
             wf.wf_forecast_readiness(ctx, rel, comp, stream)
@@ -680,7 +688,7 @@ def run_gpu(args, rank, world, local):
             "data": "synthetic",
             "config": {"workload": f"{WORKLOAD}: {w.description} plans per GPU (here {P}), k={k}",
                        "P_per_gpu": P, "N": prob.N, "k": k,
-                       "l2": "flushed between timed steps (256 MiB write)",
+                       "l2": "flushed between timed steps (256 MiB write, then read back)",
                        "ctx_create_ms": ctx_ms,
                        "stage_ms": {"forecast": forecast_ms, "eval": eval_ms_mean, "topk": topk_ms}},
             "e2e": {"value": P * world / (e2e_ms * 1e-3), "unit": "plans/s",
