@@ -233,7 +233,10 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
         noderec[2 * n + 1] = make_int4(a, len, (int32_t)(c0 | (c1 << 16)), 0);
         for (int32_t d = 0; d < D; ++d) {
             const int64_t i = (int64_t)n * D + d;
-            lk[i] = make_int2(pb->lat_us[i], adm[i] - pb->weight_mib[pb->model[n]]);
+            // KV admission, or -1 where the activation does not fit the device
+            // (Eq. 8): the sweep's producers read the pair for every unit anyway.
+            lk[i] = make_int2(pb->lat_us[i],
+                              adm[i] <= pb->cap_mib[d] ? adm[i] - pb->weight_mib[pb->model[n]] : -1);
         }
     }
     size_t o_rec = img.add(noderec.data(), sizeof(int4) * noderec.size());

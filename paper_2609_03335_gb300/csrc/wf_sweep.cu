@@ -157,6 +157,10 @@ constexpr uint32_t kPrefetch = 1u << 9;
 constexpr uint32_t kWasEmpty = 1u << 10;   // after residency: a miss on an empty device
 constexpr uint32_t kEmptied = 1u << 15;    // after residency: the unit's reclaim empties the device
 constexpr uint32_t kRunCap = 0xFFFFFFFFu;  // saturation of w0
+// A plan's open word in shared memory: the devices still occupied at its end
+// (residency, low bits) and, from bit kOpenBad, the placement status bits
+// (WF_ST_DEVICE, WF_ST_CAPACITY) its producers found.
+constexpr int kOpenBad = 24;
 
 // Residency lanes per plan: a device group each (d = g mod kG), or one lane
 // for every device under reclamation by next use.
@@ -372,6 +376,13 @@ __device__ __forceinline__ const uint32_t *bits_row(const uint32_t *base, int64_
     return (const uint32_t *)((const uint8_t *)base + boff);
 }
 
+// Bulk prefetch of [p, p + bytes) into L2 (p 16-byte aligned, bytes a
+// multiple of 16); no completion to wait for.
+__device__ __forceinline__ void l2_prefetch(const void *p, uint32_t bytes)
+{
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+
 // The records of kI (plan, position) pairs at once, with the gathers of all
 // pairs issued together in three dependent rounds: the head's own tables
 // (placement, node record, fusion / prefetch / retain words, third and
@@ -383,10 +394,10 @@ __device__ __forceinline__ const uint32_t *bits_row(const uint32_t *base, int64_
 template <int kI, int kPitch>
 __device__ __forceinline__ void produce_batch(const wf_dev_problem &dp, const wf_plans &pl, const RowPtrs *rp,
                                               const bool *act, const int32_t *hh, uint2 *rb, int pos,
-                                              const int *qq, uint32_t *dev)
+                                              const int *qq, uint32_t *dev, uint32_t *open)
 {
     const int32_t D = dp.D;
-    uint32_t d[kI], fw[kI], pw[kI], rw[kI], c2[kI];
+    uint32_t d[kI], fw[kI], pw[kI], rw[kI], c2[kI], bad[kI];
     uint4 hr[kI];
 #pragma unroll
     for (int j = 0; j < kI; ++j) {
@@ -397,6 +408,15 @@ __device__ __forceinline__ void produce_batch(const wf_dev_problem &dp, const wf
         pw[j] = act[j] ? __ldg(bits_row(pl.prefetch, rp[j].boff) + (h >> 5)) : 0u;
         rw[j] = act[j] && pl.retain ? __ldg(bits_row(pl.retain, rp[j].boff) + (h >> 5)) : 0xFFFFFFFFu;
         c2[j] = act[j] ? __ldg(dp.wc23 + h) : 0u;
+    }
+    // Placement and fit (Eq. 8) of every position's activation: a device
+    // index beyond D here, a device it does not fit (KV entry -1 in lk) with
+    // the next gathers.  A plan with either gets the status bits, and the
+    // record a skip, so no later stage indexes by it.
+#pragma unroll
+    for (int j = 0; j < kI; ++j) {
+        bad[j] = act[j] && d[j] >= (uint32_t)D ? (uint32_t)WF_ST_DEVICE : 0u;
+        if (bad[j]) d[j] = 0u;
     }
     int2 lk0[kI];
     uint32_t pprev[kI], fnx[kI], pnx[kI];
@@ -415,7 +435,9 @@ __device__ __forceinline__ void produce_batch(const wf_dev_problem &dp, const wf
         uint2 *dst = rb + pos * kPitch + qq[j];
         const int32_t h = hh[j];
         const uint32_t s0 = hr[j].x >> 16;
-        if (!act[j] || (((fw[j] >> (h & 31)) & 1u) && pprev[j] == d[j])) {  // no unit, or inside its head's
+        if (act[j] && !bad[j] && lk0[j].y < 0) bad[j] = (uint32_t)WF_ST_CAPACITY;  // (d was cleared for a bad device)
+        if (bad[j]) atomicOr(open + qq[j], bad[j] << kOpenBad);
+        if (!act[j] || bad[j] || (((fw[j] >> (h & 31)) & 1u) && pprev[j] == d[j])) {  // no unit, or inside its head's
             dst[0] = make_uint2(0u, 0u);
             dst[1 * kChunk * kPitch] = make_uint2(0u, kSkip);
             dst[2 * kChunk * kPitch] = make_uint2(0u, 0u);
@@ -424,11 +446,13 @@ __device__ __forceinline__ void produce_batch(const wf_dev_problem &dp, const wf
         uint32_t run = (uint32_t)lk0[j].x + (uint32_t)dp.grant, ovf = 0;  // both < 2^31: no wrap
         int32_t kv = lk0[j].y, tail = h;
         uint32_t ty = hr[j].y, tw = hr[j].w, c2t = c2[j], rwt = rw[j];
+        uint32_t cbad = 0;  // a member that does not fit the head's device
         if (s0 != 0xFFFFu && ((fnx[j] >> (s0 & 31)) & 1u) && pnx[j] == d[j]) {  // Eq. 3 chain
             const uint32_t *fuse = bits_row(pl.fuse, rp[j].boff);
             for (uint32_t s = s0; s != 0xFFFFu;) {
                 if (s != s0 && (!bit_of_g(fuse, s) || __ldg(rp[j].place + s) != d[j])) break;
                 const int2 lk = __ldg(dp.lk + s * D + d[j]);
+                cbad |= lk.y < 0;
                 const uint4 sr = __ldg(dp.hrec + s);
                 const uint32_t r2 = run + (uint32_t)lk.x;
                 ovf |= r2 < run;
@@ -441,6 +465,13 @@ __device__ __forceinline__ void produce_batch(const wf_dev_problem &dp, const wf
             }
             c2t = __ldg(dp.wc23 + tail);
             rwt = pl.retain ? __ldg(bits_row(pl.retain, rp[j].boff) + (tail >> 5)) : 0xFFFFFFFFu;
+        }
+        if (cbad) {  // (the member's own position flags the plan as well)
+            atomicOr(open + qq[j], (uint32_t)WF_ST_CAPACITY << kOpenBad);
+            dst[0] = make_uint2(0u, 0u);
+            dst[1 * kChunk * kPitch] = make_uint2(0u, kSkip);
+            dst[2 * kChunk * kPitch] = make_uint2(0u, 0u);
+            continue;
         }
         const uint32_t nwl = (ty >> 20) & 7u;
         const uint32_t pf = (pw[j] >> (h & 31)) & 1u;
@@ -587,6 +618,18 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
                 rp[j].boff = pq * pl.bits_stride;
             }
         }
+        // The node-indexed rows (placement, fusion and prefetch bits) are
+        // gathered all through the sweep; one bulk L2 prefetch per row up
+        // front streams them in rather than sector by sector.  (Rows are
+        // 16-byte aligned, and their 16-byte-rounded sizes fit the strides.)
+        const uint32_t place_bytes = (uint32_t)((N + 15) & ~15), bits_bytes = (uint32_t)((((N + 31) >> 5) * 4 + 15) & ~15);
+#pragma unroll
+        for (int j = 0; j < kIters; ++j)
+            if (pos == 0 && okq[j]) {
+                l2_prefetch(rp[j].place, place_bytes);
+                l2_prefetch(bits_row(pl.fuse, rp[j].boff), bits_bytes);
+                l2_prefetch(bits_row(pl.prefetch, rp[j].boff), bits_bytes);
+            }
         // Dispatch entries are read one chunk ahead of their use.
         int32_t h0[kIters];
 #pragma unroll
@@ -610,7 +653,7 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
                         make_uint2(act[j] ? (uint32_t)__ldg(dp.nextuse + qplan[j] * (int64_t)N + i) : 0xFFFFu, 0u);
             }
             uint32_t dev[kIters];
-            produce_batch<kIters, kPitch>(dp, pl, rp, act, h0, rb, pos, qq, dev);
+            produce_batch<kIters, kPitch>(dp, pl, rp, act, h0, rb, pos, qq, dev, open);
             // For each residency lane, the chunk's units on its devices: one
             // ballot per device group; each half-warp holds one plan.
 #pragma unroll
@@ -876,7 +919,12 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
     }
     if (kNarrow) ovf |= end == (TT)kRunCap;
     named_sync(kOpen, kResThreads + 32);  // the residency stage's final device counts
-    if (live && ovf) {  // handed to the next path
+    const uint32_t bad = live ? open[lane] >> kOpenBad : 0u;  // placement bits found by the producers
+    if (bad) {  // an invalid plan: its status bits and INT64_MAX metrics
+        out.status[p] = bad;
+        out.makespan_us[p] = out.p95_us[p] = out.gpu_us[p] = WF_INF64;
+        if (kPhi) dp.phi_timely[p] = dp.phi_life[p] = WF_INF64;
+    } else if (live && ovf) {  // handed to the next path
         const int32_t kk = atomicAdd(ovf_count, 1);
         ovf_list[kk] = (int32_t)p;
     } else if (live) {
@@ -1248,7 +1296,7 @@ __host__ __device__ inline uint32_t status_warp_bytes(int32_t N)
 
 // kByte: every device index is below 8, so one byte per node holds its fit
 // mask (fit8): a quarter of the table reads of the 32-bit masks.
-template <bool kByte, int kU>
+template <bool kByte, int kU, bool kPlace>
 __global__ void __launch_bounds__(128)
 status_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out)
 {
@@ -1271,51 +1319,6 @@ status_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out)
         // Every loop issues kU 16-byte reads per lane before it uses any: on
         // long rows a warp keeps a plan's reads in flight rather than one
         // round trip per 512 bytes (kU = 1 on short rows, whose loops run once).
-        for (int32_t b16 = 16 * lane; b16 < N; b16 += kU * 512) {
-            uint4 pw[kU], fb[kU], fm[kU][4];
-#pragma unroll
-            for (int u = 0; u < kU; ++u) {
-                const int32_t n16 = b16 + 512 * u;
-                const bool in = n16 < N;
-                pw[u] = in ? __ldg((const uint4 *)(place + n16)) : make_uint4(0u, 0u, 0u, 0u);
-                if (kByte) {
-                    fb[u] = in ? __ldg((const uint4 *)(dp.fit8 + n16)) : make_uint4(0u, 0u, 0u, 0u);
-                } else {
-#pragma unroll
-                    for (int q = 0; q < 4; ++q)
-                        fm[u][q] = in ? __ldg((const uint4 *)(dp.fitmask + n16 + 4 * q)) : make_uint4(0u, 0u, 0u, 0u);
-                }
-            }
-#pragma unroll
-            for (int u = 0; u < kU; ++u) {
-                const int32_t n16 = b16 + 512 * u;
-                const uint32_t pws[4] = {pw[u].x, pw[u].y, pw[u].z, pw[u].w};
-                if (kByte) {
-                    const uint32_t fbs[4] = {fb[u].x, fb[u].y, fb[u].z, fb[u].w};
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-#pragma unroll
-                        for (int j = 0; j < 4; ++j) {
-                            const uint32_t d = (pws[q] >> (8 * j)) & 255u, f = (fbs[q] >> (8 * j)) & 255u;
-                            if (n16 + 4 * q + j < N)
-                                st |= d >= (uint32_t)D ? WF_ST_DEVICE
-                                                       : (((f >> (d & 7u)) & 1u) ? 0u : WF_ST_CAPACITY);
-                        }
-                    }
-                } else {
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const uint32_t f[4] = {fm[u][q].x, fm[u][q].y, fm[u][q].z, fm[u][q].w};
-#pragma unroll
-                        for (int j = 0; j < 4; ++j) {
-                            const uint32_t d = (pws[q] >> (8 * j)) & 255u;
-                            if (n16 + 4 * q + j < N)
-                                st |= d >= (uint32_t)D ? WF_ST_DEVICE : (((f[j] >> d) & 1u) ? 0u : WF_ST_CAPACITY);
-                        }
-                    }
-                }
-            }
-        }
         // The inverse permutation, 8 dispatch entries a lane at a time, then
         // read back: a repeated node leaves some entry unmatched.
         for (int32_t b8 = 8 * lane; b8 < N; b8 += kU * 256) {
@@ -1372,6 +1375,57 @@ status_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out)
             }
             st = __reduce_or_sync(0xFFFFFFFFu, st);
         }
+        // Placement and fit (Eq. 8): here when asked (kPlace), else only for
+        // a plan whose order is already invalid; the sweep's producers check
+        // the placement of every other plan as they read it.
+        if (kPlace || st) {
+            for (int32_t b16 = 16 * lane; b16 < N; b16 += kU * 512) {
+                uint4 pw[kU], fb[kU], fm[kU][4];
+#pragma unroll
+                for (int u = 0; u < kU; ++u) {
+                    const int32_t n16 = b16 + 512 * u;
+                    const bool in = n16 < N;
+                    pw[u] = in ? __ldg((const uint4 *)(place + n16)) : make_uint4(0u, 0u, 0u, 0u);
+                    if (kByte) {
+                        fb[u] = in ? __ldg((const uint4 *)(dp.fit8 + n16)) : make_uint4(0u, 0u, 0u, 0u);
+                    } else {
+#pragma unroll
+                        for (int q = 0; q < 4; ++q)
+                            fm[u][q] = in ? __ldg((const uint4 *)(dp.fitmask + n16 + 4 * q)) : make_uint4(0u, 0u, 0u, 0u);
+                    }
+                }
+#pragma unroll
+                for (int u = 0; u < kU; ++u) {
+                    const int32_t n16 = b16 + 512 * u;
+                    const uint32_t pws[4] = {pw[u].x, pw[u].y, pw[u].z, pw[u].w};
+                    if (kByte) {
+                        const uint32_t fbs[4] = {fb[u].x, fb[u].y, fb[u].z, fb[u].w};
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+#pragma unroll
+                            for (int j = 0; j < 4; ++j) {
+                                const uint32_t d = (pws[q] >> (8 * j)) & 255u, f = (fbs[q] >> (8 * j)) & 255u;
+                                if (n16 + 4 * q + j < N)
+                                    st |= d >= (uint32_t)D ? WF_ST_DEVICE
+                                                           : (((f >> (d & 7u)) & 1u) ? 0u : WF_ST_CAPACITY);
+                            }
+                        }
+                    } else {
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            const uint32_t f[4] = {fm[u][q].x, fm[u][q].y, fm[u][q].z, fm[u][q].w};
+#pragma unroll
+                            for (int j = 0; j < 4; ++j) {
+                                const uint32_t d = (pws[q] >> (8 * j)) & 255u;
+                                if (n16 + 4 * q + j < N)
+                                    st |= d >= (uint32_t)D ? WF_ST_DEVICE : (((f[j] >> d) & 1u) ? 0u : WF_ST_CAPACITY);
+                            }
+                        }
+                    }
+                }
+            }
+        }
+        st = __reduce_or_sync(0xFFFFFFFFu, st);
         if (lane == 0) {
             out.status[p] = st;
             if (st) out.makespan_us[p] = out.p95_us[p] = out.gpu_us[p] = WF_INF64;
@@ -1381,27 +1435,38 @@ status_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out)
     }
 }
 
-template <bool kByte, int kU>
+template <bool kByte, int kU, bool kPlace>
 int launch_status_as(const wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, cudaStream_t st)
 {
     const wf_dev_problem &dp = ctx->dp;
     const size_t wbytes = status_warp_bytes(dp.N);
     const int swarps = (int)std::max<size_t>(1, std::min<size_t>(4, (227 * 1024) / wbytes));
     const size_t ssmem = wbytes * swarps;
-    int rc = wf_cuda_check(cudaFuncSetAttribute(status_kernel<kByte, kU>,
+    int rc = wf_cuda_check(cudaFuncSetAttribute(status_kernel<kByte, kU, kPlace>,
                                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ssmem),
                            "status smem attribute");
     if (rc) return rc;
     const int64_t sblocks = std::min<int64_t>((pl->P + swarps - 1) / swarps, (int64_t)ctx->sms * 16);
-    status_kernel<kByte, kU><<<(unsigned)sblocks, 32 * swarps, ssmem, st>>>(dp, *pl, *out);
+    status_kernel<kByte, kU, kPlace><<<(unsigned)sblocks, 32 * swarps, ssmem, st>>>(dp, *pl, *out);
     return WF_OK;
 }
 
-int launch_status(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, cudaStream_t st)
+template <bool kPlace>
+int launch_status_p(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, cudaStream_t st)
 {
     const bool byte = ctx->dp.D <= 8, wide = ctx->dp.N >= 1024;
-    if (wide) return byte ? launch_status_as<true, 4>(ctx, pl, out, st) : launch_status_as<false, 4>(ctx, pl, out, st);
-    return byte ? launch_status_as<true, 1>(ctx, pl, out, st) : launch_status_as<false, 1>(ctx, pl, out, st);
+    if (wide)
+        return byte ? launch_status_as<true, 4, kPlace>(ctx, pl, out, st)
+                    : launch_status_as<false, 4, kPlace>(ctx, pl, out, st);
+    return byte ? launch_status_as<true, 1, kPlace>(ctx, pl, out, st)
+                : launch_status_as<false, 1, kPlace>(ctx, pl, out, st);
+}
+
+// The status pass; with place false the placement and fit checks of a plan
+// whose order is valid are left to the deterministic sweep's producers.
+int launch_status(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, cudaStream_t st, bool place)
+{
+    return place ? launch_status_p<true>(ctx, pl, out, st) : launch_status_p<false>(ctx, pl, out, st);
 }
 
 }  // namespace
@@ -1423,7 +1488,7 @@ int wf_launch_stoch(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, siz
                     int32_t *ovf_list, int32_t *ovf_count, cudaStream_t st)
 {
     const wf_dev_problem &dp = ctx->dp;
-    int rc = launch_status(ctx, pl, out, st);
+    int rc = launch_status(ctx, pl, out, st, true);
     if (rc) return rc;
     const unsigned blocks = (unsigned)pl->P;
     if (dp.M <= 8) {
@@ -1639,7 +1704,9 @@ int wf_launch_sweep(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, con
                     bool wide_first, int32_t *counts, int32_t *list1, int32_t *list2, cudaStream_t st,
                     const int32_t **rest_list, const int32_t **rest_count)
 {
-    int rc = launch_status(ctx, pl, out, st);
+    // The next-use pass reads every plan's placement before the sweep, so
+    // under that policy the status pass checks placement itself.
+    int rc = launch_status(ctx, pl, out, st, ctx->dp.reclaim != 0);
     if (!rc && ctx->dp.reclaim) rc = wf_launch_nextuse(ctx, pl, out, st);
     if (rc) return rc;
     if (cfg.smem32 && !(wide_first && cfg.smem64)) {
