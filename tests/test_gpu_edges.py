@@ -198,3 +198,39 @@ def test_bounded_wait_expiry_is_reported():
     wf.wf_ctx_status(ctx)
     for a, b in zip(res.numpy(), oracle.eval_plans(w.problem, host)):
         assert np.array_equal(a, b)
+
+
+@pytest.mark.parametrize("reclaim", [0, 1])
+def test_placement_errors_found_by_the_sweep(reclaim):
+    """Placement and fit errors the sweep's producers find (the status pass
+    checks only the order of such plans): a fused chain member that does not
+    fit its head's device, a device index beyond D, valid plans beside them.
+    Under next-use reclamation the status pass checks placement itself."""
+    N, D = 15, 2
+    prob = chains_window([5, 5, 5], D=D, M=1, seed=9)  # one model: every chain edge is fusible
+    peak = np.full((N, D), 3, np.int32)
+    peak[2, 0] = peak[7, 0] = 20  # nodes 2 and 7 fit device 1 only
+    prob = prob.with_(peak_mib=peak.reshape(-1), cap_mib=np.array([12, 30], np.int32), reclaim=reclaim)
+    P = 96
+    plans = wfgen.Plans.empty(P, N)
+    rng = np.random.default_rng(3)
+    for p in range(P):
+        nxt, order = [0, 5, 10], []
+        while len(order) < N:  # the three chains interleaved in a random order
+            c = int(rng.choice([i for i in range(3) if nxt[i] < 5 * i + 5]))
+            order.append(nxt[c])
+            nxt[c] += 1
+        plans.order[p, :N] = order
+        place = rng.integers(0, D, size=N)
+        if p % 4 == 0:
+            place[:] = 0  # whole chains fused on device 0, with members 2 and 7 that do not fit it
+        elif p % 4 == 1:
+            place[rng.integers(N)] = D + int(rng.integers(0, 200))
+        elif p % 4 == 2:
+            place[:] = 1
+        plans.place[p, :N] = place
+        plans.fuse[p, :] = 0xFFFFFFFF
+        plans.prefetch[p, :] = rng.integers(0, 2**32, size=plans.prefetch.shape[1], dtype=np.uint64).astype(np.uint32)
+    want = oracle_eval(prob, plans)
+    assert (want["status"] & 2).any() and (want["status"] & 1).any() and (want["status"] == 0).any()
+    assert_same(gpu_eval(prob, plans, k=8), want)
