@@ -217,6 +217,18 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
     size_t o_br = img.add(stoch ? pb->bm_r : nullptr, stoch ? sizeof(int32_t) * pb->bm_rn : 0);
     size_t o_bc = img.add(stoch ? pb->bm_c : nullptr, stoch ? sizeof(int32_t) * pb->bm_cn : 0);
     size_t o_be = img.add(stoch ? pb->bm_e : nullptr, stoch ? sizeof(int32_t) * pb->bm_en : 0);
+    // The radius and angle tables again as int16 when every value fits: half
+    // the L1 footprint for the stochastic sweep's per-sample lookups.
+    std::vector<int16_t> br16, bc16;
+    bool t16 = stoch;
+    for (int32_t i = 0; t16 && i < pb->bm_rn; ++i) t16 = pb->bm_r[i] >= -32768 && pb->bm_r[i] <= 32767;
+    for (int32_t i = 0; t16 && i < pb->bm_cn; ++i) t16 = pb->bm_c[i] >= -32768 && pb->bm_c[i] <= 32767;
+    if (t16) {
+        br16.assign(pb->bm_r, pb->bm_r + pb->bm_rn);
+        bc16.assign(pb->bm_c, pb->bm_c + pb->bm_cn);
+    }
+    size_t o_br16 = img.add(t16 ? br16.data() : nullptr, t16 ? sizeof(int16_t) * br16.size() : 0);
+    size_t o_bc16 = img.add(t16 ? bc16.data() : nullptr, t16 ? sizeof(int16_t) * bc16.size() : 0);
     size_t o_err = img.add(nullptr, 256);
     // Slot tables of the shared-memory sweep.
     std::vector<int32_t> rslot(N), wl_off;
@@ -358,6 +370,8 @@ extern "C" int wf_ctx_create(const wf_problem *pb, int device, int64_t max_P, wf
     dp.bm_r = (const int32_t *)(base + o_br);
     dp.bm_c = (const int32_t *)(base + o_bc);
     dp.bm_e = (const int32_t *)(base + o_be);
+    dp.bm_r16 = t16 ? (const int16_t *)(base + o_br16) : nullptr;
+    dp.bm_c16 = t16 ? (const int16_t *)(base + o_bc16) : nullptr;
     dp.err = (int *)(base + o_err);
     c->err = dp.err;
     dp.nslots = nslots > 0 ? nslots : 0;

@@ -33,6 +33,7 @@ struct wf_dev_problem {
     const int32_t *lev_nodes;   // [N]
     int32_t nlev;
     const int32_t *bm_r, *bm_c, *bm_e;
+    const int16_t *bm_r16, *bm_c16;  // bm_r, bm_c as int16 when every value fits (else null)
     int *err;                   // device error word (0 = ok)
 
     // Finish-time slots of the per-plan sweep (see wf_slots.cpp).  Slots

@@ -994,7 +994,9 @@ __device__ __forceinline__ uint64_t splitmix64(uint64_t x)
     return x ^ (x >> 31);
 }
 
-template <typename Q>
+// BT: the element type of the radius and angle tables read per sample
+// (int16 copies when every value fits, else the int32 tables).
+template <typename Q, typename BT>
 __global__ void __launch_bounds__(32 * kSWarps)
 stoch_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list, int32_t *ovf_count)
 {
@@ -1121,6 +1123,9 @@ stoch_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list,
     const uint64_t key = splitmix64(splitmix64(dp.seed ^ (uint64_t)(pl.plan_base + p)) ^ (uint64_t)t);
     const uint64_t rmask = (uint64_t)(dp.bm_rn - 1), cmask = (uint64_t)(dp.bm_cn - 1);
     const int64_t zoff = (dp.bm_en - 1) >> 1;
+    const BT *bmr, *bmc;
+    if constexpr (sizeof(BT) == 2) { bmr = dp.bm_r16; bmc = dp.bm_c16; }
+    else { bmr = dp.bm_r; bmc = dp.bm_c; }
     const uint32_t grant = (uint32_t)dp.grant;
     uint32_t end = 0, ovf = 0;
     int64_t gsum = 0;
@@ -1144,7 +1149,7 @@ stoch_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list,
             uint64_t run = 0;
             for (int32_t j = (int32_t)rb[kRecWords * kSChunk + k];; j = (int32_t)(__ldg(dp.links + j) >> 16)) {
                 const uint64_t hh = splitmix64(key ^ (uint64_t)j);
-                const int64_t prod = (int64_t)__ldg(dp.bm_r + (hh & rmask)) * (int64_t)__ldg(dp.bm_c + ((hh >> 32) & cmask));
+                const int64_t prod = (int64_t)__ldg(bmr + (hh & rmask)) * (int64_t)__ldg(bmc + ((hh >> 32) & cmask));
                 const int64_t mult = __ldg(dp.bm_e + ((prod >> 18) + zoff));
                 run += ((uint64_t)(uint32_t)__ldg(&dp.lk[j * D + d].x) * (uint64_t)mult + 32768u) >> 16;
                 if (j == tail) break;
@@ -1484,6 +1489,21 @@ size_t wf_stoch_smem(const wf_dev_problem &dp)
     return s <= 227 * 1024 ? s : 0;
 }
 
+namespace {
+
+template <typename Q, typename BT>
+int stoch_launch(const wf_dev_problem &dp, unsigned blocks, size_t smem, const wf_plans *pl, const wf_eval_out *out,
+                 int32_t *ovf_list, int32_t *ovf_count, cudaStream_t st)
+{
+    int rc = wf_cuda_check(cudaFuncSetAttribute(stoch_kernel<Q, BT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                (int)smem), "stochastic smem attribute");
+    if (rc) return rc;
+    stoch_kernel<Q, BT><<<blocks, 32 * kSWarps, smem, st>>>(dp, *pl, *out, ovf_list, ovf_count);
+    return WF_OK;
+}
+
+}  // namespace
+
 int wf_launch_stoch(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, size_t smem,
                     int32_t *ovf_list, int32_t *ovf_count, cudaStream_t st)
 {
@@ -1491,17 +1511,14 @@ int wf_launch_stoch(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, siz
     int rc = launch_status(ctx, pl, out, st, true);
     if (rc) return rc;
     const unsigned blocks = (unsigned)pl->P;
-    if (dp.M <= 8) {
-        rc = wf_cuda_check(cudaFuncSetAttribute(stoch_kernel<uint32_t>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                (int)smem), "stochastic smem attribute");
-        if (rc) return rc;
-        stoch_kernel<uint32_t><<<blocks, 32 * kSWarps, smem, st>>>(dp, *pl, *out, ovf_list, ovf_count);
-    } else {
-        rc = wf_cuda_check(cudaFuncSetAttribute(stoch_kernel<uint64_t>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                (int)smem), "stochastic smem attribute");
-        if (rc) return rc;
-        stoch_kernel<uint64_t><<<blocks, 32 * kSWarps, smem, st>>>(dp, *pl, *out, ovf_list, ovf_count);
-    }
+    const bool t16 = dp.bm_r16 != nullptr;
+    if (dp.M <= 8)
+        rc = t16 ? stoch_launch<uint32_t, int16_t>(dp, blocks, smem, pl, out, ovf_list, ovf_count, st)
+                 : stoch_launch<uint32_t, int32_t>(dp, blocks, smem, pl, out, ovf_list, ovf_count, st);
+    else
+        rc = t16 ? stoch_launch<uint64_t, int16_t>(dp, blocks, smem, pl, out, ovf_list, ovf_count, st)
+                 : stoch_launch<uint64_t, int32_t>(dp, blocks, smem, pl, out, ovf_list, ovf_count, st);
+    if (rc) return rc;
     return wf_cuda_check(cudaGetLastError(), "stochastic launch");
 }
 
