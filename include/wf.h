@@ -462,9 +462,11 @@ int wf_ctx_set_eval_path(wf_ctx *ctx, int32_t path);
  * for the next running unit to end); a unit of another model waits for the
  * device to drain, then hits or loads as without the limit.  B_q = 1 gives
  * the same results as 0.  Deterministic problems with least-recently-used
- * reclamation only; evaluation calls then take the exact int64 path (a
- * thread per plan) and reject retain rows when B_q > 1 and the window terms
- * of Eq. 12 (WF_EINVAL).  The first increase may reallocate the evaluation
+ * reclamation only.  Evaluation calls then play the plans in a shared-memory
+ * sweep of their own (the exact int64 path for a unit whose summed run time
+ * saturates 32 bits, or for every plan when the window's state does not fit
+ * a CTA), and reject retain rows when B_q > 1 and the window terms of Eq. 12
+ * (WF_EINVAL).  The first increase may reallocate the evaluation
  * scratch; not thread-safe with calls in flight on the context.  Returns
  * WF_EINVAL for a value outside 0..64 or such a problem.
  */

@@ -569,7 +569,17 @@ int wf_launch_eval(wf_ctx *ctx, const wf_plans *plans, const wf_eval_out *out, c
         return wf_set_error(WF_EINVAL, "the window terms of Eq. 12 are not modelled with a replica batch limit");
     if (dp.S == 0) {
         const int64_t blocks = (units + kEvalThreads - 1) / kEvalThreads;
-        // The replica batch limit is played by the int64 path only.
+        // The replica batch limit: its own sweep in shared memory, the int64
+        // path for what it hands on (or for everything, when it does not fit).
+        const size_t bsm = dp.batch > 0 && !ctx->force_int64 ? wf_batch_smem(dp) : 0;
+        if (bsm) {
+            int rc = wf_cuda_check(cudaMemsetAsync(ctx->ovf_count, 0, sizeof(int32_t), st), "reset overflow count");
+            if (!rc) rc = wf_launch_batch(ctx, plans, out, bsm, ctx->ovf_list, ctx->ovf_count, st);
+            if (rc) return rc;
+            eval_list_kernel<<<(unsigned)blocks, kEvalThreads, 0, st>>>(dp, *plans, *out, scratch, ctx->eval_row_bytes,
+                                                                       units, ctx->ovf_list, ctx->ovf_count);
+            return wf_cuda_check(cudaGetLastError(), "int64 pass launch");
+        }
         const wf_sweep_cfg cfg = ctx->force_int64 || dp.batch > 0 ? wf_sweep_cfg{} : wf_sweep_config(dp);
         if (dp.reclaim && !cfg.smem64)
             return wf_set_error(WF_EINVAL, "reclamation by next use runs only in the shared-memory sweep");

@@ -152,6 +152,9 @@ struct wf_sweep_cfg {
 wf_sweep_cfg wf_sweep_config(const wf_dev_problem &dp);
 int wf_launch_nextuse(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, cudaStream_t st);
 size_t wf_stoch_smem(const wf_dev_problem &dp);
+size_t wf_batch_smem(const wf_dev_problem &dp);
+int wf_launch_batch(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, size_t smem, int32_t *ovf_list,
+                    int32_t *ovf_count, cudaStream_t st);
 int wf_launch_stoch(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, size_t smem,
                     int32_t *ovf_list, int32_t *ovf_count, cudaStream_t st);
 // Status pass, then the sweeps (u32 first unless wide_first); on return

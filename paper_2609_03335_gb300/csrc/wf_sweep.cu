@@ -945,6 +945,294 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
 }
 
 // ---------------------------------------------------------------------------
+// Replica batch limit B_q (Eq. 11 over the running units, Section 3.5; the
+// reading of the oracle's simulate_batched): the same producer warps build
+// the unit records, and one play warp (lane = plan) settles each unit's
+// admission and timing together -- under the limit an admission waits for
+// running units to end, so residency cannot be settled ahead of the times.
+// Per plan and device: the current replica's model, up to B_q slots (end
+// time, KV), the last admission, residency stamps (dispatch position + 1 of
+// the last use, 0 = not resident), resident weights and count, and the
+// occupancy interval; 64-bit times, finish slots as in the sweep.
+// ---------------------------------------------------------------------------
+constexpr int kBqPlans = 8;                        // plans per CTA (play lanes)
+constexpr int kBqProducers = kBqPlans / kPlansPerIter;  // one plan pair per producer warp
+constexpr int kBqWarps = 1 + kBqProducers;
+constexpr int kBqBuffers = 4;
+constexpr int kBqPitch = kBqPlans | 1;
+constexpr int kBqFull = 1, kBqEmpty = kBqFull + kBqBuffers;  // named barriers
+static_assert(kBqEmpty + kBqBuffers <= 16, "named barriers");
+
+struct BqLayout {
+    uint32_t weight, cap, load, arr, ring, slots, stamp, se, sk, used, nres, cur, adm, occ, gpu, open, total;
+};
+
+__host__ __device__ inline BqLayout bq_layout(int32_t D, int32_t M, int32_t W, int32_t B, int32_t NS)
+{
+    constexpr uint32_t P = kBqPlans;
+    BqLayout l;
+    uint32_t o = 0;
+    l.weight = o; o += round16(4u * M);
+    l.cap = o; o += round16(4u * D);
+    l.load = o; o += round16(4u * M * D);
+    l.arr = o; o += round16(4u * W);
+    l.ring = o; o += 8u * kBqBuffers * 3 * kChunk * kBqPitch;
+    l.slots = o; o += 8u * (uint32_t)NS * P;
+    l.stamp = o; o += 4u * D * M * P;
+    l.se = o; o += 8u * D * B * P;
+    l.sk = o; o += round16(4u * D * B * P);
+    l.used = o; o += 4u * D * P;
+    l.nres = o; o += 4u * D * P;
+    l.cur = o; o += round16(4u * D * P);
+    l.adm = o; o += 8u * D * P;
+    l.occ = o; o += 8u * D * P;
+    l.gpu = o; o += 8u * D * P;
+    l.open = o; o += 16u * ((P + 3) / 4);
+    l.total = o;
+    return l;
+}
+
+__global__ void __launch_bounds__(32 * kBqWarps)
+bq_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, int32_t *ovf_list, int32_t *ovf_count)
+{
+    constexpr int kP = kBqPlans, kPitch = kBqPitch;
+    constexpr int kProdThreads = 32 * kBqProducers;
+    extern __shared__ __align__(128) uint8_t sm[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int32_t N = dp.N, D = dp.D, M = dp.M, W = dp.W, B = dp.batch;
+    const BqLayout L = bq_layout(D, M, W, B, dp.nslots + 2);
+    const int64_t j0 = (int64_t)blockIdx.x * kP;
+    const int ng = (int)(pl.P - j0 < kP ? pl.P - j0 : kP);
+    uint2 *ring = (uint2 *)(sm + L.ring);
+    const int32_t chunks = (N + kChunk - 1) / kChunk;
+    int32_t *weight = (int32_t *)(sm + L.weight);
+    int32_t *cap = (int32_t *)(sm + L.cap);
+    int32_t *load = (int32_t *)(sm + L.load);
+    uint32_t *arrival = (uint32_t *)(sm + L.arr);
+    uint32_t *open = (uint32_t *)(sm + L.open);  // placement status bits from the producers (bit kOpenBad on)
+    for (int32_t k = threadIdx.x; k < M; k += blockDim.x) weight[k] = __ldg(dp.weight + k);
+    for (int32_t k = threadIdx.x; k < D; k += blockDim.x) cap[k] = __ldg(dp.cap + k);
+    for (int32_t k = threadIdx.x; k < M * D; k += blockDim.x) load[k] = __ldg(dp.load + k);
+    for (int32_t k = threadIdx.x; k < W; k += blockDim.x) arrival[k] = (uint32_t)__ldg(dp.arrival + k);
+    if (threadIdx.x < kP) open[threadIdx.x] = 0;
+
+    if (warp >= 1) {
+        // ---------------- producers: lane = dispatch position (as in pc_kernel) ----------------
+        __syncthreads();
+        const int pw = warp - 1;
+        const int pos = lane % kChunk, sub = lane / kChunk;
+        const int q = pw * kPlansPerIter + sub;  // one plan per half-warp
+        RowPtrs rp[1];
+        int qq[1] = {q};
+        bool ok = q < ng;
+        rp[0].place = nullptr;
+        rp[0].order = nullptr;
+        rp[0].boff = 0;
+        if (ok) {
+            const int64_t pq = j0 + q;
+            ok = __ldg(out.status + pq) == 0;
+            rp[0].place = pl.place + pq * pl.place_stride;
+            rp[0].order = (const uint16_t *)((const uint8_t *)pl.order + pq * pl.order_stride);
+            rp[0].boff = pq * pl.bits_stride;
+        }
+        const uint32_t place_bytes = (uint32_t)((N + 15) & ~15), bits_bytes = (uint32_t)((((N + 31) >> 5) * 4 + 15) & ~15);
+        if (pos == 0 && ok) {
+            l2_prefetch(rp[0].place, place_bytes);
+            l2_prefetch(bits_row(pl.fuse, rp[0].boff), bits_bytes);
+            l2_prefetch(bits_row(pl.prefetch, rp[0].boff), bits_bytes);
+        }
+        int32_t h0[1] = {ok && pos < N ? (int32_t)__ldg(rp[0].order + pos) : 0};
+        for (int32_t c = 0; c < chunks; ++c) {
+            const int b = c % kBqBuffers;
+            if (c >= kBqBuffers) named_sync(kBqEmpty + b, kProdThreads + 32);  // the play warp released buffer b
+            uint2 *rb = ring + b * 3 * kChunk * kPitch;
+            const int32_t i = c * kChunk + pos;
+            const int32_t h1 = ok && i + kChunk < N ? (int32_t)__ldg(rp[0].order + i + kChunk) : 0;
+            bool act[1] = {ok && i < N};
+            uint32_t dev[1];
+            produce_batch<1, kPitch>(dp, pl, rp, act, h0, rb, pos, qq, dev, open);
+            h0[0] = h1;
+            named_arrive(kBqFull + b, kProdThreads + 32);  // buffer b is full
+        }
+        for (int32_t c = chunks; c < chunks + kBqBuffers; ++c)
+            if (c >= kBqBuffers) named_sync(kBqEmpty + c % kBqBuffers, kProdThreads + 32);
+        return;
+    }
+
+    // ---------------- play: lane = plan (admission and timing together) ----------------
+    const int q = lane;
+    const bool mine = q < kP;
+    const int64_t p = j0 + q;
+    const bool live = mine && q < ng && out.status[p] == 0;
+    SlotArr<uint64_t, uint64_t, kP> slots;
+    slots.v = (uint64_t *)(sm + L.slots) + q;
+    uint32_t *stamp = (uint32_t *)(sm + L.stamp) + q;  // [d][m]
+    uint64_t *se = (uint64_t *)(sm + L.se) + q;        // [d][slot]
+    int32_t *sk = (int32_t *)(sm + L.sk) + q;          // [d][slot]
+    int32_t *used = (int32_t *)(sm + L.used) + q;
+    int32_t *nres = (int32_t *)(sm + L.nres) + q;
+    int32_t *cur = (int32_t *)(sm + L.cur) + q;
+    uint64_t *ladm = (uint64_t *)(sm + L.adm) + q;
+    uint64_t *occ = (uint64_t *)(sm + L.occ) + q;
+    uint64_t *gpu = (uint64_t *)(sm + L.gpu) + q;
+    constexpr uint64_t kIdle = ~0ull;  // no occupancy interval open
+    if (mine) {
+        for (int32_t k = 0; k < dp.nslots + 2; ++k) slots.set(k, 0);
+        for (int32_t k = 0; k < D * M; ++k) stamp[k * kP] = 0;
+        for (int32_t k = 0; k < D * B; ++k) { se[k * kP] = 0; sk[k * kP] = 0; }
+        for (int32_t d = 0; d < D; ++d) {
+            used[d * kP] = 0; nres[d * kP] = 0; cur[d * kP] = -1;
+            ladm[d * kP] = 0; occ[d * kP] = kIdle; gpu[d * kP] = 0;
+        }
+    }
+    __syncthreads();
+    const uint32_t trash = (uint32_t)dp.nslots;
+    uint64_t end = 0;
+    uint32_t ovf = 0;
+    // The least recently used idle model of device d other than m (-1: none).
+    auto victim_of = [&](int32_t d, uint32_t m) -> int32_t {
+        int32_t v = -1;
+        uint32_t vs = 0xFFFFFFFFu;
+        for (int32_t k = 0; k < M; ++k) {
+            const uint32_t s = stamp[(d * M + k) * kP];
+            if ((uint32_t)k != m && s != 0 && s < vs) { vs = s; v = k; }
+        }
+        return v;
+    };
+    for (int32_t c = 0; c < chunks; ++c) {
+        const int b = c % kBqBuffers;
+        named_sync(kBqFull + b, kProdThreads + 32);
+        const uint2 *rb = ring + b * 3 * kChunk * kPitch + q;
+        const int32_t kmax = min(kChunk, N - c * kChunk);
+        for (int32_t k = 0; live && k < kmax; ++k) {
+            const uint2 w0 = rb[(0 * kChunk + k) * kPitch], w1 = rb[(1 * kChunk + k) * kPitch],
+                        w2 = rb[(2 * kChunk + k) * kPitch];
+            const uint32_t r3 = w1.y;
+            if (r3 & kSkip) continue;
+            const int32_t d = (int32_t)(r3 & 31u);
+            const uint32_t m = (r3 >> 5) & 15u;
+            const uint64_t arr = w0.y, run = w0.x;  // run includes the grant
+            const int64_t kv = (int32_t)w1.x;
+            const uint32_t r4 = w2.x, r5 = w2.y;
+            ovf |= w0.x == kRunCap;  // a saturated chain run: the int64 path
+            // Release (Eq. 2, Eq. 7); an accumulator slot is reset by its reader.
+            const uint32_t rs = r5 >> 16;
+            const uint64_t rel = max(arr, slots.get(rs & 0x7FFFu));
+            slots.set((rs & 0x8000u) ? (rs & 0x7FFFu) : trash, 0);
+            const int64_t capd = cap[d], wm = weight[m];
+            uint64_t *sed = se + d * B * kP;
+            int32_t *skd = sk + d * B * kP;
+            int64_t u_d = used[d * kP];
+            uint64_t adm, start;
+            int32_t slot = 0;
+            if ((int32_t)m == cur[d * kP]) {
+                // Join the current replica: the slot that frees first, no
+                // earlier than the last admission (dispatch order), and Eq.
+                // 11 with the running units' KV; idle models go first, then
+                // the admission waits for the next running unit to end.
+                for (int32_t j = 1; j < B; ++j)
+                    if (sed[j * kP] < sed[slot * kP]) slot = j;
+                adm = max(max(rel, sed[slot * kP]), ladm[d * kP]);
+                for (;;) {
+                    int64_t running = 0;
+                    for (int32_t j = 0; j < B; ++j) running += sed[j * kP] > adm ? skd[j * kP] : 0;
+                    while (u_d + running + kv > capd) {
+                        const int32_t v = victim_of(d, m);
+                        if (v < 0) break;
+                        u_d -= weight[v];
+                        nres[d * kP] -= 1;
+                        stamp[(d * M + v) * kP] = 0;
+                    }
+                    if (u_d + running + kv <= capd) break;
+                    uint64_t next = ~0ull;  // the next running unit to end
+                    for (int32_t j = 0; j < B; ++j)
+                        if (sed[j * kP] > adm && sed[j * kP] < next) next = sed[j * kP];
+                    if (next == ~0ull) { atomicExch(dp.err, 2); break; }  // unreachable for a valid plan
+                    adm = next;
+                }
+                start = adm;
+            } else {
+                // Another model: the device drains, then the unit hits or loads.
+                uint64_t drain = 0;
+                for (int32_t j = 0; j < B; ++j) drain = max(drain, sed[j * kP]);
+                const bool hit = stamp[(d * M + m) * kP] != 0;
+                const int64_t need = hit ? kv : wm + kv;
+                while (u_d + need > capd) {
+                    const int32_t v = victim_of(d, m);
+                    if (v < 0) { atomicExch(dp.err, 2); break; }  // unreachable for a valid plan
+                    u_d -= weight[v];
+                    nres[d * kP] -= 1;
+                    stamp[(d * M + v) * kP] = 0;
+                }
+                uint64_t ready;
+                if (hit) {
+                    adm = start = max(drain, rel);
+                    ready = drain;
+                } else {
+                    const uint64_t ls = max(drain, (r3 & kPrefetch) ? arr : rel);
+                    if (occ[d * kP] == kIdle) occ[d * kP] = ls;
+                    u_d += wm;
+                    nres[d * kP] += 1;
+                    const uint64_t le = ls + (uint64_t)load[m * D + d];
+                    adm = ls;
+                    start = max(le, rel);
+                    ready = le;
+                }
+                for (int32_t j = 0; j < B; ++j) { sed[j * kP] = ready; skd[j * kP] = 0; }
+                cur[d * kP] = (int32_t)m;
+            }
+            const uint64_t cfin = start + run;
+            publish<uint64_t>(slots, r3 >> 16, cfin);  // the sink when the unit writes nothing
+            publish<uint64_t>(slots, r4 & 0xFFFFu, cfin);
+            const uint32_t nwl = (r3 >> 11) & 7u;
+            if (nwl > 2) {
+                publish<uint64_t>(slots, r4 >> 16, cfin);
+                if (nwl == 4) {
+                    publish<uint64_t>(slots, r5 & 0xFFFFu, cfin);
+                } else if (nwl > 4) {  // five or more codes: the list from global memory
+                    const int4 wr = __ldg(dp.noderec + 2 * (int32_t)(r5 & 0xFFFFu) + 1);
+                    for (int32_t e = 3; e < wr.y; ++e) publish<uint64_t>(slots, __ldg(dp.wl + wr.x + e), cfin);
+                }
+            }
+            sed[slot * kP] = cfin;
+            skd[slot * kP] = (int32_t)kv;
+            ladm[d * kP] = adm;
+            stamp[(d * M + m) * kP] = (uint32_t)(c * kChunk + k) + 1u;
+            end = max(end, cfin);
+            if ((r3 >> 10) & 1u) {  // retain bit 0 (B_q = 1 only): the model leaves after the unit
+                u_d -= wm;
+                nres[d * kP] -= 1;
+                stamp[(d * M + m) * kP] = 0;
+                cur[d * kP] = -1;
+                if (nres[d * kP] == 0) {
+                    gpu[d * kP] += cfin - occ[d * kP];
+                    occ[d * kP] = kIdle;
+                }
+            }
+            used[d * kP] = (int32_t)u_d;
+        }
+        named_arrive(kBqEmpty + b, kProdThreads + 32);  // buffer b may be refilled
+    }
+    if (!live) return;
+    const uint32_t bad = open[q] >> kOpenBad;  // placement bits found by the producers
+    if (bad) {
+        out.status[p] = bad;
+        out.makespan_us[p] = out.p95_us[p] = out.gpu_us[p] = WF_INF64;
+    } else if (ovf) {
+        ovf_list[atomicAdd(ovf_count, 1)] = (int32_t)p;
+    } else {
+        int64_t g = 0;
+        for (int32_t d = 0; d < D; ++d)
+            g += (int64_t)gpu[d * kP] + (occ[d * kP] != kIdle ? (int64_t)(end - occ[d * kP]) : 0);
+        for (int32_t w = 0; w < W; ++w) slots.set(w, slots.get(w) - arrival[w]);  // session completion latency
+        const int32_t rank = (int32_t)((95 * (int64_t)W + 99) / 100 - 1);
+        out.makespan_us[p] = (int64_t)end - dp.first_arrival;
+        out.gpu_us[p] = g;
+        out.p95_us[p] = (int64_t)select_slots<uint64_t>(slots, W, rank);
+    }
+}
+
+// ---------------------------------------------------------------------------
 // Stochastic latencies (row a11): one plan per CTA.  Model residency does not
 // depend on times, so one residency lane settles it for every sample; the
 // timing warps play kSamples samples at once (lane = sample), each drawing
@@ -1503,6 +1791,32 @@ int stoch_launch(const wf_dev_problem &dp, unsigned blocks, size_t smem, const w
 }
 
 }  // namespace
+
+// Shared memory of the replica-batch sweep for this problem, or 0 when it
+// cannot run it (the same slot and size limits as the sweep, plus room for
+// every device's B_q slots); the caller then uses the int64 path.
+size_t wf_batch_smem(const wf_dev_problem &dp)
+{
+    if (dp.batch < 1 || dp.S != 0 || dp.nslots <= 0 || dp.nslots > 32765 || dp.max_arrival >= (int64_t)1 << 32 ||
+        dp.M > 16 || dp.N > 65534 || dp.phi_life || dp.reclaim)
+        return 0;
+    const size_t s = bq_layout(dp.D, dp.M, dp.W, dp.batch, dp.nslots + 2).total;
+    return s <= 227 * 1024 ? s : 0;
+}
+
+// Status pass (placement left to the producers), then the replica-batch
+// sweep; plans with a saturated chain run are listed for the int64 path.
+int wf_launch_batch(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, size_t smem, int32_t *ovf_list,
+                    int32_t *ovf_count, cudaStream_t st)
+{
+    int rc = launch_status(ctx, pl, out, st, false);
+    if (!rc) rc = wf_cuda_check(cudaFuncSetAttribute(bq_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
+                                "batch sweep smem attribute");
+    if (rc) return rc;
+    const unsigned blocks = (unsigned)((pl->P + kBqPlans - 1) / kBqPlans);
+    bq_kernel<<<blocks, 32 * kBqWarps, smem, st>>>(ctx->dp, *pl, *out, ovf_list, ovf_count);
+    return wf_cuda_check(cudaGetLastError(), "batch sweep launch");
+}
 
 int wf_launch_stoch(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, size_t smem,
                     int32_t *ovf_list, int32_t *ovf_count, cudaStream_t st)
