@@ -329,6 +329,32 @@ def metric_of(prob):
     return f"candidate plans evaluated/sec (N={prob.N},D={prob.D}" + (f",S={prob.S})" if prob.S else ")")
 
 
+def run_step(wf, ctx, dp, res, rel, comp, ids, keys, P, k, stream, side, ev=None):
+    """One forecast / eval / top-k step.  The readiness forecast depends on the
+    window only, not on the plans, so it runs on a second stream beside the
+    evaluation, forked from and joined back into the step's stream with
+    events; the step ends when both have.  ev: timing events (start, eval
+    start, eval end, end, forecast start, forecast end) or None."""
+    import torch
+    fork = ev[0] if ev else torch.cuda.Event()
+    fork.record(stream)
+    side.wait_event(fork)
+    if ev:
+        ev[4].record(side)
+    wf.wf_forecast_readiness(ctx, rel, comp, side)
+    done = ev[5] if ev else torch.cuda.Event()
+    done.record(side)
+    if ev:
+        ev[1].record(stream)
+    wf.wf_eval_plans(ctx, dp, res, stream)
+    if ev:
+        ev[2].record(stream)
+    wf.wf_topk(ctx, res, P, k, ids, keys, stream)
+    stream.wait_event(done)
+    if ev:
+        ev[3].record(stream)
+
+
 def issue_roofline(eval_ms, clk, sms, workload=None):
     """The integer-issue roofline of the evaluation call: its warp
     instructions (ncu, same kernel source) over its CUDA-event time, against
@@ -421,28 +447,21 @@ def workload_entry(name, wf, dev, steps=5, warmup=3, with_cpu=True):
     keys = torch.empty((k, 3), dtype=torch.int64, device=dev)
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
     stream = torch.cuda.Stream(device=dev)
+    side = torch.cuda.Stream(device=dev)
     with torch.cuda.stream(stream):
         for _ in range(warmup):
             flush_l2(flush)
-            wf.wf_forecast_readiness(ctx, rel, comp, stream)
-            wf.wf_eval_plans(ctx, dp, res, stream)
-            wf.wf_topk(ctx, res, P, k, ids, keys, stream)
+            run_step(wf, ctx, dp, res, rel, comp, ids, keys, P, k, stream, side)
     wf.wf_ctx_status(ctx, stream)
     clocks = ClockSampler(dev.index)
     clocks.start()
     time.sleep(0.2)
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(steps)]
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(steps)]
     torch.cuda.synchronize()
     with torch.cuda.stream(stream):
         for e in ev:
             flush_l2(flush)
-            e[0].record(stream)
-            wf.wf_forecast_readiness(ctx, rel, comp, stream)
-            e[1].record(stream)
-            wf.wf_eval_plans(ctx, dp, res, stream)
-            e[2].record(stream)
-            wf.wf_topk(ctx, res, P, k, ids, keys, stream)
-            e[3].record(stream)
+            run_step(wf, ctx, dp, res, rel, comp, ids, keys, P, k, stream, side, e)
     torch.cuda.synchronize()
     clk = clocks.stop()
     wf.wf_ctx_status(ctx, stream)
@@ -574,10 +593,10 @@ def run_gpu(args, rank, world, local):
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
     torch.cuda.synchronize()
 
+    side = torch.cuda.Stream(device=dev)
+
     def step():
-        wf.wf_forecast_readiness(ctx, rel, comp, stream)
-        wf.wf_eval_plans(ctx, dp, res, stream)
-        wf.wf_topk(ctx, res, P, k, ids, keys, stream)
+        run_step(wf, ctx, dp, res, rel, comp, ids, keys, P, k, stream, side)
 
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
@@ -588,26 +607,19 @@ def run_gpu(args, rank, world, local):
     clocks = ClockSampler(local)
     clocks.start()
     time.sleep(0.3)
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(args.steps)]
     barrier(world)
     torch.cuda.synchronize()
     with torch.cuda.stream(stream):
         for s in range(args.steps):
             flush_l2(flush)
-            e = ev[s]
-            e[0].record(stream)
-            wf.wf_forecast_readiness(ctx, rel, comp, stream)
-            e[1].record(stream)
-            wf.wf_eval_plans(ctx, dp, res, stream)
-            e[2].record(stream)
-            wf.wf_topk(ctx, res, P, k, ids, keys, stream)
-            e[3].record(stream)
+            run_step(wf, ctx, dp, res, rel, comp, ids, keys, P, k, stream, side, ev[s])
     torch.cuda.synchronize()
     barrier(world)
     wf.wf_ctx_status(ctx, stream)
     step_ms = [e[0].elapsed_time(e[3]) for e in ev]
     eval_ms = [e[1].elapsed_time(e[2]) for e in ev]
-    forecast_ms = float(np.mean([e[0].elapsed_time(e[1]) for e in ev]))
+    forecast_ms = float(np.mean([e[4].elapsed_time(e[5]) for e in ev]))
     topk_ms = float(np.mean([e[2].elapsed_time(e[3]) for e in ev]))
     ms_per_step = max_over_ranks(float(np.mean(step_ms)), world)
     eval_ms_mean = float(np.mean(eval_ms))

@@ -230,7 +230,8 @@ int wf_topk(wf_ctx *ctx, const wf_eval_out *res, int64_t P, int32_t k,
  * The context copies the plans into one of two device staging slots on a
  * copy stream of its own, and calls alternate between the slots, so a call's
  * copy overlaps the previous call's evaluation on `stream`; each copy first
- * waits for the evaluation that last read its slot.  The results are in host
+ * waits for the call that last used its slot.  The forecast, which depends on
+ * the window only, runs on the copy stream too.  The results are in host
  * memory once `stream` has passed the call (synchronize or record an event
  * after it).  The host plan arrays must stay unchanged until the call's copy
  * has run (at the latest, when `stream` has passed the call).  Host memory

@@ -1,14 +1,15 @@
 // One step of the hot path from and to host memory (wf_eval_topk_host):
-// host plan rows -> a device staging slot -> forecast / evaluation / top-k on
-// the caller's stream -> results back to the host.
+// host plan rows -> a device staging slot -> evaluation / top-k on the
+// caller's stream (the forecast beside them) -> results back to the host.
 //
 // The context holds two staging slots and a copy stream.  A call takes the
 // slot the previous call did not use, so its copy (on the copy stream) runs
 // while the previous call evaluates (on the caller's stream); the copy first
-// waits for the event recorded after the evaluation that last read the slot,
+// waits for the event recorded at the end of the call that last used the slot,
 // and the evaluation waits for the event recorded after the copy.  The
-// results, top-k and forecast buffers are single: everything that touches
-// them runs in order on the caller's stream.
+// forecast (which depends on the window only) runs on the copy stream too,
+// into the slot's own buffer.  The results and top-k buffers are single:
+// everything that touches them runs in order on the caller's stream.
 #include <cstdint>
 #include <cstdlib>
 
@@ -22,7 +23,7 @@ struct wf_host_stage {
     uint32_t *status;                    // [P]
     int32_t *ids;                        // [1024]
     int64_t *keys;                       // [1024][3]
-    int64_t *fc;                         // rel, comp: [2][N]
+    int64_t *fc[2];                      // per slot: rel, comp [2][N]
     cudaStream_t copy;
     cudaEvent_t copied[2], freed[2];
     int next;
@@ -78,7 +79,8 @@ int reserve(wf_ctx *c)
     if (!rc) rc = wf_cuda_check(cudaMalloc(&h->status, sizeof(uint32_t) * (size_t)P), "cudaMalloc(host status)");
     if (!rc) rc = wf_cuda_check(cudaMalloc(&h->ids, sizeof(int32_t) * 1024), "cudaMalloc(host top-k)");
     if (!rc) rc = wf_cuda_check(cudaMalloc(&h->keys, sizeof(int64_t) * 3 * 1024), "cudaMalloc(host top-k keys)");
-    if (!rc) rc = wf_cuda_check(cudaMalloc(&h->fc, sizeof(int64_t) * 2 * (size_t)N), "cudaMalloc(host forecast)");
+    for (int s = 0; s < 2 && !rc; ++s)
+        rc = wf_cuda_check(cudaMalloc(&h->fc[s], sizeof(int64_t) * 2 * (size_t)N), "cudaMalloc(host forecast)");
     if (!rc) rc = wf_cuda_check(cudaStreamCreateWithFlags(&h->copy, cudaStreamNonBlocking), "cudaStreamCreate");
     for (int s = 0; s < 2 && !rc; ++s) {
         rc = wf_cuda_check(cudaEventCreateWithFlags(&h->copied[s], cudaEventDisableTiming), "cudaEventCreate");
@@ -116,12 +118,12 @@ void wf_host_release(wf_ctx *c)
         if (h->slot[s]) cudaFree(h->slot[s]);
         if (h->copied[s]) cudaEventDestroy(h->copied[s]);
         if (h->freed[s]) cudaEventDestroy(h->freed[s]);
+        if (h->fc[s]) cudaFree(h->fc[s]);
     }
     if (h->metrics) cudaFree(h->metrics);
     if (h->status) cudaFree(h->status);
     if (h->ids) cudaFree(h->ids);
     if (h->keys) cudaFree(h->keys);
-    if (h->fc) cudaFree(h->fc);
     if (h->copy) cudaStreamDestroy(h->copy);
     free(h);
     c->host = nullptr;
@@ -168,6 +170,9 @@ extern "C" int wf_eval_topk_host(wf_ctx *c, const wf_plans *hp, int32_t k, int32
     const wf_plans d = slot_plans(h, s, P, hp->plan_base, hp->retain != nullptr);
     const cudaStream_t cp = capturing ? st : h->copy;
     if (!capturing) rc = wf_cuda_check(cudaStreamWaitEvent(cp, h->freed[s], 0), "wait for the slot");
+    // The forecast depends on the window only: it runs on the copy stream
+    // too, before the copies, beside the previous call's evaluation.
+    if (!rc && rel_host) rc = wf_launch_forecast(c, h->fc[s], h->fc[s] + N, cp);
     if (!rc) rc = copy_rows((void *)d.place, d.place_stride, hp->place, hp->place_stride, d.place_stride, P, cp);
     if (!rc) rc = copy_rows((void *)d.order, d.order_stride, hp->order, hp->order_stride, d.order_stride, P, cp);
     if (!rc) rc = copy_rows((void *)d.fuse, d.bits_stride, hp->fuse, hp->bits_stride, d.bits_stride, P, cp);
@@ -180,14 +185,12 @@ extern "C" int wf_eval_topk_host(wf_ctx *c, const wf_plans *hp, int32_t k, int32
     }
     if (rc) return rc;
 
-    if (rel_host) rc = wf_launch_forecast(c, h->fc, h->fc + N, st);
     wf_eval_out dout;
     dout.makespan_us = h->metrics;
     dout.p95_us = h->metrics + P;
     dout.gpu_us = h->metrics + 2 * P;
     dout.status = h->status;
     if (!rc) rc = wf_launch_eval(c, &d, &dout, st);
-    if (!rc && !capturing) rc = wf_cuda_check(cudaEventRecord(h->freed[s], st), "record the slot's release");
     if (!rc) rc = wf_launch_topk(c, &dout, P, k, h->ids, h->keys, st);
     if (rc) return rc;
 
@@ -207,8 +210,11 @@ extern "C" int wf_eval_topk_host(wf_ctx *c, const wf_plans *hp, int32_t k, int32
     }
     if (!rc && rel_host) {
         const size_t b = sizeof(int64_t) * (size_t)N;
-        rc = wf_cuda_check(cudaMemcpyAsync(rel_host, h->fc, b, dh, st), "forecast to host");
-        if (!rc) rc = wf_cuda_check(cudaMemcpyAsync(comp_host, h->fc + N, b, dh, st), "forecast to host");
+        rc = wf_cuda_check(cudaMemcpyAsync(rel_host, h->fc[s], b, dh, st), "forecast to host");
+        if (!rc) rc = wf_cuda_check(cudaMemcpyAsync(comp_host, h->fc[s] + N, b, dh, st), "forecast to host");
     }
+    // The slot (its rows and its forecast) may be refilled once this call's
+    // evaluation and copies back have run.
+    if (!rc && !capturing) rc = wf_cuda_check(cudaEventRecord(h->freed[s], st), "record the slot's release");
     return rc;
 }
