@@ -1,7 +1,7 @@
-"""Top-k on synthetic result arrays, at batch sizes past the single-CTA
-path: ties within and across tiles, invalid plans, a short last tile, and
-k up to its limit.  The keys are written straight into the result arrays, so
-only the top-k kernels run."""
+"""Top-k on synthetic result arrays, on both of its paths (one CTA up to
+16,384 plans, per-tile thresholds beyond): ties within and across tiles,
+invalid plans, a short last tile, and k up to its limit.  The keys are written straight into the
+result arrays, so only the top-k kernels run."""
 import numpy as np
 import pytest
 
@@ -69,3 +69,46 @@ def test_all_plans_invalid_and_tied():
     ids, keys = run_topk(mk, zeros, zeros, st, k)
     want_ids, want_keys = oracle.topk(mk, zeros, zeros, st, k)
     assert np.array_equal(ids, want_ids) and np.array_equal(keys, want_keys)
+
+
+@pytest.mark.parametrize("P,k", [
+    (1, 1), (63, 5), (1024, 1024), (1025, 1024), (1025, 1), (2049, 683),
+    (16383, 128), (16384, 128), (16384, 129), (16384, 32), (9000, 200),
+])
+def test_single_cta_batches(P, k):
+    """Batches up to the single-CTA limit, k from 1 to P: ties and invalid
+    plans."""
+    rng = np.random.default_rng(P * 7 + k)
+    mk = rng.integers(1000, 1000 + max(P // 8, 2), P).astype(np.int64)
+    p95 = rng.integers(0, 3, P).astype(np.int64)
+    gpu = rng.integers(0, 2, P).astype(np.int64)
+    st = np.where(rng.random(P) < 0.2, rng.integers(1, 16, P), 0).astype(np.uint32)
+    ids, keys = run_topk(mk, p95, gpu, st, k)
+    want_ids, want_keys = oracle.topk(mk, p95, gpu, st, k)
+    assert np.array_equal(ids, want_ids) and np.array_equal(keys, want_keys)
+
+
+def test_paths_alternate_on_one_context():
+    """The single-CTA and threshold paths alternate on one context's top-k
+    scratch."""
+    import torch
+    wf = lib()
+    P = 40000
+    rng = np.random.default_rng(11)
+    mk = rng.integers(0, 5000, P).astype(np.int64)
+    zeros = np.zeros(P, np.int64)
+    st = np.zeros(P, np.uint32)
+    ctx = wf.Ctx(wfgen.config("tiny").problem, max_P=P)
+    res = wf.Results(P)
+    res.makespan.copy_(torch.from_numpy(mk))
+    res.p95.zero_()
+    res.gpu.zero_()
+    res.status.zero_()
+    for n, k in [(16384, 32), (P, 32), (4000, 16), (16384, 500), (P, 7), (1500, 1000), (2, 2)]:
+        ids = torch.empty(k, dtype=torch.int32, device="cuda")
+        keys = torch.empty((k, 3), dtype=torch.int64, device="cuda")
+        wf.wf_topk(ctx, res, n, k, ids, keys)
+        torch.cuda.synchronize()
+        want_ids, want_keys = oracle.topk(mk[:n], zeros[:n], zeros[:n], st[:n], k)
+        assert np.array_equal(ids.cpu().numpy(), want_ids) and np.array_equal(keys.cpu().numpy(), want_keys)
+    ctx.close()
