@@ -67,8 +67,10 @@ enum {
 
 /* Evaluation path (wf_ctx_set_eval_path). */
 enum {
-    WF_PATH_AUTO = 0,   /* the shared-memory sweeps, the exact int64 path for what they hand on (the default) */
-    WF_PATH_INT64 = 1   /* every plan on the exact int64 path (a thread per plan, state in global memory) */
+    WF_PATH_AUTO = 0,     /* the shared-memory sweeps, the exact int64 path for what they hand on (the default) */
+    WF_PATH_INT64 = 1,    /* every plan on the exact int64 path (a thread per plan, state in global memory) */
+    WF_PATH_WIDE = 2,     /* every plan starts in the 64-bit sweep */
+    WF_PATH_RELATIVE = 3  /* every plan starts in the sweep with 32-bit times relative to a per-plan base */
 };
 
 /* Reclamation order (wf_ctx_set_reclaim). */
@@ -442,11 +444,26 @@ int wf_ctx_status(wf_ctx *ctx, void *stream);
 int wf_ctx_check_wait_expiry(wf_ctx *ctx, void *stream);
 
 /*
- * Which kernels later evaluation calls on this context use: WF_PATH_AUTO
- * (default) or WF_PATH_INT64, every plan on the exact int64 path.  Both give
- * the same results; the int64 path is slower and serves tests and
- * cross-checks of the sweeps.  Not thread-safe with calls in flight on the
- * context.  Returns WF_EINVAL for a NULL context or another value.
+ * Which kernels later evaluation calls on this context use.  All give the
+ * same results.
+ *   WF_PATH_AUTO (default): the 32-bit sweep, which hands a plan whose times
+ *     reach 2^32 us to the 64-bit sweep; once more than half of a batch has
+ *     left 32 bits, later calls start every plan in the relative sweep
+ *     (below), or in the 64-bit sweep where that does not apply.
+ *   WF_PATH_INT64: every plan on the exact int64 path (slower; for tests and
+ *     cross-checks of the sweeps).
+ *   WF_PATH_WIDE: every plan starts in the 64-bit sweep.
+ *   WF_PATH_RELATIVE: every plan starts in the relative sweep: 32-bit times
+ *     counted from a per-plan base that rises with the plan's devices' free
+ *     times, so a window whose times run far past 2^32 us still plays on
+ *     32-bit arithmetic; a plan whose times leave 32 bits even so goes on to
+ *     the 64-bit sweep.  Calls under next-use reclamation or for Eq. 12's
+ *     terms, and contexts too small for its scratch rows, start as
+ *     WF_PATH_WIDE.
+ * A unit whose summed run time saturates 32 bits always goes on to the int64
+ * path.  Not thread-safe with calls in flight on the context.  Returns
+ * WF_EINVAL for a NULL context or another value, and for WF_PATH_RELATIVE or
+ * WF_PATH_WIDE when the window does not fit those sweeps' shared memory.
  */
 int wf_ctx_set_eval_path(wf_ctx *ctx, int32_t path);
 

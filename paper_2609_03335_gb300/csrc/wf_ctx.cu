@@ -589,9 +589,16 @@ extern "C" int wf_ctx_status(wf_ctx *c, void *stream)
 extern "C" int wf_ctx_set_eval_path(wf_ctx *c, int32_t path)
 {
     REQUIRE(c, "NULL context");
-    REQUIRE(path == WF_PATH_AUTO || path == WF_PATH_INT64, "eval path %d is neither WF_PATH_AUTO nor WF_PATH_INT64",
-            path);
+    REQUIRE(path >= WF_PATH_AUTO && path <= WF_PATH_RELATIVE, "unknown eval path %d", path);
+    if (path == WF_PATH_WIDE || path == WF_PATH_RELATIVE) {
+        const int rc = select_device(c);
+        if (rc) return rc;
+        const wf_sweep_cfg cfg = wf_sweep_config(c->dp);
+        REQUIRE(cfg.smem64, "this window does not fit the 64-bit sweep");
+        REQUIRE(path == WF_PATH_WIDE || cfg.smemRel, "this window does not fit the relative-time sweep");
+    }
     c->force_int64 = path == WF_PATH_INT64;
+    c->start_path = path;
     return WF_OK;
 }
 

@@ -603,7 +603,7 @@ int wf_launch_eval(wf_ctx *ctx, const wf_plans *plans, const wf_eval_out *out, c
                     return wf_cuda_check(q, "overflow count event");
                 }
             }
-            const bool wide_first = ctx->prefer_wide && cfg.smem64;
+            const bool wide_first = (ctx->prefer_wide || ctx->start_path >= WF_PATH_WIDE) && cfg.smem64;
             int rc = wf_cuda_check(cudaMemsetAsync(ctx->ovf_count, 0, 2 * sizeof(int32_t), st), "reset overflow counts");
             const int32_t *rest = nullptr, *rest_count = nullptr;
             if (!rc) rc = wf_launch_sweep(ctx, plans, out, cfg, wide_first, ctx->ovf_count, ctx->ovf_list,

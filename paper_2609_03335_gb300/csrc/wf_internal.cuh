@@ -68,6 +68,10 @@ struct wf_dev_problem {
     // null outside such a call.
     int64_t *phi_timely;
     int64_t *phi_life;
+    // The relative-time sweep's exact session finishes that fell below a
+    // plan's base, [W][CTAs x plans per CTA]: the context's evaluation
+    // scratch, set for that launch only.
+    uint64_t *rel_ret;
     int64_t max_arrival;
 };
 
@@ -91,6 +95,7 @@ struct wf_ctx {
     int *err;
     int sms;                    // streaming multiprocessors of the device
     bool force_int64;           // wf_ctx_set_eval_path(WF_PATH_INT64): every plan on the int64 path
+    int32_t start_path;         // wf_ctx_set_eval_path's value (WF_PATH_WIDE / RELATIVE: the first sweep)
     int32_t *ovf_count;         // [2]: plans the u32 sweep hands on, plans left for the int64 path
     int32_t *ovf_list;          // [max_P] the u32 sweep's hand-offs (and the stochastic sweep's)
     int32_t *ovf_list2;         // [max_P] plans for the int64 path
@@ -140,14 +145,18 @@ size_t wf_eval_scratch_bytes(const wf_dev_problem &dp, int64_t max_P, int64_t *u
 size_t wf_topk_scratch_bytes(int64_t max_P);
 size_t wf_search_scratch_bytes(int64_t max_P);
 // The shared-memory sweeps that apply to a problem: u32 times with 16 plans
-// per CTA, and u64 times with plans64 plans per CTA (0 bytes = not usable);
-// res32 / res64 are the CTAs of each resident on one SM.
+// per CTA, u64 times with plans64 plans per CTA, and relative u32 times with
+// plansRel plans per CTA (0 bytes = not usable); res32 / res64 / resRel are
+// the CTAs of each resident on one SM.
 struct wf_sweep_cfg {
     size_t smem32;
     size_t smem64;
+    size_t smemRel;
     int plans64;
+    int plansRel;
     int res32;
     int res64;
+    int resRel;
 };
 wf_sweep_cfg wf_sweep_config(const wf_dev_problem &dp);
 int wf_launch_nextuse(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, cudaStream_t st);
@@ -157,8 +166,10 @@ int wf_launch_batch(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, siz
                     int32_t *ovf_count, cudaStream_t st);
 int wf_launch_stoch(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, size_t smem,
                     int32_t *ovf_list, int32_t *ovf_count, cudaStream_t st);
-// Status pass, then the sweeps (u32 first unless wide_first); on return
-// *rest_list / *rest_count name the plans left for the int64 path.
+// Status pass, then the sweeps (u32 first unless wide_first; then the
+// relative sweep where it applies and the context's path is not
+// WF_PATH_WIDE, else u64); on return *rest_list / *rest_count name the plans
+// left for the int64 path.
 int wf_launch_sweep(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, const wf_sweep_cfg &cfg,
                     bool wide_first, int32_t *counts, int32_t *list1, int32_t *list2, cudaStream_t st,
                     const int32_t **rest_list, const int32_t **rest_count);

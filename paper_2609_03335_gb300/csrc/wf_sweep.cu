@@ -180,6 +180,26 @@ struct PcGroups {
 // so more plans fit an SM.
 struct Split40 {};
 
+// Relative 32-bit times (slot storage Rel32, with TT = uint32_t): every time
+// the timing stage keeps (finish slots, device free times, the plan's end)
+// counts from a per-plan base B, which it raises now and then to one below
+// the smallest device free time.  That is exact: every later unit starts at
+// or after its device's free time, so a stored finish or arrival below B can
+// be read as B without changing any start (Eq. 2, 5, 7).  A session slot
+// that would fall below B keeps its exact value in global memory instead,
+// for the p95.
+struct Rel32 {};
+template <typename ST>
+struct IsRel {
+    static constexpr bool value = false;
+};
+template <>
+struct IsRel<Rel32> {
+    static constexpr bool value = true;
+};
+constexpr uint32_t kRebaseAt = 3u << 30;   // a plan's end above this raises its base ...
+constexpr uint32_t kRebaseMin = 1u << 28;  // ... by at least this much, else not at all
+
 template <typename ST>
 struct SlotBytes {
     static constexpr uint32_t kLo = sizeof(ST), kHi = 0;
@@ -187,6 +207,10 @@ struct SlotBytes {
 template <>
 struct SlotBytes<Split40> {
     static constexpr uint32_t kLo = 4, kHi = 1;
+};
+template <>
+struct SlotBytes<Rel32> {
+    static constexpr uint32_t kLo = 4, kHi = 0;
 };
 
 template <typename TT, typename ST, int kS>
@@ -207,6 +231,22 @@ struct SlotArr<uint64_t, Split40, kS> {
     {
         lo[i * kS] = (uint32_t)x;
         hi[i * kS] = (uint8_t)(x >> 32);
+    }
+};
+
+// Slots 2i and 2i + 1 of a 32-bit slot array read as one 64-bit value i (the
+// relative sweep's session latencies at the end of a plan).
+template <int kS>
+struct PairArr {
+    uint32_t *v;
+    __device__ __forceinline__ uint64_t get(uint32_t i) const
+    {
+        return ((uint64_t)v[(2 * i + 1) * kS] << 32) | v[2 * i * kS];
+    }
+    __device__ __forceinline__ void set(uint32_t i, uint64_t x) const
+    {
+        v[2 * i * kS] = (uint32_t)x;
+        v[(2 * i + 1) * kS] = (uint32_t)(x >> 32);
     }
 };
 
@@ -556,6 +596,8 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
     constexpr int kProdThreads = 32 * S::kProducers;
     constexpr int kResThreads = 32 * S::kRes;
     constexpr bool kNarrow = sizeof(TT) == 4;
+    constexpr bool kRel = IsRel<ST>::value;  // relative 32-bit times
+    static_assert(!kRel || (kNarrow && kReclaim == 0 && !kPhi), "relative times: u32, least recently used");
     constexpr int kG = PcGroups<kP, kReclaim>::kG;  // residency lanes per plan
     using RG = Ring<kReclaim>;
     constexpr int kBuffers = RG::kBuffers, kFullP = RG::kFullP, kFullR = RG::kFullR, kEmpty = RG::kEmpty,
@@ -848,9 +890,45 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
     int64_t gsum = 0;
     uint32_t ph_timely = 0;  // Eq. 12 window terms (kPhi)
     uint64_t ph_life = 0;
+    // Relative times (kRel): the base, the base saturated to 32 bits (for the
+    // arrivals), emptied minus newly occupied devices so far (gsum counts
+    // from the base), and the rebases so far.
+    uint64_t base = 0;
+    uint32_t bc = 0;
+    int32_t net = 0, nreb = 0;
+    const int64_t rcol = (int64_t)blockIdx.x * kP + lane, rstride = (int64_t)gridDim.x * kP;
     for (int32_t c = 0; c < chunks; ++c) {
         const int b = c % kBuffers;
         named_sync(kFullR + b, kResThreads + 32);
+        if constexpr (kRel) {
+            // Raise the base of every plan whose end nears 2^32, all lanes at
+            // once (a rare, whole-warp pass over the plan's slots).
+            if (__any_sync(0xFFFFFFFFu, live && !ovf && end > kRebaseAt)) {
+                uint32_t m = 0xFFFFFFFFu;
+                if (live && !ovf)
+                    for (int32_t d = 0; d < D; ++d) m = min(m, tfree[d * kP]);
+                const uint32_t dl = live && !ovf && m > kRebaseMin ? m - 1 : 0u;
+                if (dl) {
+                    for (int32_t w = 0; w < W; ++w) {  // session slots
+                        const uint32_t v = slots.get(w);
+                        uint64_t *r = dp.rel_ret + (int64_t)w * rstride + rcol;
+                        const uint64_t x = v && v <= dl ? base + v : 0ull;
+                        *r = nreb ? max(*r, x) : x;
+                        slots.set(w, v > dl ? v - dl : 0u);
+                    }
+                    for (int32_t k = W; k < dp.nslots + 2; ++k) {
+                        const uint32_t v = slots.get(k);
+                        slots.set(k, v > dl ? v - dl : 0u);
+                    }
+                    for (int32_t d = 0; d < D; ++d) tfree[d * kP] -= dl;
+                    end -= dl;
+                    gsum -= (int64_t)net * dl;
+                    base += dl;
+                    bc = base < 0xFFFFFFFFull ? (uint32_t)base : 0xFFFFFFFFu;
+                    ++nreb;
+                }
+            }
+        }
         const uint2 *rb = ring + b * kRW * kChunk * kPitch + lane;
         const int32_t kmax = min(kChunk, N - c * kChunk);
         if (live) {
@@ -865,7 +943,8 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
                 for (int x = 0; x < 3; ++x) nw[x] = rb[(x * kChunk + kn) * kPitch];
                 const uint32_t r3 = w[1].y;
                 if (!(r3 & kSkip)) {
-                    const uint32_t run = w[0].x, arr = w[0].y, r4 = w[2].x, r5 = w[2].y;
+                    const uint32_t run = w[0].x, arr = kRel ? max(w[0].y, bc) - bc : w[0].y, r4 = w[2].x,
+                                   r5 = w[2].y;
                     const uint32_t ld = kPhi ? w[1].x & 0x7FFFFFFFu : w[1].x;  // bit 31: a reload (kPhi)
                     TT *tf_d = tfree + (r3 & 31u) * kP;
                     // Release (Eq. 2, Eq. 7); an accumulator slot is reset by its reader.
@@ -891,8 +970,14 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
                     if (kNarrow) ovf |= (le < ls) | (cfin < start);
                     else ovf |= run == kRunCap;
                     end = max(end, cfin);
-                    if (r3 & kWasEmpty) gsum -= (int64_t)ls;   // an empty device becomes occupied
-                    if (r3 & kEmptied) gsum += (int64_t)cfin;  // the device empties after the unit
+                    if (r3 & kWasEmpty) {  // an empty device becomes occupied
+                        gsum -= (int64_t)ls;
+                        if (kRel) --net;
+                    }
+                    if (r3 & kEmptied) {  // the device empties after the unit
+                        gsum += (int64_t)cfin;
+                        if (kRel) ++net;
+                    }
 
                     publish<TT>(slots, r3 >> 16, cfin);  // the sink when the unit writes nothing
                     publish<TT>(slots, r4 & 0xFFFFu, cfin);
@@ -927,6 +1012,23 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
     } else if (live && ovf) {  // handed to the next path
         const int32_t kk = atomicAdd(ovf_count, 1);
         ovf_list[kk] = (int32_t)p;
+    } else if (live && kRel) {
+        // Back to absolute times: the session latencies as 64-bit values in
+        // slot pairs (written from the last session down, so that no pair
+        // overwrites a session slot not yet read).
+        const int64_t nopen = open[lane];
+        const uint64_t eabs = base + end;
+        const PairArr<kP> lat{(uint32_t *)(sm + L.slots) + lane};
+        for (int32_t w = W - 1; w >= 0; --w) {
+            const uint32_t v = slots.get(w);
+            uint64_t cw = v ? base + v : 0ull;
+            if (nreb) cw = max(cw, dp.rel_ret[(int64_t)w * rstride + rcol]);
+            lat.set(w, cw - arrival[w]);
+        }
+        const int32_t rank = (int32_t)((95 * (int64_t)W + 99) / 100 - 1);
+        out.makespan_us[p] = (int64_t)eabs - dp.first_arrival;
+        out.gpu_us[p] = gsum + (int64_t)net * (int64_t)base + nopen * (int64_t)eabs;
+        out.p95_us[p] = (int64_t)select_slots<uint64_t>(lat, W, rank);
     } else if (live) {
         const int64_t nopen = open[lane];
         for (int32_t w = 0; w < W; ++w) slots.set(w, slots.get(w) - arrival[w]);  // session completion latency
@@ -1849,6 +1951,13 @@ bool sweep_usable(const wf_dev_problem &dp)
 // is least recently used.
 bool split40(const wf_dev_problem &dp) { return dp.horizon < ((int64_t)1 << 40) && dp.reclaim == 0; }
 
+// The relative-time sweep: least recently used, no window terms, and room
+// for the sessions' 64-bit latencies in slot pairs at the end of a plan.
+bool rel32(const wf_dev_problem &dp)
+{
+    return sweep_usable(dp) && dp.reclaim == 0 && !dp.phi_life && 2 * (int64_t)dp.W <= (int64_t)dp.nslots + 2;
+}
+
 template <typename Q, typename TT, int kP, int kR, bool kF, typename ST = TT>
 int launch_pc(const wf_dev_problem &dp, int sms, int resident, const wf_plans *pl, const wf_eval_out *out,
               size_t smem, const int32_t *in_list, const int32_t *in_count, int32_t *list, int32_t *count, cudaStream_t st)
@@ -1925,6 +2034,60 @@ int resident(const wf_dev_problem &dp, int kp, size_t smem)
     if (dp.phi_life)
         return dp.reclaim ? resident_r<TT, 1, true>(dp, kp, smem) : resident_r<TT, 0, true>(dp, kp, smem);
     return dp.reclaim ? resident_r<TT, 1, false>(dp, kp, smem) : resident_r<TT, 0, false>(dp, kp, smem);
+}
+
+// The relative-time sweep's shapes: 16 or 6 plans per CTA.
+template <typename F>
+int rel_visit(const wf_dev_problem &dp, int kp, F &&f)
+{
+    auto by_q = [&](auto p) {
+        return dp.M <= 8 ? f(Ty<uint32_t>{}, p) : f(Ty<uint64_t>{}, p);
+    };
+    return kp == 16 ? by_q(Iv<16>{}) : by_q(Iv<6>{});
+}
+
+int resident_rel(const wf_dev_problem &dp, int kp, size_t smem)
+{
+    if (smem > 227 * 1024) return 0;
+    return rel_visit(dp, kp, [&](auto q, auto p) {
+        const auto k = pc_kernel<typename decltype(q)::type, uint32_t, decltype(p)::value, 0, false, Rel32>;
+        int n = 0;
+        if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess ||
+            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k, 32 * PcShape<decltype(p)::value>::kWarps, smem) !=
+                cudaSuccess) {
+            (void)cudaGetLastError();
+            return 0;
+        }
+        return n;
+    });
+}
+
+// Every plan of the batch, in at most as many CTAs as are resident at once
+// and as the evaluation scratch holds session rows for (each CTA walks
+// over groups); the plans that leave 32 bits go to list.
+int64_t rel_blocks(const wf_ctx *ctx, const wf_sweep_cfg &cfg, int64_t P)
+{
+    if (!cfg.smemRel) return 0;
+    const int kp = cfg.plansRel;
+    const int64_t rows = (int64_t)(ctx->eval_scratch_bytes / (8 * (size_t)std::max(ctx->dp.W, 1)));
+    return std::min<int64_t>(std::min<int64_t>((P + kp - 1) / kp, (int64_t)std::max(1, cfg.resRel) * ctx->sms),
+                             rows / kp);
+}
+
+int launch_rel(wf_ctx *ctx, const wf_sweep_cfg &cfg, int64_t blocks, const wf_plans *pl, const wf_eval_out *out,
+               int32_t *list, int32_t *count, cudaStream_t st)
+{
+    wf_dev_problem dp = ctx->dp;
+    dp.rel_ret = (uint64_t *)ctx->eval_scratch;
+    return rel_visit(dp, cfg.plansRel, [&](auto q, auto p) {
+        const auto k = pc_kernel<typename decltype(q)::type, uint32_t, decltype(p)::value, 0, false, Rel32>;
+        int rc = wf_cuda_check(cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cfg.smemRel),
+                               "sweep smem attribute");
+        if (rc) return rc;
+        k<<<(unsigned)blocks, 32 * PcShape<decltype(p)::value>::kWarps, cfg.smemRel, st>>>(dp, *pl, *out, nullptr,
+                                                                                           nullptr, list, count);
+        return wf_cuda_check(cudaGetLastError(), "sweep launch");
+    });
 }
 
 template <typename TT>
@@ -2006,6 +2169,27 @@ wf_sweep_cfg choose(const wf_dev_problem &dp)
             c.res64 = n;
         }
     }
+    // The relative-time sweep (for contexts whose plans leave 32 bits): 6 or
+    // 16 plans per CTA, whichever keeps more plans resident per SM; ties go
+    // to the smaller CTA, whose timing warp (the chain that paces the sweep)
+    // has fewer plans to play (large window: 6-plan CTAs 72.7 ms, 8-plan CTAs
+    // at the same 24 plans per SM 78.0 ms).
+    if (c.smem64 && rel32(dp)) {
+        const int rshapes[2] = {6, 16};
+        int rbest = 0;
+        for (int kp : rshapes) {
+            const int32_t NS = dp.nslots + 2;
+            const size_t sm = kp == 16 ? pc_layout<16, uint32_t, 0, false, Rel32>(dp.D, dp.M, dp.W, NS).total
+                                       : pc_layout<6, uint32_t, 0, false, Rel32>(dp.D, dp.M, dp.W, NS).total;
+            const int n = resident_rel(dp, kp, sm);
+            if (n > 0 && kp * n > rbest) {
+                rbest = kp * n;
+                c.smemRel = sm;
+                c.plansRel = kp;
+                c.resRel = n;
+            }
+        }
+    }
     return c;
 }
 
@@ -2040,7 +2224,14 @@ int wf_launch_sweep(wf_ctx *ctx, const wf_plans *pl, const wf_eval_out *out, con
     int rc = launch_status(ctx, pl, out, st, ctx->dp.reclaim != 0);
     if (!rc && ctx->dp.reclaim) rc = wf_launch_nextuse(ctx, pl, out, st);
     if (rc) return rc;
-    if (cfg.smem32 && !(wide_first && cfg.smem64)) {
+    const int64_t rblocks = wide_first && ctx->start_path != WF_PATH_WIDE ? rel_blocks(ctx, cfg, pl->P) : 0;
+    if (rblocks > 0) {
+        // Relative u32 times for every plan; the plans that leave 32 bits
+        // even so go on to the u64 sweep.
+        rc = launch_rel(ctx, cfg, rblocks, pl, out, list1, counts, st);
+        if (!rc) rc = launch_pc_q<uint64_t>(ctx, cfg.plans64, cfg.res64, pl, out, cfg.smem64, list1, counts, list2,
+                                            counts + 1, st);
+    } else if (cfg.smem32 && !(wide_first && cfg.smem64)) {
         // u32 times for every plan; the plans that leave 32 bits go on to the
         // u64 sweep, and from there (or straight) to the int64 path.
         rc = launch_pc_q<uint32_t>(ctx, kPlans32, cfg.res32, pl, out, cfg.smem32, nullptr, nullptr, list1, counts, st);

@@ -223,11 +223,13 @@ def wf_ctx_status(ctx: Ctx, stream=None):
     _check(load_library().wf_ctx_status(ctx.ptr, _stream_handle(stream)), "wf_ctx_status")
 
 
-PATH_AUTO, PATH_INT64 = 0, 1
+PATH_AUTO, PATH_INT64, PATH_WIDE, PATH_RELATIVE = 0, 1, 2, 3
 
 
 def wf_ctx_set_eval_path(ctx: Ctx, path: int):
-    """PATH_AUTO (the sweeps) or PATH_INT64 (every plan on the exact int64 path)."""
+    """PATH_AUTO (the sweeps), PATH_INT64 (every plan on the exact int64 path),
+    PATH_WIDE (every plan starts in the 64-bit sweep) or PATH_RELATIVE (in the
+    sweep with 32-bit times relative to a per-plan base)."""
     _check(load_library().wf_ctx_set_eval_path(ctx.ptr, int(path)), "wf_ctx_set_eval_path")
 
 
