@@ -20,11 +20,14 @@
 //
 // Times: the deterministic sweep first plays u32 times and lists a plan whose
 // times reach 2^32 us; a second instantiation with u64 times plays the listed
-// plans (or, once a context has seen most plans leave 32 bits, the whole
-// batch), with 16, 6 or 3 plans per CTA by occupancy and finish slots of 40
-// bits (a u32 word and a byte) while no time can reach 2^40 us.  Only a unit
-// whose summed run time saturates 32 bits goes on to the exact int64 path in
-// wf_eval.cu, as does a stochastic plan whose times leave 32 bits.
+// plans, with 16, 6 or 3 plans per CTA by occupancy and finish slots of 40
+// bits (a u32 word and a byte) while no time can reach 2^40 us.  Once a
+// context has seen most plans leave 32 bits, a third instantiation (Rel32)
+// plays the whole batch on u32 times counted from a per-plan base that rises
+// with the plan's devices' free times, and lists for the u64 sweep only what
+// leaves 32 bits even so.  Only a unit whose summed run time saturates 32
+// bits goes on to the exact int64 path in wf_eval.cu, as does a stochastic
+// plan whose times leave 32 bits.
 //
 // A compile-time variant (kPhi) also returns the window terms of Eq. 12's
 // ranking key: residency marks a reload (a model its device held before) in
