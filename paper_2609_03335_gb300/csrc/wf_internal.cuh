@@ -100,8 +100,9 @@ struct wf_ctx {
     int32_t *ovf_list;          // [max_P] the u32 sweep's hand-offs (and the stochastic sweep's)
     int32_t *ovf_list2;         // [max_P] plans for the int64 path
     // Path choice from an earlier call: when more than half of a batch left
-    // 32 bits, later calls start with the u64 sweep.  The count is read back
-    // through pinned memory and an event, never waited for.
+    // 32 bits, later calls start past the u32 sweep (the relative sweep, or
+    // the u64 one).  The count is read back through pinned memory and an
+    // event, never waited for.
     bool prefer_wide;
     bool wide_pending;
     int64_t wide_P;
