@@ -604,25 +604,34 @@ int wf_launch_eval(wf_ctx *ctx, const wf_plans *plans, const wf_eval_out *out, c
                 }
             }
             const bool wide_first = (ctx->prefer_wide || ctx->start_path >= WF_PATH_WIDE) && cfg.smem64;
-            int rc = wf_cuda_check(cudaMemsetAsync(ctx->ovf_count, 0, 2 * sizeof(int32_t), st), "reset overflow counts");
+            // Two pairs of counts, taken by calls in turn, so that a call
+            // issued before an earlier call's read-back has run does not
+            // reset the count it reads; a call that comes back to a pair
+            // whose read-back is still pending waits for that copy first.
+            const int q = capturing ? ctx->ovf_pair : (ctx->ovf_pair ^= 1);
+            int32_t *counts = ctx->ovf_count + 2 * q;
+            int rc = WF_OK;
+            if (!capturing && ctx->wide_pending && ctx->rb_pair == q)
+                rc = wf_cuda_check(cudaStreamWaitEvent(st, ctx->ovf_event, 0), "overflow read-back wait");
+            if (!rc) rc = wf_cuda_check(cudaMemsetAsync(counts, 0, 2 * sizeof(int32_t), st), "reset overflow counts");
             const int32_t *rest = nullptr, *rest_count = nullptr;
-            if (!rc) rc = wf_launch_sweep(ctx, plans, out, cfg, wide_first, ctx->ovf_count, ctx->ovf_list,
-                                          ctx->ovf_list2, st, &rest, &rest_count);
+            if (!rc) rc = wf_launch_sweep(ctx, plans, out, cfg, wide_first, counts, ctx->ovf_list, ctx->ovf_list2, st,
+                                          &rest, &rest_count);
             if (rc) return rc;
             if (cfg.smem32 && !wide_first && !ctx->wide_pending && !capturing) {
                 // The read-back runs on the context's side stream after the
-                // sweeps, so the caller's stream never waits for it.  A later
-                // call may reset the count before the copy runs; the value
-                // only picks the path, never a result.
+                // sweeps, so the caller's stream never waits for it; the
+                // value only picks the path, never a result.
                 rc = wf_cuda_check(cudaEventRecord(ctx->sweep_done, st), "sweep event");
                 if (!rc) rc = wf_cuda_check(cudaStreamWaitEvent(ctx->side, ctx->sweep_done, 0), "side stream wait");
-                if (!rc) rc = wf_cuda_check(cudaMemcpyAsync(ctx->h_ovf, ctx->ovf_count, sizeof(int32_t),
+                if (!rc) rc = wf_cuda_check(cudaMemcpyAsync(ctx->h_ovf, counts, sizeof(int32_t),
                                                             cudaMemcpyDeviceToHost, ctx->side),
                                             "overflow count read-back");
                 if (!rc) rc = wf_cuda_check(cudaEventRecord(ctx->ovf_event, ctx->side), "overflow count event");
                 if (rc) return rc;
                 ctx->wide_pending = true;
                 ctx->wide_P = plans->P;
+                ctx->rb_pair = q;
             }
             eval_list_kernel<<<(unsigned)blocks, kEvalThreads, 0, st>>>(dp, *plans, *out, scratch,
                                                                        ctx->eval_row_bytes, units,

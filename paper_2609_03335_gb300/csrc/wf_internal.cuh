@@ -96,7 +96,8 @@ struct wf_ctx {
     int sms;                    // streaming multiprocessors of the device
     bool force_int64;           // wf_ctx_set_eval_path(WF_PATH_INT64): every plan on the int64 path
     int32_t start_path;         // wf_ctx_set_eval_path's value (WF_PATH_WIDE / RELATIVE: the first sweep)
-    int32_t *ovf_count;         // [2]: plans the u32 sweep hands on, plans left for the int64 path
+    int32_t *ovf_count;         // [2]: plans the u32 sweep hands on, plans left for the int64 path (the sweep
+                                // calls use words 0-1 and 2-3 in turn)
     int32_t *ovf_list;          // [max_P] the u32 sweep's hand-offs (and the stochastic sweep's)
     int32_t *ovf_list2;         // [max_P] plans for the int64 path
     // Path choice from an earlier call: when more than half of a batch left
@@ -106,6 +107,8 @@ struct wf_ctx {
     bool prefer_wide;
     bool wide_pending;
     int64_t wide_P;
+    int ovf_pair;               // the pair of ovf_count words the last sweep call used (0 or 1)
+    int rb_pair;                // the pair whose count the pending read-back copies
     void *search_scratch;       // local search: the union's results [max_P], top-k ids, slot pairs
     void *construct_scratch;    // plan constructor: per-plan state of the plans built at once, allocated by its first call
     int64_t construct_threads;  // plans built at once (a warp each)
