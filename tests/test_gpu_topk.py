@@ -1,7 +1,7 @@
 """Top-k on synthetic result arrays, on both of its paths (one CTA up to
 16,384 plans, per-tile thresholds beyond): ties within and across tiles,
-invalid plans, a short last tile, and k up to its limit.  The keys are written straight into the
-result arrays, so only the top-k kernels run."""
+invalid plans, a short last tile, and k up to its limit.  The keys are written straight into the result
+arrays, so only the top-k kernels run."""
 import numpy as np
 import pytest
 
@@ -74,6 +74,7 @@ def test_all_plans_invalid_and_tied():
 @pytest.mark.parametrize("P,k", [
     (1, 1), (63, 5), (1024, 1024), (1025, 1024), (1025, 1), (2049, 683),
     (16383, 128), (16384, 128), (16384, 129), (16384, 32), (9000, 200),
+    (31, 31), (32, 32), (33, 32), (1024, 32), (1025, 32), (2048, 17), (5000, 32), (16384, 1), (16383, 31),
 ])
 def test_single_cta_batches(P, k):
     """Batches up to the single-CTA limit, k from 1 to P: ties and invalid
