@@ -904,25 +904,39 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
         const int b = c % kBuffers;
         named_sync(kFullR + b, kResThreads + 32);
         if constexpr (kRel) {
-            // Raise the base of every plan whose end nears 2^32, all lanes at
-            // once (a rare, whole-warp pass over the plan's slots).
+            // Raise the base of every plan whose end nears 2^32.  The whole
+            // warp walks the CTA's slot words ([slot][plan], 32 at a time,
+            // word x of plan x % kP), each lowered by its plan's rise.
             if (__any_sync(0xFFFFFFFFu, live && !ovf && end > kRebaseAt)) {
                 uint32_t m = 0xFFFFFFFFu;
                 if (live && !ovf)
                     for (int32_t d = 0; d < D; ++d) m = min(m, tfree[d * kP]);
                 const uint32_t dl = live && !ovf && m > kRebaseMin ? m - 1 : 0u;
+                uint32_t *sw = (uint32_t *)(sm + L.slots);
+                __syncwarp();  // every lane's slot writes are seen by the others
+                const int32_t nw = W * kP, nall = (dp.nslots + 2) * kP;
+                for (int32_t x0 = 0; x0 < nw; x0 += 32) {  // session slots: keep what falls below the base
+                    const int32_t x = x0 + lane, q = x % kP;
+                    const uint32_t dq = __shfl_sync(0xFFFFFFFFu, dl, q);
+                    const uint64_t bq = __shfl_sync(0xFFFFFFFFu, base, q);
+                    const int32_t rq = __shfl_sync(0xFFFFFFFFu, nreb, q);
+                    if (x < nw && dq) {
+                        const uint32_t v = sw[x];
+                        uint64_t *r = dp.rel_ret + (int64_t)(x / kP) * rstride + (int64_t)blockIdx.x * kP + q;
+                        const uint64_t keep = v && v <= dq ? bq + v : 0ull;
+                        *r = rq ? max(*r, keep) : keep;
+                        sw[x] = v > dq ? v - dq : 0u;
+                    }
+                }
+                for (int32_t x0 = nw; x0 < nall; x0 += 32) {
+                    const int32_t x = x0 + lane;
+                    const uint32_t dq = __shfl_sync(0xFFFFFFFFu, dl, x % kP);
+                    if (x < nall && dq) {
+                        const uint32_t v = sw[x];
+                        sw[x] = v > dq ? v - dq : 0u;
+                    }
+                }
                 if (dl) {
-                    for (int32_t w = 0; w < W; ++w) {  // session slots
-                        const uint32_t v = slots.get(w);
-                        uint64_t *r = dp.rel_ret + (int64_t)w * rstride + rcol;
-                        const uint64_t x = v && v <= dl ? base + v : 0ull;
-                        *r = nreb ? max(*r, x) : x;
-                        slots.set(w, v > dl ? v - dl : 0u);
-                    }
-                    for (int32_t k = W; k < dp.nslots + 2; ++k) {
-                        const uint32_t v = slots.get(k);
-                        slots.set(k, v > dl ? v - dl : 0u);
-                    }
                     for (int32_t d = 0; d < D; ++d) tfree[d * kP] -= dl;
                     end -= dl;
                     gsum -= (int64_t)net * dl;
@@ -930,6 +944,7 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
                     bc = base < 0xFFFFFFFFull ? (uint32_t)base : 0xFFFFFFFFu;
                     ++nreb;
                 }
+                __syncwarp();
             }
         }
         const uint2 *rb = ring + b * kRW * kChunk * kPitch + lane;
