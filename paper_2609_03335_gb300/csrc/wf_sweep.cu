@@ -203,6 +203,10 @@ struct IsRel<Rel32> {
 constexpr uint32_t kRebaseAt = 3u << 30;   // a plan's end above this raises its base ...
 constexpr uint32_t kRebaseMin = 1u << 28;  // ... by at least this much, else not at all
 
+// Up to this many sessions the timing lane selects its plan's p95 itself;
+// beyond, a warp per plan does after the sweep (warp_select).
+constexpr int32_t kLaneSelect = 32;
+
 template <typename ST>
 struct SlotBytes {
     static constexpr uint32_t kLo = sizeof(ST), kHi = 0;
@@ -303,27 +307,7 @@ __device__ __forceinline__ void named_arrive(int id, int threads)
     asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(threads) : "memory");
 }
 
-// r-th smallest (0-based) of the kS-strided values v[0], v[kS], ...
-template <typename TT, int kS>
-__device__ TT select_strided(TT *v, int32_t n, int32_t r)
-{
-    int32_t lo = 0, hi = n - 1;
-    while (lo < hi) {
-        const TT pivot = v[(lo + (hi - lo) / 2) * kS];
-        int32_t i = lo, j = hi;
-        while (i <= j) {
-            while (v[i * kS] < pivot) ++i;
-            while (v[j * kS] > pivot) --j;
-            if (i <= j) { TT t = v[i * kS]; v[i * kS] = v[j * kS]; v[j * kS] = t; ++i; --j; }
-        }
-        if (r <= j) hi = j;
-        else if (r >= i) lo = i;
-        else return v[r * kS];
-    }
-    return v[r * kS];
-}
-
-// The same over slots 0 .. n-1 of a slot array.
+// The r-th smallest (0-based) of slots 0 .. n-1 of a slot array (one thread).
 template <typename TT, typename SA>
 __device__ TT select_slots(const SA &v, int32_t n, int32_t r)
 {
@@ -341,6 +325,80 @@ __device__ TT select_slots(const SA &v, int32_t n, int32_t r)
         else return v.get(r);
     }
     return v.get(r);
+}
+
+// The same by a whole warp.  The p95's rank is near the top (the
+// (n - r)-th largest: 4th of 64, 13th of 256), so the warp takes maxima: the
+// largest value below the last maximum and how many equal it, until the
+// count reaches n - r.  For a rank further down, a radix selection from the
+// highest bit set in any value, each bit decided by a ballot.  Up to 32
+// kCache values are read once into registers (a column of the slot array is
+// a strided read with bank conflicts); more are read again for every step.
+template <int kCache, typename SA, typename F>
+__device__ __forceinline__ void each_value(const SA &a, int32_t n, bool cached, const uint64_t (&c)[kCache], F &&f)
+{
+    const int lane = threadIdx.x & 31;
+    if (cached) {
+#pragma unroll
+        for (int j = 0; j < kCache; ++j)
+            if (32 * j < n) f(c[j], 32 * j + lane < n);
+    } else {
+        for (int32_t i0 = 0; i0 < n; i0 += 32) {
+            const int32_t i = i0 + lane;
+            f(i < n ? (uint64_t)a.get(i) : 0ull, i < n);
+        }
+    }
+}
+
+template <typename SA>
+__device__ uint64_t warp_select(const SA &a, int32_t n, int32_t r)
+{
+    constexpr int kCache = 8;
+    constexpr int32_t kMaxSteps = 32;
+    const int lane = threadIdx.x & 31;
+    const bool cached = n <= 32 * kCache;
+    uint64_t c[kCache];  // the values, 0 beyond n (never above the answer when taking maxima)
+#pragma unroll
+    for (int j = 0; j < kCache; ++j) {
+        const int32_t i = 32 * j + lane;
+        c[j] = cached && i < n ? (uint64_t)a.get(i) : 0ull;
+    }
+    if (n - r <= kMaxSteps) {
+        int32_t need = n - r;  // the need-th largest of the values below thr
+        uint64_t thr = ~0ull;
+        for (;;) {
+            uint64_t mx = 0;
+            each_value(a, n, cached, c, [&](uint64_t v, bool) {
+                if (v < thr) mx = max(mx, v);
+            });
+            const uint32_t hi = __reduce_max_sync(0xFFFFFFFFu, (uint32_t)(mx >> 32));
+            const uint32_t lo = __reduce_max_sync(0xFFFFFFFFu, (uint32_t)(mx >> 32) == hi ? (uint32_t)mx : 0u);
+            const uint64_t m = ((uint64_t)hi << 32) | lo;
+            int32_t cnt = 0;
+            each_value(a, n, cached, c, [&](uint64_t v, bool in) {
+                cnt += __popc(__ballot_sync(0xFFFFFFFFu, in && v == m));
+            });
+            if (cnt >= need) return m;
+            need -= cnt;
+            thr = m;
+        }
+    }
+    uint64_t any = 0;
+    each_value(a, n, cached, c, [&](uint64_t v, bool) { any |= v; });
+    any = ((uint64_t)__reduce_or_sync(0xFFFFFFFFu, (uint32_t)(any >> 32)) << 32) |
+          __reduce_or_sync(0xFFFFFFFFu, (uint32_t)any);
+    uint64_t prefix = 0;
+    for (int bit = any ? 63 - __clzll((long long)any) : -1; bit >= 0; --bit) {
+        int32_t zeros = 0;  // values that match prefix above bit and have a 0 there
+        each_value(a, n, cached, c, [&](uint64_t v, bool in) {
+            zeros += __popc(__ballot_sync(0xFFFFFFFFu, in && ((v ^ prefix) >> bit) == 0));
+        });
+        if (r >= zeros) {
+            r -= zeros;
+            prefix |= 1ull << bit;
+        }
+    }
+    return prefix;
 }
 
 // Two extra slots follow a plan's nslots slots: a sink that absorbs writes
@@ -608,6 +666,7 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
     extern __shared__ __align__(128) uint8_t sm[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int32_t N = dp.N, D = dp.D, M = dp.M, W = dp.W;
+    const int32_t rank = (int32_t)((95 * (int64_t)W + 99) / 100 - 1);  // the p95's nearest rank (Section 4.2)
     const PcLayout L = pc_layout<kP, TT, kReclaim, kPhi, ST>(D, M, W, dp.nslots + 2);
     const int64_t total = in_list ? (int64_t)*in_count : pl.P;
     if ((int64_t)blockIdx.x * kP >= total) return;  // the whole CTA: no plan
@@ -1043,22 +1102,43 @@ pc_kernel(wf_dev_problem dp, wf_plans pl, wf_eval_out out, const int32_t *in_lis
             if (nreb) cw = max(cw, dp.rel_ret[(int64_t)w * rstride + rcol]);
             lat.set(w, cw - arrival[w]);
         }
-        const int32_t rank = (int32_t)((95 * (int64_t)W + 99) / 100 - 1);
         out.makespan_us[p] = (int64_t)eabs - dp.first_arrival;
         out.gpu_us[p] = gsum + (int64_t)net * (int64_t)base + nopen * (int64_t)eabs;
-        out.p95_us[p] = (int64_t)select_slots<uint64_t>(lat, W, rank);
+        if (W <= kLaneSelect) out.p95_us[p] = (int64_t)select_slots<uint64_t>(lat, W, rank);
     } else if (live) {
         const int64_t nopen = open[lane];
         for (int32_t w = 0; w < W; ++w) slots.set(w, slots.get(w) - arrival[w]);  // session completion latency
-        const int32_t rank = (int32_t)((95 * (int64_t)W + 99) / 100 - 1);
         out.makespan_us[p] = (int64_t)end - dp.first_arrival;
         out.gpu_us[p] = gsum + nopen * (int64_t)end;
-        out.p95_us[p] = (int64_t)select_slots<TT>(slots, W, rank);
+        if (W <= kLaneSelect) out.p95_us[p] = (int64_t)select_slots<TT>(slots, W, rank);
         if (kPhi) {
             dp.phi_timely[p] = ph_timely;
             dp.phi_life[p] = (int64_t)ph_life;
         }
     }
+    // A plan whose p95 is still to be selected (more than kLaneSelect sessions).
+    if (mine) open[lane] = live && !bad && !ovf && W > kLaneSelect;
+    }
+    __syncthreads();  // every stage is done with the group
+    // The p95 of every plan played to the end with more than kLaneSelect
+    // sessions (Section 4.2, nearest rank): the whole CTA, a warp per plan,
+    // over the session latencies the timing stage left in the plan's slots.
+    for (int q = warp; q < kP && W > kLaneSelect; q += S::kWarps) {
+        if (!open[q]) continue;
+        uint64_t v;
+        if constexpr (kRel) {
+            v = warp_select(PairArr<kP>{(uint32_t *)(sm + L.slots) + q}, W, rank);
+        } else {
+            SlotArr<TT, ST, kP> sq;
+            if constexpr (SlotBytes<ST>::kHi) {
+                sq.lo = (uint32_t *)(sm + L.slots) + q;
+                sq.hi = sm + L.slots_hi + q;
+            } else {
+                sq.v = (TT *)(sm + L.slots) + q;
+            }
+            v = warp_select(sq, W, rank);
+        }
+        if (lane == 0) out.p95_us[in_list ? (int64_t)in_list[j0 + q] : j0 + q] = (int64_t)v;
     }
     __syncthreads();  // the group's shared state is free for the next group
   }

@@ -443,3 +443,27 @@ def test_admission_margin(seed):
     assert_same(got, want)
     rel, comp = oracle.forecast(prob)
     assert np.array_equal(got["rel"], rel) and np.array_equal(got["comp"], comp)
+
+
+@pytest.mark.parametrize("n_sessions,path", [(33, "auto"), (70, "auto"), (256, "auto"), (300, "auto"),
+                                             (70, "wide"), (300, "wide"), (70, "relative"), (300, "relative")])
+def test_many_sessions_p95(n_sessions, path):
+    """More than 32 sessions: a warp per plan selects the p95 after the sweep
+    (up to 256 latencies held in registers, more read from shared memory for
+    every bit), on each sweep; equal latencies from sessions with equal
+    shapes and arrivals."""
+    wf = lib()
+    rng = np.random.default_rng(6100 + n_sessions)
+    prob = random_problem(rng, n_sessions=n_sessions, sizes=(4, 6), D=4, M=3, arrivals=n_sessions % 2 == 0)
+    if path == "relative":
+        lat = (prob.lat_us.astype(np.int64) % 1000 + (1 << 26)).astype(np.int32)
+        prob = prob.with_(lat_us=lat)
+    plans = wfgen.make_plans(prob, 400, n_sessions, p_retain=0.5)
+    inject_invalid(plans, prob, rng)
+    want = oracle_eval(prob, plans)
+    ctx = wf.Ctx(prob, max_P=plans.P)
+    if path != "auto":
+        wf.wf_ctx_set_eval_path(ctx, wf.PATH_RELATIVE if path == "relative" else wf.PATH_WIDE)
+    for _ in range(2):
+        assert_same(gpu_eval(prob, plans, k=8, ctx=ctx), want)
+    ctx.close()
