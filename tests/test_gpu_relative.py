@@ -3,8 +3,10 @@ times relative to a per-plan base (PATH_RELATIVE) and in the 64-bit sweep
 (PATH_WIDE), against the oracle.  The cases cover bases raised while
 sessions still arrive (arrivals up to 4e9 us), sessions that finish long
 before their plan ends, devices that empty and fill again (retain rows),
-invalid plans, and plans that leave 32 bits even so (one device left idle
-keeps the base at zero; a fused chain's summed run saturates)."""
+invalid plans, and the plans that leave 32 bits even so (a device left idle
+keeps a plan's base at zero; a fused chain's summed run time of 2^32 or more
+sends its plan to the int64 path), whichever of those the random windows
+produce."""
 import numpy as np
 import pytest
 
