@@ -283,33 +283,67 @@ def test_int64_path_matches_oracle(name):
     assert_same(got, oracle_eval(w.problem, plans))
 
 
-def test_times_beyond_u32_take_the_int64_path():
+def _eval_on_path(prob, plans, k, path):
+    wf = lib()
+    ctx = wf.Ctx(prob, max_P=plans.P)
+    if path != "auto":
+        wf.wf_ctx_set_eval_path(ctx, wf.PATH_RELATIVE if path == "relative" else wf.PATH_WIDE)
+    got = gpu_eval(prob, plans, k=k, ctx=ctx)
+    ctx.close()
+    return got
+
+
+@pytest.mark.parametrize("path", ["auto", "wide", "relative"])
+def test_times_beyond_u32_take_the_int64_path(path):
     """Run times near 2^30 us make every makespan exceed 2^32 us; those plans
-    must still match the oracle exactly."""
+    must still match the oracle exactly, started in any sweep."""
     rng = np.random.default_rng(31)
     prob = random_problem(rng, n_sessions=5, sizes=(6, 10), D=3, M=3)
     lat = (prob.lat_us.astype(np.int64) % 1000 + (1 << 30) - 5000).astype(np.int32)
     prob = prob.with_(lat_us=lat)
     plans = wfgen.make_plans(prob, 300, 3, p_retain=0.5)
-    got = gpu_eval(prob, plans, k=10)
+    got = _eval_on_path(prob, plans, 10, path)
     want = oracle_eval(prob, plans)
     assert (want["makespan"][want["status"] == 0] >= (1 << 32)).all()
     assert_same(got, want)
 
 
-def test_fused_run_time_beyond_u32():
+@pytest.mark.parametrize("path", ["auto", "wide", "relative"])
+def test_fused_run_time_beyond_u32(path):
     """Fused chains of near-2^31 us members: a unit's summed run time alone
-    leaves 32 bits, with a start of 0 on some plans."""
+    leaves 32 bits, with a start of 0 on some plans; started in any sweep."""
     rng = np.random.default_rng(43)
     prob = random_problem(rng, n_sessions=3, sizes=(6, 9), D=2, M=2)
     lat = np.full(prob.N * prob.D, (1 << 31) - 1, np.int32)
     prob = prob.with_(lat_us=lat, arrival_us=np.zeros(prob.W, np.int64),
                       load_us=np.zeros_like(prob.load_us), grant_us=0)
     plans = wfgen.make_plans(prob, 300, 8, p_fuse=0.95)
-    got = gpu_eval(prob, plans, k=4)
+    got = _eval_on_path(prob, plans, 4, path)
     want = oracle_eval(prob, plans)
     assert (want["makespan"][want["status"] == 0] >= (1 << 32)).all()
     assert_same(got, want)
+
+
+def test_relative_sweep_with_an_idle_device():
+    """Plans that leave a device unused keep their base at zero in the
+    relative sweep (the smallest free time is that device's 0), so their times
+    leave 32 bits and go on to the 64-bit sweep; the others rebase."""
+    wf = lib()
+    rng = np.random.default_rng(59)
+    prob = random_problem(rng, n_sessions=8, sizes=(8, 14), D=3, M=3, tight=False)
+    lat = (prob.lat_us.astype(np.int64) % 1000 + (1 << 27)).astype(np.int32)
+    prob = prob.with_(lat_us=lat, peak_mib=np.minimum(prob.peak_mib, np.repeat(prob.cap_mib[None, :], prob.N, 0)
+                                                      .reshape(-1)).astype(np.int32))
+    plans = wfgen.make_plans(prob, 400, 21, p_retain=0.5)
+    plans.place[::2, :prob.N] %= 2  # every other plan on devices 0 and 1 only
+    want = oracle_eval(prob, plans)
+    ok = want["status"] == 0
+    assert ok[::2].sum() > 100 and (want["makespan"][ok] >= 1 << 32).mean() > 0.9
+    ctx = wf.Ctx(prob, max_P=plans.P)
+    wf.wf_ctx_set_eval_path(ctx, wf.PATH_RELATIVE)
+    for _ in range(2):
+        assert_same(gpu_eval(prob, plans, k=8, ctx=ctx), want)
+    ctx.close()
 
 
 def test_horizon_beyond_2_40_uses_8_byte_slots():
